@@ -1,0 +1,185 @@
+/*
+ * pf16 -- pure-FP16 ResNet-50 training kernels for NVIDIA GB300 (sm_103a).
+ *
+ * The library implements the hot path of "Distributed low-precision Training
+ * Without Mixed Precision" (arXiv 1911.07384): ResNet-50 trained with every
+ * activation, weight and gradient stored in IEEE binary16 and every
+ * arithmetic operation done in binary16, with no FP32 master copy of any
+ * parameter (Sec. 5.2) and with the x0.25 scaling after each BatchNorm of a
+ * residual block (Sec. 4.2).  Convolutions accumulate in FP16 inside the
+ * tensor cores (tcgen05, FP16 accumulators in tensor memory).
+ *
+ * Conventions shared by every entry point
+ *  - Tensors are dense binary16 bit patterns (uint16_t) in DEVICE memory,
+ *    owned and allocated by the caller.  Activations are NHWC (C innermost),
+ *    convolution weights KRSC.  Every tensor pointer must be 16-byte aligned.
+ *  - Calls are asynchronous and stream-ordered on `stream` (a cudaStream_t;
+ *    NULL = the legacy default stream).  The library never allocates or frees
+ *    memory and keeps no tensors between calls; scratch memory is the
+ *    caller's `ws` buffer, sized by the matching *_workspace_size function.
+ *    Calls on distinct streams may run concurrently; calls that share a
+ *    workspace must be ordered by the caller.
+ *  - Every argument is validated on the host before anything is launched; an
+ *    invalid call returns a negative status and launches nothing.
+ *  - Device-side waits are bounded; one that runs out records PF16_ERR_TIMEOUT
+ *    in a device status word, read (and cleared) by pf16_sync_status.
+ *  - Rounding: IEEE roundTiesToEven for every binary16 operation, subnormals
+ *    kept (no flush to zero), never a fused multiply-add unless stated.
+ */
+#ifndef PF16_H
+#define PF16_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---------------------------------------------------------------- status */
+enum {
+  PF16_OK = 0,
+  PF16_ERR_NULL = -1,        /* a required pointer is NULL */
+  PF16_ERR_ALIGN = -2,       /* a tensor pointer is not 16-byte aligned */
+  PF16_ERR_SHAPE = -3,       /* non-positive, inconsistent or too-large sizes */
+  PF16_ERR_UNSUPPORTED = -4, /* well-formed but outside what the kernels cover */
+  PF16_ERR_WORKSPACE = -5,   /* workspace NULL or smaller than required */
+  PF16_ERR_CUDA = -6,        /* a CUDA runtime or driver call failed */
+  PF16_ERR_TIMEOUT = -7,     /* a bounded device-side wait expired */
+  PF16_ERR_ARG = -8          /* invalid flag, phase or enum value */
+};
+
+/* ----------------------------------------------------------------- flags */
+#define PF16_ACCUMULATE 0x1u  /* conv: out = rn(out + result) instead of out = result */
+#define PF16_BN_RELU 0x1u     /* BN: apply ReLU to the output */
+#define PF16_BN_RESIDUAL 0x2u /* BN: add the residual tensor before the ReLU */
+
+/* ------------------------------------------------------------ convolution
+ * Convolution of the ResNet-50 layers (Sec. 5.1) in pure FP16 (Sec. 5.2):
+ * dilation 1, one group, the same stride and padding on both axes.
+ *   x  [n][h][w][c]    input activations (NHWC)
+ *   w  [k][r][s][c]    weights (KRSC)
+ *   y  [n][p][q][k]    output, p = (h + 2 pad - r)/stride + 1, q likewise
+ * Supported: c and k multiples of 64 (any n, h, w), or c == 3 with k == 64
+ * (the ResNet-50 stem; its 7x7 patches are staged through the workspace),
+ * or h == w == r == s == 1 with c a multiple of 64 and k a multiple of 8
+ * (the fully connected layer).  r, s <= 7; stride 1 or 2; pad < r. */
+typedef struct {
+  int32_t n, h, w, c, k, r, s, stride, pad;
+} pf16_conv_desc;
+
+#define PF16_PASS_FWD 0
+#define PF16_PASS_DGRAD 1
+#define PF16_PASS_WGRAD 2
+
+/* Bytes of workspace the given pass needs (0 if none).  Returns 0 for an
+ * invalid descriptor as well; the call then reports the error. */
+size_t pf16_conv_workspace_size(const pf16_conv_desc* d, int pass);
+
+/* Forward: y[n,p,q,k] = sum_{r,s,c} x[n, p*st+r-pad, q*st+s-pad, c] * w[k,r,s,c]
+ * (zero outside x).  FP16 products, FP16 accumulation in the tensor core,
+ * FP16 result.  flags: PF16_ACCUMULATE. */
+int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                  void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
+/* Data gradient: dx[n,h,w,c] = sum over the (k,r,s) with h+pad-r = p*st and
+ * w+pad-s = q*st in range of dy[n,p,q,k] * w[k,r,s,c]; stride 2 is split into
+ * its stride-phase sub-problems, so no zero-insertion work is done.  Every
+ * element of dx is written (zeros included) unless PF16_ACCUMULATE, in which
+ * case dx = rn(dx + result) and positions no tap reaches are left unchanged.
+ * Not available for c == 3 (the stem needs no input gradient). */
+int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
+/* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*st+r-pad, q*st+s-pad, c].
+ * The reduction over n*p*q pixels is split into chunks, each accumulated in
+ * FP16 by the tensor core into FP16 partials in the workspace, which are then
+ * summed by a balanced pairwise FP16 tree.  flags must be 0. */
+int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream);
+
+/* ------------------------------------------------------------------- SGD
+ * One step of SGD with momentum and coupled weight decay, the PyTorch
+ * ImageNet recipe the paper adopts (Sec. 5.1), done entirely in FP16 with no
+ * master copy (Sec. 5.2).  In place on w[n] and v[n] (the momentum buffer,
+ * start it at +0), gradient g[n]; lr, momentum and wd are binary16 bit
+ * patterns.  Per element, each op rounded once to binary16, no FMA:
+ *   g' = rn(g + rn(wd*w))   (skipped entirely when wd is +0)
+ *   v  = rn(rn(momentum*v) + g')
+ *   w  = rn(w - rn(lr*v))
+ * flags must be 0.  n may be 0 (nothing is launched). */
+int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
+                    uint16_t momentum, uint16_t wd, uint32_t flags, void* stream);
+
+/* ------------------------------------------------------------- BatchNorm
+ * BatchNorm with batch statistics over the n*h*w rows of each of c channels
+ * (Eq. 1, Eq. 2), each output then multiplied by post_scale (0x3400 = 0.25
+ * inside residual blocks, 0x3C00 = 1 for the stem, Sec. 4.2), optionally
+ * plus a residual tensor and followed by ReLU (flags).  All arithmetic FP16:
+ * the mean and the (biased, two-pass) variance are balanced pairwise
+ * "halving" trees (each node rn(rn(a+b) * 0.5) over zero-padded power-of-two
+ * leaves, scaled once by the padding ratio), so no partial sum can overflow.
+ *   phase 0 (forward, training):  reads x, gamma, beta[, residual];
+ *       writes y, mean, invstd (per channel, saved for the backward).
+ *   phase 1 (backward): reads x, gamma, mean, invstd, dy[, y_saved when
+ *       PF16_BN_RELU]; writes dx, dgamma, dbeta and, if non-NULL, dresidual
+ *       (= dy masked by ReLU, the gradient flowing to the residual input).
+ * c must be a multiple of 8 and at most 2048. */
+typedef struct {
+  int32_t n, h, w, c;
+  uint16_t eps;        /* binary16 bits, e.g. 0x00A8 (1e-5, subnormal) */
+  uint16_t post_scale; /* binary16 bits */
+  uint32_t flags;      /* PF16_BN_RELU | PF16_BN_RESIDUAL */
+} pf16_bn_desc;
+
+typedef struct {
+  const uint16_t *x, *gamma, *beta, *residual, *dy, *y_saved;
+  uint16_t *y, *mean, *invstd, *dx, *dgamma, *dbeta, *dresidual;
+} pf16_bn_tensors;
+
+size_t pf16_bn_workspace_size(const pf16_bn_desc* d);
+int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, void* ws,
+                    size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------- rest of the train step
+ * The remaining ops of the ResNet-50 training step (Sec. 5.1), all FP16. */
+
+/* 3x3 max pooling, stride 2, padding 1 (padding never wins), NHWC. */
+int pf16_maxpool_fwd(const uint16_t* x, uint16_t* y, int32_t n, int32_t h, int32_t w, int32_t c,
+                     void* stream);
+/* Backward: each window's gradient goes to the first cell (scan r then s)
+ * holding the window maximum; a cell's contributions are added in FP16 in
+ * window order.  Writes every element of dx. */
+int pf16_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int32_t n, int32_t h,
+                     int32_t w, int32_t c, void* stream);
+/* Global average pooling: y[n][c] = mean over hw pixels (halving tree). */
+int pf16_avgpool_fwd(const uint16_t* x, uint16_t* y, int32_t n, int32_t hw, int32_t c,
+                     void* stream);
+/* Backward: dx[n][i][c] = rn(dy[n][c] * rn(1/hw)). */
+int pf16_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int32_t n, int32_t hw, int32_t c,
+                     void* stream);
+
+/* Softmax cross-entropy on logits[b][k] + bias[k] (bias may be NULL) with
+ * int32 labels[b] in [0, k): loss (one binary16 scalar, mean over the batch),
+ * dlogits[b][k] = (softmax - onehot) / b and dbias[k] = sum_b dlogits (if
+ * non-NULL).  k <= 4096; the workspace holds per-row losses. */
+size_t pf16_softmax_xent_workspace_size(int32_t b, int32_t k);
+int pf16_softmax_xent(const uint16_t* logits, const uint16_t* bias, const int32_t* labels,
+                      int32_t b, int32_t k, uint16_t* loss, uint16_t* dlogits, uint16_t* dbias,
+                      void* ws, size_t ws_bytes, void* stream);
+
+/* --------------------------------------------------------------- status
+ * Waits for `stream`, then returns and clears the device status word of the
+ * current device: PF16_OK, PF16_ERR_TIMEOUT after a bounded wait ran out, or
+ * PF16_ERR_CUDA if the stream itself reports an error. */
+int pf16_sync_status(void* stream);
+/* Static, human-readable text for a status code. */
+const char* pf16_status_string(int status);
+/* Compute capability major*10+minor of the current device, or a negative
+ * status if no device is usable.  The kernels need 103 (sm_103a). */
+int pf16_device_arch(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PF16_H */

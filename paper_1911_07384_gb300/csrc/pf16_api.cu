@@ -1,0 +1,760 @@
+// C-ABI of libpf16 (declared in include/pf16.h): argument validation, the
+// per-call plan of each convolution pass (tile width, split-K, stride phases),
+// TMA tensor-map encoding and kernel dispatch.  Nothing here allocates device
+// memory; every call is asynchronous on the caller's stream.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/pf16.h"
+#include "pf16_internal.h"
+#include "pf16_ptx.cuh"
+
+namespace pf16 {
+
+// Device status word: bounded device waits that expire record PF16_ERR_TIMEOUT here.
+__device__ int g_pf16_status = 0;
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+typedef CUresult (*EncodeIm2colFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const int*, const int*,
+                                   cuuint32_t, cuuint32_t, const cuuint32_t*,
+                                   CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+std::once_flag g_fn_once;
+EncodeTiledFn g_encode_tiled = nullptr;
+EncodeIm2colFn g_encode_im2col = nullptr;
+
+bool driver_fns() {
+  std::call_once(g_fn_once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode_tiled = reinterpret_cast<EncodeTiledFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode_im2col = reinterpret_cast<EncodeIm2colFn>(p);
+  });
+  return g_encode_tiled && g_encode_im2col;
+}
+
+constexpr int kMaxDevices = 64;
+std::mutex g_dev_mu;
+int* g_status_ptr[kMaxDevices] = {nullptr};
+int g_num_sms[kMaxDevices] = {0};
+
+// Per-device constants: status-word address and SM count.
+int device_consts(int** status, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return PF16_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_pf16_status) != cudaSuccess) return PF16_ERR_CUDA;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return PF16_ERR_CUDA;
+    g_status_ptr[dev] = static_cast<int*>(p);
+    g_num_sms[dev] = n;
+  }
+  *status = g_status_ptr[dev];
+  *sms = g_num_sms[dev];
+  return PF16_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+// 2-D tiled map over a row-major [rows][cols] FP16 matrix with row stride ld (elements).
+bool map_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld,
+            uint32_t box_cols, uint32_t box_rows) {
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return g_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 3-D tiled map: dims (d0 contiguous, d1, d2) with byte strides s1, s2.
+bool map_3d(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
+            uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2) {
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1, s2};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t es[3] = {1, 1, 1};
+  return g_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// im2col map over an NHWC tensor.  The bounding box of filter-corner positions
+// starts at (lo_h, lo_w) and holds gh x gw points at `step`; each load yields
+// `pixels` consecutive grid points x 64 channels.
+bool map_im2col(CUtensorMap* m, const void* base, int N, int H, int W, int C, int lo_h, int lo_w,
+                int gh, int gw, int step, int pixels) {
+  const int up_h = lo_h + (gh - 1) * step - (H - 1);
+  const int up_w = lo_w + (gw - 1) * step - (W - 1);
+  if (lo_h < -128 || lo_h > 127 || lo_w < -128 || lo_w > 127 || up_h < -128 || up_h > 127 ||
+      up_w < -128 || up_w > 127)
+    return false;
+  cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+  int lower[2] = {lo_w, lo_h};
+  int upper[2] = {up_w, up_h};
+  cuuint32_t es[4] = {1, (cuuint32_t)step, (cuuint32_t)step, 1};
+  return g_encode_im2col(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(base), dims,
+                         strides, lower, upper, 64, (cuuint32_t)pixels, es,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ---------------------------------------------------------------- conv plans
+enum ConvKind { KIND_GENERIC = 0, KIND_STEM = 1, KIND_FC = 2 };
+
+struct Shape {
+  long long N, H, W, C, K, R, S, st, pad, P, Q;
+  ConvKind kind;
+};
+
+int conv_shape(const pf16_conv_desc* d, Shape* s) {
+  if (!d) return PF16_ERR_NULL;
+  if (d->n <= 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->k <= 0 || d->r <= 0 || d->s <= 0 ||
+      d->pad < 0 || d->stride <= 0)
+    return PF16_ERR_SHAPE;
+  if (d->stride > 2 || d->r > 7 || d->s > 7 || d->pad >= std::max(d->r, d->s))
+    return PF16_ERR_UNSUPPORTED;
+  s->N = d->n;
+  s->H = d->h;
+  s->W = d->w;
+  s->C = d->c;
+  s->K = d->k;
+  s->R = d->r;
+  s->S = d->s;
+  s->st = d->stride;
+  s->pad = d->pad;
+  if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s) return PF16_ERR_SHAPE;
+  s->P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+  s->Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+  const long long lim = (1ll << 31) - 1;
+  if (s->N * s->H * s->W * s->C > lim * 8 || s->N * s->P * s->Q > lim / 2 ||
+      s->N * s->H * s->W > lim / 2 || s->K * s->R * s->S * s->C > lim)
+    return PF16_ERR_SHAPE;
+  if (d->c == 3) {
+    if (d->k % 64 != 0) return PF16_ERR_UNSUPPORTED;
+    s->kind = KIND_STEM;
+  } else if (d->h == 1 && d->w == 1 && d->r == 1 && d->s == 1 && d->pad == 0 && d->stride == 1) {
+    if (d->c % 64 != 0 || d->k % 8 != 0) return PF16_ERR_UNSUPPORTED;
+    s->kind = KIND_FC;
+  } else {
+    if (d->c % 64 != 0 || d->k % 64 != 0) return PF16_ERR_UNSUPPORTED;
+    s->kind = KIND_GENERIC;
+  }
+  return PF16_OK;
+}
+
+int pick_bn_out(long long n) {  // tile width for an output of n columns
+  if (n <= 64) return 64;
+  if (n <= 128) return 128;
+  if (n % 256 == 0 || n > 192) return 256;
+  return 192;
+}
+int pick_bn_wgrad(long long n) {
+  if (n % 256 == 0) return 256;
+  if (n % 192 == 0) return 192;
+  if (n % 128 == 0) return 128;
+  if (n <= 64) return 64;
+  return n <= 192 ? 192 : 256;
+}
+
+long long stem_kcol(const Shape& s) { return (long long)round_up((size_t)(s.R * s.S * s.C), 8); }
+
+struct WgradSplit {
+  int bn, m_tiles, n_tiles, num_kb, kb_per_split, splits;
+  long long ncols;  // GEMM N
+};
+
+// Split-K plan of the weight gradient.  Independent of the device so that
+// pf16_conv_workspace_size and the call always agree: about two units of work
+// per SM of a 152-SM GB300, at least 4 and at most 64 K-blocks (4096 pixels)
+// accumulated in one FP16 tensor-memory accumulator, at most 1024 splits.
+constexpr int kWgradTargetUnits = 2 * 152;
+
+WgradSplit wgrad_split(const Shape& s) {
+  WgradSplit w;
+  w.ncols = s.kind == KIND_STEM ? stem_kcol(s) : s.R * s.S * s.C;
+  w.bn = pick_bn_wgrad(w.ncols);
+  w.m_tiles = cdiv(s.K, kBM);
+  w.n_tiles = cdiv(w.ncols, w.bn);
+  w.num_kb = cdiv(s.N * s.P * s.Q, kBK);
+  const int units = w.m_tiles * w.n_tiles;
+  int splits = std::max(1, cdiv(kWgradTargetUnits, units));
+  int kps = std::max(4, cdiv(w.num_kb, splits));
+  kps = std::min(kps, 64);  // at most 4096 pixels accumulated in one FP16 accumulator
+  w.kb_per_split = std::min(kps, w.num_kb);
+  w.splits = cdiv(w.num_kb, w.kb_per_split);
+  if (w.splits > 1024) {
+    w.kb_per_split = cdiv(w.num_kb, 1024);
+    w.splits = cdiv(w.num_kb, w.kb_per_split);
+  }
+  return w;
+}
+
+size_t ws_fwd(const Shape& s) {
+  if (s.kind != KIND_STEM) return 0;
+  const long long kc = stem_kcol(s);
+  return round_up((size_t)(s.N * s.P * s.Q * kc * 2), 256) + round_up((size_t)(s.K * kc * 2), 256);
+}
+size_t ws_wgrad(const Shape& s) {
+  const WgradSplit w = wgrad_split(s);
+  size_t b = 0;
+  if (w.splits > 1 || s.kind == KIND_STEM) b += round_up((size_t)w.splits * s.K * w.ncols * 2, 256);
+  if (s.kind == KIND_STEM) b += round_up((size_t)(s.N * s.P * s.Q * w.ncols * 2), 256);
+  return b;
+}
+
+// Taps of one stride phase of the data gradient.  For output row h = st*i + ph
+// the contributing filter rows r satisfy (ph + pad - r) % st == 0 and read dy
+// row i + (ph + pad - r) / st; likewise for columns.
+struct Phase {
+  int gh, gw;           // output grid of the phase
+  int nr, ns;           // contributing filter rows / columns
+  int rr[7], ar[7];     // filter row and dy-row offset
+  int ss[7], bs[7];     // filter column and dy-column offset
+  bool empty() const { return nr == 0 || ns == 0 || gh <= 0 || gw <= 0; }
+};
+
+Phase make_phase(const Shape& s, int ph, int pw) {
+  Phase f;
+  f.gh = (int)((s.H - ph + s.st - 1) / s.st);
+  f.gw = (int)((s.W - pw + s.st - 1) / s.st);
+  f.nr = f.ns = 0;
+  for (int r = 0; r < s.R; ++r) {
+    const long long t = ph + s.pad - r;
+    if (((t % s.st) + s.st) % s.st == 0) {
+      f.rr[f.nr] = r;
+      f.ar[f.nr++] = (int)(t >= 0 ? t / s.st : -((-t) / s.st));
+    }
+  }
+  for (int c = 0; c < s.S; ++c) {
+    const long long t = pw + s.pad - c;
+    if (((t % s.st) + s.st) % s.st == 0) {
+      f.ss[f.ns] = c;
+      f.bs[f.ns++] = (int)(t >= 0 ? t / s.st : -((-t) / s.st));
+    }
+  }
+  return f;
+}
+
+void set_kmajor(GemmParams& p, bool a, bool b) {
+  if (a) {
+    p.a_lbo = 16;
+    p.a_sbo = 1024;
+    p.a_kstep = 32;
+  }
+  if (b) {
+    p.b_lbo = 16;
+    p.b_sbo = 1024;
+    p.b_kstep = 32;
+  }
+}
+void set_mnmajor(GemmParams& p, bool a, bool b) {
+  if (a) {
+    p.a_lbo = 8192;
+    p.a_sbo = 1024;
+    p.a_kstep = 2048;
+  }
+  if (b) {
+    p.b_lbo = 8192;
+    p.b_sbo = 1024;
+    p.b_kstep = 2048;
+  }
+}
+
+GemmParams base_params(int* status) {
+  GemmParams p;
+  memset(&p, 0, sizeof(p));
+  p.kb_per_split = 1 << 30;
+  p.splits = 1;
+  p.status = status;
+  p.wait_limit_ns = 4000000000ull;
+  return p;
+}
+
+int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int sms,
+        cudaStream_t st) {
+  p.m_tiles = cdiv(p.M, kBM);
+  p.n_tiles = cdiv(p.N, BN);
+  if (p.splits == 1) p.kb_per_split = p.num_kb;
+  p.idesc = idesc_f16(kBM, BN, p.a_mode == LD_TILED_MN,
+                      p.b_mode == LD_TILED_MN || p.b_mode == LD_IM2COL_MN || p.b_mode == LD_TAP3D_MN,
+                      false);
+  const long long units = (long long)p.m_tiles * p.n_tiles * p.splits;
+  if (units <= 0 || p.num_kb <= 0) return PF16_OK;
+  const int grid = (int)std::min<long long>(units, sms);
+  return launch_gemm(BN, a, b, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
+int check_common(const void* a, const void* b, const void* c) {
+  if (!a || !b || !c) return PF16_ERR_NULL;
+  if (!aligned16(a) || !aligned16(b) || !aligned16(c)) return PF16_ERR_ALIGN;
+  return PF16_OK;
+}
+
+}  // namespace
+}  // namespace pf16
+
+using namespace pf16;
+
+extern "C" {
+
+size_t pf16_conv_workspace_size(const pf16_conv_desc* d, int pass) {
+  Shape s;
+  if (conv_shape(d, &s) != PF16_OK) return 0;
+  if (pass == PF16_PASS_FWD) return ws_fwd(s);
+  if (pass == PF16_PASS_DGRAD) return 0;
+  if (pass == PF16_PASS_WGRAD) return ws_wgrad(s);
+  return 0;
+}
+
+int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                  void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  Shape s;
+  int rc = conv_shape(d, &s);
+  if (rc != PF16_OK) return rc;
+  if ((rc = check_common(x, w, y)) != PF16_OK) return rc;
+  if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  const size_t need = ws_fwd(s);
+  if (need && (!ws || ws_bytes < need)) return PF16_ERR_WORKSPACE;
+  if (need && !aligned16(ws)) return PF16_ERR_ALIGN;
+  if (!driver_fns()) return PF16_ERR_CUDA;
+  int* status;
+  int sms;
+  if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  GemmParams p = base_params(status);
+  CUtensorMap ma, mb;
+  p.M = (int)(s.N * s.P * s.Q);
+  p.N = (int)s.K;
+  p.out = y;
+  p.ldo = s.K;
+  p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
+  const int BN = pick_bn_out(s.K);
+  p.a_mode = LD_TILED_K;
+  p.b_mode = LD_TILED_K;
+  set_kmajor(p, true, true);
+  if (s.kind == KIND_STEM) {
+    const long long kc = stem_kcol(s);
+    uint16_t* col = static_cast<uint16_t*>(ws);
+    uint16_t* wpad = col + round_up((size_t)(p.M * kc * 2), 256) / 2;
+    if (launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
+                           (int)s.S, (int)s.C, (int)s.st, (int)s.pad, (int)kc, st) != cudaSuccess)
+      return PF16_ERR_CUDA;
+    if (launch_pad_rows(w, wpad, (int)s.K, (int)(s.R * s.S * s.C), (int)kc, st) != cudaSuccess)
+      return PF16_ERR_CUDA;
+    if (!map_2d(&ma, col, kc, p.M, kc, 64, kBM) || !map_2d(&mb, wpad, kc, s.K, kc, 64, BN))
+      return PF16_ERR_CUDA;
+    p.num_kb = cdiv(kc, kBK);
+  } else {
+    const bool dense = s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0;
+    if (dense) {
+      if (!map_2d(&ma, x, s.C, s.N * s.H * s.W, s.C, 64, kBM)) return PF16_ERR_CUDA;
+    } else {
+      p.a_mode = LD_IM2COL_K;
+      p.ga = PixGrid{(int)s.P, (int)s.Q, (int)s.st, (int)-s.pad, (int)-s.pad};
+      if (!map_im2col(&ma, x, (int)s.N, (int)s.H, (int)s.W, (int)s.C, (int)-s.pad, (int)-s.pad,
+                      (int)s.P, (int)s.Q, (int)s.st, kBM))
+        return PF16_ERR_CUDA;
+      p.ntaps = (int)(s.R * s.S);
+      for (int r = 0; r < s.R; ++r)
+        for (int c = 0; c < s.S; ++c) {
+          p.tap_dr[r * s.S + c] = (int8_t)r;
+          p.tap_ds[r * s.S + c] = (int8_t)c;
+          p.tap_w[r * s.S + c] = (int8_t)(r * s.S + c);
+        }
+      p.a_cpt = (int)(s.C / 64);
+    }
+    if (!map_2d(&mb, w, s.R * s.S * s.C, s.K, s.R * s.S * s.C, 64, BN)) return PF16_ERR_CUDA;
+    p.num_kb = (int)(s.R * s.S * s.C / 64);
+  }
+  return run(BN, ma, mb, p, sms, st);
+}
+
+int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  Shape s;
+  int rc = conv_shape(d, &s);
+  if (rc != PF16_OK) return rc;
+  if (s.kind == KIND_STEM) return PF16_ERR_UNSUPPORTED;
+  if ((rc = check_common(dy, w, dx)) != PF16_OK) return rc;
+  if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  if (!driver_fns()) return PF16_ERR_CUDA;
+  int* status;
+  int sms;
+  if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const bool accum = (flags & PF16_ACCUMULATE) != 0;
+  const int BN = pick_bn_out(s.C);
+  const size_t dx_elems = (size_t)(s.N * s.H * s.W * s.C);
+
+  if (s.R == 1 && s.S == 1 && s.pad == 0) {
+    // 1x1: dx[n, st*p, st*q, :] = dy[n,p,q,:] . w ; other positions receive nothing
+    GemmParams p = base_params(status);
+    CUtensorMap ma, mb;
+    p.M = (int)(s.N * s.P * s.Q);
+    p.N = (int)s.C;
+    p.a_mode = LD_TILED_K;
+    p.b_mode = LD_TILED_MN;
+    set_kmajor(p, true, false);
+    set_mnmajor(p, false, true);
+    if (!map_2d(&ma, dy, s.K, s.N * s.P * s.Q, s.K, 64, kBM) ||
+        !map_2d(&mb, w, s.C, s.K, s.C, 64, 64))
+      return PF16_ERR_CUDA;
+    p.num_kb = cdiv(s.K, kBK);
+    p.out = dx;
+    p.ldo = s.C;
+    p.out_mode = accum ? OUT_ACCUM : OUT_STORE;
+    if (s.st != 1) {
+      if (!accum && launch_fill_zero(dx, dx_elems, st) != cudaSuccess) return PF16_ERR_CUDA;
+      p.remap = 1;
+      p.rm_gh = (int)s.P;
+      p.rm_gw = (int)s.Q;
+      p.rm_H = (int)s.H;
+      p.rm_W = (int)s.W;
+      p.rm_step = (int)s.st;
+    }
+    return run(BN, ma, mb, p, sms, st);
+  }
+
+  // R x S filters: one implicit GEMM per stride phase (ph, pw); positions no
+  // phase reaches are zero-filled first (unless accumulating).
+  bool any_empty = false;
+  for (int ph = 0; ph < s.st; ++ph)
+    for (int pw = 0; pw < s.st; ++pw) any_empty |= make_phase(s, ph, pw).empty();
+  if (any_empty && !accum && launch_fill_zero(dx, dx_elems, st) != cudaSuccess)
+    return PF16_ERR_CUDA;
+  for (int ph = 0; ph < s.st; ++ph)
+    for (int pw = 0; pw < s.st; ++pw) {
+      const Phase f = make_phase(s, ph, pw);
+      if (f.empty()) continue;
+      const int gh = f.gh, gw = f.gw, nr = f.nr, ns = f.ns;
+      const int *ar = f.ar, *bs = f.bs, *rr = f.rr, *ss = f.ss;
+      const int amin = *std::min_element(ar, ar + nr), bmin = *std::min_element(bs, bs + ns);
+      GemmParams p = base_params(status);
+      CUtensorMap ma, mb;
+      p.M = (int)(s.N * gh * gw);
+      p.N = (int)s.C;
+      p.a_mode = LD_IM2COL_K;
+      p.b_mode = LD_TAP3D_MN;
+      set_kmajor(p, true, false);
+      set_mnmajor(p, false, true);
+      p.ga = PixGrid{gh, gw, 1, amin, bmin};
+      if (!map_im2col(&ma, dy, (int)s.N, (int)s.P, (int)s.Q, (int)s.K, amin, bmin, gh, gw, 1, kBM))
+        return PF16_ERR_CUDA;
+      if (!map_3d(&mb, w, s.C, s.R * s.S, s.K, s.C * 2, s.R * s.S * s.C * 2, 64, 1, 64))
+        return PF16_ERR_CUDA;
+      p.ntaps = nr * ns;
+      for (int i = 0; i < nr; ++i)
+        for (int j = 0; j < ns; ++j) {
+          p.tap_dr[i * ns + j] = (int8_t)(ar[i] - amin);
+          p.tap_ds[i * ns + j] = (int8_t)(bs[j] - bmin);
+          p.tap_w[i * ns + j] = (int8_t)(rr[i] * s.S + ss[j]);
+        }
+      p.a_cpt = p.b_cpt = (int)(s.K / 64);
+      p.num_kb = p.ntaps * p.a_cpt;
+      p.out = dx;
+      p.ldo = s.C;
+      p.out_mode = accum ? OUT_ACCUM : OUT_STORE;
+      p.remap = (s.st != 1) ? 1 : 0;
+      p.rm_gh = gh;
+      p.rm_gw = gw;
+      p.rm_H = (int)s.H;
+      p.rm_W = (int)s.W;
+      p.rm_step = (int)s.st;
+      p.rm_ph = ph;
+      p.rm_pw = pw;
+      if ((rc = run(BN, ma, mb, p, sms, st)) != PF16_OK) return rc;
+    }
+  return PF16_OK;
+}
+
+int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  Shape s;
+  int rc = conv_shape(d, &s);
+  if (rc != PF16_OK) return rc;
+  if ((rc = check_common(x, dy, dw)) != PF16_OK) return rc;
+  if (flags != 0) return PF16_ERR_ARG;
+  int* status;
+  int sms;
+  if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
+  const size_t need = ws_wgrad(s);
+  if (need && (!ws || ws_bytes < need)) return PF16_ERR_WORKSPACE;
+  if (need && !aligned16(ws)) return PF16_ERR_ALIGN;
+  if (!driver_fns()) return PF16_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WgradSplit wsp = wgrad_split(s);
+
+  GemmParams p = base_params(status);
+  CUtensorMap ma, mb;
+  const long long pixels = s.N * s.P * s.Q;
+  p.M = (int)s.K;
+  p.N = (int)wsp.ncols;
+  p.num_kb = wsp.num_kb;
+  p.splits = wsp.splits;
+  p.kb_per_split = wsp.kb_per_split;
+  p.a_mode = LD_TILED_MN;
+  set_mnmajor(p, true, true);
+  if (!map_2d(&ma, dy, s.K, pixels, s.K, 64, 64)) return PF16_ERR_CUDA;
+  uint16_t* parts = static_cast<uint16_t*>(ws);
+  const bool partial = wsp.splits > 1 || s.kind == KIND_STEM;
+  if (s.kind == KIND_STEM) {
+    uint16_t* col = parts + round_up((size_t)wsp.splits * s.K * wsp.ncols * 2, 256) / 2;
+    if (launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
+                           (int)s.S, (int)s.C, (int)s.st, (int)s.pad, (int)wsp.ncols,
+                           st) != cudaSuccess)
+      return PF16_ERR_CUDA;
+    p.b_mode = LD_TILED_MN;
+    if (!map_2d(&mb, col, wsp.ncols, pixels, wsp.ncols, 64, 64)) return PF16_ERR_CUDA;
+  } else if (s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0) {
+    p.b_mode = LD_TILED_MN;
+    if (!map_2d(&mb, x, s.C, pixels, s.C, 64, 64)) return PF16_ERR_CUDA;
+  } else {
+    p.b_mode = LD_IM2COL_MN;
+    p.gb = PixGrid{(int)s.P, (int)s.Q, (int)s.st, (int)-s.pad, (int)-s.pad};
+    if (!map_im2col(&mb, x, (int)s.N, (int)s.H, (int)s.W, (int)s.C, (int)-s.pad, (int)-s.pad,
+                    (int)s.P, (int)s.Q, (int)s.st, 64))
+      return PF16_ERR_CUDA;
+    p.ntaps = (int)(s.R * s.S);
+    for (int r = 0; r < s.R; ++r)
+      for (int c = 0; c < s.S; ++c) {
+        p.tap_dr[r * s.S + c] = (int8_t)r;
+        p.tap_ds[r * s.S + c] = (int8_t)c;
+      }
+    p.b_cin = (int)s.C;
+    p.b_oob_c = (int)round_up((size_t)s.C, 64);
+  }
+  if (partial) {
+    p.out = parts;
+    p.ldo = wsp.ncols;
+    p.out_mode = OUT_PARTIAL;
+  } else {
+    p.out = dw;
+    p.ldo = wsp.ncols;
+    p.out_mode = OUT_STORE;
+  }
+  if ((rc = run(wsp.bn, ma, mb, p, sms, st)) != PF16_OK) return rc;
+  if (partial) {
+    const long long rsc = s.R * s.S * s.C;
+    if (launch_splitk_reduce(parts, wsp.splits, s.K, (int)wsp.ncols, dw, rsc, (int)rsc, st) !=
+        cudaSuccess)
+      return PF16_ERR_CUDA;
+  }
+  return PF16_OK;
+}
+
+int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
+                    uint16_t momentum, uint16_t wd, uint32_t flags, void* stream) {
+  if (flags != 0) return PF16_ERR_ARG;
+  if (n == 0) return PF16_OK;
+  if (!w || !v || !g) return PF16_ERR_NULL;
+  if (!aligned16(w) || !aligned16(v) || !aligned16(g)) return PF16_ERR_ALIGN;
+  return launch_sgd(w, v, g, n, lr, momentum, wd, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+static int bn_validate(const pf16_bn_desc* d, BnLaunch* b) {
+  if (!d) return PF16_ERR_NULL;
+  if (d->n <= 0 || d->h <= 0 || d->w <= 0 || d->c <= 0) return PF16_ERR_SHAPE;
+  if (d->c % 8 != 0 || d->c > 2048) return PF16_ERR_UNSUPPORTED;
+  if (d->flags & ~(uint32_t)(PF16_BN_RELU | PF16_BN_RESIDUAL)) return PF16_ERR_ARG;
+  const long long R = (long long)d->n * d->h * d->w;
+  if (R * d->c > (1ll << 34) || R > (1ll << 31) - 1) return PF16_ERR_SHAPE;
+  bn_plan((int)R, d->c, b);
+  b->eps = d->eps;
+  b->post_scale = d->post_scale;
+  b->relu = (d->flags & PF16_BN_RELU) ? 1 : 0;
+  b->residual = (d->flags & PF16_BN_RESIDUAL) ? 1 : 0;
+  return PF16_OK;
+}
+
+size_t pf16_bn_workspace_size(const pf16_bn_desc* d) {
+  BnLaunch b;
+  if (bn_validate(d, &b) != PF16_OK) return 0;
+  return bn_ws_bytes(b);
+}
+
+int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, void* ws,
+                    size_t ws_bytes, void* stream) {
+  BnLaunch b;
+  int rc = bn_validate(d, &b);
+  if (rc != PF16_OK) return rc;
+  if (!t) return PF16_ERR_NULL;
+  if (phase != 0 && phase != 1) return PF16_ERR_ARG;
+  if (!ws) return PF16_ERR_WORKSPACE;
+  if (ws_bytes < bn_ws_bytes(b)) return PF16_ERR_WORKSPACE;
+  if (!aligned16(ws)) return PF16_ERR_ALIGN;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (phase == 0) {
+    const void* req[] = {t->x, t->gamma, t->beta, t->y, t->mean, t->invstd};
+    for (const void* p : req) {
+      if (!p) return PF16_ERR_NULL;
+      if (!aligned16(p)) return PF16_ERR_ALIGN;
+    }
+    if (b.residual && !t->residual) return PF16_ERR_NULL;
+    if (b.residual && !aligned16(t->residual)) return PF16_ERR_ALIGN;
+    return launch_bn_fwd(b, t->x, t->gamma, t->beta, b.residual ? t->residual : nullptr, t->y,
+                         t->mean, t->invstd, static_cast<uint16_t*>(ws), st) == cudaSuccess
+               ? PF16_OK
+               : PF16_ERR_CUDA;
+  }
+  const void* req[] = {t->x, t->gamma, t->mean, t->invstd, t->dy, t->dx, t->dgamma, t->dbeta};
+  for (const void* p : req) {
+    if (!p) return PF16_ERR_NULL;
+    if (!aligned16(p)) return PF16_ERR_ALIGN;
+  }
+  if (b.relu && !t->y_saved) return PF16_ERR_NULL;
+  if (b.relu && !aligned16(t->y_saved)) return PF16_ERR_ALIGN;
+  if (t->dresidual && !aligned16(t->dresidual)) return PF16_ERR_ALIGN;
+  return launch_bn_bwd(b, t->x, t->gamma, t->mean, t->invstd, t->dy, b.relu ? t->y_saved : nullptr,
+                       t->dx, t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws),
+                       st) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+static int pool_check(const void* a, const void* b, int32_t n, int32_t h, int32_t w, int32_t c) {
+  if (!a || !b) return PF16_ERR_NULL;
+  if (!aligned16(a) || !aligned16(b)) return PF16_ERR_ALIGN;
+  if (n <= 0 || h <= 0 || w <= 0 || c <= 0) return PF16_ERR_SHAPE;
+  if (c % 8 != 0) return PF16_ERR_UNSUPPORTED;
+  if ((long long)n * h * w * c > (1ll << 34)) return PF16_ERR_SHAPE;
+  return PF16_OK;
+}
+
+int pf16_maxpool_fwd(const uint16_t* x, uint16_t* y, int32_t n, int32_t h, int32_t w, int32_t c,
+                     void* stream) {
+  int rc = pool_check(x, y, n, h, w, c);
+  if (rc != PF16_OK) return rc;
+  return launch_maxpool_fwd(x, y, n, h, w, c, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int32_t n, int32_t h,
+                     int32_t w, int32_t c, void* stream) {
+  int rc = pool_check(x, dx, n, h, w, c);
+  if (rc != PF16_OK) return rc;
+  if (!dy) return PF16_ERR_NULL;
+  if (!aligned16(dy)) return PF16_ERR_ALIGN;
+  return launch_maxpool_bwd(x, dy, dx, n, h, w, c, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_avgpool_fwd(const uint16_t* x, uint16_t* y, int32_t n, int32_t hw, int32_t c,
+                     void* stream) {
+  int rc = pool_check(x, y, n, hw, 1, c);
+  if (rc != PF16_OK) return rc;
+  if (hw > 4096) return PF16_ERR_UNSUPPORTED;
+  return launch_avgpool_fwd(x, y, n, hw, c, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int32_t n, int32_t hw, int32_t c,
+                     void* stream) {
+  int rc = pool_check(dy, dx, n, hw, 1, c);
+  if (rc != PF16_OK) return rc;
+  return launch_avgpool_bwd(dy, dx, n, hw, c, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+size_t pf16_softmax_xent_workspace_size(int32_t b, int32_t k) {
+  if (b <= 0 || k <= 0) return 0;
+  return round_up((size_t)b * 2, 256);
+}
+
+int pf16_softmax_xent(const uint16_t* logits, const uint16_t* bias, const int32_t* labels,
+                      int32_t b, int32_t k, uint16_t* loss, uint16_t* dlogits, uint16_t* dbias,
+                      void* ws, size_t ws_bytes, void* stream) {
+  if (!logits || !labels || !loss || !dlogits) return PF16_ERR_NULL;
+  if (b <= 0 || k <= 0 || b > 65535) return PF16_ERR_SHAPE;
+  if (k > 4096) return PF16_ERR_UNSUPPORTED;
+  if (!ws || ws_bytes < pf16_softmax_xent_workspace_size(b, k)) return PF16_ERR_WORKSPACE;
+  return launch_softmax_xent(logits, bias, labels, b, k, loss, dlogits, dbias,
+                             static_cast<uint16_t*>(ws), static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_sync_status(void* stream) {
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return PF16_ERR_CUDA;
+  int* status;
+  int sms;
+  int rc = device_consts(&status, &sms);
+  if (rc != PF16_OK) return rc;
+  int v = 0;
+  if (cudaMemcpy(&v, status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return PF16_ERR_CUDA;
+  if (v != 0) {
+    const int zero = 0;
+    if (cudaMemcpy(status, &zero, sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess)
+      return PF16_ERR_CUDA;
+  }
+  return v;
+}
+
+const char* pf16_status_string(int status) {
+  switch (status) {
+    case PF16_OK: return "ok";
+    case PF16_ERR_NULL: return "a required pointer is NULL";
+    case PF16_ERR_ALIGN: return "a tensor pointer is not 16-byte aligned";
+    case PF16_ERR_SHAPE: return "invalid or inconsistent sizes";
+    case PF16_ERR_UNSUPPORTED: return "sizes or options outside what the kernels support";
+    case PF16_ERR_WORKSPACE: return "workspace missing or too small";
+    case PF16_ERR_CUDA: return "a CUDA runtime or driver call failed";
+    case PF16_ERR_TIMEOUT: return "a bounded device-side wait expired";
+    case PF16_ERR_ARG: return "invalid flag, phase or enum value";
+    default: return "unknown status";
+  }
+}
+
+int pf16_device_arch(void) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return PF16_ERR_CUDA;
+  int maj = 0, min = 0;
+  if (cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&min, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return PF16_ERR_CUDA;
+  return maj * 10 + min;
+}
+
+}  // extern "C"

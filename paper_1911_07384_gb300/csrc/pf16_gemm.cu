@@ -1,0 +1,357 @@
+// tcgen05 implicit-GEMM engine for the pure-FP16 convolutions (forward, data
+// gradient, weight gradient) of the ResNet-50 training step: FP16 operands,
+// FP16 accumulation in tensor memory, FP16 results -- no FP32 anywhere
+// (paper Sec. 5.2: all arithmetic and storage in FP16).
+//
+// One persistent CTA per SM, 6 warps:
+//   warp 0    TMA producer: one elected lane streams 64-wide K-blocks of A
+//             and B into a ring of shared-memory stages (mbarrier full/empty).
+//   warp 1    allocates tensor memory; one lane issues tcgen05.mma
+//             (kind::f16, D = f16, M = 128, N = BN, K = 16) and commits each
+//             stage back to the producer and each finished tile to the
+//             epilogue.  Two TMEM accumulators alternate so the epilogue of
+//             tile i overlaps the MMAs of tile i + 1.
+//   warps 2-5 epilogue: tcgen05.ld of one accumulator row per thread, pack to
+//             FP16, store (or FP16-accumulate, or write a split-K partial).
+// Every mbarrier wait is bounded; on expiry the CTA records PF16_ERR_TIMEOUT
+// and all roles leave their loops, so the kernel always terminates.
+#include <cstdio>
+
+#include "pf16_internal.h"
+#include "pf16_ptx.cuh"
+
+namespace pf16 {
+
+template <int BN>
+struct GemmCfg {
+  static constexpr int A_BYTES = kBM * kBK * 2;
+  static constexpr int B_BYTES = BN * kBK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : (BN == 192 ? 5 : 4));
+  static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES;
+};
+
+static constexpr int kErrTimeout = -7;  // PF16_ERR_TIMEOUT
+
+__device__ __forceinline__ void record_timeout(const GemmParams& p, volatile int* abort_flag) {
+  *abort_flag = 1;
+  atomicCAS(p.status, 0, kErrTimeout);
+}
+
+__device__ __forceinline__ void grid_decompose(int m, const PixGrid& g, int& n, int& i, int& j) {
+  const int per = g.gh * g.gw;
+  n = m / per;
+  const int rem = m - n * per;
+  i = rem / g.gw;
+  j = rem - i * g.gw;
+}
+
+__device__ __forceinline__ void load_a(const GemmParams& p, const CUtensorMap* map, uint32_t dst,
+                                       uint32_t bar, int m0, int kb) {
+  switch (p.a_mode) {
+    case LD_TILED_K:
+      tma_load_2d(dst, map, bar, kb * kBK, m0);
+      break;
+    case LD_TILED_MN:
+      tma_load_2d(dst, map, bar, m0, kb * kBK);
+      tma_load_2d(dst + 8192, map, bar, m0 + 64, kb * kBK);
+      break;
+    case LD_IM2COL_K: {
+      const int tap = kb / p.a_cpt;
+      const int c0 = (kb - tap * p.a_cpt) * 64;
+      int n, i, j;
+      grid_decompose(m0, p.ga, n, i, j);
+      tma_load_im2col_4d(dst, map, bar, c0, j * p.ga.step + p.ga.base_w,
+                         i * p.ga.step + p.ga.base_h, n, (uint16_t)p.tap_ds[tap],
+                         (uint16_t)p.tap_dr[tap]);
+    } break;
+    default:
+      break;
+  }
+}
+
+template <int BN>
+__device__ __forceinline__ void load_b(const GemmParams& p, const CUtensorMap* map, uint32_t dst,
+                                       uint32_t bar, int n0, int kb) {
+  switch (p.b_mode) {
+    case LD_TILED_K:
+      tma_load_2d(dst, map, bar, kb * kBK, n0);
+      break;
+    case LD_TILED_MN:
+#pragma unroll
+      for (int j = 0; j < BN / 64; ++j) tma_load_2d(dst + j * 8192, map, bar, n0 + 64 * j, kb * kBK);
+      break;
+    case LD_IM2COL_MN: {
+      int n, i, jj;
+      grid_decompose(kb * kBK, p.gb, n, i, jj);
+      const int bw = jj * p.gb.step + p.gb.base_w, bh = i * p.gb.step + p.gb.base_h;
+#pragma unroll
+      for (int j = 0; j < BN / 64; ++j) {
+        const int col = n0 + 64 * j;
+        int tap = col / p.b_cin;
+        int c0 = col - tap * p.b_cin;
+        if (tap >= p.ntaps) {  // past the last tap: an all-out-of-bounds box (zeros)
+          tap = 0;
+          c0 = p.b_oob_c;
+        }
+        tma_load_im2col_4d(dst + j * 8192, map, bar, c0, bw, bh, n, (uint16_t)p.tap_ds[tap],
+                           (uint16_t)p.tap_dr[tap]);
+      }
+    } break;
+    case LD_TAP3D_MN: {
+      const int t = kb / p.b_cpt;
+      const int k0 = (kb - t * p.b_cpt) * 64;
+#pragma unroll
+      for (int j = 0; j < BN / 64; ++j) tma_load_3d(dst + j * 8192, map, bar, n0 + 64 * j, p.tap_w[t], k0);
+    } break;
+    default:
+      break;
+  }
+}
+
+__device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0, int& n0, int& split,
+                                            int& kb0, int& kb1, int BN) {
+  const int per = p.m_tiles * p.n_tiles;
+  split = u / per;
+  const int rem = u - split * per;
+  const int mt = rem / p.n_tiles;
+  m0 = mt * kBM;
+  n0 = (rem - mt * p.n_tiles) * BN;
+  kb0 = split * p.kb_per_split;
+  kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+}
+
+__device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int split) {
+  long long row;
+  if (p.out_mode == OUT_PARTIAL) {
+    row = (long long)split * p.M + m;
+  } else if (p.remap) {
+    const int per = p.rm_gh * p.rm_gw;
+    const int n = m / per;
+    const int rem = m - n * per;
+    const int i = rem / p.rm_gw, j = rem - (rem / p.rm_gw) * p.rm_gw;
+    row = ((long long)n * p.rm_H + (long long)(i * p.rm_step + p.rm_ph)) * p.rm_W +
+          (j * p.rm_step + p.rm_pw);
+  } else {
+    row = m;
+  }
+  return p.out + row * p.ldo;
+}
+
+// low halves of two 32-bit TMEM words -> one f16x2
+__device__ __forceinline__ uint32_t pack_lo(uint32_t a, uint32_t b) { return __byte_perm(a, b, 0x5410); }
+
+template <int BN>
+__global__ void __launch_bounds__(192, 1)
+    k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+           const __grid_constant__ GemmParams p) {
+  using Cfg = GemmCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + Cfg::STAGES;
+  uint64_t* tfull = bars + 2 * Cfg::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < Cfg::STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&mapA);
+    tma_prefetch_desc(&mapB);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total = p.m_tiles * p.n_tiles * p.splits;
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
+        int m0, n0, split, kb0, kb1;
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim)) {
+            record_timeout(p, abort_flag);
+            break;
+          }
+          const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
+          load_a(p, &mapA, sa, fb, m0, kb);
+          load_b<BN>(p, &mapB, sa + Cfg::A_BYTES, fb, n0, kb);
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
+        int m0, n0, split, kb0, kb1;
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim)) {
+          record_timeout(p, abort_flag);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        bool ok = true;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, lim)) {
+            record_timeout(p, abort_flag);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
+          const uint32_t sb = sa + Cfg::A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = smem_desc(sa + kk * p.a_kstep, p.a_lbo, p.a_sbo, 2);
+            const uint64_t bd = smem_desc(sb + kk * p.b_kstep, p.b_lbo, p.b_sbo, 2);
+            tc_mma_f16(d_tmem, ad, bd, p.idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(smem_u32(&empty[stage]));
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(&tfull[acc]));
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+    }
+  } else {
+    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1
+    const int sub = warp & 3;
+    const int row = sub * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
+    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      int m0, n0, split, kb0, kb1;
+      unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+      const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) record_timeout(p, abort_flag);
+        break;
+      }
+      tc_fence_after();
+      const int m = m0 + row;
+      const bool row_ok = m < p.M;
+      uint16_t* orow = row_ok ? out_row(p, m, split) : nullptr;
+      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld16(tbase + c, r);
+        tmem_ld16(tbase + c + 16, r + 16);
+        tmem_ld_wait();
+        if (row_ok) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            const int n = n0 + c + g * 8;
+            if (n + 8 <= p.N) {
+              uint4 v;
+              v.x = pack_lo(r[g * 8 + 0], r[g * 8 + 1]);
+              v.y = pack_lo(r[g * 8 + 2], r[g * 8 + 3]);
+              v.z = pack_lo(r[g * 8 + 4], r[g * 8 + 5]);
+              v.w = pack_lo(r[g * 8 + 6], r[g * 8 + 7]);
+              uint4* dst = reinterpret_cast<uint4*>(orow + n);
+              if (p.out_mode == OUT_ACCUM) {
+                const uint4 o = *dst;
+                v.x = hadd2_rn(o.x, v.x);
+                v.y = hadd2_rn(o.y, v.y);
+                v.z = hadd2_rn(o.z, v.z);
+                v.w = hadd2_rn(o.w, v.w);
+              }
+              *dst = v;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+int gemm_smem_bytes(int BN) {
+  switch (BN) {
+    case 64: return GemmCfg<64>::SMEM;
+    case 128: return GemmCfg<128>::SMEM;
+    case 192: return GemmCfg<192>::SMEM;
+    case 256: return GemmCfg<256>::SMEM;
+    default: return -1;
+  }
+}
+
+template <int BN>
+static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const GemmParams& p,
+                               int grid, cudaStream_t s) {
+  static bool attr_set[64] = {false};  // per device ordinal
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         GemmCfg<BN>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  k_gemm<BN><<<grid, 192, GemmCfg<BN>::SMEM, s>>>(mA, mB, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const GemmParams& p,
+                        int grid, cudaStream_t s) {
+  switch (BN) {
+    case 64: return launch_bn_t<64>(mA, mB, p, grid, s);
+    case 128: return launch_bn_t<128>(mA, mB, p, grid, s);
+    case 192: return launch_bn_t<192>(mA, mB, p, grid, s);
+    case 256: return launch_bn_t<256>(mA, mB, p, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace pf16

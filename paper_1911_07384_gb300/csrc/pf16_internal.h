@@ -1,0 +1,137 @@
+// Internal interfaces of libpf16 shared between the C-ABI layer (pf16_api.cu)
+// and the kernels (pf16_gemm.cu, pf16_elementwise.cu).  Not installed.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace pf16 {
+
+// ---------------------------------------------------------------------------
+// tcgen05 implicit-GEMM engine.
+//
+// D[m][n] = sum_k A[m][k] * B[n][k], D in FP16, accumulated in FP16 inside the
+// tensor core (tcgen05.mma kind::f16, D type f16) into tensor memory.  Tiles
+// are 128 (M) x BN (N) x 64 (K-block).  Each K-block of each operand is
+// brought into shared memory by TMA in one of the load modes below, always as
+// 128-byte-swizzled atoms of 8 rows x 128 bytes:
+//   LD_TILED_K    2-D tiled box (64 k, rows): K-major operand, e.g. weights
+//                 [K][R*S*C] or a dense [pixels][channels] activation.
+//   LD_TILED_MN   2-D tiled boxes (64 mn, 64 k-rows): MN-major operand whose
+//                 K-block is 64 consecutive rows, e.g. dy as [pixels][K].
+//   LD_IM2COL_K   TMA im2col box (64 channels x 128 pixels) at one filter tap:
+//                 K-major activation patch, the implicit-GEMM A of the
+//                 forward and of the stride-phase data gradient.
+//   LD_IM2COL_MN  TMA im2col boxes (64 channels x 64 pixels): MN-major
+//                 activation patch for the weight gradient (K = pixels).
+//   LD_TAP3D_MN   3-D tiled boxes over weights viewed as (C, R*S, K): the
+//                 64(k) x 64(c) slice of one tap, MN-major B of the data
+//                 gradient (no transposed weight copy is needed).
+// ---------------------------------------------------------------------------
+enum LoadMode : int {
+  LD_TILED_K = 0,
+  LD_TILED_MN = 1,
+  LD_IM2COL_K = 2,
+  LD_IM2COL_MN = 3,
+  LD_TAP3D_MN = 4
+};
+enum OutMode : int { OUT_STORE = 0, OUT_ACCUM = 1, OUT_PARTIAL = 2 };
+
+constexpr int kMaxTaps = 49;
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+
+// Pixel grid that GEMM rows (or K-block pixels) enumerate, image-major, and
+// how a grid point maps to the im2col base coordinate (filter corner).
+struct PixGrid {
+  int gh, gw;             // grid points per image along h and w
+  int step;               // input step between grid points (conv stride)
+  int base_h, base_w;     // input coordinate of grid point (0, 0)
+};
+
+struct GemmParams {
+  int M, N;               // GEMM output extent
+  int num_kb;             // K-blocks in the whole reduction
+  int kb_per_split;       // K-blocks per split (split-K)
+  int splits;
+  int m_tiles, n_tiles;
+  int a_mode, b_mode;
+  int a_cpt;              // IM2COL_K: channel chunks (of 64) per tap
+  int b_cpt;              // TAP3D_MN: K chunks (of 64) per tap
+  int b_cin;              // IM2COL_MN: input channels (n -> tap, channel)
+  int b_oob_c;            // IM2COL_MN: a channel coordinate past the tensor (zero fill)
+  PixGrid ga, gb;         // pixel grids of the im2col operands
+  int ntaps;
+  int8_t tap_dr[kMaxTaps], tap_ds[kMaxTaps];  // im2col offsets (h, w) of each tap
+  int8_t tap_w[kMaxTaps];                     // weight tap index r*S+s (TAP3D_MN)
+  // epilogue
+  int out_mode;
+  uint16_t* out;
+  long long ldo;          // output row stride (elements)
+  int remap;              // rows -> strided positions of a stride phase
+  int rm_gh, rm_gw, rm_H, rm_W, rm_step, rm_ph, rm_pw;
+  // MMA
+  uint32_t idesc;
+  uint32_t a_lbo, a_sbo, a_kstep;  // smem-descriptor strides, bytes per 16-wide k step
+  uint32_t b_lbo, b_sbo, b_kstep;
+  int* status;            // device status word
+  unsigned long long wait_limit_ns;
+};
+
+// Launch the engine (BN in {64, 128, 192, 256}).  Returns a cudaError_t.
+cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,
+                        const GemmParams& p, int grid, cudaStream_t stream);
+int gemm_smem_bytes(int BN);
+
+// ---------------------------------------------------------------------------
+// Memory-bound kernels (pf16_elementwise.cu).  All return cudaError_t of the
+// launch.
+// ---------------------------------------------------------------------------
+cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
+                       uint16_t mom, uint16_t wd, cudaStream_t s);
+// sum of `splits` FP16 partial matrices [splits][rows][cols] by a balanced
+// pairwise tree; the result row r goes to out + r*ldo (only cols_out columns).
+cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long rows, int cols,
+                                 uint16_t* out, long long ldo, int cols_out, cudaStream_t s);
+// stem patches: col[m][j] = x[n, 2p+r-3, 2q+s-3, c] for j = (r*7+s)*3+c < 147, 0 up to kcol.
+cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, int W, int P,
+                               int Q, int R, int S, int C, int stride, int pad, int kcol,
+                               cudaStream_t s);
+// w[K][kin] -> wpad[K][kcol] (zero padded)
+cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wpad, int K, int kin, int kcol,
+                            cudaStream_t s);
+// zero the positions of a strided output no stride phase reaches (or all)
+cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s);
+
+struct BnLaunch {
+  int R, C;
+  uint16_t eps, post_scale;
+  int relu, residual;
+  int rows_per_block;     // power of two
+  int blocks;             // ceil(R / rows_per_block)
+  int blocks_pow2;
+};
+cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
+                          const uint16_t* beta, const uint16_t* residual, uint16_t* y,
+                          uint16_t* mean, uint16_t* invstd, uint16_t* ws, cudaStream_t s);
+cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
+                          const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
+                          const uint16_t* y_saved, uint16_t* dx, uint16_t* dgamma,
+                          uint16_t* dbeta, uint16_t* dres, uint16_t* ws, cudaStream_t s);
+void bn_plan(int R, int C, BnLaunch* b);
+size_t bn_ws_bytes(const BnLaunch& b);
+
+cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, int N, int H, int W, int C,
+                               cudaStream_t s);
+cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int N, int H,
+                               int W, int C, cudaStream_t s);
+cudaError_t launch_avgpool_fwd(const uint16_t* x, uint16_t* y, int N, int HW, int C,
+                               cudaStream_t s);
+cudaError_t launch_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int N, int HW, int C,
+                               cudaStream_t s);
+cudaError_t launch_softmax_xent(const uint16_t* logits, const uint16_t* bias,
+                                const int32_t* labels, int B, int K, uint16_t* loss,
+                                uint16_t* dlogits, uint16_t* dbias, uint16_t* ws,
+                                cudaStream_t s);
+
+}  // namespace pf16

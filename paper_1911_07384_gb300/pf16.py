@@ -1,0 +1,220 @@
+"""Thin ctypes binding of libpf16 (include/pf16.h): the same entry points,
+argument marshalling only.  Tensors are torch CUDA tensors (any 2-byte dtype;
+the bits are binary16); every computation happens in the library's kernels.
+A non-zero status raises PF16Error.  If the library cannot be built or
+loaded, importing the entry points raises: there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from . import build as _build
+
+PF16_OK = 0
+PF16_ERR_NULL = -1
+PF16_ERR_ALIGN = -2
+PF16_ERR_SHAPE = -3
+PF16_ERR_UNSUPPORTED = -4
+PF16_ERR_WORKSPACE = -5
+PF16_ERR_CUDA = -6
+PF16_ERR_TIMEOUT = -7
+PF16_ERR_ARG = -8
+
+PF16_ACCUMULATE = 0x1
+PF16_BN_RELU = 0x1
+PF16_BN_RESIDUAL = 0x2
+PF16_PASS_FWD, PF16_PASS_DGRAD, PF16_PASS_WGRAD = 0, 1, 2
+
+EXPORTS = [
+    "pf16_conv_workspace_size", "pf16_conv_fwd", "pf16_conv_dgrad", "pf16_conv_wgrad",
+    "pf16_sgd_update", "pf16_bn_workspace_size", "pf16_bn_fwd_bwd", "pf16_maxpool_fwd",
+    "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
+    "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
+    "pf16_status_string", "pf16_device_arch",
+]
+
+
+class PF16Error(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: pf16 status {code} ({status_string(code)})")
+
+
+class ConvDesc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("n", "h", "w", "c", "k", "r", "s", "stride", "pad")]
+
+    def out_hw(self):
+        return ((self.h + 2 * self.pad - self.r) // self.stride + 1,
+                (self.w + 2 * self.pad - self.s) // self.stride + 1)
+
+
+class BnDesc(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("h", ctypes.c_int32), ("w", ctypes.c_int32),
+                ("c", ctypes.c_int32), ("eps", ctypes.c_uint16), ("post_scale", ctypes.c_uint16),
+                ("flags", ctypes.c_uint32)]
+
+
+_BN_T = ("x", "gamma", "beta", "residual", "dy", "y_saved", "y", "mean", "invstd", "dx", "dgamma",
+         "dbeta", "dresidual")
+
+
+class BnTensors(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in _BN_T]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def lib():
+    """Load (building first if needed) libpf16.so."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build()
+            L = ctypes.CDLL(path)
+            vp, sz, u16, u32, i32, I = (ctypes.c_void_p, ctypes.c_size_t, ctypes.c_uint16,
+                                       ctypes.c_uint32, ctypes.c_int32, ctypes.c_int)
+            cdp = ctypes.POINTER(ConvDesc)
+            L.pf16_conv_workspace_size.argtypes = [cdp, I]
+            L.pf16_conv_workspace_size.restype = sz
+            for nm in ("pf16_conv_fwd", "pf16_conv_dgrad", "pf16_conv_wgrad"):
+                getattr(L, nm).argtypes = [cdp, vp, vp, vp, vp, sz, u32, vp]
+                getattr(L, nm).restype = I
+            L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
+            L.pf16_sgd_update.restype = I
+            L.pf16_bn_workspace_size.argtypes = [ctypes.POINTER(BnDesc)]
+            L.pf16_bn_workspace_size.restype = sz
+            L.pf16_bn_fwd_bwd.argtypes = [ctypes.POINTER(BnDesc), I, ctypes.POINTER(BnTensors), vp,
+                                          sz, vp]
+            L.pf16_bn_fwd_bwd.restype = I
+            L.pf16_maxpool_fwd.argtypes = [vp, vp, i32, i32, i32, i32, vp]
+            L.pf16_maxpool_bwd.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
+            L.pf16_avgpool_fwd.argtypes = [vp, vp, i32, i32, i32, vp]
+            L.pf16_avgpool_bwd.argtypes = [vp, vp, i32, i32, i32, vp]
+            for nm in ("pf16_maxpool_fwd", "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd"):
+                getattr(L, nm).restype = I
+            L.pf16_softmax_xent_workspace_size.argtypes = [i32, i32]
+            L.pf16_softmax_xent_workspace_size.restype = sz
+            L.pf16_softmax_xent.argtypes = [vp, vp, vp, i32, i32, vp, vp, vp, vp, sz, vp]
+            L.pf16_softmax_xent.restype = I
+            L.pf16_sync_status.argtypes = [vp]
+            L.pf16_sync_status.restype = I
+            L.pf16_status_string.argtypes = [I]
+            L.pf16_status_string.restype = ctypes.c_char_p
+            L.pf16_device_arch.argtypes = []
+            L.pf16_device_arch.restype = I
+            _lib = L
+    return _lib
+
+
+def status_string(code: int) -> str:
+    return lib().pf16_status_string(int(code)).decode()
+
+
+def _check(rc: int, where: str) -> None:
+    if rc != PF16_OK:
+        raise PF16Error(rc, where)
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def conv_desc(n, h, w, c, k, r, s, stride, pad) -> ConvDesc:
+    return ConvDesc(n, h, w, c, k, r, s, stride, pad)
+
+
+def conv_workspace_size(d: ConvDesc, pass_: int) -> int:
+    return int(lib().pf16_conv_workspace_size(ctypes.byref(d), pass_))
+
+
+def conv_fwd(d, x, w, y, ws=None, flags=0, stream=None):
+    _check(lib().pf16_conv_fwd(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(y), _ptr(ws), _nbytes(ws),
+                               flags, _stream(stream)), "pf16_conv_fwd")
+
+
+def conv_dgrad(d, dy, w, dx, ws=None, flags=0, stream=None):
+    _check(lib().pf16_conv_dgrad(ctypes.byref(d), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws),
+                                 _nbytes(ws), flags, _stream(stream)), "pf16_conv_dgrad")
+
+
+def conv_wgrad(d, x, dy, dw, ws=None, flags=0, stream=None):
+    _check(lib().pf16_conv_wgrad(ctypes.byref(d), _ptr(x), _ptr(dy), _ptr(dw), _ptr(ws),
+                                 _nbytes(ws), flags, _stream(stream)), "pf16_conv_wgrad")
+
+
+def sgd_update(w, v, g, lr_bits, momentum_bits, wd_bits, flags=0, stream=None):
+    _check(lib().pf16_sgd_update(_ptr(w), _ptr(v), _ptr(g), w.numel(), lr_bits, momentum_bits,
+                                 wd_bits, flags, _stream(stream)), "pf16_sgd_update")
+
+
+def bn_desc(n, h, w, c, eps_bits=0x00A8, post_scale_bits=0x3400, flags=0) -> BnDesc:
+    return BnDesc(n, h, w, c, eps_bits, post_scale_bits, flags)
+
+
+def bn_workspace_size(d: BnDesc) -> int:
+    return int(lib().pf16_bn_workspace_size(ctypes.byref(d)))
+
+
+def bn_fwd_bwd(d, phase, ws, stream=None, **tensors):
+    t = BnTensors(**{k: (v.data_ptr() if v is not None else None) for k, v in tensors.items()})
+    _check(lib().pf16_bn_fwd_bwd(ctypes.byref(d), phase, ctypes.byref(t), _ptr(ws), _nbytes(ws),
+                                 _stream(stream)), "pf16_bn_fwd_bwd")
+
+
+def maxpool_fwd(x, y, n, h, w, c, stream=None):
+    _check(lib().pf16_maxpool_fwd(_ptr(x), _ptr(y), n, h, w, c, _stream(stream)), "pf16_maxpool_fwd")
+
+
+def maxpool_bwd(x, dy, dx, n, h, w, c, stream=None):
+    _check(lib().pf16_maxpool_bwd(_ptr(x), _ptr(dy), _ptr(dx), n, h, w, c, _stream(stream)),
+           "pf16_maxpool_bwd")
+
+
+def avgpool_fwd(x, y, n, hw, c, stream=None):
+    _check(lib().pf16_avgpool_fwd(_ptr(x), _ptr(y), n, hw, c, _stream(stream)), "pf16_avgpool_fwd")
+
+
+def avgpool_bwd(dy, dx, n, hw, c, stream=None):
+    _check(lib().pf16_avgpool_bwd(_ptr(dy), _ptr(dx), n, hw, c, _stream(stream)), "pf16_avgpool_bwd")
+
+
+def softmax_xent_workspace_size(b, k) -> int:
+    return int(lib().pf16_softmax_xent_workspace_size(b, k))
+
+
+def softmax_xent(logits, bias, labels, b, k, loss, dlogits, dbias, ws, stream=None):
+    _check(lib().pf16_softmax_xent(_ptr(logits), _ptr(bias), _ptr(labels), b, k, _ptr(loss),
+                                   _ptr(dlogits), _ptr(dbias), _ptr(ws), _nbytes(ws),
+                                   _stream(stream)), "pf16_softmax_xent")
+
+
+def sync_status(stream=None) -> int:
+    return int(lib().pf16_sync_status(_stream(stream)))
+
+
+def device_arch() -> int:
+    return int(lib().pf16_device_arch())
+
+
+def loaded_path() -> str:
+    return os.path.abspath(_build.LIB)

@@ -1,0 +1,91 @@
+"""The C-ABI library builds for sm_103a, loads without a GPU, exports every
+entry point include/pf16.h declares, and rejects invalid calls on the host
+with the documented status codes before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_1911_07384_gb300 import pf16
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "pf16.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(pf16_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_and_binding_agree():
+    assert declared_functions() == sorted(pf16.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol():
+    L = pf16.lib()
+    for name in declared_functions():
+        assert hasattr(L, name), name
+        assert ctypes.cast(getattr(L, name), ctypes.c_void_p).value
+
+
+def test_status_strings():
+    for code in range(-8, 1):
+        assert pf16.status_string(code) != "unknown status"
+    assert pf16.status_string(-99) == "unknown status"
+
+
+FAKE = ctypes.c_void_p(0x10000)      # aligned, never dereferenced: validation fails first
+FAKE_MIS = ctypes.c_void_p(0x10002)  # misaligned
+
+
+def test_conv_validation_errors():
+    L = pf16.lib()
+    good = pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 1, 1)
+    assert L.pf16_conv_fwd(None, FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_NULL
+    bad = pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 1, 1)
+    bad.h = 0
+    assert L.pf16_conv_fwd(ctypes.byref(bad), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_SHAPE
+    odd = pf16.conv_desc(2, 8, 8, 48, 64, 3, 3, 1, 1)
+    assert L.pf16_conv_fwd(ctypes.byref(odd), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_UNSUPPORTED
+    s3 = pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 3, 1)
+    assert L.pf16_conv_fwd(ctypes.byref(s3), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_UNSUPPORTED
+    assert L.pf16_conv_fwd(ctypes.byref(good), None, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_conv_fwd(ctypes.byref(good), FAKE_MIS, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_ALIGN
+    assert L.pf16_conv_fwd(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, 0x80, None) == pf16.PF16_ERR_ARG
+    assert L.pf16_conv_wgrad(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, 1, None) == pf16.PF16_ERR_ARG
+    stem = pf16.conv_desc(2, 32, 32, 3, 64, 7, 7, 2, 3)
+    assert L.pf16_conv_dgrad(ctypes.byref(stem), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_UNSUPPORTED
+    # stem forward needs its patch workspace
+    assert L.pf16_conv_fwd(ctypes.byref(stem), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_WORKSPACE
+
+
+def test_workspace_sizes_are_host_computable():
+    cfg3 = pf16.conv_desc(256, 56, 56, 256, 64, 1, 1, 1, 0)
+    assert pf16.conv_workspace_size(cfg3, pf16.PF16_PASS_FWD) == 0
+    assert pf16.conv_workspace_size(cfg3, pf16.PF16_PASS_DGRAD) == 0
+    w = pf16.conv_workspace_size(cfg3, pf16.PF16_PASS_WGRAD)
+    assert w > 0 and w % 256 == 0
+    stem = pf16.conv_desc(256, 224, 224, 3, 64, 7, 7, 2, 3)
+    assert pf16.conv_workspace_size(stem, pf16.PF16_PASS_FWD) >= 256 * 112 * 112 * 147 * 2
+    bad = pf16.conv_desc(0, 56, 56, 256, 64, 1, 1, 1, 0)
+    assert pf16.conv_workspace_size(bad, pf16.PF16_PASS_WGRAD) == 0
+
+
+def test_other_validation_errors():
+    L = pf16.lib()
+    assert L.pf16_sgd_update(FAKE, FAKE, FAKE, 16, 0, 0, 0, 1, None) == pf16.PF16_ERR_ARG
+    assert L.pf16_sgd_update(None, FAKE, FAKE, 16, 0, 0, 0, 0, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_sgd_update(FAKE_MIS, FAKE, FAKE, 16, 0, 0, 0, 0, None) == pf16.PF16_ERR_ALIGN
+    assert L.pf16_sgd_update(None, None, None, 0, 0, 0, 0, 0, None) == pf16.PF16_OK  # n = 0: no-op
+    d = pf16.bn_desc(2, 4, 4, 12)
+    assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, None, FAKE, 1 << 20, None) == pf16.PF16_ERR_UNSUPPORTED
+    d = pf16.bn_desc(2, 4, 4, 64)
+    t = pf16.BnTensors()
+    assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 2, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_ARG
+    assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1, None) == pf16.PF16_ERR_WORKSPACE
+    assert L.pf16_maxpool_fwd(FAKE, FAKE, 1, 8, 8, 12, None) == pf16.PF16_ERR_UNSUPPORTED
+    assert L.pf16_avgpool_fwd(FAKE, None, 1, 49, 64, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_softmax_xent(FAKE, None, FAKE, 4, 5000, FAKE, FAKE, None, FAKE, 1 << 20,
+                               None) == pf16.PF16_ERR_UNSUPPORTED

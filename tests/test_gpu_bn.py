@@ -1,0 +1,104 @@
+"""GPU parity of pf16_bn_fwd_bwd (Eq. 1, Eq. 2, x post_scale, residual, ReLU)
+against the oracle's binary64 BatchNorm on the same binary16 inputs.
+
+Tolerance (no bound is given by the paper; derived from the FP16 schedule):
+the statistics are halving trees of depth L = ceil(log2 R) (one rounding per
+level), the normalisation and affine steps add a fixed number of roundings.
+Per element of the forward output
+    |err| <= (4 L + 8) u * (s (|gamma| (|xhat| + 1) + |beta|) + |residual|) + 2^-24
+and of the data gradient
+    |err| <= (4 L + 8) u * |s gamma invstd| * (|dy'| + max|dy'| (|xhat| + 1)) + 2^-24,
+u = 2^-11; dgamma / dbeta within (4 L + 8) u * s * sum|terms| + 2^-24."""
+import numpy as np
+import pytest
+
+from paper_1911_07384_gb300 import pf16
+from paper_1911_07384_gb300 import synthetic as syn
+from gpu_util import U, dev, empty16, f64, host, workspace
+
+pytestmark = pytest.mark.gpu
+
+EPS = 0x00A8
+EPS_F = float(np.uint16(EPS).view(np.float16))
+
+
+def f16(a):
+    return np.asarray(a, np.float64).astype(np.float16).view(np.uint16)
+
+
+CASES = [
+    # N, H, W, C, post_scale, relu, residual
+    (4, 14, 14, 64, 0.25, True, True),
+    (2, 7, 7, 2048, 0.25, False, False),
+    (8, 56, 56, 64, 1.0, True, False),
+    (3, 5, 7, 24, 0.25, True, True),      # C not a power of two, ragged rows
+    (256, 14, 14, 256, 0.25, True, True),  # R = 50,176
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: "N{}_{}x{}_C{}_s{}_relu{}_res{}".format(*c))
+def test_bn_fwd_bwd(orc, case):
+    N, H, W, C, s, relu, res = case
+    R = N * H * W
+    L = int(np.ceil(np.log2(R)))
+    x = f16(f64(syn.normal_f16(11, (R, C), 2.0)) + 0.5)
+    gamma = f16(1.0 + 0.1 * f64(syn.normal_f16(12, (C,))))
+    beta = f16(0.1 * f64(syn.normal_f16(13, (C,))))
+    resid = syn.normal_f16(14, (R, C)) if res else None
+    dy = syn.normal_f16(15, (R, C), 0.01)
+    flags = (pf16.PF16_BN_RELU if relu else 0) | (pf16.PF16_BN_RESIDUAL if res else 0)
+    sbits = int(f16([s])[0])
+    d = pf16.bn_desc(N, H, W, C, EPS, sbits, flags)
+    ws = workspace(pf16.bn_workspace_size(d))
+    tx, tg, tb = dev(x), dev(gamma), dev(beta)
+    ty, tm, ti = empty16(R * C), empty16(C), empty16(C)
+    pf16.bn_fwd_bwd(d, 0, ws, x=tx, gamma=tg, beta=tb, residual=dev(resid) if res else None, y=ty,
+                    mean=tm, invstd=ti)
+    assert pf16.sync_status() == 0
+    y = host(ty)
+    yo, mean, var, invstd = orc.bn_fwd(x, gamma, beta, resid, R, C, EPS_F, s, relu)
+    xhat = (f64(x).reshape(R, C) - mean) * invstd
+    gf, bf = f64(gamma), f64(beta)
+    scale = s * (np.abs(gf) * (np.abs(xhat) + 1) + np.abs(bf))
+    if res:
+        scale = scale + np.abs(f64(resid).reshape(R, C))
+    tol = (4 * L + 8) * U * scale + 2.0 ** -24
+    err = np.abs(f64(y).reshape(R, C) - yo)
+    assert np.all(err <= tol), float(np.max(err / tol))
+    # saved statistics
+    assert np.all(np.abs(f64(host(tm)) - mean) <= (L + 2) * U * np.abs(f64(x).reshape(R, C)).max(0))
+    assert np.all(np.abs(f64(host(ti)) - invstd) <= (2 * L + 8) * U * invstd)
+
+    # backward, teacher-forced on the GPU's own saved output and statistics
+    tdx, tdg, tdb, tdr = empty16(R * C), empty16(C), empty16(C), empty16(R * C)
+    pf16.bn_fwd_bwd(d, 1, ws, x=tx, gamma=tg, mean=tm, invstd=ti, dy=dev(dy), y_saved=ty, dx=tdx,
+                    dgamma=tdg, dbeta=tdb, dresidual=tdr)
+    assert pf16.sync_status() == 0
+    dxo, dgo, dbo, dro = orc.bn_bwd(x, gamma, dy, y, R, C, EPS_F, s, relu)
+    assert np.array_equal(f64(host(tdr)).reshape(R, C), dro)  # masking is exact
+    dyp = np.abs(dro)
+    k = np.abs(s * gf * invstd)
+    tol = (4 * L + 8) * U * k * (dyp + dyp.max(0) * (np.abs(xhat) + 1)) + 2.0 ** -24
+    err = np.abs(f64(host(tdx)).reshape(R, C) - dxo)
+    assert np.all(err <= tol), float(np.max(err / tol))
+    tol_b = (4 * L + 8) * U * s * dyp.sum(0) + 2.0 ** -24
+    tol_g = (4 * L + 8) * U * s * (dyp * (np.abs(xhat) + 1)).sum(0) + 2.0 ** -24
+    assert np.all(np.abs(f64(host(tdb)) - dbo) <= tol_b)
+    assert np.all(np.abs(f64(host(tdg)) - dgo) <= tol_g)
+
+
+def test_bn_constant_channel_and_zero_gamma(orc):
+    """Closed forms: a constant channel normalises to 0 so y = s*beta; gamma = 0
+    gives y = s*beta exactly too."""
+    N, H, W, C = 2, 8, 8, 16
+    R = N * H * W
+    x = f16(np.tile(np.linspace(-3, 3, C), (R, 1)))
+    gamma = f16(np.where(np.arange(C) % 2 == 0, 0.0, 1.5))
+    beta = f16(np.linspace(-1, 1, C))
+    d = pf16.bn_desc(N, H, W, C, EPS, 0x3400, 0)
+    ws = workspace(pf16.bn_workspace_size(d))
+    ty = empty16(R * C)
+    pf16.bn_fwd_bwd(d, 0, ws, x=dev(x), gamma=dev(gamma), beta=dev(beta), y=ty, mean=empty16(C),
+                    invstd=empty16(C))
+    y = f64(host(ty)).reshape(R, C)
+    assert np.array_equal(y, np.tile(0.25 * f64(beta), (R, 1)))
