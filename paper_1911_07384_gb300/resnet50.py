@@ -1,0 +1,322 @@
+"""ResNet-50 v1.5 pure-FP16 training step on top of libpf16 (host code only).
+
+The network, the recipe and the FP16 rules are the paper's (Sec. 5.1, 5.2,
+4.2): ResNet-50 trained with PyTorch's ImageNet recipe -- SGD with momentum
+0.9, weight decay 1e-4 on conv/FC parameters and none on BatchNorm parameters,
+gamma of the last BatchNorm of every residual block initialised to zero --
+with every tensor and every operation in FP16, no master copy, and the output
+of every BatchNorm inside a residual block multiplied by 0.25 (the stem's
+BatchNorm is left as it is).
+
+Every op of the step is one call into libpf16 on the current CUDA stream;
+this module only lays out the buffers (torch supplies device memory) and
+issues the calls, so the whole step can be captured once in a CUDA graph and
+replayed.  Layout: activations NHWC, weights KRSC, parameters in two flat
+16-byte-aligned FP16 arenas (decayed / not decayed), each with a gradient and a
+momentum twin, so the update is two pf16_sgd_update calls.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import pf16
+from . import synthetic as syn
+
+LR = 0x2E66       # 0.1 in binary16 (0.0999755859375)
+MOMENTUM = 0x3B33  # 0.9 (0.89990234375)
+WD = 0x068E       # 1e-4 (1.00016594e-4)
+EPS = 0x00A8      # 1e-5 (subnormal, 1.00135803e-5)
+S_BLOCK = 0x3400  # 0.25: BatchNorms inside residual blocks
+S_STEM = 0x3C00   # 1.0: the stem BatchNorm
+
+STAGES = [(64, 3, 1), (128, 4, 2), (256, 6, 2), (512, 3, 2)]  # width, blocks, stride
+
+
+def _a8(n):
+    return (n + 7) // 8 * 8
+
+
+def _f16(x):
+    return torch.from_numpy(np.ascontiguousarray(x).view(np.int16))
+
+
+class Arena:
+    """Flat FP16 parameter arena with gradient and momentum twins."""
+
+    def __init__(self, name):
+        self.name = name
+        self.size = 0
+        self.slots = []
+
+    def add(self, numel):
+        off = self.size
+        self.size += _a8(numel)
+        self.slots.append((off, numel))
+        return off
+
+    def allocate(self, device):
+        n = max(self.size, 8)
+        self.w = torch.zeros(n, dtype=torch.int16, device=device)
+        self.g = torch.zeros(n, dtype=torch.int16, device=device)
+        self.v = torch.zeros(n, dtype=torch.int16, device=device)
+
+    def view(self, which, off, numel):
+        return getattr(self, which)[off:off + numel]
+
+
+class Conv:
+    def __init__(self, net, n, h, w, c, k, r, s, stride, pad):
+        self.net = net
+        self.desc = pf16.conv_desc(n, h, w, c, k, r, s, stride, pad)
+        self.P, self.Q = self.desc.out_hw()
+        self.numel = k * r * s * c
+        self.off = net.wd.add(self.numel)
+        self.flops = 2 * n * self.P * self.Q * k * c * r * s
+        net.convs.append(self)
+
+    def bind(self):
+        a = self.net.wd
+        self.w, self.gw = a.view("w", self.off, self.numel), a.view("g", self.off, self.numel)
+
+    def fwd(self, x, y):
+        self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.net.ws)
+
+    def dgrad(self, dy, dx, accumulate=False):
+        self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
+                      pf16.PF16_ACCUMULATE if accumulate else 0)
+
+    def wgrad(self, x, dy):
+        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.net.ws)
+
+
+class BN:
+    def __init__(self, net, n, h, w, c, post_scale, relu, residual=False, zero_gamma=False):
+        self.net = net
+        flags = (pf16.PF16_BN_RELU if relu else 0) | (pf16.PF16_BN_RESIDUAL if residual else 0)
+        self.desc = pf16.bn_desc(n, h, w, c, EPS, post_scale, flags)
+        self.c = c
+        self.zero_gamma = zero_gamma
+        self.g_off = net.nowd.add(c)
+        self.b_off = net.nowd.add(c)
+        self.elems = n * h * w * c
+        net.bns.append(self)
+
+    def bind(self, device):
+        a = self.net.nowd
+        self.gamma, self.beta = a.view("w", self.g_off, self.c), a.view("w", self.b_off, self.c)
+        self.dgamma, self.dbeta = a.view("g", self.g_off, self.c), a.view("g", self.b_off, self.c)
+        self.mean = torch.empty(self.c, dtype=torch.int16, device=device)
+        self.invstd = torch.empty(self.c, dtype=torch.int16, device=device)
+
+    def fwd(self, x, y, residual=None):
+        self.net.call("bn_fwd", self, pf16.bn_fwd_bwd, self.desc, 0, self.net.ws, x=x, gamma=self.gamma,
+                      beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd)
+
+    def bwd(self, x, y_saved, dy, dx, dresidual=None):
+        self.net.call("bn_bwd", self, pf16.bn_fwd_bwd, self.desc, 1, self.net.ws, x=x, gamma=self.gamma,
+                      mean=self.mean, invstd=self.invstd, dy=dy,
+                      y_saved=y_saved if self.desc.flags & pf16.PF16_BN_RELU else None, dx=dx,
+                      dgamma=self.dgamma, dbeta=self.dbeta, dresidual=dresidual)
+
+
+class Bottleneck:
+    def __init__(self, net, n, h, cin, width, stride, proj):
+        self.cin, self.width, self.stride = cin, width, stride
+        cout = 4 * width
+        self.conv1 = Conv(net, n, h, h, cin, width, 1, 1, 1, 0)
+        self.bn1 = BN(net, n, h, h, width, S_BLOCK, relu=True)
+        self.conv2 = Conv(net, n, h, h, width, width, 3, 3, stride, 1)
+        h2 = self.conv2.P
+        self.bn2 = BN(net, n, h2, h2, width, S_BLOCK, relu=True)
+        self.conv3 = Conv(net, n, h2, h2, width, cout, 1, 1, 1, 0)
+        self.bn3 = BN(net, n, h2, h2, cout, S_BLOCK, relu=True, residual=True, zero_gamma=True)
+        self.proj = proj
+        if proj:
+            self.convp = Conv(net, n, h, h, cin, cout, 1, 1, stride, 0)
+            self.bnp = BN(net, n, h2, h2, cout, S_BLOCK, relu=False)
+        self.h, self.h2, self.n, self.cout = h, h2, n, cout
+
+    def allocate(self, dev):
+        n, h, h2, w, c = self.n, self.h, self.h2, self.width, self.cout
+        e = lambda *s: torch.empty(int(np.prod(s)), dtype=torch.int16, device=dev)
+        self.a1, self.b1 = e(n, h, h, w), e(n, h, h, w)
+        self.a2, self.b2 = e(n, h2, h2, w), e(n, h2, h2, w)
+        self.a3, self.y = e(n, h2, h2, c), e(n, h2, h2, c)
+        self.dy = e(n, h2, h2, c)  # gradient w.r.t. y (written by the next block)
+        self.da3 = e(n, h2, h2, c)
+        self.db2, self.da2 = e(n, h2, h2, w), e(n, h2, h2, w)
+        self.db1, self.da1 = e(n, h, h, w), e(n, h, h, w)
+        if self.proj:
+            self.ap, self.bp = e(n, h2, h2, c), e(n, h2, h2, c)
+            self.dres, self.dap = e(n, h2, h2, c), e(n, h2, h2, c)
+
+    def forward(self, x):
+        self.x = x
+        self.conv1.fwd(x, self.a1)
+        self.bn1.fwd(self.a1, self.b1)
+        self.conv2.fwd(self.b1, self.a2)
+        self.bn2.fwd(self.a2, self.b2)
+        self.conv3.fwd(self.b2, self.a3)
+        if self.proj:
+            self.convp.fwd(x, self.ap)
+            self.bnp.fwd(self.ap, self.bp)
+            self.bn3.fwd(self.a3, self.y, residual=self.bp)
+        else:
+            self.bn3.fwd(self.a3, self.y, residual=x)
+        return self.y
+
+    def backward(self, dx):
+        """self.dy holds dL/dy; writes dL/dx into dx."""
+        if self.proj:
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=self.dres)
+        else:  # identity shortcut: its gradient is the start of dx
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=dx)
+        self.conv3.wgrad(self.b2, self.da3)
+        self.conv3.dgrad(self.da3, self.db2)
+        self.bn2.bwd(self.a2, self.b2, self.db2, self.da2)
+        self.conv2.wgrad(self.b1, self.da2)
+        self.conv2.dgrad(self.da2, self.db1)
+        self.bn1.bwd(self.a1, self.b1, self.db1, self.da1)
+        self.conv1.wgrad(self.x, self.da1)
+        if self.proj:
+            self.conv1.dgrad(self.da1, dx)
+            self.bnp.bwd(self.ap, None, self.dres, self.dap)
+            self.convp.wgrad(self.x, self.dap)
+            self.convp.dgrad(self.dap, dx, accumulate=True)
+        else:
+            self.conv1.dgrad(self.da1, dx, accumulate=True)
+
+
+class ResNet50:
+    """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
+
+    def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None):
+        self.N, self.image, self.classes, self.device = batch, image, classes, device
+        self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
+        self.wd, self.nowd = Arena("decayed"), Arena("no-decay")
+        self.convs, self.bns = [], []
+        N = batch
+        self.stem = Conv(self, N, image, image, 3, 64, 7, 7, 2, 3)
+        h = self.stem.P
+        self.bn0 = BN(self, N, h, h, 64, S_STEM, relu=True)
+        self.h0 = h
+        self.hp = (h - 1) // 2 + 1
+        h, cin = self.hp, 64
+        self.blocks = []
+        for width, nb, stride in STAGES:
+            for b in range(nb):
+                blk = Bottleneck(self, N, h, cin, width, stride if b == 0 else 1, proj=(b == 0))
+                self.blocks.append(blk)
+                h, cin = blk.h2, 4 * width
+        self.hl, self.cl = h, cin
+        self.fc = Conv(self, N, 1, 1, cin, classes, 1, 1, 1, 0)
+        self.bias_off = self.wd.add(classes)
+        self.seed_cfg = seed_cfg
+        self._allocate()
+        self._init_params()
+
+    # ------------------------------------------------------------- buffers
+    def _allocate(self):
+        dev, N = self.device, self.N
+        e = lambda *s: torch.empty(int(np.prod(s)), dtype=torch.int16, device=dev)
+        self.wd.allocate(dev)
+        self.nowd.allocate(dev)
+        for c in self.convs:
+            c.bind()
+        for b in self.bns:
+            b.bind(dev)
+        self.bias = self.wd.view("w", self.bias_off, self.classes)
+        self.dbias = self.wd.view("g", self.bias_off, self.classes)
+        h0, hp = self.h0, self.hp
+        self.x = e(N, self.image, self.image, 3)
+        self.labels = torch.zeros(N, dtype=torch.int32, device=dev)
+        self.a0, self.b0, self.p0 = e(N, h0, h0, 64), e(N, h0, h0, 64), e(N, hp, hp, 64)
+        self.dp0, self.db0, self.da0 = e(N, hp, hp, 64), e(N, h0, h0, 64), e(N, h0, h0, 64)
+        for b in self.blocks:
+            b.allocate(dev)
+        self.f = e(N, self.cl)
+        self.logits = e(N, self.classes)
+        self.dlogits = e(N, self.classes)
+        self.df = e(N, self.cl)
+        self.loss = e(1)
+        ws = 0
+        for c in self.convs:
+            ws = max(ws, pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_FWD),
+                     pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD))
+        for b in self.bns:
+            ws = max(ws, pf16.bn_workspace_size(b.desc))
+        ws = max(ws, pf16.softmax_xent_workspace_size(N, self.classes))
+        self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
+
+    def _init_params(self):
+        """He-normal conv / FC weights (std sqrt(2 / fan_in)), FC bias 0, BN gamma
+        1 and beta 0, gamma 0 in the last BatchNorm of every block; momentum +0."""
+        for i, c in enumerate(self.convs):
+            d = c.desc
+            wbits = syn.he_normal_f16(syn.seed_for(self.seed_cfg, "w", i), d.k, d.r, d.s, d.c)
+            c.w.copy_(_f16(wbits.ravel()))
+        self.bias.zero_()
+        one = int(np.float16(1.0).view(np.uint16))
+        for b in self.bns:
+            b.gamma.fill_(0 if b.zero_gamma else one)
+            b.beta.zero_()
+        self.wd.v.zero_()
+        self.nowd.v.zero_()
+
+    def set_batch(self, images_bits, labels):
+        self.x.copy_(_f16(images_bits.ravel()))
+        self.labels.copy_(torch.from_numpy(np.ascontiguousarray(labels, np.int32)))
+
+    # ------------------------------------------------------------- calls
+    def call(self, kind, layer, fn, *args, **kw):
+        if self.hook is not None:
+            return self.hook(kind, layer, fn, *args, **kw)
+        return fn(*args, **kw)
+
+    def forward(self):
+        self.stem.fwd(self.x, self.a0)
+        self.bn0.fwd(self.a0, self.b0)
+        self.call("maxpool_fwd", None, pf16.maxpool_fwd, self.b0, self.p0, self.N, self.h0, self.h0, 64)
+        h = self.p0
+        for b in self.blocks:
+            h = b.forward(h)
+        self.call("avgpool_fwd", None, pf16.avgpool_fwd, h, self.f, self.N, self.hl * self.hl, self.cl)
+        self.fc.fwd(self.f, self.logits)
+        self.call("softmax_xent", None, pf16.softmax_xent, self.logits, self.bias, self.labels, self.N,
+                  self.classes, self.loss, self.dlogits, self.dbias, self.ws)
+
+    def backward(self):
+        self.fc.wgrad(self.f, self.dlogits)
+        self.fc.dgrad(self.dlogits, self.df)
+        last = self.blocks[-1]
+        self.call("avgpool_bwd", None, pf16.avgpool_bwd, self.df, last.dy, self.N, self.hl * self.hl,
+                  self.cl)
+        for i in range(len(self.blocks) - 1, -1, -1):
+            dx = self.blocks[i - 1].dy if i > 0 else self.dp0
+            self.blocks[i].backward(dx)
+        self.call("maxpool_bwd", None, pf16.maxpool_bwd, self.b0, self.dp0, self.db0, self.N, self.h0,
+                  self.h0, 64)
+        self.bn0.bwd(self.a0, self.b0, self.db0, self.da0)
+        self.stem.wgrad(self.x, self.da0)
+
+    def update(self):
+        self.call("sgd", None, pf16.sgd_update, self.wd.w, self.wd.v, self.wd.g, LR, MOMENTUM, WD)
+        self.call("sgd", None, pf16.sgd_update, self.nowd.w, self.nowd.v, self.nowd.g, LR, MOMENTUM, 0)
+
+    def step(self):
+        self.forward()
+        self.backward()
+        self.update()
+
+    # ------------------------------------------------------------- accounting
+    def conv_flops(self):
+        """Algorithmic convolution FLOPs of one step: 2*N*P*Q*K*C*R*S for each of
+        forward, data gradient (not for the stem) and weight gradient."""
+        total = 0
+        for c in self.convs:
+            total += c.flops * (2 if c is self.stem else 3)
+        return total
+
+    def param_count(self):
+        return (sum(n for _, n in self.wd.slots), sum(n for _, n in self.nowd.slots))
