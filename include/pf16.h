@@ -98,6 +98,30 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
+/* Weight gradient without any caller workspace (the paper has no counterpart:
+ * this is a convenience of the library).  Same arguments, result and error
+ * codes as pf16_conv_wgrad, minus ws / ws_bytes.  It is meant for callers that
+ * cannot give the library scratch memory: hosts that plan all device memory
+ * themselves and do not let a library request more, deployments that forbid
+ * device allocation after set-up, or bindings with no CUDA allocator at hand;
+ * it also spares a training loop the device-wide stall a cudaMalloc can cause.
+ * Its split-K scratch is one fixed array of PF16_WGRAD_NOALLOC_SCRATCH_BYTES
+ * compiled into the library; every device that loads it keeps the array until
+ * the process exits.  Nothing is allocated or freed by the call.
+ *  - A layer whose split-K scratch (pf16_conv_workspace_size(d,
+ *    PF16_PASS_WGRAD)) exceeds the array is rejected with PF16_ERR_WORKSPACE
+ *    before anything is launched; this includes the c == 3 stem, whose patch
+ *    buffer is far larger.  Every other ResNet-50 layer at batch 256 fits.
+ *  - The first call on each device looks up the array's device address (with
+ *    that device current); make that first call before any stream capture.
+ *  - All calls share the one array, which keeps the last call's contents
+ *    (no call depends on them).  Calls that can overlap on the GPU -- on
+ *    different streams, or on one device from several threads -- race on it;
+ *    order them on one stream or use pf16_conv_wgrad with separate workspaces. */
+#define PF16_WGRAD_NOALLOC_SCRATCH_BYTES (32u << 20)
+int pf16_conv_wgrad_noalloc(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy,
+                            uint16_t* dw, uint32_t flags, void* stream);
+
 /* ------------------------------------------------------------------- SGD
  * One step of SGD with momentum and coupled weight decay, the PyTorch
  * ImageNet recipe the paper adopts (Sec. 5.1), done entirely in FP16 with no

@@ -32,7 +32,7 @@ EXPORTS = [
     "pf16_sgd_update", "pf16_bn_workspace_size", "pf16_bn_fwd_bwd", "pf16_maxpool_fwd",
     "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
-    "pf16_status_string", "pf16_device_arch",
+    "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
 ]
 
 
@@ -83,6 +83,8 @@ def lib():
             for nm in ("pf16_conv_fwd", "pf16_conv_dgrad", "pf16_conv_wgrad"):
                 getattr(L, nm).argtypes = [cdp, vp, vp, vp, vp, sz, u32, vp]
                 getattr(L, nm).restype = I
+            L.pf16_conv_wgrad_noalloc.argtypes = [cdp, vp, vp, vp, u32, vp]
+            L.pf16_conv_wgrad_noalloc.restype = I
             L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
             L.pf16_sgd_update.restype = I
             L.pf16_bn_workspace_size.argtypes = [ctypes.POINTER(BnDesc)]
@@ -160,6 +162,16 @@ def conv_dgrad(d, dy, w, dx, ws=None, flags=0, stream=None):
 def conv_wgrad(d, x, dy, dw, ws=None, flags=0, stream=None):
     _check(lib().pf16_conv_wgrad(ctypes.byref(d), _ptr(x), _ptr(dy), _ptr(dw), _ptr(ws),
                                  _nbytes(ws), flags, _stream(stream)), "pf16_conv_wgrad")
+
+
+def conv_wgrad_noalloc(d, x, dy, dw, flags=0, stream=None):
+    """Weight gradient with the library's fixed internal scratch instead of a
+    caller workspace (for callers that cannot provide device memory)."""
+    _check(lib().pf16_conv_wgrad_noalloc(ctypes.byref(d), _ptr(x), _ptr(dy), _ptr(dw), flags,
+                                         _stream(stream)), "pf16_conv_wgrad_noalloc")
+
+
+WGRAD_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 def sgd_update(w, v, g, lr_bits, momentum_bits, wd_bits, flags=0, stream=None):
