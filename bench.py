@@ -162,10 +162,22 @@ def main():
     ap.add_argument("--impl", default="pf16", choices=["pf16", "reference"])
     ap.add_argument("--batch", type=int, default=BATCH)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--conv", default=None,
+                    help="time one conv pass instead of the step: N,H,W,C,K,R,S,stride,pad")
+    ap.add_argument("--pass", dest="conv_pass", default="fwd", choices=["fwd", "dgrad", "wgrad"])
+    ap.add_argument("--sweep", default=None, choices=["cfg2", "cfg3"],
+                    help="per-layer conv lines: cfg2 = every distinct ResNet-50 conv at N=64, "
+                         "cfg3 = the N=256 pure-GEMM 1x1 layers")
     args = ap.parse_args()
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.conv:
+        print(json.dumps(time_conv(tuple(int(v) for v in args.conv.split(",")), args.conv_pass,
+                                   args.steps, args.warmup)), flush=True)
+        return 0
+    if args.sweep:
+        return run_sweep(args)
     if args.warmup < 3:
         args.warmup = 3
 
@@ -290,6 +302,92 @@ def main():
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+CFG3 = [(256, 56, 56, 256, 64, 1, 1, 1, 0), (256, 28, 28, 512, 128, 1, 1, 1, 0),
+        (256, 14, 14, 1024, 256, 1, 1, 1, 0), (256, 7, 7, 512, 2048, 1, 1, 1, 0)]
+
+
+def run_sweep(args):
+    from paper_1911_07384_gb300.resnet50 import conv_shapes
+
+    if args.sweep == "cfg3":
+        shapes = [(f"cfg3_{i}", s) for i, s in enumerate(CFG3)]
+    else:
+        seen, shapes = set(), []
+        for name, s in conv_shapes(64):
+            if s not in seen:
+                seen.add(s)
+                shapes.append((name, s))
+    for name, s in shapes:
+        for ps in ("fwd", "dgrad", "wgrad"):
+            if ps == "dgrad" and s[3] == 3:
+                continue
+            r = time_conv(s, ps, args.steps, args.warmup)
+            r["layer"] = name
+            print(json.dumps(r), flush=True)
+    return 0
+
+
+def time_conv(shape, conv_pass, steps, warmup):
+    """One convolution pass on synthetic N(0,1) inputs, He weights, dy ~ N(0, 0.01^2):
+    `steps` launches timed with CUDA events on the launching stream; when the
+    operands fit in L2 a 256 MiB buffer is rewritten between launches."""
+    import torch
+
+    from paper_1911_07384_gb300 import pf16
+    from paper_1911_07384_gb300 import synthetic as syn
+
+    N, H, W, C, K, R, S, st, pd = shape
+    d = pf16.conv_desc(*shape)
+    P, Q = d.out_hw()
+    dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).cuda()
+    x = dev(syn.normal_f16(syn.seed_for(2, "x"), (N, H, W, C)))
+    w = dev(syn.he_normal_f16(syn.seed_for(2, "w"), K, R, S, C))
+    dy = dev(syn.normal_f16(syn.seed_for(2, "dy"), (N, P, Q, K), 0.01))
+    y = torch.empty(N * P * Q * K, dtype=torch.int16, device="cuda")
+    dx = torch.empty(N * H * W * C, dtype=torch.int16, device="cuda")
+    dw = torch.empty(K * R * S * C, dtype=torch.int16, device="cuda")
+    p = {"fwd": pf16.PF16_PASS_FWD, "dgrad": pf16.PF16_PASS_DGRAD, "wgrad": pf16.PF16_PASS_WGRAD}[conv_pass]
+    wsb = pf16.conv_workspace_size(d, p)
+    ws = torch.empty(max(wsb, 1), dtype=torch.uint8, device="cuda")
+    flush = None
+    io_bytes = 2 * (x.numel() + w.numel() + (y.numel() if conv_pass != "dgrad" else dy.numel()))
+    if io_bytes < 2 * 135 * 2 ** 20:
+        flush = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")
+    fn = {"fwd": lambda: pf16.conv_fwd(d, x, w, y, ws),
+          "dgrad": lambda: pf16.conv_dgrad(d, dy, w, dx),
+          "wgrad": lambda: pf16.conv_wgrad(d, x, dy, dw, ws)}[conv_pass]
+    for _ in range(max(warmup, 3)):
+        fn()
+    torch.cuda.synchronize()
+    times = []
+    s = torch.cuda.current_stream()
+    for _ in range(steps):
+        if flush is not None:
+            flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        fn()
+        e1.record(s)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    assert pf16.sync_status() == 0
+    ms = float(np.median(times))
+    flops = 2.0 * N * P * Q * K * C * R * S
+    byts = 2.0 * {"fwd": N * H * W * C + K * R * S * C + N * P * Q * K,
+                  "dgrad": N * P * Q * K + K * R * S * C + N * H * W * C,
+                  "wgrad": N * H * W * C + N * P * Q * K + K * R * S * C}[conv_pass]
+    pk = peaks()
+    tf = flops / ms / 1e9
+    gbs = byts / ms / 1e6
+    attainable = min(pk["bf16_tflops"], byts and flops / byts * pk["hbm_gbs"] / 1e3)
+    del x, w, dy, y, dx, dw, ws, flush
+    return {"metric": "conv pass TFLOP/s", "conv": list(shape), "pass": conv_pass, "ms": ms,
+            "ms_best": float(np.min(times)), "tflops": tf, "gbs": gbs,
+            "frac_of_dense_peak": tf / pk["bf16_tflops"],
+            "frac_of_attainable": tf / attainable, "arith_intensity": flops / byts,
+            "workspace_bytes": wsb, "l2_flush": io_bytes < 2 * 135 * 2 ** 20}
 
 
 def count_launches(net):

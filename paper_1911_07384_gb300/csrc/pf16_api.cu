@@ -161,6 +161,8 @@ int conv_shape(const pf16_conv_desc* d, Shape* s) {
     return PF16_ERR_SHAPE;
   if (d->c == 3) {
     if (d->k % 64 != 0) return PF16_ERR_UNSUPPORTED;
+    // the patch gather stages r padded input rows in shared memory
+    if ((long long)d->r * (d->w + 2 * d->pad) * 3 * 2 > 200 * 1024) return PF16_ERR_UNSUPPORTED;
     s->kind = KIND_STEM;
   } else if (d->h == 1 && d->w == 1 && d->r == 1 && d->s == 1 && d->pad == 0 && d->stride == 1) {
     if (d->c % 64 != 0 || d->k % 8 != 0) return PF16_ERR_UNSUPPORTED;
@@ -310,8 +312,20 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
                       false);
   const long long units = (long long)p.m_tiles * p.n_tiles * p.splits;
   if (units <= 0 || p.num_kb <= 0) return PF16_OK;
+  // Row-major outputs leave through TMA stores of 32-row x 64-column boxes; the
+  // split-K partials use a 3-D map so each split's plane is clipped on its own.
+  CUtensorMap c = a;
+  p.tma_store = 0;
+  if (p.out_mode == OUT_STORE && !p.remap) {
+    if (!map_2d(&c, p.out, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+    p.tma_store = 1;
+  } else if (p.out_mode == OUT_PARTIAL) {
+    if (!map_3d(&c, p.out, p.N, p.M, p.splits, p.ldo * 2, (uint64_t)p.M * p.ldo * 2, 64, 32, 1))
+      return PF16_ERR_CUDA;
+    p.tma_store = 1;
+  }
   const int grid = (int)std::min<long long>(units, sms);
-  return launch_gemm(BN, a, b, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+  return launch_gemm(BN, a, b, c, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
 int check_common(const void* a, const void* b, const void* c) {
@@ -668,6 +682,7 @@ int pf16_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int32_
                      int32_t w, int32_t c, void* stream) {
   int rc = pool_check(x, dx, n, h, w, c);
   if (rc != PF16_OK) return rc;
+  if (w > 1024) return PF16_ERR_UNSUPPORTED;  // a band of 11 input rows is staged in shared memory
   if (!dy) return PF16_ERR_NULL;
   if (!aligned16(dy)) return PF16_ERR_ALIGN;
   return launch_maxpool_bwd(x, dy, dx, n, h, w, c, static_cast<cudaStream_t>(stream)) ==

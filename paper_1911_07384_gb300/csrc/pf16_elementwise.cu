@@ -6,6 +6,8 @@
 // f16x2, never contracted), subnormals kept.  Global traffic is 128-bit.
 #include <cuda_fp16.h>
 
+#include <cstring>
+
 #include "pf16_internal.h"
 #include "pf16_ptx.cuh"
 
@@ -14,7 +16,6 @@ namespace pf16 {
 namespace {
 
 constexpr uint32_t kHalfHalf2 = 0x38003800u;  // {0.5, 0.5}
-constexpr uint32_t kZero2 = 0u;
 
 __host__ __device__ __forceinline__ uint32_t dup2(uint16_t h) { return (uint32_t)h | ((uint32_t)h << 16); }
 
@@ -166,20 +167,52 @@ cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, ui
 // Split-K weight-gradient reduction: out = balanced pairwise FP16 tree over
 // the `splits` partial matrices.
 // ============================================================================
-__global__ void k_splitk_reduce(const uint16_t* __restrict__ parts, int splits, long long rows,
-                                int cols, uint16_t* __restrict__ out, long long ldo,
-                                int cols_out) {
+// A CTA of 256 threads = cl output chunks (8 columns each) x grp split groups;
+// each thread sums a contiguous power-of-two run of splits (zero past the
+// last split) with batched independent loads, then the groups are summed
+// pairwise in shared memory: a balanced tree over the padded splits.
+__global__ void __launch_bounds__(256)
+    k_splitk_reduce(const uint16_t* __restrict__ parts, int splits, int splits_pow2, int grp,
+                    long long rows, int cols, uint16_t* __restrict__ out, long long ldo,
+                    int cols_out) {
+  __shared__ uint4 sh[256];
+  const int cl = 256 / grp;
+  const int t = threadIdx.x;
+  const int lane = t % cl, g = t / cl;
   const int cpr = cols / 8;
   const long long total = rows * cpr;
-  const long long plane = rows * (long long)cols;
-  for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (long long)gridDim.x * blockDim.x) {
-    const long long r = t / cpr;
-    const int cg = (int)(t - r * cpr);
+  const long long chunk = (long long)blockIdx.x * cl + lane;
+  const long long plane = rows * (long long)cols / 8;  // uint4 per partial plane
+  const int seg = splits_pow2 / grp;
+  uint4 acc = zero4();
+  if (chunk < total) {
+    const long long r = chunk / cpr;
+    const int cg = (int)(chunk - r * cpr);
     const uint4* src = reinterpret_cast<const uint4*>(parts + r * cols + cg * 8);
     Tree4<11, false> tree;
-    for (int s = 0; s < splits; ++s) tree.push(__ldg(src + (s * plane) / 8));
-    const uint4 v = tree.finish(ceil_log2(splits));
+    for (int i0 = 0; i0 < seg; i0 += 4) {
+      uint4 v[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int sp = g * seg + i0 + i;
+        v[i] = (i0 + i < seg && sp < splits) ? __ldg(src + sp * plane) : zero4();
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i0 + i < seg) tree.push(v[i]);
+    }
+    acc = tree.finish(ceil_log2(seg));
+  }
+  sh[t] = acc;
+  __syncthreads();
+  for (int half = grp / 2; half >= 1; half /= 2) {
+    if (g < half) sh[t] = add4(sh[t], sh[t + half * cl]);
+    __syncthreads();
+  }
+  if (g == 0 && chunk < total) {
+    const long long r = chunk / cpr;
+    const int cg = (int)(chunk - r * cpr);
+    const uint4 v = sh[t];
     const uint16_t* h = reinterpret_cast<const uint16_t*>(&v);
     uint16_t* o = out + r * ldo + cg * 8;
 #pragma unroll
@@ -190,55 +223,78 @@ __global__ void k_splitk_reduce(const uint16_t* __restrict__ parts, int splits, 
 
 cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long rows, int cols,
                                  uint16_t* out, long long ldo, int cols_out, cudaStream_t s) {
+  int sp2 = 1;
+  while (sp2 < splits) sp2 *= 2;
+  const int grp = sp2 < 32 ? sp2 : 32;
+  const int cl = 256 / grp;
   const long long total = rows * (cols / 8);
-  long long blocks = (total + 255) / 256;
-  if (blocks > 152 * 32) blocks = 152 * 32;
-  if (blocks < 1) blocks = 1;
-  k_splitk_reduce<<<(unsigned)blocks, 256, 0, s>>>(parts, splits, rows, cols, out, ldo, cols_out);
+  const long long blocks = (total + cl - 1) / cl;
+  k_splitk_reduce<<<(unsigned)blocks, 256, 0, s>>>(parts, splits, sp2, grp, rows, cols, out, ldo, cols_out);
   return cudaGetLastError();
 }
 
 // ============================================================================
 // Stem patch gather (c = 3 cannot be fetched by TMA: a pixel is 6 bytes).
 // col[m][j], m = (n, p, q), j = (r*S + s)*C + c < R*S*C, zero-padded to kcol.
+// One CTA per output row (n, p): the R input rows it needs are staged in
+// shared memory with `pad` zero pixels on each side, then each thread builds
+// the patch row of one output pixel and writes it with 16-byte stores.
 // ============================================================================
 __global__ void k_stem_im2col(const uint16_t* __restrict__ x, uint16_t* __restrict__ col, int N,
                               int H, int W, int P, int Q, int R, int S, int C, int stride, int pad,
                               int kcol) {
-  const int groups = kcol / 8;
-  const long long total = (long long)N * P * Q * groups;
+  extern __shared__ uint16_t rows[];  // [R][W + 2 pad][C], then the patch offset table
+  const int WP = W + 2 * pad;
+  const int rowlen = WP * C;
+  int* offs = reinterpret_cast<int*>(rows + ((R * rowlen + 1) & ~1));
+  const int n = blockIdx.x / P, p = blockIdx.x - n * P;
   const int kin = R * S * C;
-  for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (long long)gridDim.x * blockDim.x) {
-    const long long m = t / groups;
-    const int g = (int)(t - m * groups);
-    const int q = (int)(m % Q);
-    const int p = (int)((m / Q) % P);
-    const int n = (int)(m / ((long long)P * Q));
-    uint16_t v[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const int j = g * 8 + e;
-      uint16_t val = 0;
-      if (j < kin) {
-        const int c = j % C, rs = j / C;
-        const int s = rs % S, r = rs / S;
-        const int h = p * stride + r - pad, w = q * stride + s - pad;
-        if (h >= 0 && h < H && w >= 0 && w < W) val = x[(((long long)n * H + h) * W + w) * C + c];
-      }
-      v[e] = val;
+  for (int j = threadIdx.x; j < kcol; j += blockDim.x) {
+    if (j < kin) {
+      const int c = j % C, rs = j / C;
+      offs[j] = (rs / S) * rowlen + (rs % S) * C + c;
+    } else {
+      offs[j] = -1;
     }
-    *reinterpret_cast<uint4*>(col + m * kcol + g * 8) = *reinterpret_cast<uint4*>(v);
+  }
+  for (int r = 0; r < R; ++r) {
+    const int h = p * stride + r - pad;
+    uint16_t* dst = rows + r * rowlen;
+    const bool in = h >= 0 && h < H;
+    const uint16_t* src = x + ((long long)n * H + (in ? h : 0)) * W * C;
+    for (int e = threadIdx.x; e < rowlen; e += blockDim.x) {
+      const int src_e = e - pad * C;
+      dst[e] = (in && src_e >= 0 && src_e < W * C) ? src[src_e] : (uint16_t)0;
+    }
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < Q; q += blockDim.x) {
+    uint16_t* out = col + ((long long)blockIdx.x * Q + q) * kcol;
+    const uint16_t* base = rows + q * stride * C;
+    for (int g = 0; g < kcol; g += 8) {
+      uint16_t v[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const int o = offs[g + e];
+        v[e] = o >= 0 ? base[o] : (uint16_t)0;
+      }
+      *reinterpret_cast<uint4*>(out + g) = *reinterpret_cast<uint4*>(v);
+    }
   }
 }
 
 cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, int W, int P, int Q,
                                int R, int S, int C, int stride, int pad, int kcol,
                                cudaStream_t s) {
-  const long long total = (long long)N * P * Q * (kcol / 8);
-  long long blocks = (total + 255) / 256;
-  if (blocks > 152 * 64) blocks = 152 * 64;
-  k_stem_im2col<<<(unsigned)blocks, 256, 0, s>>>(x, col, N, H, W, P, Q, R, S, C, stride, pad, kcol);
+  const size_t shm = (((size_t)R * (W + 2 * pad) * C + 1) & ~(size_t)1) * sizeof(uint16_t) +
+                     (size_t)kcol * sizeof(int);
+  if (shm > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_stem_im2col, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)shm);
+    if (e != cudaSuccess) return e;
+  }
+  k_stem_im2col<<<(unsigned)((long long)N * P), 128, shm, s>>>(x, col, N, H, W, P, Q, R, S, C, stride,
+                                                               pad, kcol);
   return cudaGetLastError();
 }
 
@@ -266,193 +322,362 @@ cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s) {
 // BatchNorm (Eq. 1, Eq. 2, then x post_scale, + residual, ReLU), FP16 only.
 //
 // Statistics are means over the R rows of each channel computed as balanced
-// "halving" trees (node = rn(rn(a/2) + rn(b/2))) over R zero-padded to 2^L
-// leaves: thread-level trees over rows_per_thread leaves, a shared-memory
-// tree over the block's row groups, then a tree over the blocks' results in a
-// second kernel, and one final multiplication by rn(2^L / R).  Sums (for
-// dgamma, dbeta) are the same tree scaled back by 2^L exactly.
+// "halving" trees (node = rn(rn(a/2) + rn(b/2)), which cannot overflow).  A
+// CTA owns RB = rpb * 16 consecutive-ish rows (each thread 16 rows of one
+// group of 8 channels, kept in registers) and produces, per channel,
+//   forward:  its mean mu_b over its actual rows and the mean of (x - mu_b)^2
+//             over them (a second tree over the same registers: one HBM pass);
+//   backward: the padded means of dy' and dy' * xhat.
+// A second small kernel combines the per-CTA results over a balanced tree:
+// forward by the pairwise parallel-variance rule (counts kept exactly, so the
+// partial last CTA is weighted right), backward by halving trees scaled once
+// by rn(Bpow2*RB/R) for the means and by 2^L (exact power-of-two steps) for
+// the sums behind dgamma / dbeta.  Then one elementwise pass applies.
 // ============================================================================
 namespace {
 
 constexpr int kBnThreads = 256;
-constexpr int kBnMaxL = 8;  // rows per thread <= 256
+constexpr int kBnRpt = 16;  // rows per thread in the statistics kernels
 
 struct BnGeom {
   int tc;   // threads per row (channel groups of 8)
-  int rpb;  // row groups per block (power of two)
-  int rpt;  // rows per thread (power of two)
+  int rpb;  // row groups per CTA (power of two)
 };
 
-__host__ __device__ inline BnGeom bn_geom(int C, int rows_per_block) {
+__host__ __device__ inline BnGeom bn_geom(int C) {
   BnGeom g;
   g.tc = C / 8;
   int rpb = 1;
   while (rpb * 2 * g.tc <= kBnThreads) rpb *= 2;
   g.rpb = rpb;
-  g.rpt = rows_per_block / rpb;
   return g;
 }
 
-enum { BN_STAT_MEAN = 0, BN_STAT_VAR = 1, BN_STAT_BWD = 2 };
+struct BnStatArgs {
+  const uint16_t* x;
+  const uint16_t* dy;
+  const uint16_t* y_saved;
+  const uint16_t* mean_in;    // backward: saved mean
+  const uint16_t* invstd_in;  // backward: saved invstd
+  int R, C, blocks, blocks_pow2, total_levels;
+  uint16_t ratio;       // rn(Bpow2 * RB / R)
+  uint16_t last_scale;  // rn(RB / n_last): padded mean -> actual mean of the last CTA
+  uint16_t eps, post_scale;
+  int relu;
+  uint16_t* ws1;        // [blocks][C]
+  uint16_t* ws2;        // [blocks][C]
+  // outputs
+  uint16_t* mean_out;
+  uint16_t* invstd_out;
+  uint16_t* dgamma;
+  uint16_t* dbeta;
+  uint16_t* mm;         // backward: mean(dy'), mean(dy' xhat) for the apply pass, [2][C]
+};
 
-// Partial per-block means.  ws_out[block][C] (and ws_out2 for the backward).
-template <int MODE>
-__global__ void __launch_bounds__(kBnThreads)
-    k_bn_partial(const uint16_t* __restrict__ x, const uint16_t* __restrict__ dy,
-                 const uint16_t* __restrict__ y_saved, const uint16_t* __restrict__ mean,
-                 const uint16_t* __restrict__ invstd, int R, int C, int rows_per_block, int relu,
-                 uint16_t* __restrict__ ws_out, uint16_t* __restrict__ ws_out2) {
-  extern __shared__ uint4 sh[];
-  const BnGeom g = bn_geom(C, rows_per_block);
-  const int t = threadIdx.x;
-  const bool active = t < g.tc * g.rpb;
-  const int cg = t % g.tc, rg = t / g.tc;
-  const long long row0 = (long long)blockIdx.x * rows_per_block;
-  Tree4<kBnMaxL, true> t1, t2;
-  uint4 mu = zero4(), is = zero4();
-  if (active && MODE != BN_STAT_MEAN) mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
-  if (active && MODE == BN_STAT_BWD) is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
-  if (active) {
-    for (int i = 0; i < g.rpt; ++i) {
-      const long long r = row0 + rg + (long long)i * g.rpb;
-      uint4 l1 = zero4(), l2 = zero4();
-      if (r < R) {
-        const long long off = (r * C) / 8 + cg;
-        const uint4 xv = __ldg(reinterpret_cast<const uint4*>(x) + off);
-        if (MODE == BN_STAT_MEAN) {
-          l1 = xv;
-        } else if (MODE == BN_STAT_VAR) {
-          const uint4 d = sub4(xv, mu);
-          l1 = mul4v(d, d);
-        } else {
-          uint4 d = __ldg(reinterpret_cast<const uint4*>(dy) + off);
-          if (relu) {
-            const uint4 ys = __ldg(reinterpret_cast<const uint4*>(y_saved) + off);
-            d.x &= relu_mask2(ys.x);
-            d.y &= relu_mask2(ys.y);
-            d.z &= relu_mask2(ys.z);
-            d.w &= relu_mask2(ys.w);
-          }
-          const uint4 xh = mul4v(sub4(xv, mu), is);
-          l1 = d;
-          l2 = mul4v(d, xh);
-        }
-      }
-      t1.push(l1);
-      if (MODE == BN_STAT_BWD) t2.push(l2);
-    }
-  }
-  const int lv = 31 - __clz(g.rpt);
-  uint4* s1 = sh;
-  uint4* s2 = sh + kBnThreads;
-  if (active) {
-    s1[t] = t1.finish(lv);
-    if (MODE == BN_STAT_BWD) s2[t] = t2.finish(lv);
-  }
-  __syncthreads();
-  // tree over row groups: partner rg ^ half
-  for (int half = g.rpb / 2; half >= 1; half /= 2) {
-    if (active && rg < half) {
-      const int o = (rg + half) * g.tc + cg;
-      s1[t] = hmerge4(s1[t], s1[o]);
-      if (MODE == BN_STAT_BWD) s2[t] = hmerge4(s2[t], s2[o]);
-    }
+__device__ __forceinline__ uint4 tree16(uint4* v) {
+#pragma unroll
+  for (int w = 8; w >= 1; w /= 2)
+#pragma unroll
+    for (int i = 0; i < w; ++i) v[i] = hmerge4(v[2 * i], v[2 * i + 1]);
+  return v[0];
+}
+
+// halving tree over the rpb row groups of the CTA, in shared memory
+__device__ __forceinline__ void smem_tree(uint4* sh, int t, int tc, int rg, int rpb, bool active) {
+  for (int half = rpb / 2; half >= 1; half /= 2) {
+    if (active && rg < half) sh[t] = hmerge4(sh[t], sh[(rg + half) * tc + (t % tc)]);
     __syncthreads();
-  }
-  if (active && rg == 0) {
-    reinterpret_cast<uint4*>(ws_out)[(long long)blockIdx.x * g.tc + cg] = s1[t];
-    if (MODE == BN_STAT_BWD) reinterpret_cast<uint4*>(ws_out2)[(long long)blockIdx.x * g.tc + cg] = s2[t];
   }
 }
 
-// Tree over the per-block results (blocks zero-padded to blocks_pow2).  One
-// CTA of 256 threads per channel group of 8.
-template <int MODE>
-__global__ void __launch_bounds__(256)
-    k_bn_final(const uint16_t* __restrict__ ws1, const uint16_t* __restrict__ ws2, int C,
-               int blocks, int blocks_pow2, int total_levels, uint16_t ratio, uint16_t eps,
-               uint16_t post_scale, const uint16_t* __restrict__ gamma, uint16_t* __restrict__ out1,
-               uint16_t* __restrict__ out2, uint16_t* __restrict__ dgamma,
-               uint16_t* __restrict__ dbeta, uint16_t* __restrict__ m_out) {
-  __shared__ uint4 s1[256], s2[256];
-  const int tc = C / 8;
-  const int cg = blockIdx.x;
+__global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a) {
+  __shared__ uint4 sh[kBnThreads];
+  const BnGeom g = bn_geom(a.C);
   const int t = threadIdx.x;
-  const int nthr = blocks_pow2 < 256 ? blocks_pow2 : 256;
-  const int per = blocks_pow2 / nthr;  // power of two
+  const int cg = t % g.tc, rg = t / g.tc;
+  const bool active = t < g.tc * g.rpb;
+  const long long RB = (long long)g.rpb * kBnRpt;
+  const long long row0 = (long long)blockIdx.x * RB;
+  const bool last_cta = blockIdx.x == a.blocks - 1;
+  uint4 v[kBnRpt], d[kBnRpt];
+  bool ok[kBnRpt];
+#pragma unroll
+  for (int i = 0; i < kBnRpt; ++i) {
+    const long long r = row0 + rg + (long long)i * g.rpb;
+    ok[i] = active && r < a.R;
+    v[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
+    d[i] = v[i];
+  }
+  if (active) sh[t] = tree16(d);
+  __syncthreads();
+  smem_tree(sh, t, g.tc, rg, g.rpb, active);
+  uint4 mu = sh[cg];  // padded mean of this CTA
+  __syncthreads();
+  if (last_cta) mu = mul4(mu, dup2(a.last_scale));
+#pragma unroll
+  for (int i = 0; i < kBnRpt; ++i) {
+    const uint4 e = sub4(v[i], mu);
+    d[i] = ok[i] ? mul4v(e, e) : zero4();
+  }
+  if (active) sh[t] = tree16(d);
+  __syncthreads();
+  smem_tree(sh, t, g.tc, rg, g.rpb, active);
+  uint4 var = sh[cg];
+  if (last_cta) var = mul4(var, dup2(a.last_scale));
+  if (active && rg == 0) {
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = mu;
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = var;
+  }
+}
+
+// Combination of per-CTA (mean, variance) pairs by the pairwise parallel
+// variance rule: merging groups a and b with counts na, nb gives
+//   mean = wa*mean_a + wb*mean_b,  var = wa*var_a + wb*var_b + wa*wb*(mean_b - mean_a)^2,
+// wa = na/(na+nb).  For equal counts (every merge away from the partial last
+// CTA) this is exactly the halving merge of the means and of the variances
+// plus ((mean_b - mean_a)/2)^2.  Weights are constants of the counts.
+struct MV {
+  uint4 mu, v;
+  long long n;
+};
+
+__device__ __forceinline__ MV mv_merge(const MV& a, const MV& b) {
+  if (b.n == 0) return a;
+  if (a.n == 0) return b;
+  MV r;
+  r.n = a.n + b.n;
+  const uint4 d = sub4(b.mu, a.mu);
+  if (a.n == b.n) {
+    r.mu = hmerge4(a.mu, b.mu);
+    const uint4 dh = mul4(d, kHalfHalf2);
+    r.v = add4(hmerge4(a.v, b.v), mul4v(dh, dh));
+  } else {
+    const __half wa = __float2half_rn((float)((double)a.n / (double)r.n));
+    const __half wb = __float2half_rn((float)((double)b.n / (double)r.n));
+    const uint32_t wa2 = dup2(__half_as_ushort(wa)), wb2 = dup2(__half_as_ushort(wb));
+    const uint32_t wab2 = hmul2_rn(wa2, wb2);
+    r.mu = add4(mul4(a.mu, wa2), mul4(b.mu, wb2));
+    r.v = add4(add4(mul4(a.v, wa2), mul4(b.v, wb2)), mul4(mul4v(d, d), wab2));
+  }
+  return r;
+}
+
+constexpr int kFinalThreads = 256;
+
+// One CTA per group of 8 channels: each thread merges a contiguous run of
+// per-CTA results (loaded together), then the threads are merged in pairs in
+// shared memory; both levels follow a balanced binary tree.
+__global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs a, int rows_per_block) {
+  __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
+  __shared__ long long sn[kFinalThreads];
+  const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
+  const int nthr = a.blocks_pow2 < kFinalThreads ? a.blocks_pow2 : kFinalThreads;
+  const int seg = a.blocks_pow2 / nthr;
+  const long long n_last = (long long)a.R - (long long)(a.blocks - 1) * rows_per_block;
+  auto count = [&](int b) -> long long {
+    return b < a.blocks - 1 ? (long long)rows_per_block : (b == a.blocks - 1 ? n_last : 0);
+  };
   if (t < nthr) {
-    Tree4<12, true> a, b;
-    for (int i = 0; i < per; ++i) {
-      const int blk = t * per + i;
-      uint4 v1 = zero4(), v2 = zero4();
-      if (blk < blocks) {
-        v1 = __ldg(reinterpret_cast<const uint4*>(ws1) + (long long)blk * tc + cg);
-        if (MODE == BN_STAT_BWD) v2 = __ldg(reinterpret_cast<const uint4*>(ws2) + (long long)blk * tc + cg);
+    // binary-counter tree over this thread's seg slots (seg is a power of two)
+    MV st[12];
+    unsigned cnt = 0;
+    for (int i0 = 0; i0 < seg; i0 += 4) {
+      uint4 m[4], q[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int b = t * seg + i0 + i;
+        const bool ok = (i0 + i < seg) && b < a.blocks;
+        m[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws1) + (long long)b * tc + cg) : zero4();
+        q[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws2) + (long long)b * tc + cg) : zero4();
       }
-      a.push(v1);
-      if (MODE == BN_STAT_BWD) b.push(v2);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (i0 + i >= seg) break;
+        MV node{m[i], q[i], count(t * seg + i0 + i)};
+#pragma unroll
+        for (int l = 0; l < 12; ++l) {
+          if (cnt & (1u << l)) {
+            node = mv_merge(st[l], node);
+          } else {
+            st[l] = node;
+            break;
+          }
+        }
+        ++cnt;
+      }
     }
-    const int lv = 31 - __clz(per);
-    s1[t] = a.finish(lv);
-    if (MODE == BN_STAT_BWD) s2[t] = b.finish(lv);
+    const int lv = 31 - __clz(seg);  // seg == 2^lv, cnt == seg: the tree is st[lv]
+    MV res = st[0];
+#pragma unroll
+    for (int l = 0; l < 12; ++l)
+      if (l == lv) res = st[l];
+    smu[t] = res.mu;
+    sv[t] = res.v;
+    sn[t] = res.n;
+  }
+  __syncthreads();
+  for (int half = nthr / 2; half >= 1; half /= 2) {
+    if (t < half) {
+      const MV r = mv_merge(MV{smu[t], sv[t], sn[t]}, MV{smu[t + half], sv[t + half], sn[t + half]});
+      smu[t] = r.mu;
+      sv[t] = r.v;
+      sn[t] = r.n;
+    }
+    __syncthreads();
+  }
+  if (t == 0) {
+    const uint4 ve = add4(sv[0], make_uint4(dup2(a.eps), dup2(a.eps), dup2(a.eps), dup2(a.eps)));
+    uint4 is;
+    const __half2* hv = reinterpret_cast<const __half2*>(&ve);
+    __half2* hi = reinterpret_cast<__half2*>(&is);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) hi[j] = h2rsqrt(hv[j]);
+    reinterpret_cast<uint4*>(a.mean_out)[cg] = smu[0];
+    reinterpret_cast<uint4*>(a.invstd_out)[cg] = is;
+  }
+}
+
+// Backward: halving trees over the per-CTA padded means (zero padding is
+// exact for sums), then means (x rn(2^L/R)) and sums (x 2^L exactly).
+__global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs a) {
+  __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
+  const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
+  const int nthr = a.blocks_pow2 < kFinalThreads ? a.blocks_pow2 : kFinalThreads;
+  const int seg = a.blocks_pow2 / nthr;
+  if (t < nthr) {
+    Tree4<12, true> t1, t2;
+    for (int i0 = 0; i0 < seg; i0 += 4) {
+      uint4 p[4], q[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int b = t * seg + i0 + i;
+        const bool ok = (i0 + i < seg) && b < a.blocks;
+        p[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws1) + (long long)b * tc + cg) : zero4();
+        q[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws2) + (long long)b * tc + cg) : zero4();
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (i0 + i >= seg) break;
+        t1.push(p[i]);
+        t2.push(q[i]);
+      }
+    }
+    const int lv = 31 - __clz(seg);
+    s1[t] = t1.finish(lv);
+    s2[t] = t2.finish(lv);
   }
   __syncthreads();
   for (int half = nthr / 2; half >= 1; half /= 2) {
     if (t < half) {
       s1[t] = hmerge4(s1[t], s1[t + half]);
-      if (MODE == BN_STAT_BWD) s2[t] = hmerge4(s2[t], s2[t + half]);
+      s2[t] = hmerge4(s2[t], s2[t + half]);
     }
     __syncthreads();
   }
-  if (t != 0) return;
-  const uint32_t ratio2 = dup2(ratio);
-  if (MODE == BN_STAT_MEAN) {
-    reinterpret_cast<uint4*>(out1)[cg] = mul4(s1[0], ratio2);
-  } else if (MODE == BN_STAT_VAR) {
-    const uint4 var = mul4(s1[0], ratio2);
-    const uint4 ve = add4(var, make_uint4(dup2(eps), dup2(eps), dup2(eps), dup2(eps)));
-    uint4 r;
-    const __half2* hv = reinterpret_cast<const __half2*>(&ve);
-    __half2* hr = reinterpret_cast<__half2*>(&r);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) hr[j] = h2rsqrt(hv[j]);
-    reinterpret_cast<uint4*>(out2)[cg] = r;
-  } else {
-    // means for the elementwise pass, and the sums (tree * 2^L) for dbeta / dgamma
-    const uint4 m1 = mul4(s1[0], ratio2), m2 = mul4(s2[0], ratio2);
-    reinterpret_cast<uint4*>(m_out)[cg] = m1;
-    reinterpret_cast<uint4*>(m_out)[tc + cg] = m2;
-    const uint32_t ps = dup2(post_scale);
-    reinterpret_cast<uint4*>(dbeta)[cg] = mul4(ldexp4(s1[0], total_levels), ps);
-    reinterpret_cast<uint4*>(dgamma)[cg] = mul4(ldexp4(s2[0], total_levels), ps);
+  if (t == 0) {
+    const uint32_t ratio2 = dup2(a.ratio), ps = dup2(a.post_scale);
+    reinterpret_cast<uint4*>(a.mm)[cg] = mul4(s1[0], ratio2);
+    reinterpret_cast<uint4*>(a.mm)[tc + cg] = mul4(s2[0], ratio2);
+    reinterpret_cast<uint4*>(a.dbeta)[cg] = mul4(ldexp4(s1[0], a.total_levels), ps);
+    reinterpret_cast<uint4*>(a.dgamma)[cg] = mul4(ldexp4(s2[0], a.total_levels), ps);
   }
 }
+
+__global__ void __launch_bounds__(kBnThreads) k_bn_bwd_stats(const BnStatArgs a) {
+  __shared__ uint4 sh[kBnThreads];
+  const BnGeom g = bn_geom(a.C);
+  const int t = threadIdx.x;
+  const int cg = t % g.tc, rg = t / g.tc;
+  const bool active = t < g.tc * g.rpb;
+  const long long RB = (long long)g.rpb * kBnRpt;
+  const long long row0 = (long long)blockIdx.x * RB;
+  uint4 mu = zero4(), is = zero4();
+  if (active) {
+    mu = __ldg(reinterpret_cast<const uint4*>(a.mean_in) + cg);
+    is = __ldg(reinterpret_cast<const uint4*>(a.invstd_in) + cg);
+  }
+  Tree4<5, true> tr1, tr2;  // 16 leaves each, pushed in row order
+#pragma unroll
+  for (int h = 0; h < kBnRpt; h += 4) {
+    uint4 xs[4], ds[4], ys[4];
+    bool ok[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const long long r = row0 + rg + (long long)(h + i) * g.rpb;
+      ok[i] = active && r < a.R;
+      const long long off = (r * a.C) / 8 + cg;
+      xs[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + off) : zero4();
+      ds[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.dy) + off) : zero4();
+      ys[i] = (ok[i] && a.relu) ? __ldg(reinterpret_cast<const uint4*>(a.y_saved) + off) : zero4();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      uint4 dd = ds[i];
+      if (a.relu) {
+        dd.x &= relu_mask2(ys[i].x);
+        dd.y &= relu_mask2(ys[i].y);
+        dd.z &= relu_mask2(ys[i].z);
+        dd.w &= relu_mask2(ys[i].w);
+      }
+      const uint4 xh = mul4v(sub4(xs[i], mu), is);
+      tr1.push(dd);
+      tr2.push(ok[i] ? mul4v(dd, xh) : zero4());
+    }
+  }
+  if (active) sh[t] = tr1.finish(4);
+  __syncthreads();
+  smem_tree(sh, t, g.tc, rg, g.rpb, active);
+  const uint4 p1 = sh[cg];
+  __syncthreads();
+  if (active) sh[t] = tr2.finish(4);
+  __syncthreads();
+  smem_tree(sh, t, g.tc, rg, g.rpb, active);
+  const uint4 p2 = sh[cg];
+  if (active && rg == 0) {
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = p1;
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = p2;
+  }
+}
+
+constexpr int kApplyRows = 8;  // rows per thread per CTA in the apply passes
 
 __global__ void __launch_bounds__(256)
     k_bn_apply(const uint16_t* __restrict__ x, const uint16_t* __restrict__ gamma,
                const uint16_t* __restrict__ beta, const uint16_t* __restrict__ mean,
                const uint16_t* __restrict__ invstd, const uint16_t* __restrict__ residual,
-               uint16_t* __restrict__ y, long long total_vec, int tc, uint16_t post_scale,
-               int relu) {
+               uint16_t* __restrict__ y, int R, int C, int rpb, uint16_t post_scale, int relu) {
+  const int tc = C / 8;
+  const int t = threadIdx.x;
+  if (t >= tc * rpb) return;
+  const int cg = t % tc, rg = t / tc;
   const uint32_t ps = dup2(post_scale);
-  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total_vec;
-       i += (long long)gridDim.x * blockDim.x) {
-    const int cg = (int)(i % tc);
-    const uint4 xv = __ldg(reinterpret_cast<const uint4*>(x) + i);
-    const uint4 mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
-    const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
-    const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
-    const uint4 be = __ldg(reinterpret_cast<const uint4*>(beta) + cg);
-    const uint4 xh = mul4v(sub4(xv, mu), is);         // Eq. 1
+  const uint4 mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
+  const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
+  const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
+  const uint4 be = __ldg(reinterpret_cast<const uint4*>(beta) + cg);
+  const long long row0 = (long long)blockIdx.x * rpb * kApplyRows;
+  uint4 xv[kApplyRows], rv[kApplyRows];
+#pragma unroll
+  for (int i = 0; i < kApplyRows; ++i) {
+    const long long r = row0 + rg + (long long)i * rpb;
+    const long long off = (r * C) / 8 + cg;
+    xv[i] = r < R ? __ldg(reinterpret_cast<const uint4*>(x) + off) : zero4();
+    rv[i] = (r < R && residual) ? __ldg(reinterpret_cast<const uint4*>(residual) + off) : zero4();
+  }
+#pragma unroll
+  for (int i = 0; i < kApplyRows; ++i) {
+    const long long r = row0 + rg + (long long)i * rpb;
+    if (r >= R) break;
+    const uint4 xh = mul4v(sub4(xv[i], mu), is);      // Eq. 1
     uint4 z = mul4(add4(mul4v(ga, xh), be), ps);      // Eq. 2, then x post_scale
-    if (residual) z = add4(z, __ldg(reinterpret_cast<const uint4*>(residual) + i));
+    if (residual) z = add4(z, rv[i]);
     if (relu) {
       z.x = relu2(z.x);
       z.y = relu2(z.y);
       z.z = relu2(z.z);
       z.w = relu2(z.w);
     }
-    reinterpret_cast<uint4*>(y)[i] = z;
+    reinterpret_cast<uint4*>(y)[(r * C) / 8 + cg] = z;
   }
 }
 
@@ -461,31 +686,49 @@ __global__ void __launch_bounds__(256)
                    const uint16_t* __restrict__ mean, const uint16_t* __restrict__ invstd,
                    const uint16_t* __restrict__ dy, const uint16_t* __restrict__ y_saved,
                    const uint16_t* __restrict__ mm, uint16_t* __restrict__ dx,
-                   uint16_t* __restrict__ dres, long long total_vec, int tc, uint16_t post_scale,
+                   uint16_t* __restrict__ dres, int R, int C, int rpb, uint16_t post_scale,
                    int relu) {
+  const int tc = C / 8;
+  const int t = threadIdx.x;
+  if (t >= tc * rpb) return;
+  const int cg = t % tc, rg = t / tc;
   const uint32_t ps = dup2(post_scale);
-  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total_vec;
-       i += (long long)gridDim.x * blockDim.x) {
-    const int cg = (int)(i % tc);
-    uint4 d = __ldg(reinterpret_cast<const uint4*>(dy) + i);
-    if (relu) {
-      const uint4 ys = __ldg(reinterpret_cast<const uint4*>(y_saved) + i);
-      d.x &= relu_mask2(ys.x);
-      d.y &= relu_mask2(ys.y);
-      d.z &= relu_mask2(ys.z);
-      d.w &= relu_mask2(ys.w);
+  const uint4 mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
+  const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
+  const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
+  const uint4 m1 = __ldg(reinterpret_cast<const uint4*>(mm) + cg);
+  const uint4 m2 = __ldg(reinterpret_cast<const uint4*>(mm) + tc + cg);
+  const uint4 k = mul4v(mul4(ga, ps), is);  // s * gamma * invstd
+  const long long row0 = (long long)blockIdx.x * rpb * kApplyRows;
+#pragma unroll
+  for (int h = 0; h < kApplyRows; h += 4) {
+    uint4 xs[4], ds[4], ys[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const long long r = row0 + rg + (long long)(h + i) * rpb;
+      const long long off = (r * C) / 8 + cg;
+      const bool ok = r < R;
+      ds[i] = ok ? __ldg(reinterpret_cast<const uint4*>(dy) + off) : zero4();
+      xs[i] = ok ? __ldg(reinterpret_cast<const uint4*>(x) + off) : zero4();
+      ys[i] = (ok && relu) ? __ldg(reinterpret_cast<const uint4*>(y_saved) + off) : zero4();
     }
-    const uint4 xv = __ldg(reinterpret_cast<const uint4*>(x) + i);
-    const uint4 mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
-    const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
-    const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
-    const uint4 m1 = __ldg(reinterpret_cast<const uint4*>(mm) + cg);
-    const uint4 m2 = __ldg(reinterpret_cast<const uint4*>(mm) + tc + cg);
-    const uint4 xh = mul4v(sub4(xv, mu), is);
-    const uint4 k = mul4v(mul4(ga, ps), is);          // s * gamma * invstd
-    const uint4 t = sub4(sub4(d, m1), mul4v(xh, m2));  // dy' - mean(dy') - xhat*mean(dy'*xhat)
-    reinterpret_cast<uint4*>(dx)[i] = mul4v(k, t);
-    if (dres) reinterpret_cast<uint4*>(dres)[i] = d;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const long long r = row0 + rg + (long long)(h + i) * rpb;
+      if (r >= R) break;
+      uint4 d = ds[i];
+      if (relu) {
+        d.x &= relu_mask2(ys[i].x);
+        d.y &= relu_mask2(ys[i].y);
+        d.z &= relu_mask2(ys[i].z);
+        d.w &= relu_mask2(ys[i].w);
+      }
+      const uint4 xh = mul4v(sub4(xs[i], mu), is);
+      const uint4 tt = sub4(sub4(d, m1), mul4v(xh, m2));  // dy' - mean(dy') - xhat*mean(dy'*xhat)
+      const long long off = (r * C) / 8 + cg;
+      reinterpret_cast<uint4*>(dx)[off] = mul4v(k, tt);
+      if (dres) reinterpret_cast<uint4*>(dres)[off] = d;
+    }
   }
 }
 
@@ -501,20 +744,18 @@ unsigned grid_for(long long work, int per_block, int cap) {
 void bn_plan(int R, int C, BnLaunch* b) {
   b->R = R;
   b->C = C;
-  const BnGeom g0 = bn_geom(C, 1);
-  // rows per thread: aim for about 4 CTAs per SM, 8..128 rows per thread
-  int rpt = 8;
-  while (rpt < 128 && (long long)R / ((long long)g0.rpb * rpt * 2) >= 152 * 4) rpt *= 2;
-  b->rows_per_block = g0.rpb * rpt;
+  const BnGeom g = bn_geom(C);
+  b->rows_per_block = g.rpb * kBnRpt;
   b->blocks = (int)(((long long)R + b->rows_per_block - 1) / b->rows_per_block);
   int p2 = 1;
   while (p2 < b->blocks) p2 *= 2;
   b->blocks_pow2 = p2;
 }
 
+// [ws1: blocks*C] [ws2: blocks*C] [mm: 2*C]
 size_t bn_ws_bytes(const BnLaunch& b) {
-  // two per-block partial planes + the two per-channel means of the backward
-  return (size_t)2 * b.blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) + 256;
+  return 256 + (size_t)2 * b.blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) +
+         256;
 }
 
 static uint16_t f16_bits_host(float f) {
@@ -522,37 +763,42 @@ static uint16_t f16_bits_host(float f) {
   return *reinterpret_cast<uint16_t*>(&h);
 }
 
-static void bn_scale_consts(const BnLaunch& b, uint16_t* ratio, int* levels) {
+static BnStatArgs bn_args(const BnLaunch& b, uint16_t* ws) {
+  BnStatArgs a;
+  memset(&a, 0, sizeof(a));
+  a.R = b.R;
+  a.C = b.C;
+  a.blocks = b.blocks;
+  a.blocks_pow2 = b.blocks_pow2;
   const long long leaves = (long long)b.rows_per_block * b.blocks_pow2;
   int L = 0;
   while ((1ll << L) < leaves) ++L;
-  *levels = L;
-  *ratio = f16_bits_host((float)((double)leaves / (double)b.R));
+  a.total_levels = L;
+  a.ratio = f16_bits_host((float)((double)leaves / (double)b.R));
+  const long long n_last = (long long)b.R - (long long)(b.blocks - 1) * b.rows_per_block;
+  a.last_scale = f16_bits_host((float)((double)b.rows_per_block / (double)n_last));
+  a.eps = b.eps;
+  a.post_scale = b.post_scale;
+  a.relu = b.relu;
+  a.ws1 = ws;
+  a.ws2 = a.ws1 + (size_t)b.blocks * b.C;
+  a.mm = a.ws2 + (size_t)b.blocks * b.C;
+  return a;
 }
 
 cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* beta, const uint16_t* residual, uint16_t* y,
                           uint16_t* mean, uint16_t* invstd, uint16_t* ws, cudaStream_t s) {
-  uint16_t ratio;
-  int L;
-  bn_scale_consts(b, &ratio, &L);
-  const size_t shm = 2 * kBnThreads * sizeof(uint4);
-  uint16_t* part = ws;
-  k_bn_partial<BN_STAT_MEAN><<<b.blocks, kBnThreads, shm, s>>>(x, nullptr, nullptr, nullptr, nullptr,
-                                                               b.R, b.C, b.rows_per_block, 0, part,
-                                                               nullptr);
-  k_bn_final<BN_STAT_MEAN><<<b.C / 8, 256, 0, s>>>(part, nullptr, b.C, b.blocks, b.blocks_pow2, L,
-                                                   ratio, b.eps, b.post_scale, gamma, mean, nullptr,
-                                                   nullptr, nullptr, nullptr);
-  k_bn_partial<BN_STAT_VAR><<<b.blocks, kBnThreads, shm, s>>>(x, nullptr, nullptr, mean, nullptr, b.R,
-                                                              b.C, b.rows_per_block, 0, part,
-                                                              nullptr);
-  k_bn_final<BN_STAT_VAR><<<b.C / 8, 256, 0, s>>>(part, nullptr, b.C, b.blocks, b.blocks_pow2, L,
-                                                  ratio, b.eps, b.post_scale, gamma, nullptr, invstd,
-                                                  nullptr, nullptr, nullptr);
-  const long long tv = (long long)b.R * b.C / 8;
-  k_bn_apply<<<grid_for(tv, 256, 152 * 16), 256, 0, s>>>(x, gamma, beta, mean, invstd, residual, y, tv, b.C / 8,
-                                                         b.post_scale, b.relu);
+  BnStatArgs a = bn_args(b, ws);
+  a.x = x;
+  a.mean_out = mean;
+  a.invstd_out = invstd;
+  k_bn_fwd_stats<<<b.blocks, kBnThreads, 0, s>>>(a);
+  k_bn_fwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a, b.rows_per_block);
+  const BnGeom g = bn_geom(b.C);
+  const int rows = g.rpb * kApplyRows;
+  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, beta, mean, invstd, residual, y,
+                                                              b.R, b.C, g.rpb, b.post_scale, b.relu);
   return cudaGetLastError();
 }
 
@@ -560,21 +806,21 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
                           const uint16_t* y_saved, uint16_t* dx, uint16_t* dgamma,
                           uint16_t* dbeta, uint16_t* dres, uint16_t* ws, cudaStream_t s) {
-  uint16_t ratio;
-  int L;
-  bn_scale_consts(b, &ratio, &L);
-  const size_t shm = 2 * kBnThreads * sizeof(uint4);
-  uint16_t* p1 = ws;
-  uint16_t* p2 = ws + (size_t)b.blocks * b.C;
-  uint16_t* mm = ws + (size_t)2 * b.blocks * b.C;
-  k_bn_partial<BN_STAT_BWD><<<b.blocks, kBnThreads, shm, s>>>(x, dy, y_saved, mean, invstd, b.R, b.C,
-                                                              b.rows_per_block, b.relu, p1, p2);
-  k_bn_final<BN_STAT_BWD><<<b.C / 8, 256, 0, s>>>(p1, p2, b.C, b.blocks, b.blocks_pow2, L, ratio,
-                                                  b.eps, b.post_scale, gamma, nullptr, nullptr,
-                                                  dgamma, dbeta, mm);
-  const long long tv = (long long)b.R * b.C / 8;
-  k_bn_bwd_apply<<<grid_for(tv, 256, 152 * 16), 256, 0, s>>>(x, gamma, mean, invstd, dy, y_saved, mm, dx,
-                                                             dres, tv, b.C / 8, b.post_scale, b.relu);
+  BnStatArgs a = bn_args(b, ws);
+  a.x = x;
+  a.dy = dy;
+  a.y_saved = y_saved;
+  a.mean_in = mean;
+  a.invstd_in = invstd;
+  a.dgamma = dgamma;
+  a.dbeta = dbeta;
+  k_bn_bwd_stats<<<b.blocks, kBnThreads, 0, s>>>(a);
+  k_bn_bwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a);
+  const BnGeom g = bn_geom(b.C);
+  const int rows = g.rpb * kApplyRows;
+  k_bn_bwd_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, mean, invstd, dy, y_saved,
+                                                                  a.mm, dx, dres, b.R, b.C, g.rpb,
+                                                                  b.post_scale, b.relu);
   return cudaGetLastError();
 }
 
@@ -616,60 +862,98 @@ __global__ void k_maxpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restri
   }
 }
 
-__global__ void k_maxpool_bwd(const uint16_t* __restrict__ x, const uint16_t* __restrict__ dy,
-                              uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
+// Backward.  A CTA owns output-window rows [p0, p0 + kPoolTP) of one image
+// and one group of 8 channels, i.e. input rows [2 p0, 2 p0 + 2 kPoolTP).  It
+// stages input rows 2 p0 - 1 .. 2 p0 + 2 kPoolTP + 1 in shared memory, finds
+// each window's first maximum once (code r*3+s per channel, 0xFF if the
+// window has no valid cell), then every owned cell sums, in window order, the
+// gradients of the windows whose maximum it holds.
+constexpr int kPoolTP = 4;
+
+__global__ void __launch_bounds__(256)
+    k_maxpool_bwd(const uint16_t* __restrict__ x, const uint16_t* __restrict__ dy,
+                  uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
+  extern __shared__ uint4 band[];  // [2*kPoolTP + 3][W] cells of 8 channels
   const int tc = C / 8;
-  const long long total = (long long)N * H * W * tc;
-  for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (long long)gridDim.x * blockDim.x) {
-    const int cg = (int)(t % tc);
-    const long long pix = t / tc;
-    const int w = (int)(pix % W), h = (int)((pix / W) % H), n = (int)(pix / ((long long)H * W));
-    uint32_t acc[4] = {0, 0, 0, 0};
-    const int p_lo = h / 2, p_hi = min(P - 1, (h + 1) / 2);
-    const int q_lo = w / 2, q_hi = min(Q - 1, (w + 1) / 2);
-    for (int p = p_lo; p <= p_hi; ++p) {
-      if (h < 2 * p - 1 || h > 2 * p + 1) continue;
-      for (int q = q_lo; q <= q_hi; ++q) {
-        if (w < 2 * q - 1 || w > 2 * q + 1) continue;
-        // argmax of window (p, q): first maximum in r-then-s order
-        float m[8];
-        int arg[8];
+  const int bands = (P + kPoolTP - 1) / kPoolTP;
+  const int cg = blockIdx.x % tc;
+  const int rest = blockIdx.x / tc;
+  const int pb = rest % bands, n = rest / bands;
+  const int p0 = pb * kPoolTP;
+  const int h0 = 2 * p0 - 1;  // input row held in band row 0
+  constexpr int BR = 2 * kPoolTP + 3;
+  uint8_t* codes = reinterpret_cast<uint8_t*>(band + BR * W);  // [kPoolTP + 1][Q][8]
+  for (int i = threadIdx.x; i < BR * W; i += blockDim.x) {
+    const int br = i / W, w = i - br * W;
+    const int h = h0 + br;
+    band[i] = (h >= 0 && h < H) ? __ldg(reinterpret_cast<const uint4*>(x + (((long long)n * H + h) * W + w) * C) + cg)
+                                : make_uint4(0, 0, 0, 0);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < (kPoolTP + 1) * Q; i += blockDim.x) {
+    const int pp = i / Q, q = i - pp * Q;
+    const int p = p0 + pp;
+    float m[8];
+    uint8_t code[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          m[e] = -INFINITY;
-          arg[e] = -1;
-        }
-        for (int r = 0; r < 3; ++r) {
-          const int hh = 2 * p + r - 1;
-          if (hh < 0 || hh >= H) continue;
-          for (int s = 0; s < 3; ++s) {
-            const int ww = 2 * q + s - 1;
-            if (ww < 0 || ww >= W) continue;
-            const uint4 v =
-                __ldg(reinterpret_cast<const uint4*>(x + (((long long)n * H + hh) * W + ww) * C) + cg);
-            const __half* hv = reinterpret_cast<const __half*>(&v);
+    for (int e = 0; e < 8; ++e) {
+      m[e] = -INFINITY;
+      code[e] = 0xFF;
+    }
+    if (p < P) {
+      for (int r = 0; r < 3; ++r) {
+        const int h = 2 * p + r - 1;
+        if (h < 0 || h >= H) continue;
+        for (int c = 0; c < 3; ++c) {
+          const int w = 2 * q + c - 1;
+          if (w < 0 || w >= W) continue;
+          const uint4 v = band[(h - h0) * W + w];
+          const __half* hv = reinterpret_cast<const __half*>(&v);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float f = __half2float(hv[e]);
-              if (f > m[e]) {
-                m[e] = f;
-                arg[e] = hh * W + ww;
-              }
+          for (int e = 0; e < 8; ++e) {
+            const float f = __half2float(hv[e]);
+            if (f > m[e]) {
+              m[e] = f;
+              code[e] = (uint8_t)(r * 3 + c);
             }
           }
         }
-        const uint4 g = __ldg(reinterpret_cast<const uint4*>(dy + (((long long)n * P + p) * Q + q) * C) + cg);
-        const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g);
-        const int me = h * W + w;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t sel = (arg[2 * j] == me ? 0x0000FFFFu : 0u) | (arg[2 * j + 1] == me ? 0xFFFF0000u : 0u);
-          if (sel) acc[j] = hadd2_rn(acc[j], gw[j] & sel);
-        }
       }
     }
-    reinterpret_cast<uint4*>(dx)[t] = make_uint4(acc[0], acc[1], acc[2], acc[3]);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) codes[i * 8 + e] = code[e];
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 2 * kPoolTP * W; i += blockDim.x) {
+    const int hh = i / W, w = i - hh * W;
+    const int h = 2 * p0 + hh;
+    if (h >= H) continue;
+    uint32_t acc[4] = {0, 0, 0, 0};
+    const int p_lo = h / 2, p_hi = (h + 1) / 2;  // windows covering row h
+    for (int p = p_lo; p <= p_hi; ++p) {
+      if (p >= P || h < 2 * p - 1 || h > 2 * p + 1) continue;
+      const int pp = p - p0;  // 0 .. kPoolTP
+      for (int q = w / 2; q <= (w + 1) / 2; ++q) {
+        if (q >= Q || w < 2 * q - 1 || w > 2 * q + 1) continue;
+        const uint8_t* cd = codes + (pp * Q + q) * 8;
+        const uint8_t mine = (uint8_t)((h - (2 * p - 1)) * 3 + (w - (2 * q - 1)));
+        uint32_t sel[4];
+        bool any = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          sel[j] = (cd[2 * j] == mine ? 0x0000FFFFu : 0u) | (cd[2 * j + 1] == mine ? 0xFFFF0000u : 0u);
+          any |= sel[j] != 0;
+        }
+        if (!any) continue;
+        const uint4 g = __ldg(reinterpret_cast<const uint4*>(dy + (((long long)n * P + p) * Q + q) * C) + cg);
+        const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (sel[j]) acc[j] = hadd2_rn(acc[j], gw[j] & sel[j]);
+      }
+    }
+    reinterpret_cast<uint4*>(dx + (((long long)n * H + h) * W + w) * C)[cg] =
+        make_uint4(acc[0], acc[1], acc[2], acc[3]);
   }
 }
 
@@ -684,8 +968,13 @@ cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, int N, int H, int
 cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int N, int H,
                                int W, int C, cudaStream_t s) {
   const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
-  const long long total = (long long)N * H * W * (C / 8);
-  k_maxpool_bwd<<<grid_for(total, 256, 152 * 16), 256, 0, s>>>(x, dy, dx, N, H, W, C, P, Q);
+  const int bands = (P + kPoolTP - 1) / kPoolTP;
+  const size_t shm = (size_t)(2 * kPoolTP + 3) * W * sizeof(uint4) + (size_t)(kPoolTP + 1) * Q * 8;
+  if (shm > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_maxpool_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    if (e != cudaSuccess) return e;
+  }
+  k_maxpool_bwd<<<(unsigned)((long long)N * bands * (C / 8)), 256, shm, s>>>(x, dy, dx, N, H, W, C, P, Q);
   return cudaGetLastError();
 }
 

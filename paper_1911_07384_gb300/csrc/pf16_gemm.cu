@@ -29,8 +29,9 @@ struct GemmCfg {
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : (BN == 192 ? 5 : 4));
   static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
+  static constexpr int STAGING_BYTES = 4 * 4096;  // per epilogue warp: 32 rows x 64 cols
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
-  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES;
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
 };
 
 static constexpr int kErrTimeout = -7;  // PF16_ERR_TIMEOUT
@@ -146,12 +147,13 @@ __device__ __forceinline__ uint32_t pack_lo(uint32_t a, uint32_t b) { return __b
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-           const __grid_constant__ GemmParams p) {
+           const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
   using Cfg = GemmCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES);
+  uint8_t* staging = smem + Cfg::STAGES * Cfg::STAGE_BYTES;  // 1024-aligned, 4 KB per epilogue warp
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + Cfg::STAGES;
   uint64_t* tfull = bars + 2 * Cfg::STAGES;
@@ -173,6 +175,7 @@ __global__ void __launch_bounds__(192, 1)
     fence_mbar_init();
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapB);
+    if (p.tma_store) tma_prefetch_desc(&mapC);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
@@ -189,6 +192,7 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
+      uint32_t issued = 0;  // stages loaded so far (for the drain below)
       for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
         int m0, n0, split, kb0, kb1;
         unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
@@ -202,10 +206,25 @@ __global__ void __launch_bounds__(192, 1)
           mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
           load_a(p, &mapA, sa, fb, m0, kb);
           load_b<BN>(p, &mapB, sa + Cfg::A_BYTES, fb, n0, kb);
+          ++issued;
           if (++stage == Cfg::STAGES) {
             stage = 0;
             phase ^= 1;
           }
+        }
+      }
+      if (*abort_flag) {
+        // Another role gave up: let the copies this thread started land before
+        // the CTA's shared memory is released (each wait bounded on its own).
+        const uint32_t n = issued < (uint32_t)Cfg::STAGES ? issued : (uint32_t)Cfg::STAGES;
+        int s = stage;
+        uint32_t ph = phase;
+        for (uint32_t i = 0; i < n; ++i) {
+          if (--s < 0) {
+            s = Cfg::STAGES - 1;
+            ph ^= 1;
+          }
+          mbar_wait(smem_u32(&full[s]), ph, 1000000000ull);
         }
       }
     }
@@ -269,10 +288,51 @@ __global__ void __launch_bounds__(192, 1)
         break;
       }
       tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
+      if (p.tma_store) {
+        // 64-column chunks: TMEM -> registers -> 128B-swizzled staging -> TMA store
+        const uint32_t stg = smem_u32(staging) + (uint32_t)(sub * 4096);
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 64) {
+          uint32_t r[64];
+          tmem_ld16(tbase + c, r);
+          tmem_ld16(tbase + c + 16, r + 16);
+          tmem_ld16(tbase + c + 32, r + 32);
+          tmem_ld16(tbase + c + 48, r + 48);
+          tmem_ld_wait();
+          if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+          }
+          if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            uint4 v;
+            v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
+            v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
+            v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
+            v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
+            st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            if (p.out_mode == OUT_PARTIAL)
+              tma_store_3d(&mapC, stg, n0 + c, m0 + sub * 32, split);
+            else
+              tma_store_2d(&mapC, stg, n0 + c, m0 + sub * 32);
+            bulk_commit();
+          }
+        }
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+        continue;
+      }
       const int m = m0 + row;
       const bool row_ok = m < p.M;
       uint16_t* orow = row_ok ? out_row(p, m, split) : nullptr;
-      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll 1
       for (int c = 0; c < BN; c += 32) {
         uint32_t r[32];
@@ -308,6 +368,7 @@ __global__ void __launch_bounds__(192, 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
+    if (p.tma_store && lane == 0) bulk_wait0();
   }
   tc_fence_before();
   __syncthreads();
@@ -328,8 +389,8 @@ int gemm_smem_bytes(int BN) {
 }
 
 template <int BN>
-static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const GemmParams& p,
-                               int grid, cudaStream_t s) {
+static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                               const GemmParams& p, int grid, cudaStream_t s) {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
@@ -339,17 +400,17 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  k_gemm<BN><<<grid, 192, GemmCfg<BN>::SMEM, s>>>(mA, mB, p);
+  k_gemm<BN><<<grid, 192, GemmCfg<BN>::SMEM, s>>>(mA, mB, mC, p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const GemmParams& p,
-                        int grid, cudaStream_t s) {
+cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                        const GemmParams& p, int grid, cudaStream_t s) {
   switch (BN) {
-    case 64: return launch_bn_t<64>(mA, mB, p, grid, s);
-    case 128: return launch_bn_t<128>(mA, mB, p, grid, s);
-    case 192: return launch_bn_t<192>(mA, mB, p, grid, s);
-    case 256: return launch_bn_t<256>(mA, mB, p, grid, s);
+    case 64: return launch_bn_t<64>(mA, mB, mC, p, grid, s);
+    case 128: return launch_bn_t<128>(mA, mB, mC, p, grid, s);
+    case 192: return launch_bn_t<192>(mA, mB, mC, p, grid, s);
+    case 256: return launch_bn_t<256>(mA, mB, mC, p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

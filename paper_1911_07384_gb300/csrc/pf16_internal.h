@@ -66,6 +66,7 @@ struct GemmParams {
   int8_t tap_w[kMaxTaps];                     // weight tap index r*S+s (TAP3D_MN)
   // epilogue
   int out_mode;
+  int tma_store;          // 1: rows written by TMA stores through mapC (row-major, no remap)
   uint16_t* out;
   long long ldo;          // output row stride (elements)
   int remap;              // rows -> strided positions of a stride phase
@@ -80,7 +81,8 @@ struct GemmParams {
 
 // Launch the engine (BN in {64, 128, 192, 256}).  Returns a cudaError_t.
 cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmParams& p, int grid, cudaStream_t stream);
+                        const CUtensorMap& mapC, const GemmParams& p, int grid,
+                        cudaStream_t stream);
 int gemm_smem_bytes(int BN);
 
 // ---------------------------------------------------------------------------

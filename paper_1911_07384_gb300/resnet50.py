@@ -33,6 +33,28 @@ S_STEM = 0x3C00   # 1.0: the stem BatchNorm
 STAGES = [(64, 3, 1), (128, 4, 2), (256, 6, 2), (512, 3, 2)]  # width, blocks, stride
 
 
+def conv_shapes(batch=256, image=224, classes=1000):
+    """(name, (N, H, W, C, K, R, S, stride, pad)) of every conv of the network, in
+    forward order, without allocating anything."""
+    out = [("stem", (batch, image, image, 3, 64, 7, 7, 2, 3))]
+    h = (image + 6 - 7) // 2 + 1
+    h = (h - 1) // 2 + 1
+    cin = 64
+    for si, (width, nb, stride) in enumerate(STAGES):
+        for b in range(nb):
+            st = stride if b == 0 else 1
+            h2 = (h + 2 - 3) // st + 1
+            nm = f"s{si + 1}b{b}"
+            out.append((nm + ".conv1", (batch, h, h, cin, width, 1, 1, 1, 0)))
+            out.append((nm + ".conv2", (batch, h, h, width, width, 3, 3, st, 1)))
+            out.append((nm + ".conv3", (batch, h2, h2, width, 4 * width, 1, 1, 1, 0)))
+            if b == 0:
+                out.append((nm + ".proj", (batch, h, h, cin, 4 * width, 1, 1, st, 0)))
+            h, cin = h2, 4 * width
+    out.append(("fc", (batch, 1, 1, cin, classes, 1, 1, 1, 0)))
+    return out
+
+
 def _a8(n):
     return (n + 7) // 8 * 8
 
