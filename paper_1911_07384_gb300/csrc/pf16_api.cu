@@ -312,11 +312,12 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
                       false);
   const long long units = (long long)p.m_tiles * p.n_tiles * p.splits;
   if (units <= 0 || p.num_kb <= 0) return PF16_OK;
-  // Row-major outputs leave through TMA stores of 32-row x 64-column boxes; the
+  // Row-major outputs leave through TMA stores of 32-row x 64-column boxes
+  // (PF16_ACCUMULATE through TMA reduce-add stores, out = rn(out + tile)); the
   // split-K partials use a 3-D map so each split's plane is clipped on its own.
   CUtensorMap c = a;
   p.tma_store = 0;
-  if (p.out_mode == OUT_STORE && !p.remap) {
+  if ((p.out_mode == OUT_STORE || p.out_mode == OUT_ACCUM) && !p.remap) {
     if (!map_2d(&c, p.out, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
     p.tma_store = 1;
   } else if (p.out_mode == OUT_PARTIAL) {

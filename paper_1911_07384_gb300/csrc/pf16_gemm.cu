@@ -321,6 +321,8 @@ __global__ void __launch_bounds__(192, 1)
           if (lane == 0) {
             if (p.out_mode == OUT_PARTIAL)
               tma_store_3d(&mapC, stg, n0 + c, m0 + sub * 32, split);
+            else if (p.out_mode == OUT_ACCUM)
+              tma_reduce_add_2d(&mapC, stg, n0 + c, m0 + sub * 32);
             else
               tma_store_2d(&mapC, stg, n0 + c, m0 + sub * 32);
             bulk_commit();
