@@ -360,6 +360,7 @@ struct BnStatArgs {
   const uint16_t* mean_in;    // backward: saved mean
   const uint16_t* invstd_in;  // backward: saved invstd
   int R, C, blocks, blocks_pow2, total_levels;
+  int chunks_per_cta;   // row chunks (of rpb * 16 rows) per statistics CTA, a power of two
   uint16_t ratio;       // rn(Bpow2 * RB / R)
   uint16_t last_scale;  // rn(RB / n_last): padded mean -> actual mean of the last CTA
   uint16_t eps, post_scale;
@@ -387,46 +388,6 @@ __device__ __forceinline__ void smem_tree(uint4* sh, int t, int tc, int rg, int 
   for (int half = rpb / 2; half >= 1; half /= 2) {
     if (active && rg < half) sh[t] = hmerge4(sh[t], sh[(rg + half) * tc + (t % tc)]);
     __syncthreads();
-  }
-}
-
-__global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a) {
-  __shared__ uint4 sh[kBnThreads];
-  const BnGeom g = bn_geom(a.C);
-  const int t = threadIdx.x;
-  const int cg = t % g.tc, rg = t / g.tc;
-  const bool active = t < g.tc * g.rpb;
-  const long long RB = (long long)g.rpb * kBnRpt;
-  const long long row0 = (long long)blockIdx.x * RB;
-  const bool last_cta = blockIdx.x == a.blocks - 1;
-  uint4 v[kBnRpt], d[kBnRpt];
-  bool ok[kBnRpt];
-#pragma unroll
-  for (int i = 0; i < kBnRpt; ++i) {
-    const long long r = row0 + rg + (long long)i * g.rpb;
-    ok[i] = active && r < a.R;
-    v[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
-    d[i] = v[i];
-  }
-  if (active) sh[t] = tree16(d);
-  __syncthreads();
-  smem_tree(sh, t, g.tc, rg, g.rpb, active);
-  uint4 mu = sh[cg];  // padded mean of this CTA
-  __syncthreads();
-  if (last_cta) mu = mul4(mu, dup2(a.last_scale));
-#pragma unroll
-  for (int i = 0; i < kBnRpt; ++i) {
-    const uint4 e = sub4(v[i], mu);
-    d[i] = ok[i] ? mul4v(e, e) : zero4();
-  }
-  if (active) sh[t] = tree16(d);
-  __syncthreads();
-  smem_tree(sh, t, g.tc, rg, g.rpb, active);
-  uint4 var = sh[cg];
-  if (last_cta) var = mul4(var, dup2(a.last_scale));
-  if (active && rg == 0) {
-    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = mu;
-    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = var;
   }
 }
 
@@ -460,6 +421,72 @@ __device__ __forceinline__ MV mv_merge(const MV& a, const MV& b) {
     r.v = add4(add4(mul4(a.v, wa2), mul4(b.v, wb2)), mul4(mul4v(d, d), wab2));
   }
   return r;
+}
+
+__global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a) {
+  __shared__ uint4 sh[kBnThreads];
+  const BnGeom g = bn_geom(a.C);
+  const int t = threadIdx.x;
+  const int cg = t % g.tc, rg = t / g.tc;
+  const bool active = t < g.tc * g.rpb;
+  const long long RB = (long long)g.rpb * kBnRpt;  // rows of one chunk
+  const long long total_chunks = (a.R + RB - 1) / RB;
+  MV st[8];  // binary counter over this CTA's chunks (held by the rg == 0 threads)
+  unsigned cnt = 0;
+  for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
+    const long long chunk = (long long)blockIdx.x * a.chunks_per_cta + ci;
+    if (chunk >= total_chunks) break;
+    const long long row0 = chunk * RB;
+    const bool last_chunk = chunk == total_chunks - 1;
+    uint4 v[kBnRpt], d[kBnRpt];
+    bool ok[kBnRpt];
+#pragma unroll
+    for (int i = 0; i < kBnRpt; ++i) {
+      const long long r = row0 + rg + (long long)i * g.rpb;
+      ok[i] = active && r < a.R;
+      v[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
+      d[i] = v[i];
+    }
+    if (active) sh[t] = tree16(d);
+    __syncthreads();
+    smem_tree(sh, t, g.tc, rg, g.rpb, active);
+    uint4 mu = sh[cg];  // padded mean of the chunk
+    __syncthreads();
+    if (last_chunk) mu = mul4(mu, dup2(a.last_scale));
+#pragma unroll
+    for (int i = 0; i < kBnRpt; ++i) {
+      const uint4 e = sub4(v[i], mu);
+      d[i] = ok[i] ? mul4v(e, e) : zero4();
+    }
+    if (active) sh[t] = tree16(d);
+    __syncthreads();
+    smem_tree(sh, t, g.tc, rg, g.rpb, active);
+    uint4 var = sh[cg];
+    __syncthreads();
+    if (last_chunk) var = mul4(var, dup2(a.last_scale));
+    if (active && rg == 0) {
+      MV node{mu, var, last_chunk ? a.R - row0 : RB};
+#pragma unroll
+      for (int l = 0; l < 8; ++l) {
+        if (cnt & (1u << l)) {
+          node = mv_merge(st[l], node);
+        } else {
+          st[l] = node;
+          break;
+        }
+      }
+      ++cnt;
+    }
+  }
+  if (active && rg == 0 && cnt) {
+    // fold the counter: remaining nodes from the lowest level (the latest rows) up
+    MV acc{zero4(), zero4(), 0};
+#pragma unroll
+    for (int l = 0; l < 8; ++l)
+      if (cnt & (1u << l)) acc = mv_merge(st[l], acc);
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = acc.mu;
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = acc.v;
+  }
 }
 
 constexpr int kFinalThreads = 256;
@@ -590,52 +617,61 @@ __global__ void __launch_bounds__(kBnThreads) k_bn_bwd_stats(const BnStatArgs a)
   const int cg = t % g.tc, rg = t / g.tc;
   const bool active = t < g.tc * g.rpb;
   const long long RB = (long long)g.rpb * kBnRpt;
-  const long long row0 = (long long)blockIdx.x * RB;
   uint4 mu = zero4(), is = zero4();
   if (active) {
     mu = __ldg(reinterpret_cast<const uint4*>(a.mean_in) + cg);
     is = __ldg(reinterpret_cast<const uint4*>(a.invstd_in) + cg);
   }
-  Tree4<5, true> tr1, tr2;  // 16 leaves each, pushed in row order
+  Tree4<8, true> c1, c2;  // halving trees over this CTA's chunks (rg == 0 threads)
+  for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
+    const long long row0 = ((long long)blockIdx.x * a.chunks_per_cta + ci) * RB;
+    Tree4<5, true> tr1, tr2;  // 16 leaves each, pushed in row order
 #pragma unroll
-  for (int h = 0; h < kBnRpt; h += 4) {
-    uint4 xs[4], ds[4], ys[4];
-    bool ok[4];
+    for (int h = 0; h < kBnRpt; h += 4) {
+      uint4 xs[4], ds[4], ys[4];
+      bool ok[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const long long r = row0 + rg + (long long)(h + i) * g.rpb;
-      ok[i] = active && r < a.R;
-      const long long off = (r * a.C) / 8 + cg;
-      xs[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + off) : zero4();
-      ds[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.dy) + off) : zero4();
-      ys[i] = (ok[i] && a.relu) ? __ldg(reinterpret_cast<const uint4*>(a.y_saved) + off) : zero4();
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      uint4 dd = ds[i];
-      if (a.relu) {
-        dd.x &= relu_mask2(ys[i].x);
-        dd.y &= relu_mask2(ys[i].y);
-        dd.z &= relu_mask2(ys[i].z);
-        dd.w &= relu_mask2(ys[i].w);
+      for (int i = 0; i < 4; ++i) {
+        const long long r = row0 + rg + (long long)(h + i) * g.rpb;
+        ok[i] = active && r < a.R;
+        const long long off = (r * a.C) / 8 + cg;
+        xs[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + off) : zero4();
+        ds[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.dy) + off) : zero4();
+        ys[i] = (ok[i] && a.relu) ? __ldg(reinterpret_cast<const uint4*>(a.y_saved) + off) : zero4();
       }
-      const uint4 xh = mul4v(sub4(xs[i], mu), is);
-      tr1.push(dd);
-      tr2.push(ok[i] ? mul4v(dd, xh) : zero4());
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        uint4 dd = ds[i];
+        if (a.relu) {
+          dd.x &= relu_mask2(ys[i].x);
+          dd.y &= relu_mask2(ys[i].y);
+          dd.z &= relu_mask2(ys[i].z);
+          dd.w &= relu_mask2(ys[i].w);
+        }
+        const uint4 xh = mul4v(sub4(xs[i], mu), is);
+        tr1.push(dd);
+        tr2.push(ok[i] ? mul4v(dd, xh) : zero4());
+      }
+    }
+    if (active) sh[t] = tr1.finish(4);
+    __syncthreads();
+    smem_tree(sh, t, g.tc, rg, g.rpb, active);
+    const uint4 p1 = sh[cg];
+    __syncthreads();
+    if (active) sh[t] = tr2.finish(4);
+    __syncthreads();
+    smem_tree(sh, t, g.tc, rg, g.rpb, active);
+    const uint4 p2 = sh[cg];
+    __syncthreads();
+    if (active && rg == 0) {
+      c1.push(p1);
+      c2.push(p2);
     }
   }
-  if (active) sh[t] = tr1.finish(4);
-  __syncthreads();
-  smem_tree(sh, t, g.tc, rg, g.rpb, active);
-  const uint4 p1 = sh[cg];
-  __syncthreads();
-  if (active) sh[t] = tr2.finish(4);
-  __syncthreads();
-  smem_tree(sh, t, g.tc, rg, g.rpb, active);
-  const uint4 p2 = sh[cg];
   if (active && rg == 0) {
-    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = p1;
-    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = p2;
+    const int lv = 31 - __clz(a.chunks_per_cta);
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = c1.finish(lv);
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = c2.finish(lv);
   }
 }
 
@@ -745,8 +781,14 @@ void bn_plan(int R, int C, BnLaunch* b) {
   b->R = R;
   b->C = C;
   const BnGeom g = bn_geom(C);
-  b->rows_per_block = g.rpb * kBnRpt;
-  b->blocks = (int)(((long long)R + b->rows_per_block - 1) / b->rows_per_block);
+  const long long chunk = (long long)g.rpb * kBnRpt;
+  const long long chunks = ((long long)R + chunk - 1) / chunk;
+  // about four statistics CTAs per SM, each over a power-of-two number of chunks
+  int cpc = 1;
+  while (cpc < 128 && chunks > (long long)cpc * 152 * 4) cpc *= 2;
+  b->chunks_per_cta = cpc;
+  b->rows_per_block = (int)(chunk * cpc);
+  b->blocks = (int)((chunks + cpc - 1) / cpc);
   int p2 = 1;
   while (p2 < b->blocks) p2 *= 2;
   b->blocks_pow2 = p2;
@@ -770,13 +812,15 @@ static BnStatArgs bn_args(const BnLaunch& b, uint16_t* ws) {
   a.C = b.C;
   a.blocks = b.blocks;
   a.blocks_pow2 = b.blocks_pow2;
+  a.chunks_per_cta = b.chunks_per_cta;
   const long long leaves = (long long)b.rows_per_block * b.blocks_pow2;
   int L = 0;
   while ((1ll << L) < leaves) ++L;
   a.total_levels = L;
   a.ratio = f16_bits_host((float)((double)leaves / (double)b.R));
-  const long long n_last = (long long)b.R - (long long)(b.blocks - 1) * b.rows_per_block;
-  a.last_scale = f16_bits_host((float)((double)b.rows_per_block / (double)n_last));
+  const long long chunk_rows = b.rows_per_block / b.chunks_per_cta;
+  const long long n_last = (long long)b.R - (((long long)b.R - 1) / chunk_rows) * chunk_rows;
+  a.last_scale = f16_bits_host((float)((double)chunk_rows / (double)n_last));
   a.eps = b.eps;
   a.post_scale = b.post_scale;
   a.relu = b.relu;

@@ -49,45 +49,34 @@ __device__ __forceinline__ void grid_decompose(int m, const PixGrid& g, int& n, 
   j = rem - i * g.gw;
 }
 
-__device__ __forceinline__ void load_a(const GemmParams& p, const CUtensorMap* map, uint32_t dst,
-                                       uint32_t bar, int m0, int kb) {
-  switch (p.a_mode) {
-    case LD_TILED_K:
-      tma_load_2d(dst, map, bar, kb * kBK, m0);
-      break;
-    case LD_TILED_MN:
-      tma_load_2d(dst, map, bar, m0, kb * kBK);
-      tma_load_2d(dst + 8192, map, bar, m0 + 64, kb * kBK);
-      break;
-    case LD_IM2COL_K: {
-      const int tap = kb / p.a_cpt;
-      const int c0 = (kb - tap * p.a_cpt) * 64;
+// Producer state of one work unit: everything that depends only on the tile
+// is decomposed once, and the per-K-block coordinates advance incrementally
+// (no integer divisions on the single issuing thread's critical path).
+template <int BN>
+struct Cursor {
+  int kb;
+  // A, im2col: input coordinates of the tile's first pixel; current tap / chunk
+  int a_w, a_h, a_n, a_tap, a_c;
+  // B, im2col (weight gradient): grid point of the K-block's first pixel and
+  // the (tap, channel) of each 64-wide column chunk of the tile
+  int b_n, b_i, b_j;
+  int b_tap[BN / 64], b_c[BN / 64];
+  // B, per-tap weight slices (data gradient): current tap / K chunk
+  int b_t, b_k;
+
+  __device__ __forceinline__ void init(const GemmParams& p, int m0, int n0, int kb0) {
+    kb = kb0;
+    if (p.a_mode == LD_IM2COL_K) {
       int n, i, j;
       grid_decompose(m0, p.ga, n, i, j);
-      tma_load_im2col_4d(dst, map, bar, c0, j * p.ga.step + p.ga.base_w,
-                         i * p.ga.step + p.ga.base_h, n, (uint16_t)p.tap_ds[tap],
-                         (uint16_t)p.tap_dr[tap]);
-    } break;
-    default:
-      break;
-  }
-}
-
-template <int BN>
-__device__ __forceinline__ void load_b(const GemmParams& p, const CUtensorMap* map, uint32_t dst,
-                                       uint32_t bar, int n0, int kb) {
-  switch (p.b_mode) {
-    case LD_TILED_K:
-      tma_load_2d(dst, map, bar, kb * kBK, n0);
-      break;
-    case LD_TILED_MN:
-#pragma unroll
-      for (int j = 0; j < BN / 64; ++j) tma_load_2d(dst + j * 8192, map, bar, n0 + 64 * j, kb * kBK);
-      break;
-    case LD_IM2COL_MN: {
-      int n, i, jj;
-      grid_decompose(kb * kBK, p.gb, n, i, jj);
-      const int bw = jj * p.gb.step + p.gb.base_w, bh = i * p.gb.step + p.gb.base_h;
+      a_w = j * p.ga.step + p.ga.base_w;
+      a_h = i * p.ga.step + p.ga.base_h;
+      a_n = n;
+      a_tap = kb0 / p.a_cpt;
+      a_c = (kb0 - a_tap * p.a_cpt) * 64;
+    }
+    if (p.b_mode == LD_IM2COL_MN) {
+      grid_decompose(kb0 * kBK, p.gb, b_n, b_i, b_j);
 #pragma unroll
       for (int j = 0; j < BN / 64; ++j) {
         const int col = n0 + 64 * j;
@@ -97,20 +86,85 @@ __device__ __forceinline__ void load_b(const GemmParams& p, const CUtensorMap* m
           tap = 0;
           c0 = p.b_oob_c;
         }
-        tma_load_im2col_4d(dst + j * 8192, map, bar, c0, bw, bh, n, (uint16_t)p.tap_ds[tap],
-                           (uint16_t)p.tap_dr[tap]);
+        b_tap[j] = tap;
+        b_c[j] = c0;
       }
-    } break;
-    case LD_TAP3D_MN: {
-      const int t = kb / p.b_cpt;
-      const int k0 = (kb - t * p.b_cpt) * 64;
-#pragma unroll
-      for (int j = 0; j < BN / 64; ++j) tma_load_3d(dst + j * 8192, map, bar, n0 + 64 * j, p.tap_w[t], k0);
-    } break;
-    default:
-      break;
+    }
+    if (p.b_mode == LD_TAP3D_MN) {
+      b_t = kb0 / p.b_cpt;
+      b_k = (kb0 - b_t * p.b_cpt) * 64;
+    }
   }
-}
+
+  __device__ __forceinline__ void advance(const GemmParams& p) {
+    ++kb;
+    if (p.a_mode == LD_IM2COL_K) {
+      a_c += 64;
+      if (a_c == p.a_cpt * 64) {
+        a_c = 0;
+        ++a_tap;
+      }
+    }
+    if (p.b_mode == LD_IM2COL_MN) {
+      b_j += kBK;
+      while (b_j >= p.gb.gw) {
+        b_j -= p.gb.gw;
+        if (++b_i == p.gb.gh) {
+          b_i = 0;
+          ++b_n;
+        }
+      }
+    }
+    if (p.b_mode == LD_TAP3D_MN) {
+      b_k += 64;
+      if (b_k == p.b_cpt * 64) {
+        b_k = 0;
+        ++b_t;
+      }
+    }
+  }
+
+  __device__ __forceinline__ void load(const GemmParams& p, const CUtensorMap* ma, const CUtensorMap* mb,
+                                       uint32_t sa, uint32_t sb, uint32_t bar, int m0, int n0) const {
+    switch (p.a_mode) {
+      case LD_TILED_K:
+        tma_load_2d(sa, ma, bar, kb * kBK, m0);
+        break;
+      case LD_TILED_MN:
+        tma_load_2d(sa, ma, bar, m0, kb * kBK);
+        tma_load_2d(sa + 8192, ma, bar, m0 + 64, kb * kBK);
+        break;
+      case LD_IM2COL_K:
+        tma_load_im2col_4d(sa, ma, bar, a_c, a_w, a_h, a_n, (uint16_t)p.tap_ds[a_tap],
+                           (uint16_t)p.tap_dr[a_tap]);
+        break;
+      default:
+        break;
+    }
+    switch (p.b_mode) {
+      case LD_TILED_K:
+        tma_load_2d(sb, mb, bar, kb * kBK, n0);
+        break;
+      case LD_TILED_MN:
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK);
+        break;
+      case LD_IM2COL_MN: {
+        const int bw = b_j * p.gb.step + p.gb.base_w, bh = b_i * p.gb.step + p.gb.base_h;
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j)
+          tma_load_im2col_4d(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
+                             (uint16_t)p.tap_dr[b_tap[j]]);
+      } break;
+      case LD_TAP3D_MN:
+#pragma unroll
+        for (int j = 0; j < BN / 64; ++j) tma_load_3d(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k);
+        break;
+      default:
+        break;
+    }
+  }
+};
 
 __device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0, int& n0, int& split,
                                             int& kb0, int& kb1, int BN) {
@@ -196,7 +250,9 @@ __global__ void __launch_bounds__(192, 1)
       for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
         int m0, n0, split, kb0, kb1;
         unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
-        for (int kb = kb0; kb < kb1; ++kb) {
+        Cursor<BN> cur;
+        cur.init(p, m0, n0, kb0);
+        for (int kb = kb0; kb < kb1; ++kb, cur.advance(p)) {
           if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim)) {
             record_timeout(p, abort_flag);
             break;
@@ -204,8 +260,7 @@ __global__ void __launch_bounds__(192, 1)
           const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
-          load_a(p, &mapA, sa, fb, m0, kb);
-          load_b<BN>(p, &mapB, sa + Cfg::A_BYTES, fb, n0, kb);
+          cur.load(p, &mapA, &mapB, sa, sa + Cfg::A_BYTES, fb, m0, n0);
           ++issued;
           if (++stage == Cfg::STAGES) {
             stage = 0;

@@ -109,7 +109,8 @@ struct BnLaunch {
   int R, C;
   uint16_t eps, post_scale;
   int relu, residual;
-  int rows_per_block;     // power of two
+  int rows_per_block;     // rows per statistics CTA (chunks_per_cta chunks), a power of two
+  int chunks_per_cta;
   int blocks;             // ceil(R / rows_per_block)
   int blocks_pow2;
 };
