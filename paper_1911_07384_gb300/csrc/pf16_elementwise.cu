@@ -423,49 +423,51 @@ __device__ __forceinline__ MV mv_merge(const MV& a, const MV& b) {
   return r;
 }
 
+// Forward statistics: every thread streams cpc chunks of 16 of its rows; per
+// chunk it forms the mean of its valid rows and the mean squared deviation
+// from it (register trees), and merges chunks into a running node with the
+// count-aware pairwise rule.  One shared-memory merge across the CTA's row
+// groups closes the CTA.
 __global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a) {
-  __shared__ uint4 sh[kBnThreads];
+  __shared__ uint4 smu[kBnThreads], sv[kBnThreads];
+  __shared__ long long sn[kBnThreads];
   const BnGeom g = bn_geom(a.C);
   const int t = threadIdx.x;
   const int cg = t % g.tc, rg = t / g.tc;
   const bool active = t < g.tc * g.rpb;
-  const long long RB = (long long)g.rpb * kBnRpt;  // rows of one chunk
-  const long long total_chunks = (a.R + RB - 1) / RB;
-  MV st[8];  // binary counter over this CTA's chunks (held by the rg == 0 threads)
+  const long long RB = (long long)g.rpb * kBnRpt;
+  MV st[8];
   unsigned cnt = 0;
-  for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
-    const long long chunk = (long long)blockIdx.x * a.chunks_per_cta + ci;
-    if (chunk >= total_chunks) break;
-    const long long row0 = chunk * RB;
-    const bool last_chunk = chunk == total_chunks - 1;
-    uint4 v[kBnRpt], d[kBnRpt];
-    bool ok[kBnRpt];
+  if (active) {
+    for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
+      const long long row0 = ((long long)blockIdx.x * a.chunks_per_cta + ci) * RB;
+      if (row0 >= a.R) break;
+      uint4 v[kBnRpt], d[kBnRpt];
+      int nv = 0;
 #pragma unroll
-    for (int i = 0; i < kBnRpt; ++i) {
-      const long long r = row0 + rg + (long long)i * g.rpb;
-      ok[i] = active && r < a.R;
-      v[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
-      d[i] = v[i];
-    }
-    if (active) sh[t] = tree16(d);
-    __syncthreads();
-    smem_tree(sh, t, g.tc, rg, g.rpb, active);
-    uint4 mu = sh[cg];  // padded mean of the chunk
-    __syncthreads();
-    if (last_chunk) mu = mul4(mu, dup2(a.last_scale));
+      for (int i = 0; i < kBnRpt; ++i) {
+        const long long r = row0 + rg + (long long)i * g.rpb;
+        const bool ok = r < a.R;
+        nv += ok;
+        v[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
+        d[i] = v[i];
+      }
+      if (nv == 0) break;
+      // mean of the valid rows: padded halving tree, rescaled when rows are missing
+      uint4 mu = tree16(d);
+      uint32_t sc = 0;
+      if (nv < kBnRpt) {
+        sc = dup2(__half_as_ushort(__float2half_rn((float)kBnRpt / (float)nv)));
+        mu = mul4(mu, sc);
+      }
 #pragma unroll
-    for (int i = 0; i < kBnRpt; ++i) {
-      const uint4 e = sub4(v[i], mu);
-      d[i] = ok[i] ? mul4v(e, e) : zero4();
-    }
-    if (active) sh[t] = tree16(d);
-    __syncthreads();
-    smem_tree(sh, t, g.tc, rg, g.rpb, active);
-    uint4 var = sh[cg];
-    __syncthreads();
-    if (last_chunk) var = mul4(var, dup2(a.last_scale));
-    if (active && rg == 0) {
-      MV node{mu, var, last_chunk ? a.R - row0 : RB};
+      for (int i = 0; i < kBnRpt; ++i) {
+        const uint4 e = sub4(v[i], mu);
+        d[i] = (i < nv) ? mul4v(e, e) : zero4();  // valid rows are the first nv
+      }
+      uint4 var = tree16(d);
+      if (nv < kBnRpt) var = mul4(var, sc);
+      MV node{mu, var, nv};
 #pragma unroll
       for (int l = 0; l < 8; ++l) {
         if (cnt & (1u << l)) {
@@ -478,14 +480,27 @@ __global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a)
       ++cnt;
     }
   }
-  if (active && rg == 0 && cnt) {
-    // fold the counter: remaining nodes from the lowest level (the latest rows) up
-    MV acc{zero4(), zero4(), 0};
+  MV acc{zero4(), zero4(), 0};
 #pragma unroll
-    for (int l = 0; l < 8; ++l)
-      if (cnt & (1u << l)) acc = mv_merge(st[l], acc);
-    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = acc.mu;
-    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = acc.v;
+  for (int l = 0; l < 8; ++l)
+    if (cnt & (1u << l)) acc = mv_merge(st[l], acc);
+  smu[t] = acc.mu;
+  sv[t] = acc.v;
+  sn[t] = acc.n;
+  __syncthreads();
+  for (int half = g.rpb / 2; half >= 1; half /= 2) {
+    if (active && rg < half) {
+      const int o = (rg + half) * g.tc + cg;
+      const MV r = mv_merge(MV{smu[t], sv[t], sn[t]}, MV{smu[o], sv[o], sn[o]});
+      smu[t] = r.mu;
+      sv[t] = r.v;
+      sn[t] = r.n;
+    }
+    __syncthreads();
+  }
+  if (active && rg == 0) {
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = smu[t];
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = sv[t];
   }
 }
 
