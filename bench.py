@@ -165,11 +165,18 @@ def main():
     ap.add_argument("--conv", default=None,
                     help="time one conv pass instead of the step: N,H,W,C,K,R,S,stride,pad")
     ap.add_argument("--pass", dest="conv_pass", default="fwd", choices=["fwd", "dgrad", "wgrad"])
+    ap.add_argument("--bn", default=None,
+                    help="time one BatchNorm pass instead of the step: N,H,W,C (ReLU + residual, s=0.25)")
+    ap.add_argument("--bn-pass", default="fwd", choices=["fwd", "bwd"])
+    ap.add_argument("--ingest-traffic", default=None, metavar="CSV",
+                    help="store k_gemm DRAM bytes per launch from an ncu CSV of one step, then exit")
     ap.add_argument("--sweep", default=None, choices=["cfg2", "cfg3"],
                     help="per-layer conv lines: cfg2 = every distinct ResNet-50 conv at N=64, "
                          "cfg3 = the N=256 pure-GEMM 1x1 layers")
     args = ap.parse_args()
     rank, world, local = dist_env()
+    if args.ingest_traffic:
+        return ingest_traffic(args.ingest_traffic)
     if args.impl == "reference":
         return run_reference(args, rank, world)
     if args.conv:
@@ -178,6 +185,10 @@ def main():
         return 0
     if args.sweep:
         return run_sweep(args)
+    if args.bn:
+        print(json.dumps(time_bn(tuple(int(v) for v in args.bn.split(",")), args.bn_pass, args.steps,
+                                 args.warmup)), flush=True)
+        return 0
     if args.warmup < 3:
         args.warmup = 3
 
@@ -212,9 +223,13 @@ def main():
     if rc != 0:
         raise RuntimeError(f"device status {rc} after warm-up step")
     graph = torch.cuda.CUDAGraph()
+    n0 = pf16.kernel_launches()
     with torch.cuda.graph(graph, stream=stream):
         net.step()
-    launches = count_launches(net)
+    launches = pf16.kernel_launches() - n0  # libpf16 kernels recorded into the step graph
+    if launches != count_launches(net):
+        raise RuntimeError(f"step graph holds {launches} libpf16 kernels, the call plan "
+                           f"predicts {count_launches(net)}")
 
     for _ in range(args.warmup):
         graph.replay()
@@ -273,7 +288,8 @@ def main():
     pk = peaks()
     peak = pk["bf16_tflops_sustained"]  # FP16 and BF16 share the dense tensor rate
     roof = {"bound": "tensor", "achieved": conv["tflops"], "peak": peak, "unit": "TFLOP/s",
-            "frac": conv["tflops"] / peak, "traffic": None,
+            "frac": conv["tflops"] / peak, "traffic": gemm_traffic(),
+            "algorithmic_bytes_per_launch": conv["bytes_per_launch"],
             "kernel": "k_gemm (all conv passes of the step, split-K reduce included)",
             "peak_src": f"{pk['src']} bf16 dense sustained"}
 
@@ -390,11 +406,124 @@ def time_conv(shape, conv_pass, steps, warmup):
             "workspace_bytes": wsb, "l2_flush": io_bytes < 2 * 135 * 2 ** 20}
 
 
+def time_bn(shape, bn_pass, steps, warmup):
+    """One BatchNorm pass (x0.25, residual, ReLU) timed with CUDA events.  Bytes
+    are the algorithmic minimum of the pass: forward reads x and the residual
+    and writes y; backward reads x, dy and the saved output and writes dx and
+    the residual gradient."""
+    import torch
+
+    from paper_1911_07384_gb300 import pf16
+    from paper_1911_07384_gb300 import synthetic as syn
+
+    N, H, W, C = shape
+    R = N * H * W
+    dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).cuda()
+    e = lambda n: torch.empty(n, dtype=torch.int16, device="cuda")
+    x, res, dy = dev(syn.normal_f16(11, (R * C,))), dev(syn.normal_f16(12, (R * C,))), dev(
+        syn.normal_f16(13, (R * C,), 0.01))
+    one = np.float16(1.0).view(np.uint16)
+    g, b = dev(np.full(C, one, np.uint16)), dev(np.zeros(C, np.uint16))
+    y, mean, inv, dx, dg, db, dr = e(R * C), e(C), e(C), e(R * C), e(C), e(C), e(R * C)
+    d = pf16.bn_desc(N, H, W, C, 0x00A8, 0x3400, pf16.PF16_BN_RELU | pf16.PF16_BN_RESIDUAL)
+    ws = torch.empty(pf16.bn_workspace_size(d), dtype=torch.uint8, device="cuda")
+    fwd = lambda: pf16.bn_fwd_bwd(d, 0, ws, x=x, gamma=g, beta=b, residual=res, y=y, mean=mean, invstd=inv)
+    bwd = lambda: pf16.bn_fwd_bwd(d, 1, ws, x=x, gamma=g, mean=mean, invstd=inv, dy=dy, y_saved=y, dx=dx,
+                                  dgamma=dg, dbeta=db, dresidual=dr)
+    fwd()
+    fn = fwd if bn_pass == "fwd" else bwd
+    for _ in range(max(warmup, 3)):
+        fn()
+    torch.cuda.synchronize()
+    times = []
+    s = torch.cuda.current_stream()
+    for _ in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        fn()
+        e1.record(s)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    assert pf16.sync_status() == 0
+    ms = float(np.median(times))
+    byts = 2.0 * R * C * (3 if bn_pass == "fwd" else 5)
+    pk = peaks()
+    return {"metric": "BatchNorm pass GB/s", "bn": list(shape), "pass": bn_pass, "ms": ms,
+            "ms_best": float(np.min(times)), "gbs": byts / ms / 1e6,
+            "frac_of_hbm": byts / ms / 1e6 / pk["hbm_gbs"], "algorithmic_bytes": byts}
+
+
+TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_resnet50_b256_step_traffic.json")
+GEMM_SOURCES = ["pf16_gemm.cu", "pf16_api.cu", "pf16_internal.h", "pf16_ptx.cuh"]
+
+
+def gemm_source_digest():
+    """sha256 over the conv GEMM kernel and the code that plans its launches."""
+    import hashlib
+
+    h = hashlib.sha256()
+    for nm in GEMM_SOURCES:
+        with open(os.path.join(ROOT, "paper_1911_07384_gb300", "csrc", nm), "rb") as f:
+            h.update(nm.encode() + b"\0" + f.read())
+    return h.hexdigest()
+
+
+def ingest_traffic(csv_path):
+    """Per-launch DRAM traffic of k_gemm from an ncu CSV of one bench step
+    (metrics gpu__time_duration.sum, dram__bytes_read.sum, dram__bytes_write.sum),
+    stored with the digest of the sources it was measured on."""
+    import csv as _csv
+
+    with open(csv_path) as f:
+        rows = [r for r in _csv.reader(f)]
+    hi = next(i for i, r in enumerate(rows) if "Kernel Name" in r)
+    h = rows[hi]
+    ki, mi, ui, vi, ii = (h.index("Kernel Name"), h.index("Metric Name"), h.index("Metric Unit"),
+                          h.index("Metric Value"), h.index("ID"))
+    scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "ns": 1, "nsecond": 1,
+             "usecond": 1e3, "msecond": 1e6}
+    per = {}
+    for r in rows[hi + 1:]:
+        if len(r) <= vi or "k_gemm" not in r[ki]:
+            continue
+        per.setdefault(r[ii], {})[r[mi]] = float(r[vi].replace(",", "")) * scale[r[ui]]
+    from paper_1911_07384_gb300.resnet50 import conv_shapes
+
+    step = sum(2 + (0 if c == 3 else (st * st if r > 1 else 1))
+               for _, (_, _, _, c, _, r, _, st, _) in conv_shapes(BATCH))
+    ids = sorted(per, key=int)[:step]  # the first whole step (the eager warm-up step)
+    if len(ids) < step:
+        raise SystemExit(f"{csv_path}: {len(ids)} k_gemm launches, one step has {step}")
+    per = {i: per[i] for i in ids}
+    n = len(per)
+    rd = sum(v["dram__bytes_read.sum"] for v in per.values())
+    wr = sum(v["dram__bytes_write.sum"] for v in per.values())
+    ns = sum(v["gpu__time_duration.sum"] for v in per.values())
+    out = {"kernel": "k_gemm", "workload": WORKLOAD, "launches": n, "dram_read_bytes": rd,
+           "dram_write_bytes": wr, "time_ns": ns, "traffic_per_launch": (rd + wr) / n,
+           "source_sha256": gemm_source_digest()}
+    with open(TRAFFIC_JSON, "w") as f:
+        json.dump(out, f, indent=1)
+        f.write("\n")
+    print(json.dumps(out))
+    return 0
+
+
+def gemm_traffic():
+    """Stored per-launch DRAM bytes of k_gemm, or None once the sources changed."""
+    try:
+        with open(TRAFFIC_JSON) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    return t["traffic_per_launch"] if t.get("source_sha256") == gemm_source_digest() else None
+
+
 def count_launches(net):
     """Kernels of one step, counted by replaying the call sequence with a hook."""
     from paper_1911_07384_gb300 import pf16
 
-    per = {"conv_fwd": 0, "conv_dgrad": 0, "conv_wgrad": 0, "bn_fwd": 5, "bn_bwd": 3, "maxpool_fwd": 1,
+    per = {"conv_fwd": 0, "conv_dgrad": 0, "conv_wgrad": 0, "bn_fwd": 3, "bn_bwd": 3, "maxpool_fwd": 1,
            "maxpool_bwd": 1, "avgpool_fwd": 1, "avgpool_bwd": 1, "softmax_xent": 2, "sgd": 1}
     total = 0
     for c in net.convs:
@@ -403,7 +532,7 @@ def count_launches(net):
         total += 1 + (2 if stem else 0)                      # fwd (+ patch gather, weight pad)
         if not stem:
             phases = d.stride * d.stride if d.r > 1 else 1
-            total += phases + (1 if d.r == 1 and d.stride > 1 else 0)  # dgrad (+ zero fill)
+            total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
         total += 1 + (1 if ws else 0) + (1 if stem else 0)   # wgrad (+ split-K reduce, patch gather)
     total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)
@@ -425,7 +554,6 @@ def conv_roofline(net, stream, reps=3):
             e0.record(stream)
             fn(*a, **kw)
             e1.record(stream)
-            mult = 1
             recs.append((kind, layer, e0, e1))
             return None
         return fn(*a, **kw)
@@ -448,7 +576,17 @@ def conv_roofline(net, stream, reps=3):
         totals.append(ms)
     ms = float(np.median(totals))
     gflop = net.conv_flops() / 1e9
-    out = {"ms": ms, "gflop": gflop, "tflops": gflop / ms, "by_pass": {}}
+    # algorithmic bytes of a pass: |x| + |w| + |y| in FP16, each touched once
+    byts, gemms = 0, 0
+    for c in net.convs:
+        d = c.desc
+        P = (d.h + 2 * d.pad - d.r) // d.stride + 1
+        Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
+        one = 2 * (d.n * d.h * d.w * d.c + d.k * d.r * d.s * d.c + d.n * P * Q * d.k)
+        stem = d.c == 3
+        byts += one * (2 if stem else 3)
+        gemms += 2 + (0 if stem else (d.stride * d.stride if d.r > 1 else 1))
+    out = {"ms": ms, "gflop": gflop, "tflops": gflop / ms, "by_pass": {}, "bytes_per_launch": byts / gemms}
     for k, (t, f) in by_pass.items():
         out["by_pass"][k] = {"ms": t / reps, "tflops": (f / reps) / 1e9 / (t / reps) if t else None}
     return out

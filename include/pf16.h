@@ -202,6 +202,12 @@ const char* pf16_status_string(int status);
 /* Compute capability major*10+minor of the current device, or a negative
  * status if no device is usable.  The kernels need 103 (sm_103a). */
 int pf16_device_arch(void);
+/* Number of kernels this library has enqueued in this process so far, over
+ * all streams and devices; a launch recorded into a CUDA graph during stream
+ * capture counts once, when it is recorded.  Monotonic; never fails.  A
+ * diagnostic for callers that account for kernel launches (no counterpart in
+ * the paper). */
+uint64_t pf16_kernel_launches(void);
 
 #ifdef __cplusplus
 }

@@ -773,4 +773,8 @@ int pf16_device_arch(void) {
   return maj * 10 + min;
 }
 
+uint64_t pf16_kernel_launches(void) {
+  return (uint64_t)pf16::g_kernel_launches.load(std::memory_order_relaxed);
+}
+
 }  // extern "C"

@@ -160,7 +160,7 @@ cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, ui
   if (blocks < 1) blocks = 1;
   if (blocks > 152 * 16) blocks = 152 * 16;
   k_sgd<<<(unsigned)blocks, 256, 0, s>>>(w, v, g, n, dup2(lr), dup2(mom), dup2(wd), wd != 0);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 // ============================================================================
@@ -230,7 +230,7 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
   const long long total = rows * (cols / 8);
   const long long blocks = (total + cl - 1) / cl;
   k_splitk_reduce<<<(unsigned)blocks, 256, 0, s>>>(parts, splits, sp2, grp, rows, cols, out, ldo, cols_out);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 // ============================================================================
@@ -295,7 +295,7 @@ cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, i
   }
   k_stem_im2col<<<(unsigned)((long long)N * P), 128, shm, s>>>(x, col, N, H, W, P, Q, R, S, C, stride,
                                                                pad, kcol);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 __global__ void k_pad_rows(const uint16_t* __restrict__ w, uint16_t* __restrict__ wp, int K, int kin,
@@ -311,7 +311,7 @@ cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wp, int K, int kin, int
                             cudaStream_t s) {
   const int blocks = (K * kcol + 255) / 256;
   k_pad_rows<<<blocks, 256, 0, s>>>(w, wp, K, kin, kcol);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s) {
@@ -858,7 +858,7 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   const int rows = g.rpb * kApplyRows;
   k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, beta, mean, invstd, residual, y,
                                                               b.R, b.C, g.rpb, b.post_scale, b.relu);
-  return cudaGetLastError();
+  return counted_launches(3);
 }
 
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
@@ -880,7 +880,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   k_bn_bwd_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, mean, invstd, dy, y_saved,
                                                                   a.mm, dx, dres, b.R, b.C, g.rpb,
                                                                   b.post_scale, b.relu);
-  return cudaGetLastError();
+  return counted_launches(3);
 }
 
 // ============================================================================
@@ -1021,7 +1021,7 @@ cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, int N, int H, int
   const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
   const long long total = (long long)N * P * Q * (C / 8);
   k_maxpool_fwd<<<grid_for(total, 256, 152 * 16), 256, 0, s>>>(x, y, N, H, W, C, P, Q);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int N, int H,
@@ -1034,7 +1034,7 @@ cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* 
     if (e != cudaSuccess) return e;
   }
   k_maxpool_bwd<<<(unsigned)((long long)N * bands * (C / 8)), 256, shm, s>>>(x, dy, dx, N, H, W, C, P, Q);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 // ============================================================================
@@ -1074,7 +1074,7 @@ cudaError_t launch_avgpool_fwd(const uint16_t* x, uint16_t* y, int N, int HW, in
   const uint16_t ratio = f16_bits_host((float)((double)(1 << L) / HW));
   const long long total = (long long)N * (C / 8);
   k_avgpool_fwd<<<grid_for(total, 128, 152 * 16), 128, 0, s>>>(x, y, N, HW, C, L, ratio);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 cudaError_t launch_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int N, int HW, int C,
@@ -1082,7 +1082,7 @@ cudaError_t launch_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int N, int HW, 
   const uint16_t inv = f16_bits_host((float)(1.0 / HW));
   const long long total = (long long)N * HW * (C / 8);
   k_avgpool_bwd<<<grid_for(total, 256, 152 * 16), 256, 0, s>>>(dy, dx, N, HW, C, inv);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 // ============================================================================
@@ -1223,7 +1223,7 @@ cudaError_t launch_softmax_xent(const uint16_t* logits, const uint16_t* bias,
   const uint16_t ratio = f16_bits_host((float)((double)(1 << L) / B));
   k_softmax_rows<<<B, kSmThreads, 0, s>>>(logits, bias, labels, K, invB, dlogits, ws);
   k_softmax_cols<<<(K + 255) / 256, 256, 0, s>>>(dlogits, ws, B, K, L, ratio, dbias, loss);
-  return cudaGetLastError();
+  return counted_launches(2);
 }
 
 }  // namespace pf16

@@ -458,7 +458,7 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     attr_set[dev] = true;
   }
   k_gemm<BN><<<grid, 192, GemmCfg<BN>::SMEM, s>>>(mA, mB, mC, p);
-  return cudaGetLastError();
+  return counted_launches(1);
 }
 
 cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,

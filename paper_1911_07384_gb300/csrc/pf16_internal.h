@@ -1,11 +1,23 @@
 // Internal interfaces of libpf16 shared between the C-ABI layer (pf16_api.cu)
 // and the kernels (pf16_gemm.cu, pf16_elementwise.cu).  Not installed.
 #pragma once
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace pf16 {
+
+// Kernels this library has enqueued in the process (launches recorded into a
+// CUDA graph during stream capture included).  Read by pf16_kernel_launches.
+inline std::atomic<unsigned long long> g_kernel_launches{0};
+
+// Status of the n launches just made; they are counted when they succeeded.
+inline cudaError_t counted_launches(int n) {
+  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) g_kernel_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed);
+  return e;
+}
 
 // ---------------------------------------------------------------------------
 // tcgen05 implicit-GEMM engine.

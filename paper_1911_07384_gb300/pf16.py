@@ -33,6 +33,7 @@ EXPORTS = [
     "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
+    "pf16_kernel_launches",
 ]
 
 
@@ -108,6 +109,8 @@ def lib():
             L.pf16_status_string.restype = ctypes.c_char_p
             L.pf16_device_arch.argtypes = []
             L.pf16_device_arch.restype = I
+            L.pf16_kernel_launches.argtypes = []
+            L.pf16_kernel_launches.restype = ctypes.c_uint64
             _lib = L
     return _lib
 
@@ -226,6 +229,11 @@ def sync_status(stream=None) -> int:
 
 def device_arch() -> int:
     return int(lib().pf16_device_arch())
+
+
+def kernel_launches() -> int:
+    """Kernels libpf16 has enqueued in this process (graph-captured ones once)."""
+    return int(lib().pf16_kernel_launches())
 
 
 def loaded_path() -> str:
