@@ -168,6 +168,8 @@ def main():
     ap.add_argument("--bn", default=None,
                     help="time one BatchNorm pass instead of the step: N,H,W,C (ReLU + residual, s=0.25)")
     ap.add_argument("--bn-pass", default="fwd", choices=["fwd", "bwd"])
+    ap.add_argument("--layers", action="store_true",
+                    help="per-layer CUDA-event times of one eager step (median of 3), one JSON line each")
     ap.add_argument("--ingest-traffic", default=None, metavar="CSV",
                     help="store k_gemm DRAM bytes per launch from an ncu CSV of one step, then exit")
     ap.add_argument("--sweep", default=None, choices=["cfg2", "cfg3"],
@@ -185,6 +187,8 @@ def main():
         return 0
     if args.sweep:
         return run_sweep(args)
+    if args.layers:
+        return run_layers(args)
     if args.bn:
         print(json.dumps(time_bn(tuple(int(v) for v in args.bn.split(",")), args.bn_pass, args.steps,
                                  args.warmup)), flush=True)
@@ -320,6 +324,76 @@ def main():
     return 0
 
 
+def run_layers(args):
+    """Every library call of one training step timed with CUDA events on the
+    launching stream (eager, median of 3 steps), aggregated per (call, shape).
+    Convs report TFLOP/s; BatchNorm reports GB/s of its minimum bytes (forward
+    x, y, residual, ReLU mask; backward x, dy, dx, residual gradient, mask)."""
+    import collections
+
+    import torch
+
+    from paper_1911_07384_gb300 import pf16
+    from paper_1911_07384_gb300 import synthetic as syn
+    from paper_1911_07384_gb300.resnet50 import ResNet50
+
+    net = ResNet50(batch=args.batch, seed_cfg=4)
+    net.set_batch(syn.images_f16(syn.seed_for(4, "x", 0), args.batch),
+                  syn.labels(syn.seed_for(4, "labels", 0), args.batch))
+    stream = torch.cuda.Stream()
+    recs = []
+
+    def hook(kind, layer, fn, *a, **kw):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn(*a, **kw)
+        e1.record(stream)
+        recs.append((kind, layer, e0, e1))
+
+    with torch.cuda.stream(stream):
+        net.step()
+    torch.cuda.synchronize()
+    runs = []
+    for _ in range(3):
+        recs.clear()
+        net.hook = hook
+        with torch.cuda.stream(stream):
+            net.step()
+        net.hook = None
+        torch.cuda.synchronize()
+        runs.append([(k, l, e0.elapsed_time(e1)) for k, l, e0, e1 in recs])
+    if pf16.sync_status(stream) != 0:
+        raise RuntimeError("device status error")
+    agg = collections.OrderedDict()
+    for i, (kind, layer, _) in enumerate(runs[0]):
+        t = float(np.median([r[i][2] for r in runs]))
+        if kind.startswith("conv"):
+            d = layer.desc
+            key = (kind, (d.n, d.h, d.w, d.c, d.k, d.r, d.s, d.stride, d.pad))
+            work, unit = layer.flops / 1e12, "TFLOP/s"
+        elif kind.startswith("bn"):
+            d = layer.desc
+            key = (kind, (d.n, d.h, d.w, d.c, int(d.flags)))
+            relu, res = d.flags & pf16.PF16_BN_RELU, d.flags & pf16.PF16_BN_RESIDUAL
+            units = (2 + (1 if res else 0)) if kind == "bn_fwd" else (3 + (1 if res else 0))
+            work, unit = (2.0 * layer.elems * units + (layer.elems / 8 if relu else 0)) / 1e9, "GB/s"
+        else:
+            key, work, unit = (kind, ()), 0.0, ""
+        a = agg.setdefault(key, [0, 0.0, 0.0, unit])
+        a[0] += 1
+        a[1] += t
+        a[2] += work
+    total = sum(a[1] for a in agg.values())
+    for (kind, shape), (n, t, work, unit) in sorted(agg.items(), key=lambda kv: -kv[1][1]):
+        line = {"call": kind, "shape": list(shape), "n": n, "ms": t, "share": t / total}
+        if unit:
+            line["rate"] = work / (t / 1e3)
+            line["unit"] = unit
+        print(json.dumps(line), flush=True)
+    print(json.dumps({"total_ms": total, "note": "sum of per-call event times of an eager step"}))
+    return 0
+
+
 CFG3 = [(256, 56, 56, 256, 64, 1, 1, 1, 0), (256, 28, 28, 512, 128, 1, 1, 1, 0),
         (256, 14, 14, 1024, 256, 1, 1, 1, 0), (256, 7, 7, 512, 2048, 1, 1, 1, 0)]
 
@@ -409,8 +483,8 @@ def time_conv(shape, conv_pass, steps, warmup):
 def time_bn(shape, bn_pass, steps, warmup):
     """One BatchNorm pass (x0.25, residual, ReLU) timed with CUDA events.  Bytes
     are the algorithmic minimum of the pass: forward reads x and the residual
-    and writes y; backward reads x, dy and the saved output and writes dx and
-    the residual gradient."""
+    and writes y and the ReLU bit mask; backward reads x, dy and the mask and
+    writes dx and the residual gradient."""
     import torch
 
     from paper_1911_07384_gb300 import pf16
@@ -425,11 +499,13 @@ def time_bn(shape, bn_pass, steps, warmup):
     one = np.float16(1.0).view(np.uint16)
     g, b = dev(np.full(C, one, np.uint16)), dev(np.zeros(C, np.uint16))
     y, mean, inv, dx, dg, db, dr = e(R * C), e(C), e(C), e(R * C), e(C), e(C), e(R * C)
+    mask = torch.empty(R * C // 8, dtype=torch.uint8, device="cuda")
     d = pf16.bn_desc(N, H, W, C, 0x00A8, 0x3400, pf16.PF16_BN_RELU | pf16.PF16_BN_RESIDUAL)
     ws = torch.empty(pf16.bn_workspace_size(d), dtype=torch.uint8, device="cuda")
-    fwd = lambda: pf16.bn_fwd_bwd(d, 0, ws, x=x, gamma=g, beta=b, residual=res, y=y, mean=mean, invstd=inv)
-    bwd = lambda: pf16.bn_fwd_bwd(d, 1, ws, x=x, gamma=g, mean=mean, invstd=inv, dy=dy, y_saved=y, dx=dx,
-                                  dgamma=dg, dbeta=db, dresidual=dr)
+    fwd = lambda: pf16.bn_fwd_bwd(d, 0, ws, x=x, gamma=g, beta=b, residual=res, y=y, mean=mean, invstd=inv,
+                                  relu_mask=mask)
+    bwd = lambda: pf16.bn_fwd_bwd(d, 1, ws, x=x, gamma=g, mean=mean, invstd=inv, dy=dy, relu_mask=mask,
+                                  dx=dx, dgamma=dg, dbeta=db, dresidual=dr)
     fwd()
     fn = fwd if bn_pass == "fwd" else bwd
     for _ in range(max(warmup, 3)):
@@ -446,7 +522,7 @@ def time_bn(shape, bn_pass, steps, warmup):
         times.append(e0.elapsed_time(e1))
     assert pf16.sync_status() == 0
     ms = float(np.median(times))
-    byts = 2.0 * R * C * (3 if bn_pass == "fwd" else 5)
+    byts = 2.0 * R * C * (3 if bn_pass == "fwd" else 4) + R * C / 8  # + the ReLU bit mask
     pk = peaks()
     return {"metric": "BatchNorm pass GB/s", "bn": list(shape), "pass": bn_pass, "ms": ms,
             "ms_best": float(np.min(times)), "gbs": byts / ms / 1e6,

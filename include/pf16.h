@@ -139,15 +139,28 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
  * BatchNorm with batch statistics over the n*h*w rows of each of c channels
  * (Eq. 1, Eq. 2), each output then multiplied by post_scale (0x3400 = 0.25
  * inside residual blocks, 0x3C00 = 1 for the stem, Sec. 4.2), optionally
- * plus a residual tensor and followed by ReLU (flags).  All arithmetic FP16:
- * the mean and the (biased, two-pass) variance are balanced pairwise
- * "halving" trees (each node rn(rn(a+b) * 0.5) over zero-padded power-of-two
- * leaves, scaled once by the padding ratio), so no partial sum can overflow.
+ * plus a residual tensor and followed by ReLU (flags).  All arithmetic FP16,
+ * and no partial result can overflow unless the data do: the forward mean
+ * and biased variance are balanced pairwise trees of (mean, mean squared
+ * deviation) nodes merged by the parallel-variance rule with exact counts
+ * (equal counts: mean node rn(rn(a/2) + rn(b/2))); the backward means of
+ * dy' and dy'*xhat are "halving" trees of the same node over zero-padded
+ * power-of-two leaves, scaled once by the padding ratio.  The tree shapes
+ * depend only on n*h*w and c.
  *   phase 0 (forward, training):  reads x, gamma, beta[, residual];
  *       writes y, mean, invstd (per channel, saved for the backward).
- *   phase 1 (backward): reads x, gamma, mean, invstd, dy[, y_saved when
- *       PF16_BN_RELU]; writes dx, dgamma, dbeta and, if non-NULL, dresidual
- *       (= dy masked by ReLU, the gradient flowing to the residual input).
+ *       With PF16_BN_RELU and a non-NULL relu_mask it also writes the ReLU
+ *       decisions: n*h*w*c/8 bytes, bit j of byte [row*(c/8) + g] set iff
+ *       output channel 8g+j of that row is > 0 (so y > 0).  Any alignment.
+ *   phase 1 (backward): reads x, gamma, mean, invstd, dy and, with
+ *       PF16_BN_RELU, the ReLU decisions: from relu_mask when it is non-NULL
+ *       (as written by phase 0; y_saved is then not read and may be NULL),
+ *       else from y_saved (y > 0).  Writes dx, dgamma, dbeta and, if
+ *       non-NULL, dresidual (= dy masked by ReLU, the gradient flowing to the
+ *       residual input).  Both sources give bit-identical results; the mask
+ *       moves 1/16 of the bytes.
+ * relu_mask is ignored without PF16_BN_RELU (the bit mask is a storage
+ * choice of this library, not part of the paper's method).
  * c must be a multiple of 8 and at most 2048. */
 typedef struct {
   int32_t n, h, w, c;
@@ -159,6 +172,7 @@ typedef struct {
 typedef struct {
   const uint16_t *x, *gamma, *beta, *residual, *dy, *y_saved;
   uint16_t *y, *mean, *invstd, *dx, *dgamma, *dbeta, *dresidual;
+  uint8_t* relu_mask; /* optional ReLU bit mask: written by phase 0, read by phase 1 */
 } pf16_bn_tensors;
 
 size_t pf16_bn_workspace_size(const pf16_bn_desc* d);

@@ -633,6 +633,7 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
   if (ws_bytes < bn_ws_bytes(b)) return PF16_ERR_WORKSPACE;
   if (!aligned16(ws)) return PF16_ERR_ALIGN;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int sms = 0;
   if (phase == 0) {
     const void* req[] = {t->x, t->gamma, t->beta, t->y, t->mean, t->invstd};
     for (const void* p : req) {
@@ -641,8 +642,10 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
     }
     if (b.residual && !t->residual) return PF16_ERR_NULL;
     if (b.residual && !aligned16(t->residual)) return PF16_ERR_ALIGN;
+    if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
     return launch_bn_fwd(b, t->x, t->gamma, t->beta, b.residual ? t->residual : nullptr, t->y,
-                         t->mean, t->invstd, static_cast<uint16_t*>(ws), st) == cudaSuccess
+                         t->relu_mask, t->mean, t->invstd, static_cast<uint16_t*>(ws), st) ==
+                   cudaSuccess
                ? PF16_OK
                : PF16_ERR_CUDA;
   }
@@ -651,12 +654,15 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
     if (!p) return PF16_ERR_NULL;
     if (!aligned16(p)) return PF16_ERR_ALIGN;
   }
-  if (b.relu && !t->y_saved) return PF16_ERR_NULL;
-  if (b.relu && !aligned16(t->y_saved)) return PF16_ERR_ALIGN;
+  const bool bits = b.relu && t->relu_mask;
+  if (b.relu && !bits && !t->y_saved) return PF16_ERR_NULL;
+  if (b.relu && !bits && !aligned16(t->y_saved)) return PF16_ERR_ALIGN;
   if (t->dresidual && !aligned16(t->dresidual)) return PF16_ERR_ALIGN;
-  return launch_bn_bwd(b, t->x, t->gamma, t->mean, t->invstd, t->dy, b.relu ? t->y_saved : nullptr,
-                       t->dx, t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws),
-                       st) == cudaSuccess
+  if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
+  return launch_bn_bwd(b, t->x, t->gamma, t->mean, t->invstd, t->dy,
+                       b.relu && !bits ? t->y_saved : nullptr, bits ? t->relu_mask : nullptr, t->dx,
+                       t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws), st) ==
+                 cudaSuccess
              ? PF16_OK
              : PF16_ERR_CUDA;
 }

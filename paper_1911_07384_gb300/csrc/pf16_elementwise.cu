@@ -8,6 +8,7 @@
 
 #include <cstring>
 
+#include "../../include/pf16.h"
 #include "pf16_internal.h"
 #include "pf16_ptx.cuh"
 
@@ -63,7 +64,6 @@ __device__ __forceinline__ bool h_pos(uint32_t h) {
 __device__ __forceinline__ uint32_t relu_mask2(uint32_t y) {
   return (h_pos(y) ? 0x0000FFFFu : 0u) | (h_pos(y >> 16) ? 0xFFFF0000u : 0u);
 }
-__device__ __forceinline__ uint32_t relu2(uint32_t z) { return z & relu_mask2(z); }
 
 // Balanced pairwise tree over a stream of leaves, built as a binary counter:
 // after 2^k pushes it holds exactly the perfect tree of those leaves; finish()
@@ -321,50 +321,75 @@ cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s) {
 // ============================================================================
 // BatchNorm (Eq. 1, Eq. 2, then x post_scale, + residual, ReLU), FP16 only.
 //
-// Statistics are means over the R rows of each channel computed as balanced
-// "halving" trees (node = rn(rn(a/2) + rn(b/2)), which cannot overflow).  A
-// CTA owns RB = rpb * 16 consecutive-ish rows (each thread 16 rows of one
-// group of 8 channels, kept in registers) and produces, per channel,
-//   forward:  its mean mu_b over its actual rows and the mean of (x - mu_b)^2
-//             over them (a second tree over the same registers: one HBM pass);
-//   backward: the padded means of dy' and dy' * xhat.
-// A second small kernel combines the per-CTA results over a balanced tree:
-// forward by the pairwise parallel-variance rule (counts kept exactly, so the
-// partial last CTA is weighted right), backward by halving trees scaled once
-// by rn(Bpow2*RB/R) for the means and by 2^L (exact power-of-two steps) for
-// the sums behind dgamma / dbeta.  Then one elementwise pass applies.
+// Statistics are balanced pairwise trees over the R rows of each channel.
+// Rows come in chunks of RB = rpb * 8 consecutive rows, which are contiguous
+// in memory; a statistics CTA owns chunks b, b + grid, b + 2 grid, ... (so
+// consecutive CTAs stream adjacent rows).  Its producer warp streams them
+// through a ring of shared-memory stages with one bulk copy per tensor per
+// chunk, so the bytes in flight are set by the ring, not by registers; its
+// consumer threads each reduce 8 rows (strided by rpb) of one group of 8
+// channels per chunk from shared memory:
+//   forward:  per chunk the mean of the thread's valid rows and the mean
+//             squared deviation from it (register trees over the 8 rows: x is
+//             read once), merged over the thread's chunks and then over the
+//             CTA's row groups by the count-aware pairwise parallel-variance
+//             rule;
+//   backward: the padded halving-tree means of dy' and dy' * xhat over the 8
+//             rows, a halving tree over the thread's chunks, then over the
+//             CTA's row groups (zero padded to powers of two throughout).
+// A second small kernel (one CTA per channel group) combines the per-CTA
+// results over a balanced tree: forward by the parallel-variance rule (exact
+// counts), backward by halving trees scaled once by rn(leaves / R) for the
+// means and by 2^L (exact power-of-two steps) for the sums behind dgamma and
+// dbeta.  Then one elementwise pass applies.  With ReLU the forward can also
+// store the ReLU decisions as a bit mask, which the backward then reads in
+// place of the saved output (1/16 of its bytes).
 // ============================================================================
 namespace {
 
-constexpr int kBnThreads = 256;
-constexpr int kBnRpt = 16;  // rows per thread in the statistics kernels
+constexpr int kBnThreads = 256;                 // consumer threads per CTA, at most
+constexpr int kStatRowsT = 8;                   // rows per consumer thread per chunk
+constexpr int kStatStages = 3;                  // shared-memory ring depth
+constexpr int kStatLevels = 9;                  // per-thread chunk trees: up to 256 chunks
+constexpr int kStatMaxChunks = 1 << (kStatLevels - 1);
+constexpr int kStatTensorBytes = kStatRowsT * kBnThreads * 16;  // one tensor's slot: RB rows <= 32 KB
+constexpr int kFwdCtasPerSm = 2;                // forward ring: 3 x 32 KB (x)
+constexpr int kBwdCtasPerSm = 1;                // backward ring: 3 x 64 KB (x, dy)
+constexpr int kGb300Sms = 152;
 
 struct BnGeom {
-  int tc;   // threads per row (channel groups of 8)
-  int rpb;  // row groups per CTA (power of two)
+  int tc;       // threads per row: channel groups of 8
+  int rpb;      // row groups per CTA (power of two, at most 32)
+  int threads;  // tc * rpb rounded up to whole warps
 };
 
 __host__ __device__ inline BnGeom bn_geom(int C) {
   BnGeom g;
   g.tc = C / 8;
   int rpb = 1;
-  while (rpb * 2 * g.tc <= kBnThreads) rpb *= 2;
+  while (rpb < 32 && rpb * 2 * g.tc <= kBnThreads) rpb *= 2;
   g.rpb = rpb;
+  g.threads = (g.tc * rpb + 31) / 32 * 32;
   return g;
+}
+
+__host__ __device__ constexpr int stat_smem_bytes(int ntensor) {
+  return kStatStages * ntensor * kStatTensorBytes + 16 * kStatStages;
 }
 
 struct BnStatArgs {
   const uint16_t* x;
   const uint16_t* dy;
-  const uint16_t* y_saved;
+  const uint16_t* y_saved;    // backward, ReLU from the saved output
+  const uint8_t* mask_in;     // backward, ReLU from the bit mask
   const uint16_t* mean_in;    // backward: saved mean
   const uint16_t* invstd_in;  // backward: saved invstd
   int R, C, blocks, blocks_pow2, total_levels;
-  int chunks_per_cta;   // row chunks (of rpb * 16 rows) per statistics CTA, a power of two
-  uint16_t ratio;       // rn(Bpow2 * RB / R)
-  uint16_t last_scale;  // rn(RB / n_last): padded mean -> actual mean of the last CTA
+  int chunk_levels;     // the CTA's per-thread chunk trees are padded to 2^chunk_levels
+  uint16_t ratio;       // rn(leaves / R), leaves = 2^total_levels
   uint16_t eps, post_scale;
-  int relu;
+  int* status;          // device status word
+  unsigned long long wait_limit_ns;
   uint16_t* ws1;        // [blocks][C]
   uint16_t* ws2;        // [blocks][C]
   // outputs
@@ -375,28 +400,40 @@ struct BnStatArgs {
   uint16_t* mm;         // backward: mean(dy'), mean(dy' xhat) for the apply pass, [2][C]
 };
 
-__device__ __forceinline__ uint4 tree16(uint4* v) {
+__device__ __forceinline__ uint4 tree8(uint4* v) {
 #pragma unroll
-  for (int w = 8; w >= 1; w /= 2)
+  for (int w = 4; w >= 1; w /= 2)
 #pragma unroll
     for (int i = 0; i < w; ++i) v[i] = hmerge4(v[2 * i], v[2 * i + 1]);
   return v[0];
 }
 
-// halving tree over the rpb row groups of the CTA, in shared memory
-__device__ __forceinline__ void smem_tree(uint4* sh, int t, int tc, int rg, int rpb, bool active) {
-  for (int half = rpb / 2; half >= 1; half /= 2) {
-    if (active && rg < half) sh[t] = hmerge4(sh[t], sh[(rg + half) * tc + (t % tc)]);
-    __syncthreads();
-  }
+__device__ __forceinline__ uint4 and4(uint4 a, uint4 m) {
+  return make_uint4(a.x & m.x, a.y & m.y, a.z & m.z, a.w & m.w);
+}
+// per-lane all-ones where the saved output is > 0 (the ReLU passed)
+__device__ __forceinline__ uint4 relu_mask4(uint4 y) {
+  return make_uint4(relu_mask2(y.x), relu_mask2(y.y), relu_mask2(y.z), relu_mask2(y.w));
+}
+// bit j <- lane j of z is > 0 (lane j = channel 8*cg + j)
+__device__ __forceinline__ uint32_t pos_bits8(uint4 z) {
+  return (uint32_t)h_pos(z.x) | (uint32_t)h_pos(z.x >> 16) << 1 | (uint32_t)h_pos(z.y) << 2 |
+         (uint32_t)h_pos(z.y >> 16) << 3 | (uint32_t)h_pos(z.z) << 4 | (uint32_t)h_pos(z.z >> 16) << 5 |
+         (uint32_t)h_pos(z.w) << 6 | (uint32_t)h_pos(z.w >> 16) << 7;
+}
+__device__ __forceinline__ uint32_t bits_mask2(uint32_t b) {
+  return ((b & 1u) ? 0x0000FFFFu : 0u) | ((b & 2u) ? 0xFFFF0000u : 0u);
+}
+__device__ __forceinline__ uint4 bits_mask4(uint32_t b) {
+  return make_uint4(bits_mask2(b), bits_mask2(b >> 2), bits_mask2(b >> 4), bits_mask2(b >> 6));
 }
 
-// Combination of per-CTA (mean, variance) pairs by the pairwise parallel
-// variance rule: merging groups a and b with counts na, nb gives
+// Combination of (mean, variance) pairs by the pairwise parallel variance
+// rule: merging groups a and b with counts na, nb gives
 //   mean = wa*mean_a + wb*mean_b,  var = wa*var_a + wb*var_b + wa*wb*(mean_b - mean_a)^2,
-// wa = na/(na+nb).  For equal counts (every merge away from the partial last
-// CTA) this is exactly the halving merge of the means and of the variances
-// plus ((mean_b - mean_a)/2)^2.  Weights are constants of the counts.
+// wa = na/(na+nb).  For equal counts this is exactly the halving merge of the
+// means and of the variances plus ((mean_b - mean_a)/2)^2.  Weights are
+// constants of the counts.
 struct MV {
   uint4 mu, v;
   long long n;
@@ -413,8 +450,9 @@ __device__ __forceinline__ MV mv_merge(const MV& a, const MV& b) {
     const uint4 dh = mul4(d, kHalfHalf2);
     r.v = add4(hmerge4(a.v, b.v), mul4v(dh, dh));
   } else {
-    const __half wa = __float2half_rn((float)((double)a.n / (double)r.n));
-    const __half wb = __float2half_rn((float)((double)b.n / (double)r.n));
+    // weights in binary32 (exact count ratios to 2^-24), then rounded to binary16
+    const __half wa = __float2half_rn(__fdiv_rn((float)a.n, (float)r.n));
+    const __half wb = __float2half_rn(__fdiv_rn((float)b.n, (float)r.n));
     const uint32_t wa2 = dup2(__half_as_ushort(wa)), wb2 = dup2(__half_as_ushort(wb));
     const uint32_t wab2 = hmul2_rn(wa2, wb2);
     r.mu = add4(mul4(a.mu, wa2), mul4(b.mu, wb2));
@@ -423,71 +461,136 @@ __device__ __forceinline__ MV mv_merge(const MV& a, const MV& b) {
   return r;
 }
 
-// Forward statistics: every thread streams cpc chunks of 16 of its rows; per
-// chunk it forms the mean of its valid rows and the mean squared deviation
-// from it (register trees), and merges chunks into a running node with the
-// count-aware pairwise rule.  One shared-memory merge across the CTA's row
-// groups closes the CTA.
-__global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a) {
+// Barrier over the consumer warps only (the producer warp may have left).
+__device__ __forceinline__ void consumers_sync(int n) {
+  asm volatile("bar.sync 1, %0;" ::"r"(n) : "memory");
+}
+
+// Producer (one lane): stream the CTA's chunks through the ring.  Stage s of
+// chunk ci is refilled only after every consumer warp has released it.  On a
+// wait that runs out it records the timeout and lets the copies it already
+// issued land before returning.
+__device__ __noinline__ void stat_produce(const BnStatArgs& a, long long RB, uint32_t ring, uint32_t bars,
+                                          int ntensor, const uint16_t* t0, const uint16_t* t1) {
+  const long long rowb = 2ll * a.C;
+  const uint32_t stage_bytes = (uint32_t)(ntensor * kStatTensorBytes);
+  int ci = 0;
+  bool ok = true;
+  for (;; ++ci) {
+    const long long row0 = ((long long)ci * gridDim.x + blockIdx.x) * RB;
+    if (row0 >= a.R) break;
+    const int s = ci % kStatStages;
+    const uint32_t full = bars + 8 * s, empty = bars + 8 * (kStatStages + s);
+    if (ci >= kStatStages && !mbar_wait(empty, (uint32_t)((ci / kStatStages - 1) & 1), a.wait_limit_ns)) {
+      ok = false;
+      break;
+    }
+    const long long rows = a.R - row0 < RB ? a.R - row0 : RB;
+    const uint32_t bytes = (uint32_t)(rows * rowb);
+    const uint32_t dst = ring + (uint32_t)s * stage_bytes;
+    mbar_arrive_expect_tx(full, bytes * (uint32_t)ntensor);
+    bulk_load_1d(dst, t0 + row0 * a.C, bytes, full);
+    if (ntensor == 2) bulk_load_1d(dst + kStatTensorBytes, t1 + row0 * a.C, bytes, full);
+  }
+  if (!ok) {
+    atomicExch(a.status, PF16_ERR_TIMEOUT);
+    for (int c = ci - kStatStages < 0 ? 0 : ci - kStatStages; c < ci; ++c)
+      mbar_wait(bars + 8 * (c % kStatStages), (uint32_t)((c / kStatStages) & 1), a.wait_limit_ns);
+  }
+}
+
+// Ring set-up shared by both statistics kernels; returns the barrier base.
+__device__ __forceinline__ uint32_t stat_ring_init(uint32_t ring, int ntensor, int ncons) {
+  const uint32_t bars = ring + (uint32_t)(kStatStages * ntensor * kStatTensorBytes);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStatStages; ++s) {
+      mbar_init(bars + 8 * s, 1);                            // full: the producer's expect_tx
+      mbar_init(bars + 8 * (kStatStages + s), ncons / 32);   // empty: one arrival per consumer warp
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+  return bars;
+}
+
+// Forward statistics.  Consumers: cg = t % tc (a warp reads consecutive 16-byte
+// columns of a row from shared memory), rg = t / tc.
+__global__ void __launch_bounds__(kBnThreads + 32, kFwdCtasPerSm) k_bn_fwd_stats(const BnStatArgs a) {
+  extern __shared__ __align__(128) uint8_t stat_smem[];
   __shared__ uint4 smu[kBnThreads], sv[kBnThreads];
   __shared__ long long sn[kBnThreads];
   const BnGeom g = bn_geom(a.C);
-  const int t = threadIdx.x;
+  const int t = threadIdx.x, ncons = g.threads;
+  const uint32_t ring = smem_u32(stat_smem);
+  const uint32_t bars = stat_ring_init(ring, 1, ncons);
+  const long long RB = (long long)g.rpb * kStatRowsT;
+  if (t >= ncons) {
+    if (t == ncons) stat_produce(a, RB, ring, bars, 1, a.x, nullptr);
+    return;
+  }
   const int cg = t % g.tc, rg = t / g.tc;
   const bool active = t < g.tc * g.rpb;
-  const long long RB = (long long)g.rpb * kBnRpt;
-  MV st[8];
+  MV st[kStatLevels];
   unsigned cnt = 0;
-  if (active) {
-    for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
-      const long long row0 = ((long long)blockIdx.x * a.chunks_per_cta + ci) * RB;
-      if (row0 >= a.R) break;
-      uint4 v[kBnRpt], d[kBnRpt];
-      int nv = 0;
-#pragma unroll
-      for (int i = 0; i < kBnRpt; ++i) {
-        const long long r = row0 + rg + (long long)i * g.rpb;
-        const bool ok = r < a.R;
-        nv += ok;
-        v[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.x) + (r * a.C) / 8 + cg) : zero4();
-        d[i] = v[i];
-      }
-      if (nv == 0) break;
-      // mean of the valid rows: padded halving tree, rescaled when rows are missing
-      uint4 mu = tree16(d);
-      uint32_t sc = 0;
-      if (nv < kBnRpt) {
-        sc = dup2(__half_as_ushort(__float2half_rn((float)kBnRpt / (float)nv)));
-        mu = mul4(mu, sc);
-      }
-#pragma unroll
-      for (int i = 0; i < kBnRpt; ++i) {
-        const uint4 e = sub4(v[i], mu);
-        d[i] = (i < nv) ? mul4v(e, e) : zero4();  // valid rows are the first nv
-      }
-      uint4 var = tree16(d);
-      if (nv < kBnRpt) var = mul4(var, sc);
-      MV node{mu, var, nv};
-#pragma unroll
-      for (int l = 0; l < 8; ++l) {
-        if (cnt & (1u << l)) {
-          node = mv_merge(st[l], node);
-        } else {
-          st[l] = node;
-          break;
-        }
-      }
-      ++cnt;
+  bool ok = true;
+  for (int ci = 0;; ++ci) {
+    const long long row0 = ((long long)ci * gridDim.x + blockIdx.x) * RB;
+    if (row0 >= a.R) break;
+    const int s = ci % kStatStages;
+    if (!mbar_wait(bars + 8 * s, (uint32_t)((ci / kStatStages) & 1), a.wait_limit_ns)) {
+      ok = false;
+      break;
     }
-  }
-  MV acc{zero4(), zero4(), 0};
+    const uint32_t base = ring + (uint32_t)s * kStatTensorBytes;
+    uint4 v[kStatRowsT], d[kStatRowsT];
+    int nv = 0;
 #pragma unroll
-  for (int l = 0; l < 8; ++l)
+    for (int i = 0; i < kStatRowsT; ++i) {
+      const int r = rg + i * g.rpb;
+      const bool okr = active && row0 + r < a.R;  // valid rows are a prefix of the thread's 8
+      nv += okr;
+      v[i] = zero4();
+      if (okr) ld_shared_v4(base + (uint32_t)(r * g.tc + cg) * 16u, v[i]);
+      d[i] = v[i];
+    }
+    __syncwarp();
+    if ((t & 31) == 0) mbar_arrive(bars + 8 * (kStatStages + s));
+    if (nv == 0) continue;
+    // mean of the valid rows: padded halving tree, rescaled when rows are missing
+    uint4 mu = tree8(d);
+    uint32_t sc = 0;
+    if (nv < kStatRowsT) {
+      sc = dup2(__half_as_ushort(__float2half_rn((float)kStatRowsT / (float)nv)));
+      mu = mul4(mu, sc);
+    }
+#pragma unroll
+    for (int i = 0; i < kStatRowsT; ++i) {
+      const uint4 e = sub4(v[i], mu);
+      d[i] = (i < nv) ? mul4v(e, e) : zero4();
+    }
+    uint4 var = tree8(d);
+    if (nv < kStatRowsT) var = mul4(var, sc);
+    MV node{mu, var, nv};
+#pragma unroll 1
+    for (int l = 0; l < kStatLevels; ++l) {
+      if (cnt & (1u << l)) {
+        node = mv_merge(st[l], node);
+      } else {
+        st[l] = node;
+        break;
+      }
+    }
+    ++cnt;
+  }
+  if (!ok) atomicExch(a.status, PF16_ERR_TIMEOUT);
+  MV acc{zero4(), zero4(), 0};
+#pragma unroll 1
+  for (int l = 0; l < kStatLevels; ++l)
     if (cnt & (1u << l)) acc = mv_merge(st[l], acc);
   smu[t] = acc.mu;
   sv[t] = acc.v;
   sn[t] = acc.n;
-  __syncthreads();
+  consumers_sync(ncons);
   for (int half = g.rpb / 2; half >= 1; half /= 2) {
     if (active && rg < half) {
       const int o = (rg + half) * g.tc + cg;
@@ -496,7 +599,7 @@ __global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a)
       sv[t] = r.v;
       sn[t] = r.n;
     }
-    __syncthreads();
+    consumers_sync(ncons);
   }
   if (active && rg == 0) {
     reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = smu[t];
@@ -504,20 +607,156 @@ __global__ void __launch_bounds__(kBnThreads) k_bn_fwd_stats(const BnStatArgs a)
   }
 }
 
+// ReLU source of the backward kernels
+enum BnRelu : int { BN_NO_RELU = 0, BN_RELU_SAVED = 1, BN_RELU_BITS = 2 };
+
+// Backward statistics, same consumer layout.  The ReLU decisions of the next
+// chunk (bit-mask bytes, or saved-output vectors) are loaded from global
+// memory while the current chunk is reduced.
+template <int RELU>
+__global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats(const BnStatArgs a) {
+  extern __shared__ __align__(128) uint8_t stat_smem[];
+  __shared__ uint4 s1[kBnThreads], s2[kBnThreads];
+  const BnGeom g = bn_geom(a.C);
+  const int t = threadIdx.x, ncons = g.threads;
+  const uint32_t ring = smem_u32(stat_smem);
+  const uint32_t bars = stat_ring_init(ring, 2, ncons);
+  const long long RB = (long long)g.rpb * kStatRowsT;
+  if (t >= ncons) {
+    if (t == ncons) stat_produce(a, RB, ring, bars, 2, a.x, a.dy);
+    return;
+  }
+  const int cg = t % g.tc, rg = t / g.tc;
+  const bool active = t < g.tc * g.rpb;
+  uint4 mu = zero4(), is = zero4();
+  if (active) {
+    mu = __ldg(reinterpret_cast<const uint4*>(a.mean_in) + cg);
+    is = __ldg(reinterpret_cast<const uint4*>(a.invstd_in) + cg);
+  }
+  // ReLU decisions of one chunk's rows of this thread
+  uint32_t mb[kStatRowsT];
+  uint4 ys[kStatRowsT];
+  auto load_relu = [&](int ci) {
+    const long long row0 = ((long long)ci * gridDim.x + blockIdx.x) * RB;
+#pragma unroll
+    for (int i = 0; i < kStatRowsT; ++i) {
+      const long long r = row0 + rg + (long long)i * g.rpb;
+      const bool okr = active && r < a.R;
+      const long long off = r * g.tc + cg;
+      if (RELU == BN_RELU_BITS) mb[i] = okr ? (uint32_t)__ldg(a.mask_in + off) : 0u;
+      if (RELU == BN_RELU_SAVED) ys[i] = okr ? __ldg(reinterpret_cast<const uint4*>(a.y_saved) + off) : zero4();
+    }
+  };
+  if (RELU != BN_NO_RELU) load_relu(0);
+  uint4 st1[kStatLevels], st2[kStatLevels];
+  unsigned cnt = 0;
+  bool ok = true;
+  for (int ci = 0;; ++ci) {
+    const long long row0 = ((long long)ci * gridDim.x + blockIdx.x) * RB;
+    if (row0 >= a.R) break;
+    uint32_t mcur[kStatRowsT];
+    uint4 ycur[kStatRowsT];
+#pragma unroll
+    for (int i = 0; i < kStatRowsT; ++i) {
+      if (RELU == BN_RELU_BITS) mcur[i] = mb[i];
+      if (RELU == BN_RELU_SAVED) ycur[i] = ys[i];
+    }
+    if (RELU != BN_NO_RELU) load_relu(ci + 1);  // rows past R are not read
+    const int s = ci % kStatStages;
+    if (!mbar_wait(bars + 8 * s, (uint32_t)((ci / kStatStages) & 1), a.wait_limit_ns)) {
+      ok = false;
+      break;
+    }
+    const uint32_t base = ring + (uint32_t)s * (2u * kStatTensorBytes);
+    uint4 p1[kStatRowsT], p2[kStatRowsT];
+#pragma unroll
+    for (int i = 0; i < kStatRowsT; ++i) {
+      const int r = rg + i * g.rpb;
+      const bool okr = active && row0 + r < a.R;
+      uint4 xv = zero4(), dv = zero4();
+      if (okr) {
+        const uint32_t o = (uint32_t)(r * g.tc + cg) * 16u;
+        ld_shared_v4(base + o, xv);
+        ld_shared_v4(base + kStatTensorBytes + o, dv);
+      }
+      if (RELU == BN_RELU_BITS) dv = and4(dv, bits_mask4(mcur[i]));
+      if (RELU == BN_RELU_SAVED) dv = and4(dv, relu_mask4(ycur[i]));
+      const uint4 xh = mul4v(sub4(xv, mu), is);
+      p1[i] = dv;
+      p2[i] = okr ? mul4v(dv, xh) : zero4();
+    }
+    __syncwarp();
+    if ((t & 31) == 0) mbar_arrive(bars + 8 * (kStatStages + s));
+    uint4 n1 = tree8(p1), n2 = tree8(p2);
+#pragma unroll 1
+    for (int l = 0; l < kStatLevels; ++l) {
+      if (cnt & (1u << l)) {
+        n1 = hmerge4(st1[l], n1);
+        n2 = hmerge4(st2[l], n2);
+      } else {
+        st1[l] = n1;
+        st2[l] = n2;
+        break;
+      }
+    }
+    ++cnt;
+  }
+  if (!ok) atomicExch(a.status, PF16_ERR_TIMEOUT);
+  // close the chunk trees as if zero chunks padded them to 2^chunk_levels
+  uint4 acc1 = zero4(), acc2 = zero4();
+  bool have = false;
+#pragma unroll 1
+  for (int l = 0; l < kStatLevels; ++l) {
+    if (l < a.chunk_levels) {
+      if (cnt & (1u << l)) {
+        acc1 = hmerge4(st1[l], have ? acc1 : zero4());
+        acc2 = hmerge4(st2[l], have ? acc2 : zero4());
+        have = true;
+      } else if (have) {
+        acc1 = hmerge4(acc1, zero4());
+        acc2 = hmerge4(acc2, zero4());
+      }
+    } else if (l == a.chunk_levels && (cnt & (1u << l))) {
+      acc1 = st1[l];
+      acc2 = st2[l];
+    }
+  }
+  s1[t] = acc1;
+  s2[t] = acc2;
+  consumers_sync(ncons);
+  for (int half = g.rpb / 2; half >= 1; half /= 2) {
+    if (active && rg < half) {
+      const int o = (rg + half) * g.tc + cg;
+      s1[t] = hmerge4(s1[t], s1[o]);
+      s2[t] = hmerge4(s2[t], s2[o]);
+    }
+    consumers_sync(ncons);
+  }
+  if (active && rg == 0) {
+    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = s1[t];
+    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = s2[t];
+  }
+}
+
 constexpr int kFinalThreads = 256;
 
 // One CTA per group of 8 channels: each thread merges a contiguous run of
 // per-CTA results (loaded together), then the threads are merged in pairs in
-// shared memory; both levels follow a balanced binary tree.
-__global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs a, int rows_per_block) {
+// shared memory; both levels follow a balanced binary tree.  chunk_rows is RB;
+// CTA b owns chunks b, b + blocks, ... and only the last chunk can be partial.
+__global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs a, long long chunk_rows) {
   __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
   __shared__ long long sn[kFinalThreads];
   const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
   const int nthr = a.blocks_pow2 < kFinalThreads ? a.blocks_pow2 : kFinalThreads;
   const int seg = a.blocks_pow2 / nthr;
-  const long long n_last = (long long)a.R - (long long)(a.blocks - 1) * rows_per_block;
+  const long long chunks = ((long long)a.R + chunk_rows - 1) / chunk_rows;
+  const long long last_rows = (long long)a.R - (chunks - 1) * chunk_rows;
+  const int last_owner = (int)((chunks - 1) % a.blocks);
   auto count = [&](int b) -> long long {
-    return b < a.blocks - 1 ? (long long)rows_per_block : (b == a.blocks - 1 ? n_last : 0);
+    if (b >= a.blocks) return 0;
+    const long long nb = (chunks - b + a.blocks - 1) / a.blocks;
+    return nb * chunk_rows - (b == last_owner ? chunk_rows - last_rows : 0);
   };
   if (t < nthr) {
     // binary-counter tree over this thread's seg slots (seg is a power of two)
@@ -625,78 +864,14 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
   }
 }
 
-__global__ void __launch_bounds__(kBnThreads) k_bn_bwd_stats(const BnStatArgs a) {
-  __shared__ uint4 sh[kBnThreads];
-  const BnGeom g = bn_geom(a.C);
-  const int t = threadIdx.x;
-  const int cg = t % g.tc, rg = t / g.tc;
-  const bool active = t < g.tc * g.rpb;
-  const long long RB = (long long)g.rpb * kBnRpt;
-  uint4 mu = zero4(), is = zero4();
-  if (active) {
-    mu = __ldg(reinterpret_cast<const uint4*>(a.mean_in) + cg);
-    is = __ldg(reinterpret_cast<const uint4*>(a.invstd_in) + cg);
-  }
-  Tree4<8, true> c1, c2;  // halving trees over this CTA's chunks (rg == 0 threads)
-  for (int ci = 0; ci < a.chunks_per_cta; ++ci) {
-    const long long row0 = ((long long)blockIdx.x * a.chunks_per_cta + ci) * RB;
-    Tree4<5, true> tr1, tr2;  // 16 leaves each, pushed in row order
-#pragma unroll
-    for (int h = 0; h < kBnRpt; h += 4) {
-      uint4 xs[4], ds[4], ys[4];
-      bool ok[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const long long r = row0 + rg + (long long)(h + i) * g.rpb;
-        ok[i] = active && r < a.R;
-        const long long off = (r * a.C) / 8 + cg;
-        xs[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.x) + off) : zero4();
-        ds[i] = ok[i] ? __ldg(reinterpret_cast<const uint4*>(a.dy) + off) : zero4();
-        ys[i] = (ok[i] && a.relu) ? __ldg(reinterpret_cast<const uint4*>(a.y_saved) + off) : zero4();
-      }
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        uint4 dd = ds[i];
-        if (a.relu) {
-          dd.x &= relu_mask2(ys[i].x);
-          dd.y &= relu_mask2(ys[i].y);
-          dd.z &= relu_mask2(ys[i].z);
-          dd.w &= relu_mask2(ys[i].w);
-        }
-        const uint4 xh = mul4v(sub4(xs[i], mu), is);
-        tr1.push(dd);
-        tr2.push(ok[i] ? mul4v(dd, xh) : zero4());
-      }
-    }
-    if (active) sh[t] = tr1.finish(4);
-    __syncthreads();
-    smem_tree(sh, t, g.tc, rg, g.rpb, active);
-    const uint4 p1 = sh[cg];
-    __syncthreads();
-    if (active) sh[t] = tr2.finish(4);
-    __syncthreads();
-    smem_tree(sh, t, g.tc, rg, g.rpb, active);
-    const uint4 p2 = sh[cg];
-    __syncthreads();
-    if (active && rg == 0) {
-      c1.push(p1);
-      c2.push(p2);
-    }
-  }
-  if (active && rg == 0) {
-    const int lv = 31 - __clz(a.chunks_per_cta);
-    reinterpret_cast<uint4*>(a.ws1)[(long long)blockIdx.x * g.tc + cg] = c1.finish(lv);
-    reinterpret_cast<uint4*>(a.ws2)[(long long)blockIdx.x * g.tc + cg] = c2.finish(lv);
-  }
-}
-
 constexpr int kApplyRows = 8;  // rows per thread per CTA in the apply passes
 
 __global__ void __launch_bounds__(256)
     k_bn_apply(const uint16_t* __restrict__ x, const uint16_t* __restrict__ gamma,
                const uint16_t* __restrict__ beta, const uint16_t* __restrict__ mean,
                const uint16_t* __restrict__ invstd, const uint16_t* __restrict__ residual,
-               uint16_t* __restrict__ y, int R, int C, int rpb, uint16_t post_scale, int relu) {
+               uint16_t* __restrict__ y, uint8_t* __restrict__ mask, int R, int C, int rpb,
+               uint16_t post_scale, int relu) {
   const int tc = C / 8;
   const int t = threadIdx.x;
   if (t >= tc * rpb) return;
@@ -707,38 +882,40 @@ __global__ void __launch_bounds__(256)
   const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
   const uint4 be = __ldg(reinterpret_cast<const uint4*>(beta) + cg);
   const long long row0 = (long long)blockIdx.x * rpb * kApplyRows;
-  uint4 xv[kApplyRows], rv[kApplyRows];
 #pragma unroll
-  for (int i = 0; i < kApplyRows; ++i) {
-    const long long r = row0 + rg + (long long)i * rpb;
-    const long long off = (r * C) / 8 + cg;
-    xv[i] = r < R ? __ldg(reinterpret_cast<const uint4*>(x) + off) : zero4();
-    rv[i] = (r < R && residual) ? __ldg(reinterpret_cast<const uint4*>(residual) + off) : zero4();
-  }
+  for (int h = 0; h < kApplyRows; h += 4) {
+    uint4 xv[4], rv[4];
 #pragma unroll
-  for (int i = 0; i < kApplyRows; ++i) {
-    const long long r = row0 + rg + (long long)i * rpb;
-    if (r >= R) break;
-    const uint4 xh = mul4v(sub4(xv[i], mu), is);      // Eq. 1
-    uint4 z = mul4(add4(mul4v(ga, xh), be), ps);      // Eq. 2, then x post_scale
-    if (residual) z = add4(z, rv[i]);
-    if (relu) {
-      z.x = relu2(z.x);
-      z.y = relu2(z.y);
-      z.z = relu2(z.z);
-      z.w = relu2(z.w);
+    for (int i = 0; i < 4; ++i) {
+      const long long r = row0 + rg + (long long)(h + i) * rpb;
+      const long long off = r * tc + cg;
+      xv[i] = r < R ? __ldg(reinterpret_cast<const uint4*>(x) + off) : zero4();
+      rv[i] = (r < R && residual) ? __ldg(reinterpret_cast<const uint4*>(residual) + off) : zero4();
     }
-    reinterpret_cast<uint4*>(y)[(r * C) / 8 + cg] = z;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const long long r = row0 + rg + (long long)(h + i) * rpb;
+      if (r >= R) break;
+      const uint4 xh = mul4v(sub4(xv[i], mu), is);      // Eq. 1
+      uint4 z = mul4(add4(mul4v(ga, xh), be), ps);      // Eq. 2, then x post_scale
+      if (residual) z = add4(z, rv[i]);
+      if (relu) {
+        z = and4(z, relu_mask4(z));
+        if (mask) mask[r * tc + cg] = (uint8_t)pos_bits8(z);
+      }
+      reinterpret_cast<uint4*>(y)[r * tc + cg] = z;
+    }
   }
 }
 
+template <int RELU>
 __global__ void __launch_bounds__(256)
     k_bn_bwd_apply(const uint16_t* __restrict__ x, const uint16_t* __restrict__ gamma,
                    const uint16_t* __restrict__ mean, const uint16_t* __restrict__ invstd,
                    const uint16_t* __restrict__ dy, const uint16_t* __restrict__ y_saved,
-                   const uint16_t* __restrict__ mm, uint16_t* __restrict__ dx,
-                   uint16_t* __restrict__ dres, int R, int C, int rpb, uint16_t post_scale,
-                   int relu) {
+                   const uint8_t* __restrict__ mask, const uint16_t* __restrict__ mm,
+                   uint16_t* __restrict__ dx, uint16_t* __restrict__ dres, int R, int C, int rpb,
+                   uint16_t post_scale) {
   const int tc = C / 8;
   const int t = threadIdx.x;
   if (t >= tc * rpb) return;
@@ -754,29 +931,27 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
   for (int h = 0; h < kApplyRows; h += 4) {
     uint4 xs[4], ds[4], ys[4];
+    uint32_t mb[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const long long r = row0 + rg + (long long)(h + i) * rpb;
-      const long long off = (r * C) / 8 + cg;
+      const long long off = r * tc + cg;
       const bool ok = r < R;
       ds[i] = ok ? __ldg(reinterpret_cast<const uint4*>(dy) + off) : zero4();
       xs[i] = ok ? __ldg(reinterpret_cast<const uint4*>(x) + off) : zero4();
-      ys[i] = (ok && relu) ? __ldg(reinterpret_cast<const uint4*>(y_saved) + off) : zero4();
+      if (RELU == BN_RELU_SAVED) ys[i] = ok ? __ldg(reinterpret_cast<const uint4*>(y_saved) + off) : zero4();
+      if (RELU == BN_RELU_BITS) mb[i] = ok ? (uint32_t)__ldg(mask + off) : 0u;
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const long long r = row0 + rg + (long long)(h + i) * rpb;
       if (r >= R) break;
       uint4 d = ds[i];
-      if (relu) {
-        d.x &= relu_mask2(ys[i].x);
-        d.y &= relu_mask2(ys[i].y);
-        d.z &= relu_mask2(ys[i].z);
-        d.w &= relu_mask2(ys[i].w);
-      }
+      if (RELU == BN_RELU_SAVED) d = and4(d, relu_mask4(ys[i]));
+      if (RELU == BN_RELU_BITS) d = and4(d, bits_mask4(mb[i]));
       const uint4 xh = mul4v(sub4(xs[i], mu), is);
       const uint4 tt = sub4(sub4(d, m1), mul4v(xh, m2));  // dy' - mean(dy') - xhat*mean(dy'*xhat)
-      const long long off = (r * C) / 8 + cg;
+      const long long off = r * tc + cg;
       reinterpret_cast<uint4*>(dx)[off] = mul4v(k, tt);
       if (dres) reinterpret_cast<uint4*>(dres)[off] = d;
     }
@@ -792,27 +967,33 @@ unsigned grid_for(long long work, int per_block, int cap) {
 
 }  // namespace
 
+static BnPlan bn_stat_plan(long long chunks, int ctas_per_sm) {
+  BnPlan p;
+  long long grid = (long long)kGb300Sms * ctas_per_sm;  // the fixed statistics grid
+  if (chunks > grid * kStatMaxChunks) grid = (chunks + kStatMaxChunks - 1) / kStatMaxChunks;
+  if (grid > chunks) grid = chunks;
+  p.blocks = (int)grid;
+  p.chunks_per_cta = (int)((chunks + grid - 1) / grid);
+  int p2 = 1;
+  while (p2 < p.blocks) p2 *= 2;
+  p.blocks_pow2 = p2;
+  return p;
+}
+
 void bn_plan(int R, int C, BnLaunch* b) {
   b->R = R;
   b->C = C;
   const BnGeom g = bn_geom(C);
-  const long long chunk = (long long)g.rpb * kBnRpt;
-  const long long chunks = ((long long)R + chunk - 1) / chunk;
-  // about four statistics CTAs per SM, each over a power-of-two number of chunks
-  int cpc = 1;
-  while (cpc < 128 && chunks > (long long)cpc * 152 * 4) cpc *= 2;
-  b->chunks_per_cta = cpc;
-  b->rows_per_block = (int)(chunk * cpc);
-  b->blocks = (int)((chunks + cpc - 1) / cpc);
-  int p2 = 1;
-  while (p2 < b->blocks) p2 *= 2;
-  b->blocks_pow2 = p2;
+  b->chunk_rows = g.rpb * kStatRowsT;
+  const long long chunks = ((long long)R + b->chunk_rows - 1) / b->chunk_rows;
+  b->fwd = bn_stat_plan(chunks, kFwdCtasPerSm);
+  b->bwd = bn_stat_plan(chunks, kBwdCtasPerSm);
 }
 
 // [ws1: blocks*C] [ws2: blocks*C] [mm: 2*C]
 size_t bn_ws_bytes(const BnLaunch& b) {
-  return 256 + (size_t)2 * b.blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) +
-         256;
+  const size_t blocks = (size_t)(b.fwd.blocks > b.bwd.blocks ? b.fwd.blocks : b.bwd.blocks);
+  return 256 + 2 * blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) + 256;
 }
 
 static uint16_t f16_bits_host(float f) {
@@ -820,66 +1001,116 @@ static uint16_t f16_bits_host(float f) {
   return *reinterpret_cast<uint16_t*>(&h);
 }
 
-static BnStatArgs bn_args(const BnLaunch& b, uint16_t* ws) {
+static BnStatArgs bn_args(const BnLaunch& b, const BnPlan& p, uint16_t* ws) {
   BnStatArgs a;
   memset(&a, 0, sizeof(a));
   a.R = b.R;
   a.C = b.C;
-  a.blocks = b.blocks;
-  a.blocks_pow2 = b.blocks_pow2;
-  a.chunks_per_cta = b.chunks_per_cta;
-  const long long leaves = (long long)b.rows_per_block * b.blocks_pow2;
-  int L = 0;
-  while ((1ll << L) < leaves) ++L;
-  a.total_levels = L;
+  a.blocks = p.blocks;
+  a.blocks_pow2 = p.blocks_pow2;
+  a.chunk_levels = ceil_log2(p.chunks_per_cta);
+  // leaves of the backward trees: 8 rows x 2^chunk_levels chunks x rpb row groups x CTAs
+  const long long leaves = ((long long)b.chunk_rows << a.chunk_levels) * p.blocks_pow2;
+  a.total_levels = ceil_log2(leaves);
   a.ratio = f16_bits_host((float)((double)leaves / (double)b.R));
-  const long long chunk_rows = b.rows_per_block / b.chunks_per_cta;
-  const long long n_last = (long long)b.R - (((long long)b.R - 1) / chunk_rows) * chunk_rows;
-  a.last_scale = f16_bits_host((float)((double)chunk_rows / (double)n_last));
   a.eps = b.eps;
   a.post_scale = b.post_scale;
-  a.relu = b.relu;
+  a.status = b.status;
+  a.wait_limit_ns = 4000000000ull;
   a.ws1 = ws;
-  a.ws2 = a.ws1 + (size_t)b.blocks * b.C;
-  a.mm = a.ws2 + (size_t)b.blocks * b.C;
+  a.ws2 = a.ws1 + (size_t)p.blocks * b.C;
+  a.mm = a.ws2 + (size_t)p.blocks * b.C;
   return a;
+}
+
+// Opt a statistics kernel into its dynamic shared memory once per device.
+template <typename K>
+static cudaError_t stat_smem_attr(K kernel, int bytes, bool* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* beta, const uint16_t* residual, uint16_t* y,
-                          uint16_t* mean, uint16_t* invstd, uint16_t* ws, cudaStream_t s) {
-  BnStatArgs a = bn_args(b, ws);
+                          uint8_t* relu_mask, uint16_t* mean, uint16_t* invstd, uint16_t* ws,
+                          cudaStream_t s) {
+  static bool attr[64] = {false};
+  cudaError_t e = stat_smem_attr(k_bn_fwd_stats, stat_smem_bytes(1), attr);
+  if (e != cudaSuccess) return e;
+  BnStatArgs a = bn_args(b, b.fwd, ws);
   a.x = x;
   a.mean_out = mean;
   a.invstd_out = invstd;
-  k_bn_fwd_stats<<<b.blocks, kBnThreads, 0, s>>>(a);
-  k_bn_fwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a, b.rows_per_block);
   const BnGeom g = bn_geom(b.C);
+  k_bn_fwd_stats<<<b.fwd.blocks, g.threads + 32, stat_smem_bytes(1), s>>>(a);
+  k_bn_fwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a, (long long)b.chunk_rows);
   const int rows = g.rpb * kApplyRows;
-  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, beta, mean, invstd, residual, y,
-                                                              b.R, b.C, g.rpb, b.post_scale, b.relu);
+  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), g.threads, 0, s>>>(
+      x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
+      b.post_scale, b.relu);
   return counted_launches(3);
 }
 
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
-                          const uint16_t* y_saved, uint16_t* dx, uint16_t* dgamma,
-                          uint16_t* dbeta, uint16_t* dres, uint16_t* ws, cudaStream_t s) {
-  BnStatArgs a = bn_args(b, ws);
+                          const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
+                          uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
+                          cudaStream_t s) {
+  static bool attr[3][64] = {{false}};
+  BnStatArgs a = bn_args(b, b.bwd, ws);
   a.x = x;
   a.dy = dy;
   a.y_saved = y_saved;
+  a.mask_in = relu_mask;
   a.mean_in = mean;
   a.invstd_in = invstd;
   a.dgamma = dgamma;
   a.dbeta = dbeta;
-  k_bn_bwd_stats<<<b.blocks, kBnThreads, 0, s>>>(a);
-  k_bn_bwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a);
   const BnGeom g = bn_geom(b.C);
+  const int mode = !b.relu ? BN_NO_RELU : (relu_mask ? BN_RELU_BITS : BN_RELU_SAVED);
+  const int smem = stat_smem_bytes(2);
   const int rows = g.rpb * kApplyRows;
-  k_bn_bwd_apply<<<(unsigned)((b.R + rows - 1) / rows), 256, 0, s>>>(x, gamma, mean, invstd, dy, y_saved,
-                                                                  a.mm, dx, dres, b.R, b.C, g.rpb,
-                                                                  b.post_scale, b.relu);
+  const unsigned apply_blocks = (unsigned)((b.R + rows - 1) / rows);
+  const unsigned threads = (unsigned)(g.threads + 32);
+  cudaError_t e = cudaSuccess;
+  switch (mode) {
+    case BN_NO_RELU:
+      e = stat_smem_attr(k_bn_bwd_stats<BN_NO_RELU>, smem, attr[0]);
+      if (e == cudaSuccess) k_bn_bwd_stats<BN_NO_RELU><<<b.bwd.blocks, threads, smem, s>>>(a);
+      break;
+    case BN_RELU_SAVED:
+      e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_SAVED>, smem, attr[1]);
+      if (e == cudaSuccess) k_bn_bwd_stats<BN_RELU_SAVED><<<b.bwd.blocks, threads, smem, s>>>(a);
+      break;
+    default:
+      e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_BITS>, smem, attr[2]);
+      if (e == cudaSuccess) k_bn_bwd_stats<BN_RELU_BITS><<<b.bwd.blocks, threads, smem, s>>>(a);
+      break;
+  }
+  if (e != cudaSuccess) return e;
+  k_bn_bwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a);
+  switch (mode) {
+    case BN_NO_RELU:
+      k_bn_bwd_apply<BN_NO_RELU><<<apply_blocks, g.threads, 0, s>>>(
+          x, gamma, mean, invstd, dy, nullptr, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+      break;
+    case BN_RELU_SAVED:
+      k_bn_bwd_apply<BN_RELU_SAVED><<<apply_blocks, g.threads, 0, s>>>(
+          x, gamma, mean, invstd, dy, y_saved, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+      break;
+    default:
+      k_bn_bwd_apply<BN_RELU_BITS><<<apply_blocks, g.threads, 0, s>>>(
+          x, gamma, mean, invstd, dy, nullptr, relu_mask, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+      break;
+  }
   return counted_launches(3);
 }
 

@@ -117,22 +117,31 @@ cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wpad, int K, int kin, i
 // zero the positions of a strided output no stride phase reaches (or all)
 cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s);
 
+// Statistics grid of one direction: CTA b owns row chunks b, b + blocks, ...
+struct BnPlan {
+  int blocks;
+  int chunks_per_cta;     // most chunks one CTA owns
+  int blocks_pow2;
+};
 struct BnLaunch {
   int R, C;
   uint16_t eps, post_scale;
   int relu, residual;
-  int rows_per_block;     // rows per statistics CTA (chunks_per_cta chunks), a power of two
-  int chunks_per_cta;
-  int blocks;             // ceil(R / rows_per_block)
-  int blocks_pow2;
+  int chunk_rows;         // rows per statistics chunk (contiguous in memory)
+  BnPlan fwd, bwd;
+  int* status;            // device status word (bounded waits record timeouts here)
 };
+// relu_mask (optional, ReLU only): one bit per element, byte [row][c/8].
 cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* beta, const uint16_t* residual, uint16_t* y,
-                          uint16_t* mean, uint16_t* invstd, uint16_t* ws, cudaStream_t s);
+                          uint8_t* relu_mask, uint16_t* mean, uint16_t* invstd, uint16_t* ws,
+                          cudaStream_t s);
+// ReLU decisions from relu_mask when non-null, else from y_saved.
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
-                          const uint16_t* y_saved, uint16_t* dx, uint16_t* dgamma,
-                          uint16_t* dbeta, uint16_t* dres, uint16_t* ws, cudaStream_t s);
+                          const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
+                          uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
+                          cudaStream_t s);
 void bn_plan(int R, int C, BnLaunch* b);
 size_t bn_ws_bytes(const BnLaunch& b);
 

@@ -58,7 +58,7 @@ class BnDesc(ctypes.Structure):
 
 
 _BN_T = ("x", "gamma", "beta", "residual", "dy", "y_saved", "y", "mean", "invstd", "dx", "dgamma",
-         "dbeta", "dresidual")
+         "dbeta", "dresidual", "relu_mask")
 
 
 class BnTensors(ctypes.Structure):

@@ -130,15 +130,19 @@ class BN:
         self.dgamma, self.dbeta = a.view("g", self.g_off, self.c), a.view("g", self.b_off, self.c)
         self.mean = torch.empty(self.c, dtype=torch.int16, device=device)
         self.invstd = torch.empty(self.c, dtype=torch.int16, device=device)
+        # ReLU decisions as one bit per element: the backward reads these
+        # instead of the saved output
+        relu = bool(self.desc.flags & pf16.PF16_BN_RELU)
+        self.mask = torch.empty(self.elems // 8, dtype=torch.uint8, device=device) if relu else None
 
     def fwd(self, x, y, residual=None):
         self.net.call("bn_fwd", self, pf16.bn_fwd_bwd, self.desc, 0, self.net.ws, x=x, gamma=self.gamma,
-                      beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd)
+                      beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd,
+                      relu_mask=self.mask)
 
     def bwd(self, x, y_saved, dy, dx, dresidual=None):
         self.net.call("bn_bwd", self, pf16.bn_fwd_bwd, self.desc, 1, self.net.ws, x=x, gamma=self.gamma,
-                      mean=self.mean, invstd=self.invstd, dy=dy,
-                      y_saved=y_saved if self.desc.flags & pf16.PF16_BN_RELU else None, dx=dx,
+                      mean=self.mean, invstd=self.invstd, dy=dy, relu_mask=self.mask, dx=dx,
                       dgamma=self.dgamma, dbeta=self.dbeta, dresidual=dresidual)
 
 

@@ -11,6 +11,7 @@ and of the data gradient
 u = 2^-11; dgamma / dbeta within (4 L + 8) u * s * sum|terms| + 2^-24."""
 import numpy as np
 import pytest
+import torch
 
 from paper_1911_07384_gb300 import pf16
 from paper_1911_07384_gb300 import synthetic as syn
@@ -32,7 +33,12 @@ CASES = [
     (2, 7, 7, 2048, 0.25, False, False),
     (8, 56, 56, 64, 1.0, True, False),
     (3, 5, 7, 24, 0.25, True, True),      # C not a power of two, ragged rows
-    (256, 14, 14, 256, 0.25, True, True),  # R = 50,176
+    (256, 14, 14, 256, 0.25, True, True),  # R = 50,176: two chunks on some statistics CTAs
+    # R = 9,990,500 rows of 8 channels: 39,026 statistics chunks of 256 rows,
+    # more than 152 backward CTAs take at 256 chunks each (that grid grows to
+    # 153, most CTAs closing a full 256-chunk tree); the last chunk is partial
+    # and owned by an inner CTA
+    (1, 1, 9990500, 8, 0.25, True, False),
 ]
 
 
@@ -52,10 +58,14 @@ def test_bn_fwd_bwd(orc, case):
     ws = workspace(pf16.bn_workspace_size(d))
     tx, tg, tb = dev(x), dev(gamma), dev(beta)
     ty, tm, ti = empty16(R * C), empty16(C), empty16(C)
+    tmask = torch.empty(R * C // 8, dtype=torch.uint8, device="cuda") if relu else None
     pf16.bn_fwd_bwd(d, 0, ws, x=tx, gamma=tg, beta=tb, residual=dev(resid) if res else None, y=ty,
-                    mean=tm, invstd=ti)
+                    mean=tm, invstd=ti, relu_mask=tmask)
     assert pf16.sync_status() == 0
     y = host(ty)
+    if relu:  # the bit mask holds exactly the decisions y > 0
+        bits = np.unpackbits(tmask.cpu().numpy(), bitorder="little").reshape(R, C)
+        assert np.array_equal(bits.astype(bool), f64(y).reshape(R, C) > 0)
     yo, mean, var, invstd = orc.bn_fwd(x, gamma, beta, resid, R, C, EPS_F, s, relu)
     xhat = (f64(x).reshape(R, C) - mean) * invstd
     gf, bf = f64(gamma), f64(beta)
@@ -85,6 +95,13 @@ def test_bn_fwd_bwd(orc, case):
     tol_g = (4 * L + 8) * U * s * (dyp * (np.abs(xhat) + 1)).sum(0) + 2.0 ** -24
     assert np.all(np.abs(f64(host(tdb)) - dbo) <= tol_b)
     assert np.all(np.abs(f64(host(tdg)) - dgo) <= tol_g)
+    if relu:  # the same backward reading the bit mask instead of y: bit-identical
+        mdx, mdg, mdb, mdr = empty16(R * C), empty16(C), empty16(C), empty16(R * C)
+        pf16.bn_fwd_bwd(d, 1, ws, x=tx, gamma=tg, mean=tm, invstd=ti, dy=dev(dy), relu_mask=tmask,
+                        dx=mdx, dgamma=mdg, dbeta=mdb, dresidual=mdr)
+        assert pf16.sync_status() == 0
+        for a, b in ((mdx, tdx), (mdg, tdg), (mdb, tdb), (mdr, tdr)):
+            assert np.array_equal(host(a), host(b))
 
 
 def test_bn_constant_channel_and_zero_gamma(orc):
