@@ -521,7 +521,8 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, dy, dw)) != PF16_OK) return rc;
-  if (flags != 0) return PF16_ERR_ARG;
+  if (flags & ~PF16_REUSE_PATCHES) return PF16_ERR_ARG;
+  if ((flags & PF16_REUSE_PATCHES) && s.kind != KIND_STEM) return PF16_ERR_ARG;
   int* status;
   int sms;
   if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
@@ -543,11 +544,14 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   p.a_mode = LD_TILED_MN;
   set_mnmajor(p, true, true);
   if (!map_2d(&ma, dy, s.K, pixels, s.K, 64, 64)) return PF16_ERR_CUDA;
+  // stem: [patch matrix, where pf16_conv_fwd puts it][partials]; other layers: [partials]
   uint16_t* parts = static_cast<uint16_t*>(ws);
   const bool partial = wsp.splits > 1 || s.kind == KIND_STEM;
   if (s.kind == KIND_STEM) {
-    uint16_t* col = parts + round_up((size_t)wsp.splits * s.K * wsp.ncols * 2, 256) / 2;
-    if (launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
+    uint16_t* col = static_cast<uint16_t*>(ws);
+    parts = col + round_up((size_t)(pixels * wsp.ncols * 2), 256) / 2;
+    if (!(flags & PF16_REUSE_PATCHES) &&
+        launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
                            (int)s.S, (int)s.C, (int)s.st, (int)s.pad, (int)wsp.ncols,
                            st) != cudaSuccess)
       return PF16_ERR_CUDA;
@@ -673,6 +677,7 @@ static int pool_check(const void* a, const void* b, int32_t n, int32_t h, int32_
   if (n <= 0 || h <= 0 || w <= 0 || c <= 0) return PF16_ERR_SHAPE;
   if (c % 8 != 0) return PF16_ERR_UNSUPPORTED;
   if ((long long)n * h * w * c > (1ll << 34)) return PF16_ERR_SHAPE;
+  if ((long long)w * c > (1ll << 30)) return PF16_ERR_UNSUPPORTED;  // one row's index fits 32 bits
   return PF16_OK;
 }
 
@@ -680,7 +685,32 @@ int pf16_maxpool_fwd(const uint16_t* x, uint16_t* y, int32_t n, int32_t h, int32
                      void* stream) {
   int rc = pool_check(x, y, n, h, w, c);
   if (rc != PF16_OK) return rc;
-  return launch_maxpool_fwd(x, y, n, h, w, c, static_cast<cudaStream_t>(stream)) == cudaSuccess
+  return launch_maxpool_fwd(x, y, nullptr, n, h, w, c, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_maxpool_fwd_argmax(const uint16_t* x, uint16_t* y, uint8_t* argmax, int32_t n, int32_t h,
+                            int32_t w, int32_t c, void* stream) {
+  int rc = pool_check(x, y, n, h, w, c);
+  if (rc != PF16_OK) return rc;
+  if (!argmax) return PF16_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(argmax) & 7u) != 0) return PF16_ERR_ALIGN;
+  return launch_maxpool_fwd(x, y, argmax, n, h, w, c, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
+int pf16_maxpool_bwd_argmax(const uint8_t* argmax, const uint16_t* dy, uint16_t* dx, int32_t n,
+                            int32_t h, int32_t w, int32_t c, void* stream) {
+  int rc = pool_check(dy, dx, n, h, w, c);
+  if (rc != PF16_OK) return rc;
+  if (!argmax) return PF16_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(argmax) & 7u) != 0) return PF16_ERR_ALIGN;
+  return launch_maxpool_bwd_codes(argmax, dy, dx, n, h, w, c, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
              ? PF16_OK
              : PF16_ERR_CUDA;
 }

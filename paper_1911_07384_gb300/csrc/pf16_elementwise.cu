@@ -234,67 +234,88 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
 }
 
 // ============================================================================
-// Stem patch gather (c = 3 cannot be fetched by TMA: a pixel is 6 bytes).
-// col[m][j], m = (n, p, q), j = (r*S + s)*C + c < R*S*C, zero-padded to kcol.
-// One CTA per output row (n, p): the R input rows it needs are staged in
-// shared memory with `pad` zero pixels on each side, then each thread builds
-// the patch row of one output pixel and writes it with 16-byte stores.
+// Stem patch gather (c = 3 cannot be fetched by TMA efficiently: a pixel is 6
+// bytes).  col[m][j], m = (n, p, q), j = (r*S + s)*C + c < R*S*C, zero-padded
+// to kcol.  One CTA per output row (n, p): the R input rows it needs are
+// staged in shared memory with `pad` zero pixels on each side.  The CTA's
+// output is Q * kcol contiguous halves; thread t owns the 16-byte piece
+// g = t % G (G = kcol / 8) of pixels q = t / G, t / G + T / G, ..., so a warp
+// stores consecutive 16-byte pieces and the thread's 8 source offsets stay in
+// registers.
 // ============================================================================
 __global__ void k_stem_im2col(const uint16_t* __restrict__ x, uint16_t* __restrict__ col, int N,
                               int H, int W, int P, int Q, int R, int S, int C, int stride, int pad,
                               int kcol) {
-  extern __shared__ uint16_t rows[];  // [R][W + 2 pad][C], then the patch offset table
+  extern __shared__ uint16_t rows[];  // [R][W + 2 pad][C]
   const int WP = W + 2 * pad;
   const int rowlen = WP * C;
-  int* offs = reinterpret_cast<int*>(rows + ((R * rowlen + 1) & ~1));
   const int n = blockIdx.x / P, p = blockIdx.x - n * P;
   const int kin = R * S * C;
-  for (int j = threadIdx.x; j < kcol; j += blockDim.x) {
-    if (j < kin) {
-      const int c = j % C, rs = j / C;
-      offs[j] = (rs / S) * rowlen + (rs % S) * C + c;
-    } else {
-      offs[j] = -1;
-    }
-  }
+  const int G = kcol / 8;
   for (int r = 0; r < R; ++r) {
     const int h = p * stride + r - pad;
     uint16_t* dst = rows + r * rowlen;
-    const bool in = h >= 0 && h < H;
-    const uint16_t* src = x + ((long long)n * H + (in ? h : 0)) * W * C;
-    for (int e = threadIdx.x; e < rowlen; e += blockDim.x) {
-      const int src_e = e - pad * C;
-      dst[e] = (in && src_e >= 0 && src_e < W * C) ? src[src_e] : (uint16_t)0;
+    for (int e = threadIdx.x; e < pad * C; e += blockDim.x) {
+      dst[e] = 0;
+      dst[rowlen - 1 - e] = 0;
+    }
+    if (h < 0 || h >= H) {
+      for (int e = threadIdx.x; e < W * C; e += blockDim.x) dst[pad * C + e] = 0;
+      continue;
+    }
+    const uint16_t* src = x + ((long long)n * H + h) * W * C;
+    if ((W * C) % 8 == 0) {  // every input row then starts 16-byte aligned
+      for (int v = threadIdx.x; v < W * C / 8; v += blockDim.x) {
+        const uint4 u = __ldg(reinterpret_cast<const uint4*>(src) + v);
+        const uint16_t* hv = reinterpret_cast<const uint16_t*>(&u);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) dst[pad * C + v * 8 + e] = hv[e];
+      }
+    } else {
+      for (int e = threadIdx.x; e < W * C; e += blockDim.x) dst[pad * C + e] = src[e];
     }
   }
   __syncthreads();
-  for (int q = threadIdx.x; q < Q; q += blockDim.x) {
-    uint16_t* out = col + ((long long)blockIdx.x * Q + q) * kcol;
-    const uint16_t* base = rows + q * stride * C;
-    for (int g = 0; g < kcol; g += 8) {
-      uint16_t v[8];
+  const int g = threadIdx.x % G;
+  const int q0 = threadIdx.x / G, qs = blockDim.x / G;
+  if (q0 >= qs) return;  // threads past the last whole group of G
+  int off[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const int o = offs[g + e];
-        v[e] = o >= 0 ? base[o] : (uint16_t)0;
-      }
-      *reinterpret_cast<uint4*>(out + g) = *reinterpret_cast<uint4*>(v);
+  for (int e = 0; e < 8; ++e) {
+    const int j = g * 8 + e;
+    const int c = j % C, rs = j / C;
+    off[e] = j < kin ? (rs / S) * rowlen + (rs % S) * C + c : -1;
+  }
+  uint4* out = reinterpret_cast<uint4*>(col + (long long)blockIdx.x * Q * kcol);
+  for (int q = q0; q < Q; q += qs) {
+    const uint16_t* base = rows + q * stride * C;
+    uint32_t v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t lo = off[2 * e] >= 0 ? base[off[2 * e]] : 0u;
+      const uint32_t hi = off[2 * e + 1] >= 0 ? base[off[2 * e + 1]] : 0u;
+      v[e] = lo | (hi << 16);
     }
+    out[(long long)q * G + g] = make_uint4(v[0], v[1], v[2], v[3]);
   }
 }
 
 cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, int W, int P, int Q,
                                int R, int S, int C, int stride, int pad, int kcol,
                                cudaStream_t s) {
-  const size_t shm = (((size_t)R * (W + 2 * pad) * C + 1) & ~(size_t)1) * sizeof(uint16_t) +
-                     (size_t)kcol * sizeof(int);
+  const size_t shm = (size_t)R * (W + 2 * pad) * C * sizeof(uint16_t);
   if (shm > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(k_stem_im2col, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)shm);
     if (e != cudaSuccess) return e;
   }
-  k_stem_im2col<<<(unsigned)((long long)N * P), 128, shm, s>>>(x, col, N, H, W, P, Q, R, S, C, stride,
-                                                               pad, kcol);
+  // a whole number of G-thread groups, about 160 threads, in whole warps
+  const int G = kcol / 8;
+  int threads = G * ((160 + G - 1) / G);
+  if (threads > 1024) threads = G;
+  threads = (threads + 31) / 32 * 32;
+  k_stem_im2col<<<(unsigned)((long long)N * P), threads, shm, s>>>(x, col, N, H, W, P, Q, R, S, C, stride,
+                                                                   pad, kcol);
   return counted_launches(1);
 }
 
@@ -1117,30 +1138,38 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
 // ============================================================================
 // Max pooling 3x3 / stride 2 / pad 1 and its backward (first-max rule).
 // ============================================================================
-__global__ void k_maxpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restrict__ y, int N, int H,
-                              int W, int C, int P, int Q) {
+// Forward, one CTA per output row (n, p); with `codes` it also records, per
+// output element, the position r*3+s of the window's first maximum (r then s
+// order, padding excluded).
+__global__ void __launch_bounds__(256)
+    k_maxpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restrict__ y, uint8_t* __restrict__ codes,
+                  int N, int H, int W, int C, int P, int Q) {
   const int tc = C / 8;
-  const long long total = (long long)N * P * Q * tc;
-  for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (long long)gridDim.x * blockDim.x) {
-    const int cg = (int)(t % tc);
-    const long long o = t / tc;
-    const int q = (int)(o % Q), p = (int)((o / Q) % P), n = (int)(o / ((long long)P * Q));
+  const int n = blockIdx.x / P, p = blockIdx.x - n * P;
+  const long long orow = (long long)blockIdx.x * Q * tc;  // first output vector of the row
+  for (int i = threadIdx.x; i < Q * tc; i += blockDim.x) {
+    const int q = i / tc, cg = i - q * tc;
     float m[8];
+    uint32_t code[2] = {0xFFFFFFFFu, 0xFFFFFFFFu};
 #pragma unroll
     for (int e = 0; e < 8; ++e) m[e] = -INFINITY;
     for (int r = 0; r < 3; ++r) {
       const int h = 2 * p + r - 1;
       if (h < 0 || h >= H) continue;
+      const uint4* xrow = reinterpret_cast<const uint4*>(x + ((long long)n * H + h) * W * C);
       for (int s = 0; s < 3; ++s) {
         const int w = 2 * q + s - 1;
         if (w < 0 || w >= W) continue;
-        const uint4 v = __ldg(reinterpret_cast<const uint4*>(x + (((long long)n * H + h) * W + w) * C) + cg);
+        const uint4 v = __ldg(xrow + w * tc + cg);
         const __half* hv = reinterpret_cast<const __half*>(&v);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const float f = __half2float(hv[e]);
-          if (f > m[e]) m[e] = f;
+          if (f > m[e]) {
+            m[e] = f;
+            const int sh = (e & 3) * 8;
+            code[e >> 2] = (code[e >> 2] & ~(0xFFu << sh)) | ((uint32_t)(r * 3 + s) << sh);
+          }
         }
       }
     }
@@ -1148,7 +1177,74 @@ __global__ void k_maxpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restri
     __half* ho = reinterpret_cast<__half*>(&out);
 #pragma unroll
     for (int e = 0; e < 8; ++e) ho[e] = __float2half_rn(m[e]);  // exact: m is a binary16 value
-    reinterpret_cast<uint4*>(y)[t] = out;
+    reinterpret_cast<uint4*>(y)[orow + i] = out;
+    if (codes) reinterpret_cast<uint2*>(codes)[orow + i] = make_uint2(code[0], code[1]);
+  }
+}
+
+// Backward from the recorded positions.  Input cells (2i + a, 2j + b),
+// a, b in {0, 1}, are covered exactly by the windows p in {i, i+1}, q in
+// {j, j+1} (cell row 2i only by p = i, cell column 2j only by q = j), so one
+// thread owns that 2x2 block of cells for one group of 8 channels: it loads
+// the four windows' positions and gradients once, then every cell sums, in
+// window order (p, then q), the gradients of the windows whose first maximum
+// it is.  One CTA per block row (n, i).
+__device__ __forceinline__ uint32_t code_sel2(uint32_t cw, int j, uint32_t mine) {
+  const uint32_t c0 = (cw >> ((j & 1) * 16)) & 0xFFu;
+  const uint32_t c1 = (cw >> ((j & 1) * 16 + 8)) & 0xFFu;
+  return (c0 == mine ? 0x0000FFFFu : 0u) | (c1 == mine ? 0xFFFF0000u : 0u);
+}
+
+__global__ void __launch_bounds__(512)
+    k_maxpool_bwd_codes(const uint8_t* __restrict__ codes, const uint16_t* __restrict__ dy,
+                        uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
+  const int tc = C / 8;
+  const int HB = (H + 1) / 2, WB = (W + 1) / 2;
+  const int n = blockIdx.x / HB, i = blockIdx.x - n * HB;
+  for (int t = threadIdx.x; t < WB * tc; t += blockDim.x) {
+    const int j = t / tc, cg = t - j * tc;
+    uint2 cd[2][2];
+    uint4 g[2][2];
+#pragma unroll
+    for (int a = 0; a < 2; ++a)
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const int p = i + a, q = j + b;
+        const bool ok = p < P && q < Q;
+        const long long oi = (((long long)n * P + p) * Q + q) * tc + cg;
+        cd[a][b] = ok ? __ldg(reinterpret_cast<const uint2*>(codes) + oi) : make_uint2(~0u, ~0u);
+        g[a][b] = ok ? __ldg(reinterpret_cast<const uint4*>(dy) + oi) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+    for (int ch = 0; ch < 2; ++ch) {
+      const int h = 2 * i + ch;
+      if (h >= H) break;
+#pragma unroll
+      for (int cw = 0; cw < 2; ++cw) {
+        const int w = 2 * j + cw;
+        if (w >= W) break;
+        uint32_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int a = 0; a < 2; ++a) {
+          if (a > ch) break;  // cell row 2i lies in window row i only
+#pragma unroll
+          for (int b = 0; b < 2; ++b) {
+            if (b > cw) break;
+            const int p = i + a, q = j + b;
+            const uint32_t mine = (uint32_t)((h - (2 * p - 1)) * 3 + (w - (2 * q - 1)));
+            const uint32_t cwd[2] = {cd[a][b].x, cd[a][b].y};
+            const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g[a][b]);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint32_t sel = code_sel2(cwd[k >> 1], k, mine);
+              if (sel) acc[k] = hadd2_rn(acc[k], gw[k] & sel);
+            }
+          }
+        }
+        reinterpret_cast<uint4*>(dx)[(((long long)n * H + h) * W + w) * tc + cg] =
+            make_uint4(acc[0], acc[1], acc[2], acc[3]);
+      }
+    }
   }
 }
 
@@ -1247,11 +1343,21 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, int N, int H, int W, int C,
-                               cudaStream_t s) {
+cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, uint8_t* codes, int N, int H, int W,
+                               int C, cudaStream_t s) {
   const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
-  const long long total = (long long)N * P * Q * (C / 8);
-  k_maxpool_fwd<<<grid_for(total, 256, 152 * 16), 256, 0, s>>>(x, y, N, H, W, C, P, Q);
+  k_maxpool_fwd<<<(unsigned)((long long)N * P), 256, 0, s>>>(x, y, codes, N, H, W, C, P, Q);
+  return counted_launches(1);
+}
+
+cudaError_t launch_maxpool_bwd_codes(const uint8_t* codes, const uint16_t* dy, uint16_t* dx, int N,
+                                     int H, int W, int C, cudaStream_t s) {
+  const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
+  // one thread per 2x2 cell block of a block row, where that fits in 512 threads
+  const long long per_row = (long long)((W + 1) / 2) * (C / 8);
+  const int threads = per_row >= 512 ? 512 : (int)((per_row + 31) / 32 * 32);
+  k_maxpool_bwd_codes<<<(unsigned)((long long)N * ((H + 1) / 2)), threads, 0, s>>>(codes, dy, dx, N, H,
+                                                                                     W, C, P, Q);
   return counted_launches(1);
 }
 

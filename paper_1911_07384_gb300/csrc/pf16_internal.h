@@ -145,8 +145,11 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
 void bn_plan(int R, int C, BnLaunch* b);
 size_t bn_ws_bytes(const BnLaunch& b);
 
-cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, int N, int H, int W, int C,
-                               cudaStream_t s);
+// codes (optional): per output element the window position r*3+s of its first maximum
+cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, uint8_t* codes, int N, int H, int W,
+                               int C, cudaStream_t s);
+cudaError_t launch_maxpool_bwd_codes(const uint8_t* codes, const uint16_t* dy, uint16_t* dx, int N,
+                                     int H, int W, int C, cudaStream_t s);
 cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* dx, int N, int H,
                                int W, int C, cudaStream_t s);
 cudaError_t launch_avgpool_fwd(const uint16_t* x, uint16_t* y, int N, int HW, int C,

@@ -23,6 +23,7 @@ PF16_ERR_TIMEOUT = -7
 PF16_ERR_ARG = -8
 
 PF16_ACCUMULATE = 0x1
+PF16_REUSE_PATCHES = 0x2
 PF16_BN_RELU = 0x1
 PF16_BN_RESIDUAL = 0x2
 PF16_PASS_FWD, PF16_PASS_DGRAD, PF16_PASS_WGRAD = 0, 1, 2
@@ -33,7 +34,7 @@ EXPORTS = [
     "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
-    "pf16_kernel_launches",
+    "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
 ]
 
 
@@ -95,9 +96,12 @@ def lib():
             L.pf16_bn_fwd_bwd.restype = I
             L.pf16_maxpool_fwd.argtypes = [vp, vp, i32, i32, i32, i32, vp]
             L.pf16_maxpool_bwd.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
+            L.pf16_maxpool_fwd_argmax.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
+            L.pf16_maxpool_bwd_argmax.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
             L.pf16_avgpool_fwd.argtypes = [vp, vp, i32, i32, i32, vp]
             L.pf16_avgpool_bwd.argtypes = [vp, vp, i32, i32, i32, vp]
-            for nm in ("pf16_maxpool_fwd", "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd"):
+            for nm in ("pf16_maxpool_fwd", "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
+                       "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax"):
                 getattr(L, nm).restype = I
             L.pf16_softmax_xent_workspace_size.argtypes = [i32, i32]
             L.pf16_softmax_xent_workspace_size.restype = sz
@@ -203,6 +207,16 @@ def maxpool_fwd(x, y, n, h, w, c, stream=None):
 def maxpool_bwd(x, dy, dx, n, h, w, c, stream=None):
     _check(lib().pf16_maxpool_bwd(_ptr(x), _ptr(dy), _ptr(dx), n, h, w, c, _stream(stream)),
            "pf16_maxpool_bwd")
+
+
+def maxpool_fwd_argmax(x, y, argmax, n, h, w, c, stream=None):
+    _check(lib().pf16_maxpool_fwd_argmax(_ptr(x), _ptr(y), _ptr(argmax), n, h, w, c, _stream(stream)),
+           "pf16_maxpool_fwd_argmax")
+
+
+def maxpool_bwd_argmax(argmax, dy, dx, n, h, w, c, stream=None):
+    _check(lib().pf16_maxpool_bwd_argmax(_ptr(argmax), _ptr(dy), _ptr(dx), n, h, w, c, _stream(stream)),
+           "pf16_maxpool_bwd_argmax")
 
 
 def avgpool_fwd(x, y, n, hw, c, stream=None):

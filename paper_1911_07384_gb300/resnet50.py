@@ -102,14 +102,19 @@ class Conv:
         self.w, self.gw = a.view("w", self.off, self.numel), a.view("g", self.off, self.numel)
 
     def fwd(self, x, y):
-        self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.net.ws)
+        self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.ws())
 
     def dgrad(self, dy, dx, accumulate=False):
         self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
                       pf16.PF16_ACCUMULATE if accumulate else 0)
 
+    def ws(self):
+        return self.net.stem_ws if self.desc.c == 3 else self.net.ws
+
     def wgrad(self, x, dy):
-        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.net.ws)
+        # the stem's patch matrix, gathered by its forward into its own workspace, is still there
+        flags = pf16.PF16_REUSE_PATCHES if self.desc.c == 3 else 0
+        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.ws(), flags)
 
 
 class BN:
@@ -259,6 +264,8 @@ class ResNet50:
         self.labels = torch.zeros(N, dtype=torch.int32, device=dev)
         self.a0, self.b0, self.p0 = e(N, h0, h0, 64), e(N, h0, h0, 64), e(N, hp, hp, 64)
         self.dp0, self.db0, self.da0 = e(N, hp, hp, 64), e(N, h0, h0, 64), e(N, h0, h0, 64)
+        # position of each pooling window's maximum, kept from the forward for the backward
+        self.pool_arg = torch.empty(N * hp * hp * 64, dtype=torch.uint8, device=dev)
         for b in self.blocks:
             b.allocate(dev)
         self.f = e(N, self.cl)
@@ -266,10 +273,16 @@ class ResNet50:
         self.dlogits = e(N, self.classes)
         self.df = e(N, self.cl)
         self.loss = e(1)
-        ws = 0
+        ws, stem_ws = 0, 0
         for c in self.convs:
-            ws = max(ws, pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_FWD),
-                     pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD))
+            need = max(pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_FWD),
+                       pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD))
+            if c.desc.c == 3:
+                stem_ws = max(stem_ws, need)
+            else:
+                ws = max(ws, need)
+        # the stem keeps its patch matrix from the forward to the weight gradient
+        self.stem_ws = torch.empty(stem_ws, dtype=torch.uint8, device=dev)
         for b in self.bns:
             ws = max(ws, pf16.bn_workspace_size(b.desc))
         ws = max(ws, pf16.softmax_xent_workspace_size(N, self.classes))
@@ -303,7 +316,8 @@ class ResNet50:
     def forward(self):
         self.stem.fwd(self.x, self.a0)
         self.bn0.fwd(self.a0, self.b0)
-        self.call("maxpool_fwd", None, pf16.maxpool_fwd, self.b0, self.p0, self.N, self.h0, self.h0, 64)
+        self.call("maxpool_fwd", None, pf16.maxpool_fwd_argmax, self.b0, self.p0, self.pool_arg, self.N,
+                  self.h0, self.h0, 64)
         h = self.p0
         for b in self.blocks:
             h = b.forward(h)
@@ -321,8 +335,8 @@ class ResNet50:
         for i in range(len(self.blocks) - 1, -1, -1):
             dx = self.blocks[i - 1].dy if i > 0 else self.dp0
             self.blocks[i].backward(dx)
-        self.call("maxpool_bwd", None, pf16.maxpool_bwd, self.b0, self.dp0, self.db0, self.N, self.h0,
-                  self.h0, 64)
+        self.call("maxpool_bwd", None, pf16.maxpool_bwd_argmax, self.pool_arg, self.dp0, self.db0, self.N,
+                  self.h0, self.h0, 64)
         self.bn0.bwd(self.a0, self.b0, self.db0, self.da0)
         self.stem.wgrad(self.x, self.da0)
 

@@ -86,6 +86,11 @@ def test_other_validation_errors():
     assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_NULL
     assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1, None) == pf16.PF16_ERR_WORKSPACE
     assert L.pf16_maxpool_fwd(FAKE, FAKE, 1, 8, 8, 12, None) == pf16.PF16_ERR_UNSUPPORTED
+    assert L.pf16_maxpool_fwd_argmax(FAKE, FAKE, None, 1, 8, 8, 16, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_maxpool_fwd_argmax(FAKE, FAKE, ctypes.c_void_p(0x10004), 1, 8, 8, 16,
+                                     None) == pf16.PF16_ERR_ALIGN
+    assert L.pf16_maxpool_bwd_argmax(None, FAKE, FAKE, 1, 8, 8, 16, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_maxpool_bwd_argmax(FAKE, FAKE, FAKE, 1, 8, 8, 12, None) == pf16.PF16_ERR_UNSUPPORTED
     assert L.pf16_avgpool_fwd(FAKE, None, 1, 49, 64, None) == pf16.PF16_ERR_NULL
     assert L.pf16_softmax_xent(FAKE, None, FAKE, 4, 5000, FAKE, FAKE, None, FAKE, 1 << 20,
                                None) == pf16.PF16_ERR_UNSUPPORTED

@@ -97,6 +97,28 @@ def test_conv_wgrad(orc, shape):
     assert rel < 2.0 ** -6, rel
 
 
+def test_stem_wgrad_reuses_forward_patches():
+    """PF16_REUSE_PATCHES: the stem's weight gradient on the patch matrix its
+    forward left in a shared workspace equals the one that gathers again."""
+    shape = (3, 30, 30, 3, 64, 7, 7, 2, 3)
+    x, w, dy, P, Q = inputs(shape, seed_cfg=2)
+    d = pf16.conv_desc(*shape)
+    ws = workspace(max(pf16.conv_workspace_size(d, pf16.PF16_PASS_FWD),
+                       pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)))
+    tx = dev(x)
+    pf16.conv_fwd(d, tx, dev(w), empty16(d.n * P * Q * d.k), ws)
+    dw = empty16(d.k * d.r * d.s * d.c)
+    pf16.conv_wgrad(d, tx, dev(dy), dw, ws, pf16.PF16_REUSE_PATCHES)
+    assert pf16.sync_status() == 0
+    assert np.array_equal(host(dw), run_wgrad(d, x, dy))
+    # the flag is only for the stem
+    d2 = pf16.conv_desc(2, 14, 14, 64, 64, 1, 1, 1, 0)
+    with pytest.raises(pf16.PF16Error):
+        pf16.conv_wgrad(d2, empty16(2 * 14 * 14 * 64), empty16(2 * 14 * 14 * 64), empty16(64 * 64),
+                        workspace(pf16.conv_workspace_size(d2, pf16.PF16_PASS_WGRAD)),
+                        pf16.PF16_REUSE_PATCHES)
+
+
 @pytest.mark.parametrize("shape", [(2, 9, 9, 64, 128, 3, 3, 1, 1), (2, 10, 10, 64, 64, 1, 1, 2, 0),
                                    (2, 11, 11, 64, 64, 3, 3, 2, 1)], ids=ids)
 def test_accumulate_flag(orc, shape):

@@ -8,6 +8,7 @@ L = ceil(log2 hw) and one scaling; the softmax adds the roundings of the
 bias add, the exp argument, a pairwise sum over k and the log."""
 import numpy as np
 import pytest
+import torch
 
 from paper_1911_07384_gb300 import pf16
 from paper_1911_07384_gb300 import synthetic as syn
@@ -30,6 +31,37 @@ def test_maxpool(orc, shape):
     assert pf16.sync_status() == 0
     dx, A = orc.maxpool_bwd(x, dy, N, H, W, C)
     assert np.all(np.abs(f64(host(tdx)) - dx) <= 3 * U * A)
+    # the pair that keeps the maxima's positions: same y, the first-maximum
+    # position of every window, and the very same dx
+    ty2 = empty16(N * P * Q * C)
+    targ = torch.empty(N * P * Q * C, dtype=torch.uint8, device="cuda")
+    pf16.maxpool_fwd_argmax(dev(x), ty2, targ, N, H, W, C)
+    assert np.array_equal(host(ty2), host(ty))
+    assert np.array_equal(targ.cpu().numpy().reshape(N, P, Q, C), first_max_positions(x, N, H, W, C))
+    tdx2 = empty16(N * H * W * C)
+    pf16.maxpool_bwd_argmax(targ, dev(dy), tdx2, N, H, W, C)
+    assert pf16.sync_status() == 0
+    assert np.array_equal(host(tdx2), host(tdx))
+
+
+def first_max_positions(x, N, H, W, C):
+    """r*3+s of the first maximum (r then s, padding excluded) of every 3x3 /
+    stride-2 / pad-1 window, by a scan over the nine taps in numpy."""
+    v = f64(x).reshape(N, H, W, C)
+    P, Q = (H - 1) // 2 + 1, (W - 1) // 2 + 1
+    best = np.full((N, P, Q, C), -np.inf)
+    code = np.full((N, P, Q, C), 255, np.uint8)
+    for r in range(3):
+        for s_ in range(3):
+            hs = 2 * np.arange(P) + r - 1
+            ws = 2 * np.arange(Q) + s_ - 1
+            okh, okw = (hs >= 0) & (hs < H), (ws >= 0) & (ws < W)
+            sub = v[:, np.clip(hs, 0, H - 1)][:, :, np.clip(ws, 0, W - 1)]
+            cand = np.where(okh[None, :, None, None] & okw[None, None, :, None], sub, -np.inf)
+            better = cand > best
+            best = np.where(better, cand, best)
+            code = np.where(better, np.uint8(r * 3 + s_), code)
+    return code
 
 
 def test_maxpool_ties_first_cell(orc):
@@ -41,6 +73,11 @@ def test_maxpool_ties_first_cell(orc):
     dx, A = orc.maxpool_bwd(x, dy, N, H, W, C)
     assert np.all(np.abs(f64(host(tdx)) - dx) <= 3 * U * A)
     assert np.array_equal(f64(host(tdx)) != 0, dx != 0)
+    targ = torch.empty(N * 3 * 3 * C, dtype=torch.uint8, device="cuda")
+    pf16.maxpool_fwd_argmax(dev(x), empty16(N * 3 * 3 * C), targ, N, H, W, C)
+    tdx2 = empty16(N * H * W * C)
+    pf16.maxpool_bwd_argmax(targ, dev(dy), tdx2, N, H, W, C)
+    assert np.array_equal(host(tdx2), host(tdx))
 
 
 @pytest.mark.parametrize("shape", [(256, 49, 2048), (3, 10, 64)])
