@@ -195,11 +195,16 @@ struct WgradSplit {
   long long ncols;  // GEMM N
 };
 
-// Split-K plan of the weight gradient.  Independent of the device so that
-// pf16_conv_workspace_size and the call always agree: about two units of work
-// per SM of a 152-SM GB300, at least 4 and at most 64 K-blocks (4096 pixels)
-// accumulated in one FP16 tensor-memory accumulator, at most 1024 splits.
-constexpr int kWgradTargetUnits = 2 * 152;
+// Split-K plan of the weight gradient, independent of the device so that
+// pf16_conv_workspace_size and the call always agree.  The persistent GEMM
+// runs tiles * splits units on the 152 SMs of a GB300 in ceil(units / 152)
+// rounds, so the split count is the one minimising a makespan model:
+//   rounds * (K-blocks per split * t_kb + t_unit) + partial-plane traffic,
+// with t_kb ~ 0.4 us per 128 x 256 x 64 block, t_unit ~ 1 us (pipeline fill
+// and the partial tile's store) and the splits * |dw| FP16 partials written
+// and read back at ~6 TB/s.  Between 4 and 64 K-blocks (4096 pixels) go into
+// one FP16 tensor-memory accumulator; at most 1024 splits.
+constexpr int kPlanSms = 152;
 
 WgradSplit wgrad_split(const Shape& s) {
   WgradSplit w;
@@ -208,13 +213,26 @@ WgradSplit wgrad_split(const Shape& s) {
   w.m_tiles = cdiv(s.K, kBM);
   w.n_tiles = cdiv(w.ncols, w.bn);
   w.num_kb = cdiv(s.N * s.P * s.Q, kBK);
-  const int units = w.m_tiles * w.n_tiles;
-  int splits = std::max(1, cdiv(kWgradTargetUnits, units));
-  int kps = std::max(4, cdiv(w.num_kb, splits));
-  kps = std::min(kps, 64);  // at most 4096 pixels accumulated in one FP16 accumulator
-  w.kb_per_split = std::min(kps, w.num_kb);
+  const long long tiles = (long long)w.m_tiles * w.n_tiles;
+  const double t_kb = 0.4e-6 * w.bn / 256.0, t_unit = 1.0e-6;
+  const double dw_bytes = 2.0 * (double)s.K * (double)w.ncols;
+  double best = -1.0;
+  w.kb_per_split = std::min(w.num_kb, 64);
   w.splits = cdiv(w.num_kb, w.kb_per_split);
-  if (w.splits > 1024) {
+  for (int sp = 1; sp <= 1024; ++sp) {
+    const int kps = cdiv(w.num_kb, sp);
+    if (kps > 64) continue;
+    if (kps < 4 && sp > 1) break;  // kps only shrinks from here
+    const int real = cdiv(w.num_kb, kps);
+    const long long rounds = (tiles * real + kPlanSms - 1) / kPlanSms;
+    const double t = (double)rounds * (kps * t_kb + t_unit) + (real > 1 ? real * dw_bytes * 2.0 / 6e12 : 0.0);
+    if (best < 0.0 || t < best * (1.0 - 1e-9)) {
+      best = t;
+      w.kb_per_split = kps;
+      w.splits = real;
+    }
+  }
+  if (w.splits > 1024) {  // only when more than 65,536 K-blocks: fill 1024 splits
     w.kb_per_split = cdiv(w.num_kb, 1024);
     w.splits = cdiv(w.num_kb, w.kb_per_split);
   }
