@@ -150,10 +150,10 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
  * and no partial result can overflow unless the data do: the forward mean
  * and biased variance are balanced pairwise trees of (mean, mean squared
  * deviation) nodes merged by the parallel-variance rule with exact counts
- * (equal counts: mean node rn(rn(a/2) + rn(b/2))); the backward means of
- * dy' and dy'*xhat are "halving" trees of the same node over zero-padded
- * power-of-two leaves, scaled once by the padding ratio.  The tree shapes
- * depend only on n*h*w and c.
+ * (equal counts: mean node rn(a/2 + rn(b/2)), one fused multiply-add); the
+ * backward means of dy' and dy'*xhat are "halving" trees of the same node
+ * over zero-padded power-of-two leaves, scaled once by the padding ratio.
+ * The tree shapes depend only on n*h*w and c.
  *   phase 0 (forward, training):  reads x, gamma, beta[, residual];
  *       writes y, mean, invstd (per channel, saved for the backward).
  *       With PF16_BN_RELU and a non-NULL relu_mask it also writes the ReLU

@@ -23,9 +23,12 @@ __host__ __device__ __forceinline__ uint32_t dup2(uint16_t h) { return (uint32_t
 __device__ __forceinline__ uint4 add4(uint4 a, uint4 b) {
   return make_uint4(hadd2_rn(a.x, b.x), hadd2_rn(a.y, b.y), hadd2_rn(a.z, b.z), hadd2_rn(a.w, b.w));
 }
-// halving merge: rn(rn(a/2) + rn(b/2)) -- the mean of two nodes, never overflows
+// halving merge, the mean of two nodes: rn(a/2 + rn(b/2)) as one fused
+// multiply-add.  It equals rn(rn(a/2) + rn(b/2)) whenever a/2 is exact (every
+// a but a subnormal with its last bit set) and, halving before adding, never
+// overflows.
 __device__ __forceinline__ uint32_t hmerge2(uint32_t a, uint32_t b) {
-  return hadd2_rn(hmul2_rn(a, kHalfHalf2), hmul2_rn(b, kHalfHalf2));
+  return hfma2_rn(a, kHalfHalf2, hmul2_rn(b, kHalfHalf2));
 }
 __device__ __forceinline__ uint4 hmerge4(uint4 a, uint4 b) {
   return make_uint4(hmerge2(a.x, b.x), hmerge2(a.y, b.y), hmerge2(a.z, b.z), hmerge2(a.w, b.w));

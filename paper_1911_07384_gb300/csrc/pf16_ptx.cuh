@@ -231,6 +231,12 @@ __device__ __forceinline__ uint32_t hmul2_rn(uint32_t a, uint32_t b) {
   asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
+// a * b + c with one rounding (IEEE fusedMultiplyAdd), f16x2
+__device__ __forceinline__ uint32_t hfma2_rn(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
 __device__ __forceinline__ uint32_t hmax2(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("max.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
