@@ -369,6 +369,59 @@ size_t pf16_conv_workspace_size(const pf16_conv_desc* d, int pass) {
   return 0;
 }
 
+// Padded row width of the halo engine for a 3x3 / stride 1 / pad 1 layer with
+// 64 input and 64 output channels, or 0 where it does not apply: the padded
+// grid needs ws >= W + 2 and a 128-row tile of 128 / ws whole image rows that
+// never straddles two images.
+int halo_width(const Shape& s, bool accum) {
+  if (accum || s.kind != KIND_GENERIC || s.R != 3 || s.S != 3 || s.st != 1 || s.pad != 1) return 0;
+  if (s.C != 64 || s.K != 64) return 0;
+  const int ws = s.W + 2 <= 32 ? 32 : (s.W + 2 <= 64 ? 64 : 0);
+  if (ws == 0 || s.H % (kBM / ws) != 0) return 0;
+  if ((long long)s.N * s.H * ws / kBM > (1ll << 30)) return 0;
+  return ws;
+}
+
+// 3x3 stride-1 forward (dgrad = false: in = x, weights [K][9*C]) or data
+// gradient (dgrad = true: in = dy, weights viewed (C, 9, K), taps flipped)
+// through the halo engine.  in and out are N x H x W x 64.
+int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint16_t* w, uint16_t* out,
+             int* status, int sms, cudaStream_t st) {
+  GemmParams p = base_params(status);
+  CUtensorMap ma, mb, mc;
+  const long long N = s.N, H = s.H, W = s.W;
+  cuuint64_t dims[4] = {64, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[3] = {128, (cuuint64_t)W * 128, (cuuint64_t)(H * W * 128)};
+  cuuint32_t box[4] = {64, (cuuint32_t)ws, (cuuint32_t)(kBM / ws + 2), 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  if (g_encode_tiled(&ma, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<uint16_t*>(in), dims, strides,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PF16_ERR_CUDA;
+  if (!map_3d(&mc, out, 64, W, N * H, 128, W * 128, 64, 32, 1)) return PF16_ERR_CUDA;
+  p.ntaps = 9;
+  for (int t = 0; t < 9; ++t) {
+    p.tap_dr[t] = (int8_t)(t / 3);
+    p.tap_ds[t] = (int8_t)(t % 3);
+    p.tap_w[t] = (int8_t)(dgrad ? 8 - t : t);  // the data gradient reads the filter flipped
+  }
+  if (dgrad) {
+    p.b_mode = LD_TAP3D_MN;
+    set_mnmajor(p, false, true);
+    if (!map_3d(&mb, w, 64, 9, 64, 128, 9 * 128, 64, 1, 64)) return PF16_ERR_CUDA;
+  } else {
+    p.b_mode = LD_TILED_K;
+    set_kmajor(p, false, true);
+    if (!map_2d(&mb, w, 9 * 64, 64, 9 * 64, 64, 64)) return PF16_ERR_CUDA;
+  }
+  p.idesc = idesc_f16(kBM, 64, false, dgrad, false);
+  p.halo_ws = ws;
+  p.halo_h = (int)H;
+  p.m_tiles = (int)(N * H * ws / kBM);
+  const int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
 int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
                   void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
   Shape s;
@@ -392,6 +445,8 @@ int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w,
   p.out = y;
   p.ldo = s.K;
   p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
+  if (const int ws = halo_width(s, (flags & PF16_ACCUMULATE) != 0))
+    return run_halo(s, ws, false, x, w, y, status, sms, st);
   const int BN = pick_bn_out(s.K);
   p.a_mode = LD_TILED_K;
   p.b_mode = LD_TILED_K;
@@ -449,6 +504,7 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
   if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const bool accum = (flags & PF16_ACCUMULATE) != 0;
+  if (const int ws = halo_width(s, accum)) return run_halo(s, ws, true, dy, w, dx, status, sms, st);
   const int BN = pick_bn_out(s.C);
   const size_t dx_elems = (size_t)(s.N * s.H * s.W * s.C);
 

@@ -472,4 +472,240 @@ cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, co
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Halo engine: 3x3 / stride 1 / pad 1 convolution (forward, or data gradient
+// as a convolution of dy with the flipped filter), 64 input channels, 64
+// outputs.  GEMM rows are the pixels of a padded grid whose image rows are ws
+// >= W + 2 columns wide (ws = 64 or 32), so a 128-row tile is 128/ws whole
+// image rows.  One TMA box brings the tile's input rows i0-1 .. i0+128/ws,
+// columns -1 .. ws-2 (zeros outside the image), 128-byte swizzled, one pixel
+// per 128-byte row; tap (dr, ds) is then the 128-row window that starts
+// dr*ws + ds pixels into the box.  The swizzle is a function of the absolute
+// shared-memory address, so a descriptor whose start moves by whole 128-byte
+// rows reads exactly that window (checked on the GPU: rows m + o for offsets
+// o = 1, 2, 3, 8, 9 with base offset 0).  The input is thus read once per
+// tile instead of once per tap.  The nine 64 x 64 weight slices stay in shared
+// memory for the whole launch.  Columns j >= W of the padded grid are
+// computed and then dropped by the 3-D TMA store, which clips at W.
+// Same roles and bounded waits as k_gemm.
+// ---------------------------------------------------------------------------
+struct HaloCfg {
+  static constexpr int B_TILE = 64 * kBK * 2;       // one tap's 64 x 64 weights
+  static constexpr int B_BYTES = 9 * B_TILE;        // resident
+  static constexpr int A_BOX_MAX = 64 * 4 * 128;    // ws = 64: 4 rows of 64 pixels (ws = 32: 6 x 32)
+  static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's 2-pixel over-read
+  static constexpr int STAGES = 4;
+  static constexpr int TMEM_COLS = 128;
+  static constexpr int STAGING_BYTES = 4 * 4096;
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
+  static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + BAR_BYTES;
+};
+
+__global__ void __launch_bounds__(192, 1)
+    k_gemm_halo(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
+  using Cfg = HaloCfg;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* bres = smem;                                   // 9 weight slices
+  uint8_t* astages = smem + Cfg::B_BYTES;                 // 1024-aligned stages
+  uint8_t* staging = astages + Cfg::STAGES * Cfg::A_STAGE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + Cfg::STAGES;
+  uint64_t* tfull = bars + 2 * Cfg::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* bready = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bready + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int ws = p.halo_ws, rows = kBM / ws;
+  const uint32_t box_bytes = (uint32_t)((rows + 2) * ws * 128);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < Cfg::STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    mbar_init(smem_u32(bready), 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&mapA);
+    tma_prefetch_desc(&mapB);
+    tma_prefetch_desc(&mapC);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total = p.m_tiles;
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // resident weights: the 64 x 64 slice of each of the nine taps
+      const uint32_t bb = smem_u32(bready);
+      mbar_arrive_expect_tx(bb, Cfg::B_BYTES);
+      for (int t = 0; t < 9; ++t) {
+        const uint32_t dst = smem_u32(bres + t * Cfg::B_TILE);
+        if (p.b_mode == LD_TILED_K)
+          tma_load_2d(dst, &mapB, bb, p.tap_w[t] * kBK, 0);
+        else
+          tma_load_3d(dst, &mapB, bb, 0, p.tap_w[t], 0);
+      }
+      int stage = 0;
+      uint32_t phase = 0, issued = 0;
+      for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
+        const int g = u * rows;  // first image row of the tile over all images (n*H + i0)
+        const int n = g / p.halo_h, i0 = g - n * p.halo_h;
+        if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim)) {
+          record_timeout(p, abort_flag);
+          break;
+        }
+        const uint32_t fb = smem_u32(&full[stage]);
+        mbar_arrive_expect_tx(fb, box_bytes);
+        tma_load_4d(smem_u32(astages + stage * Cfg::A_STAGE), &mapA, fb, 0, -1, i0 - 1, n);
+        ++issued;
+        if (++stage == Cfg::STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      // let every copy this thread started land before the CTA can exit
+      mbar_wait(smem_u32(bready), 0, 1000000000ull);
+      if (*abort_flag) {
+        const uint32_t nn = issued < (uint32_t)Cfg::STAGES ? issued : (uint32_t)Cfg::STAGES;
+        int s = stage;
+        uint32_t ph = phase;
+        for (uint32_t i = 0; i < nn; ++i) {
+          if (--s < 0) {
+            s = Cfg::STAGES - 1;
+            ph ^= 1;
+          }
+          mbar_wait(smem_u32(&full[s]), ph, 1000000000ull);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = mbar_wait(smem_u32(bready), 0, lim);
+      if (!ok) record_timeout(p, abort_flag);
+      tc_fence_after();
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      const uint32_t sb0 = smem_u32(bres);
+      for (int u = blockIdx.x; ok && u < total && !*abort_flag; u += gridDim.x) {
+        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim) ||
+            !mbar_wait(smem_u32(&full[stage]), phase, lim)) {
+          record_timeout(p, abort_flag);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 64);
+        const uint32_t sa = smem_u32(astages + stage * Cfg::A_STAGE);
+#pragma unroll 1
+        for (int t = 0; t < 9; ++t) {
+          const uint32_t at = sa + (uint32_t)((p.tap_dr[t] * ws + p.tap_ds[t]) * 128);
+          const uint32_t bt = sb0 + (uint32_t)(t * Cfg::B_TILE);
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            const uint64_t ad = smem_desc(at + kk * 32, 16, 1024, 2);
+            const uint64_t bd = smem_desc(bt + kk * p.b_kstep, p.b_lbo, p.b_sbo, 2);
+            tc_mma_f16(d_tmem, ad, bd, p.idesc, (t > 0 || kk > 0) ? 1u : 0u);
+          }
+        }
+        tc_commit(smem_u32(&empty[stage]));
+        if (++stage == Cfg::STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+        tc_commit(smem_u32(&tfull[acc]));
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+    }
+  } else {
+    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1; 32 rows each, which
+    // lie in one image row of the padded grid (ws is a multiple of 32)
+    const int sub = warp & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    const uint32_t stg = smem_u32(staging) + (uint32_t)(sub * 4096);
+    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) record_timeout(p, abort_flag);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * 64);
+      uint32_t r[64];
+      tmem_ld16(tbase, r);
+      tmem_ld16(tbase + 16, r + 16);
+      tmem_ld16(tbase + 32, r + 32);
+      tmem_ld16(tbase + 48, r + 48);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        uint4 v;
+        v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
+        v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
+        v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
+        v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
+        st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int mp = u * kBM + sub * 32;  // first padded-grid row of the warp
+        const int grow = mp / ws;
+        tma_store_3d(&mapC, stg, 0, mp - grow * ws, grow);
+        bulk_commit();
+      }
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+    if (lane == 0) bulk_wait0();
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                             const GemmParams& p, int grid, cudaStream_t s) {
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_halo, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         HaloCfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  k_gemm_halo<<<grid, 192, HaloCfg::SMEM, s>>>(mA, mB, mC, p);
+  return counted_launches(1);
+}
+
 }  // namespace pf16

@@ -89,6 +89,8 @@ struct GemmParams {
   uint32_t b_lbo, b_sbo, b_kstep;
   int* status;            // device status word
   unsigned long long wait_limit_ns;
+  // halo mode (launch_gemm_halo): padded row width and image height
+  int halo_ws, halo_h;
 };
 
 // Launch the engine (BN in {64, 128, 192, 256}).  Returns a cudaError_t.
@@ -96,6 +98,16 @@ cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB
                         const CUtensorMap& mapC, const GemmParams& p, int grid,
                         cudaStream_t stream);
 int gemm_smem_bytes(int BN);
+
+// Halo engine for 3x3 / stride 1 / pad 1 convolutions with 64 input and 64
+// output channels: A = one 4-D TMA box (64 channels x halo_ws columns x
+// 128/halo_ws + 2 rows) per 128-row tile of the padded pixel grid, taps as
+// row-shifted descriptor windows, the nine 64 x 64 B slices resident; the
+// output leaves through a 3-D map (64, W, N*H) clipped at W.  p.tap_dr/tap_ds
+// are the window offsets (0..2), p.tap_w the weight tap of each of the 9 taps,
+// p.b_mode LD_TILED_K (weights [K][9*64]) or LD_TAP3D_MN (weights (C, 9, K)).
+cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
+                             const GemmParams& p, int grid, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------
 // Memory-bound kernels (pf16_elementwise.cu).  All return cudaError_t of the

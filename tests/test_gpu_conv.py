@@ -16,7 +16,9 @@ pytestmark = pytest.mark.gpu
 
 SHAPES = [
     # N, H, W, C, K, R, S, stride, pad
-    (4, 56, 56, 64, 64, 3, 3, 1, 1),     # config 1
+    (4, 56, 56, 64, 64, 3, 3, 1, 1),     # config 1 (halo engine: padded rows of 64)
+    (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine, padded rows of 32
+    (3, 16, 30, 64, 64, 3, 3, 1, 1),     # halo engine, W + 2 = 32 exactly
     (1, 7, 7, 64, 64, 3, 3, 1, 1),       # one partial M tile
     (2, 9, 9, 64, 128, 3, 3, 2, 1),      # strided 3x3, odd size: unequal stride phases
     (2, 14, 14, 256, 64, 1, 1, 1, 0),    # 1x1 GEMM
@@ -120,7 +122,8 @@ def test_stem_wgrad_reuses_forward_patches():
 
 
 @pytest.mark.parametrize("shape", [(2, 9, 9, 64, 128, 3, 3, 1, 1), (2, 10, 10, 64, 64, 1, 1, 2, 0),
-                                   (2, 11, 11, 64, 64, 3, 3, 2, 1)], ids=ids)
+                                   (2, 11, 11, 64, 64, 3, 3, 2, 1), (2, 12, 10, 64, 64, 3, 3, 1, 1)],
+                         ids=ids)
 def test_accumulate_flag(orc, shape):
     N, H, W, C, K, R, S, st, pd = shape
     x, w, dy, P, Q = inputs(shape)
