@@ -27,9 +27,9 @@ struct GemmCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_BYTES = BN * kBK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : (BN == 192 ? 5 : 4));
+  static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : 4);
   static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
-  static constexpr int STAGING_BYTES = 4 * 4096;  // per epilogue warp: 32 rows x 64 cols
+  static constexpr int STAGING_BYTES = 4 * 2 * 4096;  // per epilogue warp: two 32 x 64 tiles
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
 };
@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(192, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* staging = smem + Cfg::STAGES * Cfg::STAGE_BYTES;  // 1024-aligned, 4 KB per epilogue warp
+  uint8_t* staging = smem + Cfg::STAGES * Cfg::STAGE_BYTES;  // 1024-aligned, 2 x 4 KB per epilogue warp
   uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + Cfg::STAGES;
@@ -332,6 +332,7 @@ __global__ void __launch_bounds__(192, 1)
     const int row = sub * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
+    uint32_t sbuf = 0;  // staging tile of the next chunk (two per warp, alternating)
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
@@ -346,9 +347,10 @@ __global__ void __launch_bounds__(192, 1)
       const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
       if (p.tma_store) {
         // 64-column chunks: TMEM -> registers -> 128B-swizzled staging -> TMA store
-        const uint32_t stg = smem_u32(staging) + (uint32_t)(sub * 4096);
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
+          const uint32_t stg = smem_u32(staging) + (uint32_t)((sub * 2 + sbuf) * 4096);
+          sbuf ^= 1;
           uint32_t r[64];
           tmem_ld16(tbase + c, r);
           tmem_ld16(tbase + c + 16, r + 16);
@@ -360,7 +362,7 @@ __global__ void __launch_bounds__(192, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
           }
-          if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
+          if (lane == 0) bulk_wait_read1();  // the store two chunks back has read this tile
           __syncwarp();
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -495,9 +497,9 @@ struct HaloCfg {
   static constexpr int B_BYTES = 9 * B_TILE;        // resident
   static constexpr int A_BOX_MAX = 64 * 4 * 128;    // ws = 64: 4 rows of 64 pixels (ws = 32: 6 x 32)
   static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's 2-pixel over-read
-  static constexpr int STAGES = 4;
+  static constexpr int STAGES = 3;
   static constexpr int TMEM_COLS = 128;
-  static constexpr int STAGING_BYTES = 4 * 4096;
+  static constexpr int STAGING_BYTES = 4 * 2 * 4096;  // two 32 x 64 tiles per epilogue warp
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
   static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + BAR_BYTES;
 };
@@ -642,8 +644,9 @@ __global__ void __launch_bounds__(192, 1)
     const int sub = warp & 3;
     int acc = 0;
     uint32_t acc_phase = 0;
-    const uint32_t stg = smem_u32(staging) + (uint32_t)(sub * 4096);
+    uint32_t sbuf = 0;
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
+      const uint32_t stg = smem_u32(staging) + (uint32_t)((sub * 2 + sbuf) * 4096);
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
       if (!__all_sync(0xffffffffu, got)) {
@@ -661,7 +664,7 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
-      if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
+      if (lane == 0) bulk_wait_read1();  // the store two tiles back has read this staging tile
       __syncwarp();
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -674,6 +677,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       fence_proxy_async_smem();
       __syncwarp();
+      sbuf ^= 1;
       if (lane == 0) {
         const int mp = u * kBM + sub * 32;  // first padded-grid row of the warp
         const int grow = mp / ws;
