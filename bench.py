@@ -599,7 +599,7 @@ def count_launches(net):
     """Kernels of one step, counted by replaying the call sequence with a hook."""
     from paper_1911_07384_gb300 import pf16
 
-    per = {"conv_fwd": 0, "conv_dgrad": 0, "conv_wgrad": 0, "bn_fwd": 3, "bn_bwd": 3, "maxpool_fwd": 1,
+    per = {"conv_fwd": 0, "conv_dgrad": 0, "conv_wgrad": 0, "bn_fwd": 2, "bn_bwd": 3, "maxpool_fwd": 1,
            "maxpool_bwd": 1, "avgpool_fwd": 1, "avgpool_bwd": 1, "softmax_xent": 2, "sgd": 1}
     total = 0
     for c in net.convs:
@@ -611,7 +611,7 @@ def count_launches(net):
             total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
         total += 1 + (1 if ws else 0)   # wgrad (+ split-K reduce; the stem reuses its forward's patches)
-    total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)
+    total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)  # forward statistics come from the conv
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]
     return total

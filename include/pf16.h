@@ -83,6 +83,20 @@ size_t pf16_conv_workspace_size(const pf16_conv_desc* d, int pass);
 int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
                   void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
+/* Forward with the BatchNorm statistics of its output (Eq. 1, Sec. 4.2:
+ * every conv of ResNet-50 but the FC layer feeds a BatchNorm).  Same
+ * arguments and result as pf16_conv_fwd with flags 0, and in addition each
+ * epilogue warp of the GEMM reduces the output rows it stores into a running
+ * (mean, biased variance, count) per output channel -- FP16 halving trees
+ * over 32 rows merged by the count-aware parallel-variance rule -- written to
+ * `stats` (stats_bytes >= pf16_conv_bnstats_size(d), 16-byte aligned,
+ * caller-owned; no initial contents needed).  pf16_bn_fwd_bwd phase 0 takes
+ * it through pf16_bn_tensors.conv_stats and skips its own statistics pass
+ * over y.  k must be a multiple of 64 (PF16_ERR_UNSUPPORTED otherwise). */
+size_t pf16_conv_bnstats_size(const pf16_conv_desc* d);
+int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                          void* ws, size_t ws_bytes, void* stats, size_t stats_bytes, void* stream);
+
 /* Data gradient: dx[n,h,w,c] = sum over the (k,r,s) with h+pad-r = p*st and
  * w+pad-s = q*st in range of dy[n,p,q,k] * w[k,r,s,c]; stride 2 is split into
  * its stride-phase sub-problems, so no zero-insertion work is done.  Every
@@ -168,6 +182,11 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
  *       moves 1/16 of the bytes.
  * relu_mask is ignored without PF16_BN_RELU (the bit mask is a storage
  * choice of this library, not part of the paper's method).
+ * conv_stats (phase 0, optional): when x is the output of a
+ * pf16_conv_fwd_bnstats call that filled this 16-byte-aligned buffer (and
+ * nothing has written x or the buffer since), the mean and variance are
+ * taken from its partial statistics instead of a pass over x; the result is
+ * the same BatchNorm up to the FP16 rounding of a different reduction tree.
  * c must be a multiple of 8 and at most 2048. */
 typedef struct {
   int32_t n, h, w, c;
@@ -180,6 +199,7 @@ typedef struct {
   const uint16_t *x, *gamma, *beta, *residual, *dy, *y_saved;
   uint16_t *y, *mean, *invstd, *dx, *dgamma, *dbeta, *dresidual;
   uint8_t* relu_mask; /* optional ReLU bit mask: written by phase 0, read by phase 1 */
+  const void* conv_stats; /* optional, phase 0: statistics of x from pf16_conv_fwd_bnstats */
 } pf16_bn_tensors;
 
 size_t pf16_bn_workspace_size(const pf16_bn_desc* d);

@@ -343,8 +343,24 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
       return PF16_ERR_CUDA;
     p.tma_store = 1;
   }
-  const int grid = (int)std::min<long long>(units, sms);
+  int grid = (int)std::min<long long>(units, sms);
+  if (p.st_mean) {
+    // fused statistics: every CTA keeps one n-tile (grid a multiple of n_tiles), at most
+    // kBnStatSlots / 4 CTAs per n-tile
+    grid = std::min(grid, (kBnStatSlots / 4) * p.n_tiles);
+    grid -= grid % p.n_tiles;
+  }
   return launch_gemm(BN, a, b, c, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
+// Point the GEMM's fused statistics at a conv-output statistics buffer of C channels.
+void set_stats(GemmParams& p, void* stats, long long C) {
+  if (!stats) return;
+  uint8_t* b = static_cast<uint8_t*>(stats);
+  p.st_hdr = reinterpret_cast<int*>(b);
+  p.st_mean = reinterpret_cast<uint16_t*>(b + bnstat_off_mean());
+  p.st_var = reinterpret_cast<uint16_t*>(b + bnstat_off_var(C));
+  p.st_cnt = reinterpret_cast<int*>(b + bnstat_off_cnt(C));
 }
 
 int check_common(const void* a, const void* b, const void* c) {
@@ -386,8 +402,9 @@ int halo_width(const Shape& s, bool accum) {
 // gradient (dgrad = true: in = dy, weights viewed (C, 9, K), taps flipped)
 // through the halo engine.  in and out are N x H x W x 64.
 int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint16_t* w, uint16_t* out,
-             int* status, int sms, cudaStream_t st) {
+             int* status, int sms, cudaStream_t st, void* stats = nullptr) {
   GemmParams p = base_params(status);
+  set_stats(p, stats, 64);
   CUtensorMap ma, mb, mc;
   const long long N = s.N, H = s.H, W = s.W;
   cuuint64_t dims[4] = {64, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
@@ -417,18 +434,29 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
   p.idesc = idesc_f16(kBM, 64, false, dgrad, false);
   p.halo_ws = ws;
   p.halo_h = (int)H;
+  p.halo_w = (int)W;
+  p.N = 64;
+  p.n_tiles = 1;
   p.m_tiles = (int)(N * H * ws / kBM);
-  const int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  if (stats && grid > kBnStatSlots / 4) grid = kBnStatSlots / 4;
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
-int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
-                  void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                         void* ws, size_t ws_bytes, uint32_t flags, void* stats, size_t stats_bytes,
+                         void* stream) {
   Shape s;
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, w, y)) != PF16_OK) return rc;
   if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  if (stats) {
+    if (flags != 0) return PF16_ERR_ARG;  // statistics of a plain (non-accumulating) output only
+    if (s.K % 64 != 0) return PF16_ERR_UNSUPPORTED;
+    if (!aligned16(stats)) return PF16_ERR_ALIGN;
+    if (stats_bytes < bnstat_bytes(s.K)) return PF16_ERR_WORKSPACE;
+  }
   const size_t need = ws_fwd(s);
   if (need && (!ws || ws_bytes < need)) return PF16_ERR_WORKSPACE;
   if (need && !aligned16(ws)) return PF16_ERR_ALIGN;
@@ -446,7 +474,8 @@ int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w,
   p.ldo = s.K;
   p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
   if (const int ws = halo_width(s, (flags & PF16_ACCUMULATE) != 0))
-    return run_halo(s, ws, false, x, w, y, status, sms, st);
+    return run_halo(s, ws, false, x, w, y, status, sms, st, stats);
+  set_stats(p, stats, s.K);
   const int BN = pick_bn_out(s.K);
   p.a_mode = LD_TILED_K;
   p.b_mode = LD_TILED_K;
@@ -486,6 +515,23 @@ int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w,
     p.num_kb = (int)(s.R * s.S * s.C / 64);
   }
   return run(BN, ma, mb, p, sms, st);
+}
+
+int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                  void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  return conv_fwd_impl(d, x, w, y, ws, ws_bytes, flags, nullptr, 0, stream);
+}
+
+size_t pf16_conv_bnstats_size(const pf16_conv_desc* d) {
+  Shape s;
+  if (conv_shape(d, &s) != PF16_OK || s.K % 64 != 0) return 0;
+  return bnstat_bytes(s.K);
+}
+
+int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
+                          void* ws, size_t ws_bytes, void* stats, size_t stats_bytes, void* stream) {
+  if (!stats) return PF16_ERR_NULL;
+  return conv_fwd_impl(d, x, w, y, ws, ws_bytes, 0, stats, stats_bytes, stream);
 }
 
 int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
@@ -721,6 +767,14 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
     if (b.residual && !t->residual) return PF16_ERR_NULL;
     if (b.residual && !aligned16(t->residual)) return PF16_ERR_ALIGN;
     if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
+    if (t->conv_stats) {
+      if (!aligned16(t->conv_stats)) return PF16_ERR_ALIGN;
+      return launch_bn_fwd_given_stats(b, static_cast<const uint8_t*>(t->conv_stats), t->x, t->gamma,
+                                       t->beta, b.residual ? t->residual : nullptr, t->y, t->relu_mask,
+                                       t->mean, t->invstd, st) == cudaSuccess
+                 ? PF16_OK
+                 : PF16_ERR_CUDA;
+    }
     return launch_bn_fwd(b, t->x, t->gamma, t->beta, b.residual ? t->residual : nullptr, t->y,
                          t->relu_mask, t->mean, t->invstd, static_cast<uint16_t*>(ws), st) ==
                    cudaSuccess

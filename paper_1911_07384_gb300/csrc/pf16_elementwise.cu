@@ -888,6 +888,76 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
   }
 }
 
+// Final forward statistics from a conv-output statistics buffer (written by
+// pf16_conv_fwd_bnstats): a balanced tree over the buffer's slots (padded to a
+// power of two with empty nodes), each slot a (mean, variance, count) node of
+// one epilogue warp, merged by the count-aware parallel-variance rule.  One
+// CTA per channel group of 8.
+__global__ void __launch_bounds__(kFinalThreads)
+    k_bn_fwd_final_slots(const uint8_t* __restrict__ stats, int C, uint16_t eps, uint16_t* mean_out,
+                         uint16_t* invstd_out) {
+  __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
+  __shared__ long long sn[kFinalThreads];
+  const int cg = blockIdx.x, t = threadIdx.x;
+  const int S = *reinterpret_cast<const int*>(stats);
+  const uint16_t* smean = reinterpret_cast<const uint16_t*>(stats + bnstat_off_mean());
+  const uint16_t* svar = reinterpret_cast<const uint16_t*>(stats + bnstat_off_var(C));
+  const int* scnt = reinterpret_cast<const int*>(stats + bnstat_off_cnt(C));
+  int sp2 = 1;
+  while (sp2 < S) sp2 *= 2;
+  const int nthr = sp2 < kFinalThreads ? sp2 : kFinalThreads;
+  const int seg = sp2 / nthr;
+  if (t < nthr) {
+    MV st[12];
+    unsigned cnt = 0;
+    for (int i = 0; i < seg; ++i) {
+      const int b = t * seg + i;
+      const bool ok = b < S;
+      MV node{ok ? __ldg(reinterpret_cast<const uint4*>(smean + (long long)b * C) + cg) : zero4(),
+              ok ? __ldg(reinterpret_cast<const uint4*>(svar + (long long)b * C) + cg) : zero4(),
+              ok ? (long long)__ldg(scnt + b) : 0ll};
+#pragma unroll
+      for (int l = 0; l < 12; ++l) {
+        if (cnt & (1u << l)) {
+          node = mv_merge(st[l], node);
+        } else {
+          st[l] = node;
+          break;
+        }
+      }
+      ++cnt;
+    }
+    const int lv = 31 - __clz(seg);
+    MV res = st[0];
+#pragma unroll
+    for (int l = 0; l < 12; ++l)
+      if (l == lv) res = st[l];
+    smu[t] = res.mu;
+    sv[t] = res.v;
+    sn[t] = res.n;
+  }
+  __syncthreads();
+  for (int half = nthr / 2; half >= 1; half /= 2) {
+    if (t < half) {
+      const MV r = mv_merge(MV{smu[t], sv[t], sn[t]}, MV{smu[t + half], sv[t + half], sn[t + half]});
+      smu[t] = r.mu;
+      sv[t] = r.v;
+      sn[t] = r.n;
+    }
+    __syncthreads();
+  }
+  if (t == 0) {
+    const uint4 ve = add4(sv[0], make_uint4(dup2(eps), dup2(eps), dup2(eps), dup2(eps)));
+    uint4 is;
+    const __half2* hv = reinterpret_cast<const __half2*>(&ve);
+    __half2* hi = reinterpret_cast<__half2*>(&is);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) hi[j] = h2rsqrt(hv[j]);
+    reinterpret_cast<uint4*>(mean_out)[cg] = smu[0];
+    reinterpret_cast<uint4*>(invstd_out)[cg] = is;
+  }
+}
+
 constexpr int kApplyRows = 8;  // rows per thread per CTA in the apply passes
 
 __global__ void __launch_bounds__(256)
@@ -1081,6 +1151,19 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
       b.post_scale, b.relu);
   return counted_launches(3);
+}
+
+cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_stats, const uint16_t* x,
+                                      const uint16_t* gamma, const uint16_t* beta,
+                                      const uint16_t* residual, uint16_t* y, uint8_t* relu_mask,
+                                      uint16_t* mean, uint16_t* invstd, cudaStream_t s) {
+  k_bn_fwd_final_slots<<<b.C / 8, kFinalThreads, 0, s>>>(conv_stats, b.C, b.eps, mean, invstd);
+  const BnGeom g = bn_geom(b.C);
+  const int rows = g.rpb * kApplyRows;
+  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), g.threads, 0, s>>>(
+      x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
+      b.post_scale, b.relu);
+  return counted_launches(2);
 }
 
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,

@@ -198,6 +198,146 @@ __device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int spl
 // low halves of two 32-bit TMEM words -> one f16x2
 __device__ __forceinline__ uint32_t pack_lo(uint32_t a, uint32_t b) { return __byte_perm(a, b, 0x5410); }
 
+
+// ---------------------------------------------------------------------------
+// Fused BatchNorm forward statistics of the output (GemmParams::st_mean).
+// After a warp has staged its 32 rows x 64 columns, lane l reduces channel
+// pair (2l, 2l+1) over the warp's valid rows (a prefix of the 32): the mean
+// of the 32-leaf halving tree (zero padded, scaled by rn(32/n) when rows are
+// missing) and, over the same rows, the mean squared deviation from it.  The
+// leaf is pushed into the warp's binary-counter stack of (mean, variance,
+// count) nodes merged by the count-aware parallel-variance rule -- the
+// arithmetic of the BatchNorm statistics kernels -- and the stack is closed
+// once, after the warp's last tile.  All binary16, one rounding per op.
+// ---------------------------------------------------------------------------
+constexpr int kStChunks = 4;   // 64-column chunks of a tile (BN <= 256)
+constexpr int kStLevels = 12;  // tiles per warp below 2^12
+
+__device__ __forceinline__ uint32_t hmerge2f(uint32_t a, uint32_t b) {  // rn(a/2 + rn(b/2))
+  return hfma2_rn(a, 0x38003800u, hmul2_rn(b, 0x38003800u));
+}
+__device__ __forceinline__ uint32_t dup2h(uint16_t h) { return (uint32_t)h | ((uint32_t)h << 16); }
+
+// node a <- merge(a, b) with counts na, nb (the result's count is na + nb)
+__device__ __forceinline__ void mv2_merge(uint32_t& amu, uint32_t& av, int na, uint32_t bmu, uint32_t bv,
+                                          int nb) {
+  if (nb == 0) return;
+  if (na == 0) {
+    amu = bmu;
+    av = bv;
+    return;
+  }
+  const uint32_t d = hsub2_rn(bmu, amu);
+  if (na == nb) {
+    const uint32_t dh = hmul2_rn(d, 0x38003800u);
+    amu = hmerge2f(amu, bmu);
+    av = hadd2_rn(hmerge2f(av, bv), hmul2_rn(dh, dh));
+  } else {
+    const float n = (float)(na + nb);
+    const uint32_t wa = dup2h(__half_as_ushort(__float2half_rn(__fdiv_rn((float)na, n))));
+    const uint32_t wb = dup2h(__half_as_ushort(__float2half_rn(__fdiv_rn((float)nb, n))));
+    const uint32_t wab = hmul2_rn(wa, wb);
+    amu = hadd2_rn(hmul2_rn(amu, wa), hmul2_rn(bmu, wb));
+    av = hadd2_rn(hadd2_rn(hmul2_rn(av, wa), hmul2_rn(bv, wb)), hmul2_rn(hmul2_rn(d, d), wab));
+  }
+}
+
+struct EpiStats {
+  uint32_t mu[kStChunks][kStLevels], v[kStChunks][kStLevels];
+  int n[kStLevels];
+  unsigned cnt;
+
+  __device__ __forceinline__ void init() { cnt = 0; }
+
+  // leaf of chunk c from the staged tile (row r at stg + r*128, 128B-swizzled)
+  __device__ __forceinline__ void leaf(int c, uint32_t stg, int lane, int nv) {
+    const uint32_t col = (uint32_t)(lane & 3) * 4;
+    uint32_t t[32];
+#pragma unroll
+    for (int r = 0; r < 32; ++r) {
+      uint32_t x;
+      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
+      t[r] = r < nv ? x : 0u;
+    }
+#pragma unroll
+    for (int w = 16; w >= 1; w /= 2)
+#pragma unroll
+      for (int i = 0; i < w; ++i) t[i] = hmerge2f(t[2 * i], t[2 * i + 1]);
+    uint32_t mu = t[0], sc = 0;
+    if (nv < 32) {
+      sc = dup2h(__half_as_ushort(__float2half_rn(32.0f / (float)nv)));
+      mu = hmul2_rn(mu, sc);
+    }
+#pragma unroll
+    for (int r = 0; r < 32; ++r) {
+      uint32_t x;
+      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
+      const uint32_t e = hsub2_rn(x, mu);
+      t[r] = r < nv ? hmul2_rn(e, e) : 0u;
+    }
+#pragma unroll
+    for (int w = 16; w >= 1; w /= 2)
+#pragma unroll
+      for (int i = 0; i < w; ++i) t[i] = hmerge2f(t[2 * i], t[2 * i + 1]);
+    uint32_t var = t[0];
+    if (nv < 32) var = hmul2_rn(var, sc);
+    // push into chunk c's stack (counts are updated by end_tile)
+    int nn = nv;
+#pragma unroll 1
+    for (int l = 0; l < kStLevels; ++l) {
+      if (cnt & (1u << l)) {
+        uint32_t m2 = this->mu[c][l], v2 = this->v[c][l];
+        mv2_merge(m2, v2, n[l], mu, var, nn);
+        mu = m2;
+        var = v2;
+        nn += n[l];
+      } else {
+        this->mu[c][l] = mu;
+        this->v[c][l] = var;
+        break;
+      }
+    }
+  }
+  // after all chunks of a tile with nv valid rows
+  __device__ __forceinline__ void end_tile(int nv) {
+    int nn = nv;
+#pragma unroll 1
+    for (int l = 0; l < kStLevels; ++l) {
+      if (cnt & (1u << l)) {
+        nn += n[l];
+      } else {
+        n[l] = nn;
+        break;
+      }
+    }
+    ++cnt;
+  }
+  // close the stacks and write this warp's slot for chunks c < nchunks
+  __device__ __forceinline__ void write(const GemmParams& p, int slot, int n0, int nchunks, int lane,
+                                        bool write_count) {
+    int total = 0;
+    for (int c = 0; c < nchunks; ++c) {
+      uint32_t am = 0, av = 0;
+      int an = 0;
+#pragma unroll 1
+      for (int l = 0; l < kStLevels; ++l) {
+        if (cnt & (1u << l)) {
+          uint32_t m2 = mu[c][l], v2 = v[c][l];
+          mv2_merge(m2, v2, n[l], am, av, an);
+          am = m2;
+          av = v2;
+          an += n[l];
+        }
+      }
+      const long long o = (long long)slot * p.N + n0 + c * 64 + 2 * lane;
+      *reinterpret_cast<uint32_t*>(p.st_mean + o) = am;
+      *reinterpret_cast<uint32_t*>(p.st_var + o) = av;
+      total = an;
+    }
+    if (write_count && lane == 0) p.st_cnt[slot] = total;
+  }
+};
+
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
@@ -333,6 +473,8 @@ __global__ void __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     uint32_t sbuf = 0;  // staging tile of the next chunk (two per warp, alternating)
+    EpiStats stats;
+    stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
@@ -346,6 +488,8 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
       if (p.tma_store) {
+        // valid rows of this warp (a prefix of its 32) for the fused statistics
+        const int nv = min(32, max(0, p.M - (m0 + sub * 32)));
         // 64-column chunks: TMEM -> registers -> 128B-swizzled staging -> TMA store
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
@@ -384,7 +528,9 @@ __global__ void __launch_bounds__(192, 1)
               tma_store_2d(&mapC, stg, n0 + c, m0 + sub * 32);
             bulk_commit();
           }
+          if (p.st_mean && nv > 0 && n0 + c < p.N) stats.leaf(c / 64, stg, lane, nv);
         }
+        if (p.st_mean && nv > 0) stats.end_tile(nv);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
         continue;
@@ -428,6 +574,13 @@ __global__ void __launch_bounds__(192, 1)
       if (acc == 0) acc_phase ^= 1;
     }
     if (p.tma_store && lane == 0) bulk_wait0();
+    if (p.st_mean) {
+      // this CTA's tiles all have n-tile blockIdx % n_tiles (the grid is a multiple of n_tiles)
+      const int n0 = (blockIdx.x % p.n_tiles) * BN;
+      const int nch = min(BN, p.N - n0) / 64;
+      stats.write(p, (blockIdx.x / p.n_tiles) * 4 + sub, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
+      if (blockIdx.x == 0 && sub == 0 && lane == 0) p.st_hdr[0] = 4 * ((int)gridDim.x / p.n_tiles);
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -645,6 +798,8 @@ __global__ void __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     uint32_t sbuf = 0;
+    EpiStats stats;
+    stats.init();
     for (int u = blockIdx.x; u < total; u += gridDim.x) {
       const uint32_t stg = smem_u32(staging) + (uint32_t)((sub * 2 + sbuf) * 4096);
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
@@ -684,10 +839,22 @@ __global__ void __launch_bounds__(192, 1)
         tma_store_3d(&mapC, stg, 0, mp - grow * ws, grow);
         bulk_commit();
       }
+      if (p.st_mean) {
+        const int mp = u * kBM + sub * 32;
+        const int nv = min(32, max(0, p.halo_w - mp % ws));  // columns j >= W are padding
+        if (nv > 0) {
+          stats.leaf(0, stg, lane, nv);
+          stats.end_tile(nv);
+        }
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
     if (lane == 0) bulk_wait0();
+    if (p.st_mean) {
+      stats.write(p, blockIdx.x * 4 + sub, 0, 1, lane, true);
+      if (blockIdx.x == 0 && sub == 0 && lane == 0) p.st_hdr[0] = 4 * (int)gridDim.x;
+    }
   }
   tc_fence_before();
   __syncthreads();

@@ -89,9 +89,30 @@ struct GemmParams {
   uint32_t b_lbo, b_sbo, b_kstep;
   int* status;            // device status word
   unsigned long long wait_limit_ns;
-  // halo mode (launch_gemm_halo): padded row width and image height
-  int halo_ws, halo_h;
+  // halo mode (launch_gemm_halo): padded row width, image height and width
+  int halo_ws, halo_h, halo_w;
+  // BatchNorm forward statistics of the output (OUT_STORE through TMA only;
+  // null when off): per epilogue warp a running (mean, variance, count) per
+  // output channel over all its rows, written once at the end as slot
+  // (blockIdx / n_tiles) * 4 + warp; st_hdr[0] = number of slots.
+  uint16_t* st_mean;      // [kBnStatSlots][N]
+  uint16_t* st_var;       // [kBnStatSlots][N]
+  int* st_cnt;            // [kBnStatSlots]
+  int* st_hdr;
 };
+
+// Conv-output BatchNorm statistics buffer (pf16_conv_fwd_bnstats): a header of
+// 256 bytes (int slots), then mean and variance [kBnStatSlots][C] binary16 and
+// counts [kBnStatSlots] int32, each section 256-byte aligned.
+constexpr int kBnStatSlots = 1024;
+__host__ __device__ inline size_t bnstat_off_mean() { return 256; }
+__host__ __device__ inline size_t bnstat_off_var(long long C) { return 256 + (size_t)kBnStatSlots * C * 2; }
+__host__ __device__ inline size_t bnstat_off_cnt(long long C) {
+  return 256 + (size_t)2 * kBnStatSlots * C * 2;
+}
+__host__ __device__ inline size_t bnstat_bytes(long long C) {
+  return bnstat_off_cnt(C) + (size_t)kBnStatSlots * 4;
+}
 
 // Launch the engine (BN in {64, 128, 192, 256}).  Returns a cudaError_t.
 cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,
@@ -148,6 +169,11 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
                           const uint16_t* beta, const uint16_t* residual, uint16_t* y,
                           uint8_t* relu_mask, uint16_t* mean, uint16_t* invstd, uint16_t* ws,
                           cudaStream_t s);
+// Forward from conv-output statistics (pf16_conv_fwd_bnstats): final + apply.
+cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_stats, const uint16_t* x,
+                                      const uint16_t* gamma, const uint16_t* beta,
+                                      const uint16_t* residual, uint16_t* y, uint8_t* relu_mask,
+                                      uint16_t* mean, uint16_t* invstd, cudaStream_t s);
 // ReLU decisions from relu_mask when non-null, else from y_saved.
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,

@@ -35,6 +35,7 @@ EXPORTS = [
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
+    "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats",
 ]
 
 
@@ -59,7 +60,7 @@ class BnDesc(ctypes.Structure):
 
 
 _BN_T = ("x", "gamma", "beta", "residual", "dy", "y_saved", "y", "mean", "invstd", "dx", "dgamma",
-         "dbeta", "dresidual", "relu_mask")
+         "dbeta", "dresidual", "relu_mask", "conv_stats")
 
 
 class BnTensors(ctypes.Structure):
@@ -85,6 +86,10 @@ def lib():
             for nm in ("pf16_conv_fwd", "pf16_conv_dgrad", "pf16_conv_wgrad"):
                 getattr(L, nm).argtypes = [cdp, vp, vp, vp, vp, sz, u32, vp]
                 getattr(L, nm).restype = I
+            L.pf16_conv_bnstats_size.argtypes = [cdp]
+            L.pf16_conv_bnstats_size.restype = sz
+            L.pf16_conv_fwd_bnstats.argtypes = [cdp, vp, vp, vp, vp, sz, vp, sz, vp]
+            L.pf16_conv_fwd_bnstats.restype = I
             L.pf16_conv_wgrad_noalloc.argtypes = [cdp, vp, vp, vp, u32, vp]
             L.pf16_conv_wgrad_noalloc.restype = I
             L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
@@ -159,6 +164,17 @@ def conv_workspace_size(d: ConvDesc, pass_: int) -> int:
 def conv_fwd(d, x, w, y, ws=None, flags=0, stream=None):
     _check(lib().pf16_conv_fwd(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(y), _ptr(ws), _nbytes(ws),
                                flags, _stream(stream)), "pf16_conv_fwd")
+
+
+def conv_bnstats_size(d) -> int:
+    return int(lib().pf16_conv_bnstats_size(ctypes.byref(d)))
+
+
+def conv_fwd_bnstats(d, x, w, y, stats, ws=None, stream=None):
+    """Forward conv that also writes the BatchNorm statistics of y into `stats`
+    (a device buffer of conv_bnstats_size(d) bytes) for bn_fwd_bwd(conv_stats=)."""
+    _check(lib().pf16_conv_fwd_bnstats(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(y), _ptr(ws), _nbytes(ws),
+                                       _ptr(stats), _nbytes(stats), _stream(stream)), "pf16_conv_fwd_bnstats")
 
 
 def conv_dgrad(d, dy, w, dx, ws=None, flags=0, stream=None):

@@ -100,9 +100,16 @@ class Conv:
     def bind(self):
         a = self.net.wd
         self.w, self.gw = a.view("w", self.off, self.numel), a.view("g", self.off, self.numel)
+        # BatchNorm statistics of the output, written by the forward GEMM's epilogue
+        size = pf16.conv_bnstats_size(self.desc)
+        self.stats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
 
-    def fwd(self, x, y):
-        self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.ws())
+    def fwd(self, x, y, with_stats=False):
+        if with_stats:
+            self.net.call("conv_fwd", self, pf16.conv_fwd_bnstats, self.desc, x, self.w, y, self.stats,
+                          self.ws())
+        else:
+            self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.ws())
 
     def dgrad(self, dy, dx, accumulate=False):
         self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
@@ -140,10 +147,11 @@ class BN:
         relu = bool(self.desc.flags & pf16.PF16_BN_RELU)
         self.mask = torch.empty(self.elems // 8, dtype=torch.uint8, device=device) if relu else None
 
-    def fwd(self, x, y, residual=None):
+    def fwd(self, x, y, residual=None, conv=None):
+        """conv: the layer whose fwd(with_stats=True) produced x (its statistics are used)."""
         self.net.call("bn_fwd", self, pf16.bn_fwd_bwd, self.desc, 0, self.net.ws, x=x, gamma=self.gamma,
                       beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd,
-                      relu_mask=self.mask)
+                      relu_mask=self.mask, conv_stats=conv.stats if conv is not None else None)
 
     def bwd(self, x, y_saved, dy, dx, dresidual=None):
         self.net.call("bn_bwd", self, pf16.bn_fwd_bwd, self.desc, 1, self.net.ws, x=x, gamma=self.gamma,
@@ -184,17 +192,17 @@ class Bottleneck:
 
     def forward(self, x):
         self.x = x
-        self.conv1.fwd(x, self.a1)
-        self.bn1.fwd(self.a1, self.b1)
-        self.conv2.fwd(self.b1, self.a2)
-        self.bn2.fwd(self.a2, self.b2)
-        self.conv3.fwd(self.b2, self.a3)
+        self.conv1.fwd(x, self.a1, with_stats=True)
+        self.bn1.fwd(self.a1, self.b1, conv=self.conv1)
+        self.conv2.fwd(self.b1, self.a2, with_stats=True)
+        self.bn2.fwd(self.a2, self.b2, conv=self.conv2)
+        self.conv3.fwd(self.b2, self.a3, with_stats=True)
         if self.proj:
-            self.convp.fwd(x, self.ap)
-            self.bnp.fwd(self.ap, self.bp)
-            self.bn3.fwd(self.a3, self.y, residual=self.bp)
+            self.convp.fwd(x, self.ap, with_stats=True)
+            self.bnp.fwd(self.ap, self.bp, conv=self.convp)
+            self.bn3.fwd(self.a3, self.y, residual=self.bp, conv=self.conv3)
         else:
-            self.bn3.fwd(self.a3, self.y, residual=x)
+            self.bn3.fwd(self.a3, self.y, residual=x, conv=self.conv3)
         return self.y
 
     def backward(self, dx):
@@ -314,8 +322,8 @@ class ResNet50:
         return fn(*args, **kw)
 
     def forward(self):
-        self.stem.fwd(self.x, self.a0)
-        self.bn0.fwd(self.a0, self.b0)
+        self.stem.fwd(self.x, self.a0, with_stats=True)
+        self.bn0.fwd(self.a0, self.b0, conv=self.stem)
         self.call("maxpool_fwd", None, pf16.maxpool_fwd_argmax, self.b0, self.p0, self.pool_arg, self.N,
                   self.h0, self.h0, 64)
         h = self.p0

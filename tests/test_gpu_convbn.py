@@ -1,0 +1,81 @@
+"""GPU parity of the fused BatchNorm forward statistics (pf16_conv_fwd_bnstats
+feeding pf16_bn_fwd_bwd through conv_stats; Eq. 1, Eq. 2 and Sec. 4.2).
+
+The conv output must be bit-identical to pf16_conv_fwd's.  The BatchNorm
+computed from the partial statistics is checked against the oracle's binary64
+BatchNorm of that same output, with the tolerance of tests/test_gpu_bn.py:
+per element (4L + 8) u (s (|gamma| (|xhat| + 1) + |beta|) + |residual|) + 2^-24,
+L = ceil(log2 R) -- the statistics are a different tree of the same FP16
+node operations, of depth below L + 6."""
+import numpy as np
+import pytest
+import torch
+
+from paper_1911_07384_gb300 import pf16
+from paper_1911_07384_gb300 import synthetic as syn
+from gpu_util import U, dev, empty16, f64, host, workspace
+
+pytestmark = pytest.mark.gpu
+
+EPS = 0x00A8
+EPS_F = float(np.uint16(EPS).view(np.float16))
+
+SHAPES = [
+    # N, H, W, C, K, R, S, stride, pad
+    (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine (padded rows of 32)
+    (2, 56, 56, 64, 64, 3, 3, 1, 1),     # halo engine (padded rows of 64, columns 56..63 dropped)
+    (1, 7, 7, 64, 64, 3, 3, 1, 1),       # im2col, a single partial M tile (49 rows)
+    (2, 14, 14, 256, 64, 1, 1, 1, 0),    # dense 1x1
+    (2, 13, 13, 128, 256, 3, 3, 2, 1),   # strided 3x3, 4 n-chunks in a tile
+    (2, 7, 7, 256, 512, 1, 1, 1, 0),     # two n-tiles (BN = 256)
+    (3, 7, 7, 512, 1024, 1, 1, 1, 0),    # four n-tiles
+    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem (patch matrix)
+]
+
+
+def ids(s):
+    return "N{}_{}x{}_C{}_K{}_{}x{}_s{}p{}".format(*s)
+
+
+def f16(a):
+    return np.asarray(a, np.float64).astype(np.float16).view(np.uint16)
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=ids)
+def test_conv_fwd_bnstats_then_bn(orc, shape):
+    N, H, W, C, K, R, S, st, pd = shape
+    P, Q = (H + 2 * pd - R) // st + 1, (W + 2 * pd - S) // st + 1
+    rows = N * P * Q
+    x = syn.normal_f16(syn.seed_for(6, "x"), (N, H, W, C))
+    w = syn.he_normal_f16(syn.seed_for(6, "w"), K, R, S, C)
+    d = pf16.conv_desc(*shape)
+    ws = workspace(pf16.conv_workspace_size(d, pf16.PF16_PASS_FWD))
+    tx, tw = dev(x), dev(w)
+    y_ref, y = empty16(rows * K), empty16(rows * K)
+    pf16.conv_fwd(d, tx, tw, y_ref, ws)
+    stats = torch.empty(pf16.conv_bnstats_size(d), dtype=torch.uint8, device="cuda")
+    pf16.conv_fwd_bnstats(d, tx, tw, y, stats, ws)
+    assert pf16.sync_status() == 0
+    yb = host(y)
+    assert np.array_equal(yb, host(y_ref))  # the statistics do not touch the output
+
+    gamma = f16(1.0 + 0.1 * f64(syn.normal_f16(12, (K,))))
+    beta = f16(0.1 * f64(syn.normal_f16(13, (K,))))
+    resid = syn.normal_f16(14, (rows, K))
+    s = 0.25
+    bd = pf16.bn_desc(N, P, Q, K, EPS, int(f16([s])[0]), pf16.PF16_BN_RELU | pf16.PF16_BN_RESIDUAL)
+    bws = workspace(pf16.bn_workspace_size(bd))
+    tz, tm, ti = empty16(rows * K), empty16(K), empty16(K)
+    pf16.bn_fwd_bwd(bd, 0, bws, x=y, gamma=dev(gamma), beta=dev(beta), residual=dev(resid), y=tz, mean=tm,
+                    invstd=ti, conv_stats=stats)
+    assert pf16.sync_status() == 0
+    L = int(np.ceil(np.log2(rows)))
+    zo, mean, var, invstd = orc.bn_fwd(yb, gamma, beta, resid, rows, K, EPS_F, s, True)
+    xv = f64(yb).reshape(rows, K)
+    xhat = (xv - mean) * invstd
+    scale = s * (np.abs(f64(gamma)) * (np.abs(xhat) + 1) + np.abs(f64(beta))) + np.abs(f64(resid).reshape(rows, K))
+    tol = (4 * L + 8) * U * scale + 2.0 ** -24
+    err = np.abs(f64(host(tz)).reshape(rows, K) - zo)
+    assert np.all(err <= tol), float(np.max(err / tol))
+    assert np.all(np.abs(f64(host(tm)) - mean) <= (L + 8) * U * np.abs(xv).max(0))
+    assert np.all(np.abs(f64(host(ti)) - invstd) <= (2 * L + 16) * U * invstd)
