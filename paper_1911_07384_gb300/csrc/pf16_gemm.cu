@@ -22,6 +22,12 @@
 
 namespace pf16 {
 
+// Epilogue: two warps per TMEM sub-partition (lanes 32*(warp % 4) ...), warps
+// 2-5 draining accumulator 0 (the CTA's even tiles) and warps 6-9 accumulator 1
+// (its odd tiles), so two tiles drain at once.
+constexpr int kEpiWarps = 8;
+constexpr int kGemmThreads = 32 * (2 + kEpiWarps);
+
 template <int BN>
 struct GemmCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
@@ -29,7 +35,7 @@ struct GemmCfg {
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : 4);
   static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
-  static constexpr int STAGING_BYTES = 4 * 2 * 4096;  // per epilogue warp: two 32 x 64 tiles
+  static constexpr int STAGING_BYTES = kEpiWarps * 4096;  // per epilogue warp: one 32 x 64 tile
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
 };
@@ -339,7 +345,7 @@ struct EpiStats {
 };
 
 template <int BN>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
   using Cfg = GemmCfg<BN>;
@@ -467,16 +473,16 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else {
-    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1
-    const int sub = warp & 3;
+    // epilogue warps 2..9 -> TMEM sub-partitions 2, 3, 0, 1; group grp drains accumulator grp
+    const int e = warp - 2, grp = e >> 2, sub = warp & 3;
     const int row = sub * 32 + lane;
-    int acc = 0;
+    const int acc = grp;
     uint32_t acc_phase = 0;
-    uint32_t sbuf = 0;  // staging tile of the next chunk (two per warp, alternating)
+    const uint32_t stg = smem_u32(staging) + (uint32_t)(e * 4096);
     EpiStats stats;
     stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
-    for (int u = blockIdx.x; u < total; u += gridDim.x) {
+    for (int u = blockIdx.x + grp * gridDim.x; u < total; u += 2 * gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
       unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
@@ -493,8 +499,6 @@ __global__ void __launch_bounds__(192, 1)
         // 64-column chunks: TMEM -> registers -> 128B-swizzled staging -> TMA store
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
-          const uint32_t stg = smem_u32(staging) + (uint32_t)((sub * 2 + sbuf) * 4096);
-          sbuf ^= 1;
           uint32_t r[64];
           tmem_ld16(tbase + c, r);
           tmem_ld16(tbase + c + 16, r + 16);
@@ -506,7 +510,7 @@ __global__ void __launch_bounds__(192, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
           }
-          if (lane == 0) bulk_wait_read1();  // the store two chunks back has read this tile
+          if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
           __syncwarp();
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -531,8 +535,7 @@ __global__ void __launch_bounds__(192, 1)
           if (p.st_mean && nv > 0 && n0 + c < p.N) stats.leaf(c / 64, stg, lane, nv);
         }
         if (p.st_mean && nv > 0) stats.end_tile(nv);
-        acc ^= 1;
-        if (acc == 0) acc_phase ^= 1;
+        acc_phase ^= 1;
         continue;
       }
       const int m = m0 + row;
@@ -570,16 +573,15 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1;
+      acc_phase ^= 1;
     }
     if (p.tma_store && lane == 0) bulk_wait0();
     if (p.st_mean) {
       // this CTA's tiles all have n-tile blockIdx % n_tiles (the grid is a multiple of n_tiles)
       const int n0 = (blockIdx.x % p.n_tiles) * BN;
       const int nch = min(BN, p.N - n0) / 64;
-      stats.write(p, (blockIdx.x / p.n_tiles) * 4 + sub, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
-      if (blockIdx.x == 0 && sub == 0 && lane == 0) p.st_hdr[0] = 4 * ((int)gridDim.x / p.n_tiles);
+      stats.write(p, (blockIdx.x / p.n_tiles) * kEpiWarps + e, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = kEpiWarps * ((int)gridDim.x / p.n_tiles);
     }
   }
   tc_fence_before();
@@ -612,7 +614,7 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  k_gemm<BN><<<grid, 192, GemmCfg<BN>::SMEM, s>>>(mA, mB, mC, p);
+  k_gemm<BN><<<grid, kGemmThreads, GemmCfg<BN>::SMEM, s>>>(mA, mB, mC, p);
   return counted_launches(1);
 }
 
@@ -652,12 +654,12 @@ struct HaloCfg {
   static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's 2-pixel over-read
   static constexpr int STAGES = 3;
   static constexpr int TMEM_COLS = 128;
-  static constexpr int STAGING_BYTES = 4 * 2 * 4096;  // two 32 x 64 tiles per epilogue warp
+  static constexpr int STAGING_BYTES = kEpiWarps * 4096;  // one 32 x 64 tile per epilogue warp
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
   static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + BAR_BYTES;
 };
 
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_halo(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                 const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
   using Cfg = HaloCfg;
@@ -794,14 +796,13 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1; 32 rows each, which
     // lie in one image row of the padded grid (ws is a multiple of 32)
-    const int sub = warp & 3;
-    int acc = 0;
+    const int e = warp - 2, grp = e >> 2, sub = warp & 3;
+    const int acc = grp;
     uint32_t acc_phase = 0;
-    uint32_t sbuf = 0;
+    const uint32_t stg = smem_u32(staging) + (uint32_t)(e * 4096);
     EpiStats stats;
     stats.init();
-    for (int u = blockIdx.x; u < total; u += gridDim.x) {
-      const uint32_t stg = smem_u32(staging) + (uint32_t)((sub * 2 + sbuf) * 4096);
+    for (int u = blockIdx.x + grp * gridDim.x; u < total; u += 2 * gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
       if (!__all_sync(0xffffffffu, got)) {
@@ -819,7 +820,7 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
-      if (lane == 0) bulk_wait_read1();  // the store two tiles back has read this staging tile
+      if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
       __syncwarp();
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -832,7 +833,6 @@ __global__ void __launch_bounds__(192, 1)
       }
       fence_proxy_async_smem();
       __syncwarp();
-      sbuf ^= 1;
       if (lane == 0) {
         const int mp = u * kBM + sub * 32;  // first padded-grid row of the warp
         const int grow = mp / ws;
@@ -847,13 +847,12 @@ __global__ void __launch_bounds__(192, 1)
           stats.end_tile(nv);
         }
       }
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1;
+      acc_phase ^= 1;
     }
     if (lane == 0) bulk_wait0();
     if (p.st_mean) {
-      stats.write(p, blockIdx.x * 4 + sub, 0, 1, lane, true);
-      if (blockIdx.x == 0 && sub == 0 && lane == 0) p.st_hdr[0] = 4 * (int)gridDim.x;
+      stats.write(p, blockIdx.x * kEpiWarps + e, 0, 1, lane, true);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = kEpiWarps * (int)gridDim.x;
     }
   }
   tc_fence_before();
@@ -875,7 +874,7 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  k_gemm_halo<<<grid, 192, HaloCfg::SMEM, s>>>(mA, mB, mC, p);
+  k_gemm_halo<<<grid, kGemmThreads, HaloCfg::SMEM, s>>>(mA, mB, mC, p);
   return counted_launches(1);
 }
 
