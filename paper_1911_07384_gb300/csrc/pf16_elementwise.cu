@@ -130,6 +130,7 @@ __device__ __forceinline__ void sgd2(uint32_t& w, uint32_t& v, uint32_t g, uint3
 __global__ void k_sgd(uint16_t* __restrict__ w, uint16_t* __restrict__ v,
                       const uint16_t* __restrict__ g, size_t n, uint32_t lr2, uint32_t mom2,
                       uint32_t wd2, int use_wd) {
+  pdl_wait();
   const size_t nvec = n / 8;
   const size_t stride = (size_t)gridDim.x * blockDim.x;
   uint4* W = reinterpret_cast<uint4*>(w);
@@ -162,7 +163,7 @@ cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, ui
   size_t blocks = (nvec + 255) / 256;
   if (blocks < 1) blocks = 1;
   if (blocks > 152 * 16) blocks = 152 * 16;
-  k_sgd<<<(unsigned)blocks, 256, 0, s>>>(w, v, g, n, dup2(lr), dup2(mom), dup2(wd), wd != 0);
+  launch_pdl(k_sgd, dim3((unsigned)blocks), dim3(256), 0, s, w, v, g, n, dup2(lr), dup2(mom), dup2(wd), wd != 0);
   return counted_launches(1);
 }
 
@@ -178,6 +179,7 @@ __global__ void __launch_bounds__(256)
     k_splitk_reduce(const uint16_t* __restrict__ parts, int splits, int splits_pow2, int grp,
                     long long rows, int cols, uint16_t* __restrict__ out, long long ldo,
                     int cols_out) {
+  pdl_wait();
   __shared__ uint4 sh[256];
   const int cl = 256 / grp;
   const int t = threadIdx.x;
@@ -232,7 +234,7 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
   const int cl = 256 / grp;
   const long long total = rows * (cols / 8);
   const long long blocks = (total + cl - 1) / cl;
-  k_splitk_reduce<<<(unsigned)blocks, 256, 0, s>>>(parts, splits, sp2, grp, rows, cols, out, ldo, cols_out);
+  launch_pdl(k_splitk_reduce, dim3((unsigned)blocks), dim3(256), 0, s, parts, splits, sp2, grp, rows, cols, out, ldo, cols_out);
   return counted_launches(1);
 }
 
@@ -249,6 +251,7 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
 __global__ void k_stem_im2col(const uint16_t* __restrict__ x, uint16_t* __restrict__ col, int N,
                               int H, int W, int P, int Q, int R, int S, int C, int stride, int pad,
                               int kcol) {
+  pdl_wait();
   extern __shared__ uint16_t rows[];  // [R][W + 2 pad][C]
   const int WP = W + 2 * pad;
   const int rowlen = WP * C;
@@ -317,13 +320,14 @@ cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, i
   int threads = G * ((160 + G - 1) / G);
   if (threads > 1024) threads = G;
   threads = (threads + 31) / 32 * 32;
-  k_stem_im2col<<<(unsigned)((long long)N * P), threads, shm, s>>>(x, col, N, H, W, P, Q, R, S, C, stride,
+  launch_pdl(k_stem_im2col, dim3((unsigned)((long long)N * P)), dim3(threads), shm, s, x, col, N, H, W, P, Q, R, S, C, stride,
                                                                    pad, kcol);
   return counted_launches(1);
 }
 
 __global__ void k_pad_rows(const uint16_t* __restrict__ w, uint16_t* __restrict__ wp, int K, int kin,
                            int kcol) {
+  pdl_wait();
   const int total = K * kcol;
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < total; t += gridDim.x * blockDim.x) {
     const int k = t / kcol, j = t - k * kcol;
@@ -334,7 +338,7 @@ __global__ void k_pad_rows(const uint16_t* __restrict__ w, uint16_t* __restrict_
 cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wp, int K, int kin, int kcol,
                             cudaStream_t s) {
   const int blocks = (K * kcol + 255) / 256;
-  k_pad_rows<<<blocks, 256, 0, s>>>(w, wp, K, kin, kcol);
+  launch_pdl(k_pad_rows, dim3(blocks), dim3(256), 0, s, w, wp, K, kin, kcol);
   return counted_launches(1);
 }
 
@@ -540,6 +544,7 @@ __device__ __forceinline__ uint32_t stat_ring_init(uint32_t ring, int ntensor, i
 // Forward statistics.  Consumers: cg = t % tc (a warp reads consecutive 16-byte
 // columns of a row from shared memory), rg = t / tc.
 __global__ void __launch_bounds__(kBnThreads + 32, kFwdCtasPerSm) k_bn_fwd_stats(const BnStatArgs a) {
+  pdl_wait();
   extern __shared__ __align__(128) uint8_t stat_smem[];
   __shared__ uint4 smu[kBnThreads], sv[kBnThreads];
   __shared__ long long sn[kBnThreads];
@@ -639,6 +644,7 @@ enum BnRelu : int { BN_NO_RELU = 0, BN_RELU_SAVED = 1, BN_RELU_BITS = 2 };
 // memory while the current chunk is reduced.
 template <int RELU>
 __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats(const BnStatArgs a) {
+  pdl_wait();
   extern __shared__ __align__(128) uint8_t stat_smem[];
   __shared__ uint4 s1[kBnThreads], s2[kBnThreads];
   const BnGeom g = bn_geom(a.C);
@@ -769,6 +775,7 @@ constexpr int kFinalThreads = 256;
 // shared memory; both levels follow a balanced binary tree.  chunk_rows is RB;
 // CTA b owns chunks b, b + blocks, ... and only the last chunk can be partial.
 __global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs a, long long chunk_rows) {
+  pdl_wait();
   __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
   __shared__ long long sn[kFinalThreads];
   const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
@@ -845,6 +852,7 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs
 // Backward: halving trees over the per-CTA padded means (zero padding is
 // exact for sums), then means (x rn(2^L/R)) and sums (x 2^L exactly).
 __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs a) {
+  pdl_wait();
   __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
   const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
   const int nthr = a.blocks_pow2 < kFinalThreads ? a.blocks_pow2 : kFinalThreads;
@@ -896,6 +904,7 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
 __global__ void __launch_bounds__(kFinalThreads)
     k_bn_fwd_final_slots(const uint8_t* __restrict__ stats, int C, uint16_t eps, uint16_t* mean_out,
                          uint16_t* invstd_out) {
+  pdl_wait();
   __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
   __shared__ long long sn[kFinalThreads];
   const int cg = blockIdx.x, t = threadIdx.x;
@@ -966,6 +975,7 @@ __global__ void __launch_bounds__(256)
                const uint16_t* __restrict__ invstd, const uint16_t* __restrict__ residual,
                uint16_t* __restrict__ y, uint8_t* __restrict__ mask, int R, int C, int rpb,
                uint16_t post_scale, int relu) {
+  pdl_wait();
   const int tc = C / 8;
   const int t = threadIdx.x;
   if (t >= tc * rpb) return;
@@ -1010,6 +1020,7 @@ __global__ void __launch_bounds__(256)
                    const uint8_t* __restrict__ mask, const uint16_t* __restrict__ mm,
                    uint16_t* __restrict__ dx, uint16_t* __restrict__ dres, int R, int C, int rpb,
                    uint16_t post_scale) {
+  pdl_wait();
   const int tc = C / 8;
   const int t = threadIdx.x;
   if (t >= tc * rpb) return;
@@ -1144,10 +1155,10 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   a.mean_out = mean;
   a.invstd_out = invstd;
   const BnGeom g = bn_geom(b.C);
-  k_bn_fwd_stats<<<b.fwd.blocks, g.threads + 32, stat_smem_bytes(1), s>>>(a);
-  k_bn_fwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a, (long long)b.chunk_rows);
+  launch_pdl(k_bn_fwd_stats, dim3(b.fwd.blocks), dim3(g.threads + 32), stat_smem_bytes(1), s, a);
+  launch_pdl(k_bn_fwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a, (long long)b.chunk_rows);
   const int rows = g.rpb * kApplyRows;
-  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), g.threads, 0, s>>>(
+  launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
       b.post_scale, b.relu);
   return counted_launches(3);
@@ -1157,10 +1168,10 @@ cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_sta
                                       const uint16_t* gamma, const uint16_t* beta,
                                       const uint16_t* residual, uint16_t* y, uint8_t* relu_mask,
                                       uint16_t* mean, uint16_t* invstd, cudaStream_t s) {
-  k_bn_fwd_final_slots<<<b.C / 8, kFinalThreads, 0, s>>>(conv_stats, b.C, b.eps, mean, invstd);
+  launch_pdl(k_bn_fwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, conv_stats, b.C, b.eps, mean, invstd);
   const BnGeom g = bn_geom(b.C);
   const int rows = g.rpb * kApplyRows;
-  k_bn_apply<<<(unsigned)((b.R + rows - 1) / rows), g.threads, 0, s>>>(
+  launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
       b.post_scale, b.relu);
   return counted_launches(2);
@@ -1191,30 +1202,30 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   switch (mode) {
     case BN_NO_RELU:
       e = stat_smem_attr(k_bn_bwd_stats<BN_NO_RELU>, smem, attr[0]);
-      if (e == cudaSuccess) k_bn_bwd_stats<BN_NO_RELU><<<b.bwd.blocks, threads, smem, s>>>(a);
+      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_NO_RELU>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
       break;
     case BN_RELU_SAVED:
       e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_SAVED>, smem, attr[1]);
-      if (e == cudaSuccess) k_bn_bwd_stats<BN_RELU_SAVED><<<b.bwd.blocks, threads, smem, s>>>(a);
+      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_RELU_SAVED>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
       break;
     default:
       e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_BITS>, smem, attr[2]);
-      if (e == cudaSuccess) k_bn_bwd_stats<BN_RELU_BITS><<<b.bwd.blocks, threads, smem, s>>>(a);
+      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_RELU_BITS>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
       break;
   }
   if (e != cudaSuccess) return e;
-  k_bn_bwd_final<<<b.C / 8, kFinalThreads, 0, s>>>(a);
+  launch_pdl(k_bn_bwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a);
   switch (mode) {
     case BN_NO_RELU:
-      k_bn_bwd_apply<BN_NO_RELU><<<apply_blocks, g.threads, 0, s>>>(
+      launch_pdl(k_bn_bwd_apply<BN_NO_RELU>, dim3(apply_blocks), dim3(g.threads), 0, s, 
           x, gamma, mean, invstd, dy, nullptr, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
       break;
     case BN_RELU_SAVED:
-      k_bn_bwd_apply<BN_RELU_SAVED><<<apply_blocks, g.threads, 0, s>>>(
+      launch_pdl(k_bn_bwd_apply<BN_RELU_SAVED>, dim3(apply_blocks), dim3(g.threads), 0, s, 
           x, gamma, mean, invstd, dy, y_saved, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
       break;
     default:
-      k_bn_bwd_apply<BN_RELU_BITS><<<apply_blocks, g.threads, 0, s>>>(
+      launch_pdl(k_bn_bwd_apply<BN_RELU_BITS>, dim3(apply_blocks), dim3(g.threads), 0, s, 
           x, gamma, mean, invstd, dy, nullptr, relu_mask, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
       break;
   }
@@ -1230,6 +1241,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
 __global__ void __launch_bounds__(256)
     k_maxpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restrict__ y, uint8_t* __restrict__ codes,
                   int N, int H, int W, int C, int P, int Q) {
+  pdl_wait();
   const int tc = C / 8;
   const int n = blockIdx.x / P, p = blockIdx.x - n * P;
   const long long orow = (long long)blockIdx.x * Q * tc;  // first output vector of the row
@@ -1284,6 +1296,7 @@ __device__ __forceinline__ uint32_t code_sel2(uint32_t cw, int j, uint32_t mine)
 __global__ void __launch_bounds__(512)
     k_maxpool_bwd_codes(const uint8_t* __restrict__ codes, const uint16_t* __restrict__ dy,
                         uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
+  pdl_wait();
   const int tc = C / 8;
   const int HB = (H + 1) / 2, WB = (W + 1) / 2;
   const int n = blockIdx.x / HB, i = blockIdx.x - n * HB;
@@ -1345,6 +1358,7 @@ constexpr int kPoolTP = 4;
 __global__ void __launch_bounds__(256)
     k_maxpool_bwd(const uint16_t* __restrict__ x, const uint16_t* __restrict__ dy,
                   uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
+  pdl_wait();
   extern __shared__ uint4 band[];  // [2*kPoolTP + 3][W] cells of 8 channels
   const int tc = C / 8;
   const int bands = (P + kPoolTP - 1) / kPoolTP;
@@ -1432,7 +1446,7 @@ __global__ void __launch_bounds__(256)
 cudaError_t launch_maxpool_fwd(const uint16_t* x, uint16_t* y, uint8_t* codes, int N, int H, int W,
                                int C, cudaStream_t s) {
   const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
-  k_maxpool_fwd<<<(unsigned)((long long)N * P), 256, 0, s>>>(x, y, codes, N, H, W, C, P, Q);
+  launch_pdl(k_maxpool_fwd, dim3((unsigned)((long long)N * P)), dim3(256), 0, s, x, y, codes, N, H, W, C, P, Q);
   return counted_launches(1);
 }
 
@@ -1442,7 +1456,7 @@ cudaError_t launch_maxpool_bwd_codes(const uint8_t* codes, const uint16_t* dy, u
   // one thread per 2x2 cell block of a block row, where that fits in 512 threads
   const long long per_row = (long long)((W + 1) / 2) * (C / 8);
   const int threads = per_row >= 512 ? 512 : (int)((per_row + 31) / 32 * 32);
-  k_maxpool_bwd_codes<<<(unsigned)((long long)N * ((H + 1) / 2)), threads, 0, s>>>(codes, dy, dx, N, H,
+  launch_pdl(k_maxpool_bwd_codes, dim3((unsigned)((long long)N * ((H + 1) / 2))), dim3(threads), 0, s, codes, dy, dx, N, H,
                                                                                      W, C, P, Q);
   return counted_launches(1);
 }
@@ -1456,7 +1470,7 @@ cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* 
     cudaError_t e = cudaFuncSetAttribute(k_maxpool_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
     if (e != cudaSuccess) return e;
   }
-  k_maxpool_bwd<<<(unsigned)((long long)N * bands * (C / 8)), 256, shm, s>>>(x, dy, dx, N, H, W, C, P, Q);
+  launch_pdl(k_maxpool_bwd, dim3((unsigned)((long long)N * bands * (C / 8))), dim3(256), shm, s, x, dy, dx, N, H, W, C, P, Q);
   return counted_launches(1);
 }
 
@@ -1465,6 +1479,7 @@ cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* 
 // ============================================================================
 __global__ void k_avgpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restrict__ y, int N, int HW,
                               int C, int levels, uint16_t ratio) {
+  pdl_wait();
   const int tc = C / 8;
   const long long total = (long long)N * tc;
   for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
@@ -1480,6 +1495,7 @@ __global__ void k_avgpool_fwd(const uint16_t* __restrict__ x, uint16_t* __restri
 
 __global__ void k_avgpool_bwd(const uint16_t* __restrict__ dy, uint16_t* __restrict__ dx, int N,
                               int HW, int C, uint16_t inv) {
+  pdl_wait();
   const int tc = C / 8;
   const long long total = (long long)N * HW * tc;
   for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
@@ -1496,7 +1512,7 @@ cudaError_t launch_avgpool_fwd(const uint16_t* x, uint16_t* y, int N, int HW, in
   while ((1 << L) < HW) ++L;
   const uint16_t ratio = f16_bits_host((float)((double)(1 << L) / HW));
   const long long total = (long long)N * (C / 8);
-  k_avgpool_fwd<<<grid_for(total, 128, 152 * 16), 128, 0, s>>>(x, y, N, HW, C, L, ratio);
+  launch_pdl(k_avgpool_fwd, dim3(grid_for(total, 128, 152 * 16)), dim3(128), 0, s, x, y, N, HW, C, L, ratio);
   return counted_launches(1);
 }
 
@@ -1504,7 +1520,7 @@ cudaError_t launch_avgpool_bwd(const uint16_t* dy, uint16_t* dx, int N, int HW, 
                                cudaStream_t s) {
   const uint16_t inv = f16_bits_host((float)(1.0 / HW));
   const long long total = (long long)N * HW * (C / 8);
-  k_avgpool_bwd<<<grid_for(total, 256, 152 * 16), 256, 0, s>>>(dy, dx, N, HW, C, inv);
+  launch_pdl(k_avgpool_bwd, dim3(grid_for(total, 256, 152 * 16)), dim3(256), 0, s, dy, dx, N, HW, C, inv);
   return counted_launches(1);
 }
 
@@ -1528,6 +1544,7 @@ __global__ void __launch_bounds__(kSmThreads)
     k_softmax_rows(const uint16_t* __restrict__ logits, const uint16_t* __restrict__ bias,
                    const int32_t* __restrict__ labels, int K, uint16_t invB,
                    uint16_t* __restrict__ dlogits, uint16_t* __restrict__ row_loss) {
+  pdl_wait();
   __shared__ float smax[kSmThreads / 32];
   __shared__ uint16_t ssum[kSmThreads];
   __shared__ __half s_lse;
@@ -1600,6 +1617,7 @@ __global__ void __launch_bounds__(kSmThreads)
 __global__ void k_softmax_cols(const uint16_t* __restrict__ dlogits, const uint16_t* __restrict__ row_loss,
                                int B, int K, int levels, uint16_t ratio, uint16_t* __restrict__ dbias,
                                uint16_t* __restrict__ loss) {
+  pdl_wait();
   const int k = blockIdx.x * blockDim.x + threadIdx.x;
   if (dbias && k < K) {
     uint16_t st[16];
@@ -1644,8 +1662,8 @@ cudaError_t launch_softmax_xent(const uint16_t* logits, const uint16_t* bias,
   int L = 0;
   while ((1 << L) < B) ++L;
   const uint16_t ratio = f16_bits_host((float)((double)(1 << L) / B));
-  k_softmax_rows<<<B, kSmThreads, 0, s>>>(logits, bias, labels, K, invB, dlogits, ws);
-  k_softmax_cols<<<(K + 255) / 256, 256, 0, s>>>(dlogits, ws, B, K, L, ratio, dbias, loss);
+  launch_pdl(k_softmax_rows, dim3(B), dim3(kSmThreads), 0, s, logits, bias, labels, K, invB, dlogits, ws);
+  launch_pdl(k_softmax_cols, dim3((K + 255) / 256), dim3(256), 0, s, dlogits, ws, B, K, L, ratio, dbias, loss);
   return counted_launches(2);
 }
 

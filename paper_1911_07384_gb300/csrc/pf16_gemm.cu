@@ -384,6 +384,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // set-up done: wait for the kernel this one depends on
+  pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
   const int total = p.m_tiles * p.n_tiles * p.splits;
   const uint64_t lim = p.wait_limit_ns;
@@ -614,7 +616,7 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  k_gemm<BN><<<grid, kGemmThreads, GemmCfg<BN>::SMEM, s>>>(mA, mB, mC, p);
+  launch_pdl(k_gemm<BN>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
   return counted_launches(1);
 }
 
@@ -704,6 +706,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // set-up done: wait for the kernel this one depends on
+  pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
   const int total = p.m_tiles;
   const uint64_t lim = p.wait_limit_ns;
@@ -874,7 +878,7 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  k_gemm_halo<<<grid, kGemmThreads, HaloCfg::SMEM, s>>>(mA, mB, mC, p);
+  launch_pdl(k_gemm_halo, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
   return counted_launches(1);
 }
 

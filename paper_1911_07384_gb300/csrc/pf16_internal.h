@@ -12,6 +12,25 @@ namespace pf16 {
 // CUDA graph during stream capture included).  Read by pf16_kernel_launches.
 inline std::atomic<unsigned long long> g_kernel_launches{0};
 
+// Launch with programmatic stream serialisation: the kernel may begin while
+// the previous kernel of the stream drains; every kernel of the library calls
+// pdl_wait() before it touches memory a predecessor writes.
+template <typename... K, typename... A>
+inline cudaError_t launch_pdl(void (*kernel)(K...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              A&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
+}
+
 // Status of the n launches just made; they are counted when they succeeded.
 inline cudaError_t counted_launches(int n) {
   const cudaError_t e = cudaGetLastError();

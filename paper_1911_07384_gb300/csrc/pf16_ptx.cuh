@@ -64,6 +64,16 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
 }
 
 // ----------------------------------------------------------------------------
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialisation is launched ahead of the previous kernel's completion;
+// pdl_wait() blocks until that kernel has completed and its writes are
+// visible (a no-op without a programmatic dependency).  No kernel here
+// triggers its dependents early: measured, that was slower than letting them
+// launch at completion.
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// ----------------------------------------------------------------------------
 // TMA
 // ----------------------------------------------------------------------------
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* m) {
