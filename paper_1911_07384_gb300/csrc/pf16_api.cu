@@ -347,7 +347,7 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
   if (p.st_mean) {
     // fused statistics: every CTA keeps one n-tile (grid a multiple of n_tiles), at most
     // kBnStatSlots / 4 CTAs per n-tile
-    grid = std::min(grid, (kBnStatSlots / 8) * p.n_tiles);
+    grid = std::min(grid, kBnStatSlots * p.n_tiles);
     grid -= grid % p.n_tiles;
   }
   return launch_gemm(BN, a, b, c, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
@@ -439,7 +439,7 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
   p.n_tiles = 1;
   p.m_tiles = (int)(N * H * ws / kBM);
   int grid = p.m_tiles < sms ? p.m_tiles : sms;
-  if (stats && grid > kBnStatSlots / 8) grid = kBnStatSlots / 8;
+  if (stats && grid > kBnStatSlots) grid = kBnStatSlots;
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 

@@ -318,9 +318,15 @@ struct EpiStats {
     }
     ++cnt;
   }
-  // close the stacks and write this warp's slot for chunks c < nchunks
-  __device__ __forceinline__ void write(const GemmParams& p, int slot, int n0, int nchunks, int lane,
-                                        bool write_count) {
+  // Close the stacks, merge the CTA's 8 epilogue warps (a balanced tree over
+  // warps 0..7, in shared memory `sm`, >= 8.3 KB, free of pending TMA reads)
+  // and write the CTA's node as `slot` for chunks c < nchunks.  Called by all
+  // 8 epilogue warps; uses named barrier 1.
+  __device__ __forceinline__ void write_cta(const GemmParams& p, uint8_t* sm, int e, int slot, int n0,
+                                            int nchunks, int lane, bool write_count) {
+    uint32_t* node = reinterpret_cast<uint32_t*>(sm);              // [8][kStChunks][32][2]
+    int* ncnt = reinterpret_cast<int*>(sm + 8 * kStChunks * 32 * 8);  // [8]
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
     int total = 0;
     for (int c = 0; c < nchunks; ++c) {
       uint32_t am = 0, av = 0;
@@ -335,12 +341,36 @@ struct EpiStats {
           an += n[l];
         }
       }
-      const long long o = (long long)slot * p.N + n0 + c * 64 + 2 * lane;
-      *reinterpret_cast<uint32_t*>(p.st_mean + o) = am;
-      *reinterpret_cast<uint32_t*>(p.st_var + o) = av;
+      node[((e * kStChunks + c) * 32 + lane) * 2] = am;
+      node[((e * kStChunks + c) * 32 + lane) * 2 + 1] = av;
       total = an;
     }
-    if (write_count && lane == 0) p.st_cnt[slot] = total;
+    if (lane == 0) ncnt[e] = total;
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
+    if (e != 0) return;
+    int tot = 0;
+    for (int c = 0; c < nchunks; ++c) {
+      uint32_t m[8], vv[8];
+      int nn[8];
+#pragma unroll
+      for (int w = 0; w < 8; ++w) {
+        m[w] = node[((w * kStChunks + c) * 32 + lane) * 2];
+        vv[w] = node[((w * kStChunks + c) * 32 + lane) * 2 + 1];
+        nn[w] = ncnt[w];
+      }
+#pragma unroll
+      for (int h = 1; h < 8; h *= 2)
+#pragma unroll
+        for (int w = 0; w < 8; w += 2 * h) {
+          mv2_merge(m[w], vv[w], nn[w], m[w + h], vv[w + h], nn[w + h]);
+          nn[w] += nn[w + h];
+        }
+      const long long o = (long long)slot * p.N + n0 + c * 64 + 2 * lane;
+      *reinterpret_cast<uint32_t*>(p.st_mean + o) = m[0];
+      *reinterpret_cast<uint32_t*>(p.st_var + o) = vv[0];
+      tot = nn[0];
+    }
+    if (write_count && lane == 0) p.st_cnt[slot] = tot;
   }
 };
 
@@ -582,8 +612,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // this CTA's tiles all have n-tile blockIdx % n_tiles (the grid is a multiple of n_tiles)
       const int n0 = (blockIdx.x % p.n_tiles) * BN;
       const int nch = min(BN, p.N - n0) / 64;
-      stats.write(p, (blockIdx.x / p.n_tiles) * kEpiWarps + e, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
-      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = kEpiWarps * ((int)gridDim.x / p.n_tiles);
+      stats.write_cta(p, staging, e, blockIdx.x / p.n_tiles, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = (int)gridDim.x / p.n_tiles;
     }
   }
   tc_fence_before();
@@ -855,8 +885,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     if (lane == 0) bulk_wait0();
     if (p.st_mean) {
-      stats.write(p, blockIdx.x * kEpiWarps + e, 0, 1, lane, true);
-      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = kEpiWarps * (int)gridDim.x;
+      stats.write_cta(p, staging, e, blockIdx.x, 0, 1, lane, true);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = (int)gridDim.x;
     }
   }
   tc_fence_before();

@@ -112,8 +112,8 @@ struct GemmParams {
   int halo_ws, halo_h, halo_w;
   // BatchNorm forward statistics of the output (OUT_STORE through TMA only;
   // null when off): per epilogue warp a running (mean, variance, count) per
-  // output channel over all its rows, written once at the end as slot
-  // (blockIdx / n_tiles) * 8 + epilogue warp; st_hdr[0] = number of slots.
+  // output channel over all its rows; the CTA's warps are merged at the end
+  // and written as slot blockIdx / n_tiles; st_hdr[0] = number of slots.
   uint16_t* st_mean;      // [kBnStatSlots][N]
   uint16_t* st_var;       // [kBnStatSlots][N]
   int* st_cnt;            // [kBnStatSlots]
@@ -123,7 +123,7 @@ struct GemmParams {
 // Conv-output BatchNorm statistics buffer (pf16_conv_fwd_bnstats): a header of
 // 256 bytes (int slots), then mean and variance [kBnStatSlots][C] binary16 and
 // counts [kBnStatSlots] int32, each section 256-byte aligned.
-constexpr int kBnStatSlots = 2048;
+constexpr int kBnStatSlots = 256;
 __host__ __device__ inline size_t bnstat_off_mean() { return 256; }
 __host__ __device__ inline size_t bnstat_off_var(long long C) { return 256 + (size_t)kBnStatSlots * C * 2; }
 __host__ __device__ inline size_t bnstat_off_cnt(long long C) {
