@@ -59,13 +59,10 @@ __device__ __forceinline__ uint4 ldexp4(uint4 v, int e) {
   return mul4(v, dup2(pe));
 }
 
-// positive (> 0, not NaN) test of one binary16 lane, bit-exact
-__device__ __forceinline__ bool h_pos(uint32_t h) {
-  h &= 0xFFFFu;
-  return (h & 0x8000u) == 0 && h != 0 && h <= 0x7C00u;
-}
+// per-lane all-ones where the binary16 lane is > 0 and not NaN: as an unsigned
+// 16-bit code h, 1 <= h <= 0x7C00, i.e. (h - 1) < 0x7C00 -- two SIMD ops
 __device__ __forceinline__ uint32_t relu_mask2(uint32_t y) {
-  return (h_pos(y) ? 0x0000FFFFu : 0u) | (h_pos(y >> 16) ? 0xFFFF0000u : 0u);
+  return __vcmpltu2(__vsub2(y, 0x00010001u), 0x7C007C00u);
 }
 
 // Balanced pairwise tree over a stream of leaves, built as a binary counter:
@@ -443,11 +440,13 @@ __device__ __forceinline__ uint4 and4(uint4 a, uint4 m) {
 __device__ __forceinline__ uint4 relu_mask4(uint4 y) {
   return make_uint4(relu_mask2(y.x), relu_mask2(y.y), relu_mask2(y.z), relu_mask2(y.w));
 }
-// bit j <- lane j of z is > 0 (lane j = channel 8*cg + j)
-__device__ __forceinline__ uint32_t pos_bits8(uint4 z) {
-  return (uint32_t)h_pos(z.x) | (uint32_t)h_pos(z.x >> 16) << 1 | (uint32_t)h_pos(z.y) << 2 |
-         (uint32_t)h_pos(z.y >> 16) << 3 | (uint32_t)h_pos(z.z) << 4 | (uint32_t)h_pos(z.z >> 16) << 5 |
-         (uint32_t)h_pos(z.w) << 6 | (uint32_t)h_pos(z.w >> 16) << 7;
+// the two lane bits of a per-lane all-ones mask
+__device__ __forceinline__ uint32_t mask_bits2(uint32_t m) { return (m & 1u) | ((m >> 15) & 2u); }
+// ReLU of z, and the decisions as bits (bit j: lane j of z is > 0)
+__device__ __forceinline__ uint4 relu_bits(uint4 z, uint32_t& bits) {
+  const uint4 m = relu_mask4(z);
+  bits = mask_bits2(m.x) | mask_bits2(m.y) << 2 | mask_bits2(m.z) << 4 | mask_bits2(m.w) << 6;
+  return and4(z, m);
 }
 __device__ __forceinline__ uint32_t bits_mask2(uint32_t b) {
   return ((b & 1u) ? 0x0000FFFFu : 0u) | ((b & 2u) ? 0xFFFF0000u : 0u);
@@ -1004,8 +1003,9 @@ __global__ void __launch_bounds__(256)
       uint4 z = mul4(add4(mul4v(ga, xh), be), ps);      // Eq. 2, then x post_scale
       if (residual) z = add4(z, rv[i]);
       if (relu) {
-        z = and4(z, relu_mask4(z));
-        if (mask) mask[r * tc + cg] = (uint8_t)pos_bits8(z);
+        uint32_t bits;
+        z = relu_bits(z, bits);
+        if (mask) mask[r * tc + cg] = (uint8_t)bits;
       }
       reinterpret_cast<uint4*>(y)[r * tc + cg] = z;
     }
