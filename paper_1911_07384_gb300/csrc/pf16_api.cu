@@ -202,9 +202,12 @@ struct WgradSplit {
 //   rounds * (K-blocks per split * t_kb + t_unit) + partial-plane traffic,
 // with t_kb ~ 0.4 us per 128 x 256 x 64 block, t_unit ~ 1 us (pipeline fill
 // and the partial tile's store) and the splits * |dw| FP16 partials written
-// and read back at ~6 TB/s.  Between 4 and 64 K-blocks (4096 pixels) go into
-// one FP16 tensor-memory accumulator; at most 1024 splits.
+// and read back at the reduce's effective ~2 TB/s (measured: a reduce call
+// costs several microseconds beyond its bytes).  Between 4 and 64 K-blocks
+// (4096 pixels) go into one FP16 tensor-memory accumulator; at most 1024
+// splits.
 constexpr int kPlanSms = 152;
+constexpr double kPartialBw = 2e12;  // effective partial-plane bandwidth of the reduce, bytes/s
 
 WgradSplit wgrad_split(const Shape& s) {
   WgradSplit w;
@@ -225,7 +228,7 @@ WgradSplit wgrad_split(const Shape& s) {
     if (kps < 4 && sp > 1) break;  // kps only shrinks from here
     const int real = cdiv(w.num_kb, kps);
     const long long rounds = (tiles * real + kPlanSms - 1) / kPlanSms;
-    const double t = (double)rounds * (kps * t_kb + t_unit) + (real > 1 ? real * dw_bytes * 2.0 / 6e12 : 0.0);
+    const double t = (double)rounds * (kps * t_kb + t_unit) + (real > 1 ? real * dw_bytes * 2.0 / kPartialBw : 0.0);
     if (best < 0.0 || t < best * (1.0 - 1e-9)) {
       best = t;
       w.kb_per_split = kps;
