@@ -605,12 +605,12 @@ def count_launches(net):
     for c in net.convs:
         d = c.desc
         stem = d.c == 3
-        total += 1 + (2 if stem else 0)                      # fwd (+ patch gather, weight pad)
+        total += 1 + (1 if stem else 0)                      # fwd (+ the stem's space-to-depth)
         if not stem:
             phases = d.stride * d.stride if d.r > 1 else 1
             total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
-        total += 1 + (1 if ws else 0)   # wgrad (+ split-K reduce; the stem reuses its forward's patches)
+        total += 1 + (1 if ws else 0) + (1 if stem else 0)  # wgrad (+ split-K reduce, + the stem's patch gather)
     total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)  # forward statistics come from the conv
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]

@@ -51,7 +51,6 @@ enum {
 
 /* ----------------------------------------------------------------- flags */
 #define PF16_ACCUMULATE 0x1u  /* conv: out = rn(out + result) instead of out = result */
-#define PF16_REUSE_PATCHES 0x2u /* conv wgrad, c == 3 stem: the workspace holds x's patch matrix */
 #define PF16_BN_RELU 0x1u     /* BN: apply ReLU to the output */
 #define PF16_BN_RESIDUAL 0x2u /* BN: add the residual tensor before the ReLU */
 
@@ -109,13 +108,7 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
 /* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*st+r-pad, q*st+s-pad, c].
  * The reduction over n*p*q pixels is split into chunks, each accumulated in
  * FP16 by the tensor core into FP16 partials in the workspace, which are then
- * summed by a balanced pairwise FP16 tree.  flags: 0, or PF16_REUSE_PATCHES
- * for the c == 3 stem only (PF16_ERR_ARG otherwise): the workspace already
- * holds the patch matrix of x, as pf16_conv_fwd left it when called with the
- * same descriptor, the same x and the same workspace pointer, and nothing
- * has written x or the workspace since; the gather is then skipped (a
- * storage choice of this library, no counterpart in the paper).  The library
- * cannot check this promise: a stale matrix gives a wrong gradient. */
+ * summed by a balanced pairwise FP16 tree.  flags: 0 (PF16_ERR_ARG otherwise). */
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 

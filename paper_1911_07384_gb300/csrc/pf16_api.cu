@@ -82,13 +82,14 @@ int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
 
 // 2-D tiled map over a row-major [rows][cols] FP16 matrix with row stride ld (elements).
 bool map_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint64_t ld,
-            uint32_t box_cols, uint32_t box_rows) {
+            uint32_t box_cols, uint32_t box_rows,
+            CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 2};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t es[2] = {1, 1};
   return g_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims,
-                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -242,10 +243,35 @@ WgradSplit wgrad_split(const Shape& s) {
   return w;
 }
 
+// The ResNet stem (7x7, stride 2, pad 3, 3 -> 64 channels) runs as a 4x4
+// stride-1 convolution over the 2x2 space-to-depth of its input: xs[n][I][J]
+// holds 16 channels (a*2 + b)*4 + c = x[n][2I + a - 3][2J + b - 3][c] (c < 3;
+// channel c = 3 and pixels outside x are 0), I < P + 3, J < Q + 3, and the
+// 64 x 256 packed filter ws[k][(u*4 + v)*16 + (a*2 + b)*4 + c] =
+// w[k][2u + a][2v + b][c] (0 where 2u + a or 2v + b reaches 7).  Returns the
+// halo engine's padded row width, or 0 where the stem takes the patch GEMM.
+int stem_s2d_width(const Shape& s, bool accum) {
+  if (accum || s.kind != KIND_STEM || s.R != 7 || s.S != 7 || s.st != 2 || s.pad != 3 || s.K != 64)
+    return 0;
+  int ws = 0;
+  if (s.Q + 3 <= 32 && s.P % 4 == 0)
+    ws = 32;
+  else if (s.Q + 3 <= 64 && s.P % 2 == 0)
+    ws = 64;
+  else if (s.Q + 3 <= 128)
+    ws = 128;
+  if (ws == 0 || (long long)s.N * s.P * ws / kBM > (1ll << 30)) return 0;
+  return ws;
+}
+size_t stem_s2d_bytes(const Shape& s) { return round_up((size_t)(s.N * (s.P + 3) * (s.Q + 3) * 32), 256); }
+
 size_t ws_fwd(const Shape& s) {
   if (s.kind != KIND_STEM) return 0;
   const long long kc = stem_kcol(s);
-  return round_up((size_t)(s.N * s.P * s.Q * kc * 2), 256) + round_up((size_t)(s.K * kc * 2), 256);
+  const size_t patch = round_up((size_t)(s.N * s.P * s.Q * kc * 2), 256) + round_up((size_t)(s.K * kc * 2), 256);
+  // the space-to-depth route serves plain stores; PF16_ACCUMULATE takes the patch GEMM
+  if (!stem_s2d_width(s, false)) return patch;
+  return std::max(patch, stem_s2d_bytes(s) + (size_t)(s.K * 256 * 2));
 }
 size_t ws_wgrad(const Shape& s) {
   const WgradSplit w = wgrad_split(s);
@@ -438,9 +464,63 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
   p.halo_ws = ws;
   p.halo_h = (int)H;
   p.halo_w = (int)W;
+  p.halo_cb = 128;
+  p.halo_box_rows = kBM / ws + 2;
+  p.halo_row0 = -1;
+  p.halo_col0 = -1;
   p.N = 64;
   p.n_tiles = 1;
   p.m_tiles = (int)(N * H * ws / kBM);
+  int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  if (stats && grid > kBnStatSlots) grid = kBnStatSlots;
+  return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
+// The stem through the halo engine: space-to-depth of x and the filter into
+// the workspace, then a 4x4 stride-1 convolution over 16 channels with 32-byte
+// pixel rows (layouts at stem_s2d_width).  y is N x P x Q x 64.
+int run_stem_s2d(const Shape& s, int ws, const uint16_t* x, const uint16_t* w, uint16_t* y, void* work,
+                 int* status, int sms, cudaStream_t st, void* stats) {
+  const long long N = s.N, P = s.P, Q = s.Q, Hs = P + 3, Wsd = Q + 3;
+  uint16_t* xs = static_cast<uint16_t*>(work);
+  uint16_t* wsd = xs + stem_s2d_bytes(s) / 2;
+  if (launch_stem_s2d(x, w, xs, wsd, (int)N, (int)s.H, (int)s.W, (int)Hs, (int)Wsd, (int)s.K, st) != cudaSuccess)
+    return PF16_ERR_CUDA;
+  GemmParams p = base_params(status);
+  set_stats(p, stats, 64);
+  CUtensorMap ma, mb, mc;
+  const int rows = kBM / ws;
+  cuuint64_t dims[4] = {16, (cuuint64_t)Wsd, (cuuint64_t)Hs, (cuuint64_t)N};
+  cuuint64_t strides[3] = {32, (cuuint64_t)(Wsd * 32), (cuuint64_t)(Hs * Wsd * 32)};
+  cuuint32_t box[4] = {16, (cuuint32_t)ws, (cuuint32_t)(rows + 3), 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  if (g_encode_tiled(&ma, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, xs, dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return PF16_ERR_CUDA;
+  if (!map_2d(&mb, wsd, 256, 64, 256, 16, 64, CU_TENSOR_MAP_SWIZZLE_32B)) return PF16_ERR_CUDA;
+  if (!map_3d(&mc, y, 64, Q, N * P, 128, Q * 128, 64, 32, 1)) return PF16_ERR_CUDA;
+  p.ntaps = 16;
+  for (int t = 0; t < 16; ++t) {
+    p.tap_dr[t] = (int8_t)(t / 4);
+    p.tap_ds[t] = (int8_t)(t % 4);
+    p.tap_w[t] = (int8_t)t;
+  }
+  p.b_mode = LD_TILED_K;
+  p.b_lbo = 16;
+  p.b_sbo = 256;  // 8 rows of 32 bytes
+  p.b_kstep = 32;
+  p.idesc = idesc_f16(kBM, 64, false, false, false);
+  p.halo_ws = ws;
+  p.halo_h = (int)P;
+  p.halo_w = (int)Q;
+  p.halo_cb = 32;
+  p.halo_box_rows = rows + 3;
+  p.halo_row0 = 0;
+  p.halo_col0 = 0;
+  p.N = 64;
+  p.n_tiles = 1;
+  p.m_tiles = (int)(N * P * ws / kBM);
   int grid = p.m_tiles < sms ? p.m_tiles : sms;
   if (stats && grid > kBnStatSlots) grid = kBnStatSlots;
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
@@ -478,6 +558,8 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
   if (const int ws = halo_width(s, (flags & PF16_ACCUMULATE) != 0))
     return run_halo(s, ws, false, x, w, y, status, sms, st, stats);
+  if (const int ws_s2d = stem_s2d_width(s, (flags & PF16_ACCUMULATE) != 0))
+    return run_stem_s2d(s, ws_s2d, x, w, y, ws, status, sms, st, stats);
   set_stats(p, stats, s.K);
   const int BN = pick_bn_out(s.K);
   p.a_mode = LD_TILED_K;
@@ -644,8 +726,7 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, dy, dw)) != PF16_OK) return rc;
-  if (flags & ~PF16_REUSE_PATCHES) return PF16_ERR_ARG;
-  if ((flags & PF16_REUSE_PATCHES) && s.kind != KIND_STEM) return PF16_ERR_ARG;
+  if (flags) return PF16_ERR_ARG;
   int* status;
   int sms;
   if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
@@ -667,14 +748,13 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   p.a_mode = LD_TILED_MN;
   set_mnmajor(p, true, true);
   if (!map_2d(&ma, dy, s.K, pixels, s.K, 64, 64)) return PF16_ERR_CUDA;
-  // stem: [patch matrix, where pf16_conv_fwd puts it][partials]; other layers: [partials]
+  // stem: [patch matrix][partials]; other layers: [partials]
   uint16_t* parts = static_cast<uint16_t*>(ws);
   const bool partial = wsp.splits > 1 || s.kind == KIND_STEM;
   if (s.kind == KIND_STEM) {
     uint16_t* col = static_cast<uint16_t*>(ws);
     parts = col + round_up((size_t)(pixels * wsp.ncols * 2), 256) / 2;
-    if (!(flags & PF16_REUSE_PATCHES) &&
-        launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
+    if (launch_stem_im2col(x, col, (int)s.N, (int)s.H, (int)s.W, (int)s.P, (int)s.Q, (int)s.R,
                            (int)s.S, (int)s.C, (int)s.st, (int)s.pad, (int)wsp.ncols,
                            st) != cudaSuccess)
       return PF16_ERR_CUDA;

@@ -322,6 +322,86 @@ cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, i
   return counted_launches(1);
 }
 
+// ============================================================================
+// Stem space-to-depth (7x7 / stride 2 / pad 3 over 3 channels becomes a 4x4 /
+// stride 1 convolution over 16 channels):
+//   xs[n][I][J][(a*2 + b)*4 + c] = x[n][2I + a - 3][2J + b - 3][c]   (c < 3),
+//   0 for c = 3 and outside x;  I < Hs, J < Ws;
+//   wsd[k][(u*4 + v)*16 + (a*2 + b)*4 + c] = w[k][2u + a][2v + b][c],
+//   0 for c = 3 or where 2u + a or 2v + b reaches 7.
+// Blocks below N*Hs each write one row (n, I) of xs from the two input rows
+// 2I - 3, 2I - 2 staged in shared memory, one 32-byte pixel per thread (a
+// warp stores 1 KB contiguous); the blocks after them pack the filter.
+// ============================================================================
+__global__ void k_stem_s2d(const uint16_t* __restrict__ x, const uint16_t* __restrict__ w,
+                           uint16_t* __restrict__ xs, uint16_t* __restrict__ wsd, int N, int H, int W,
+                           int Hs, int Ws, int K) {
+  pdl_wait();
+  const long long rows_total = (long long)N * Hs;
+  if ((long long)blockIdx.x >= rows_total) {
+    const int e = (int)(blockIdx.x - rows_total) * blockDim.x + threadIdx.x;
+    if (e >= K * 256) return;
+    const int k = e >> 8, j = e & 255;
+    const int t = j >> 4, ch = j & 15;
+    const int r = 2 * (t >> 2) + (ch >> 3), sc = 2 * (t & 3) + ((ch >> 2) & 1), c = ch & 3;
+    wsd[e] = (c < 3 && r < 7 && sc < 7) ? w[((k * 7 + r) * 7 + sc) * 3 + c] : (uint16_t)0;
+    return;
+  }
+  extern __shared__ uint16_t srow[];  // [2][W * 3]
+  const int n = (int)(blockIdx.x / Hs), I = (int)(blockIdx.x - (long long)n * Hs);
+  const int len = W * 3;
+  for (int a = 0; a < 2; ++a) {
+    const int h = 2 * I + a - 3;
+    uint16_t* dst = srow + a * len;
+    if (h < 0 || h >= H) {
+      for (int e = threadIdx.x; e < len; e += blockDim.x) dst[e] = 0;
+      continue;
+    }
+    const uint16_t* src = x + ((long long)n * H + h) * len;
+    if (len % 8 == 0) {  // every input row then starts 16-byte aligned
+      for (int v = threadIdx.x; v < len / 8; v += blockDim.x) {
+        const uint4 u = __ldg(reinterpret_cast<const uint4*>(src) + v);
+        *reinterpret_cast<uint4*>(dst + v * 8) = u;
+      }
+    } else {
+      for (int e = threadIdx.x; e < len; e += blockDim.x) dst[e] = src[e];
+    }
+  }
+  __syncthreads();
+  uint4* out = reinterpret_cast<uint4*>(xs + ((long long)n * Hs + I) * Ws * 16);
+  for (int J = threadIdx.x; J < Ws; J += blockDim.x) {
+    uint32_t v[8];
+#pragma unroll
+    for (int a = 0; a < 2; ++a)
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const int col = 2 * J + b - 3;
+        uint32_t c0 = 0, c1 = 0, c2 = 0;
+        if (col >= 0 && col < W) {
+          const uint16_t* q = srow + a * len + col * 3;
+          c0 = q[0];
+          c1 = q[1];
+          c2 = q[2];
+        }
+        v[(a * 2 + b) * 2] = c0 | (c1 << 16);
+        v[(a * 2 + b) * 2 + 1] = c2;
+      }
+    out[(long long)J * 2] = make_uint4(v[0], v[1], v[2], v[3]);
+    out[(long long)J * 2 + 1] = make_uint4(v[4], v[5], v[6], v[7]);
+  }
+}
+
+cudaError_t launch_stem_s2d(const uint16_t* x, const uint16_t* w, uint16_t* xs, uint16_t* wsd, int N, int H,
+                            int W, int Hs, int Ws, int K, cudaStream_t s) {
+  const size_t shm = (size_t)2 * W * 3 * sizeof(uint16_t);
+  if (shm > 48 * 1024) return cudaErrorInvalidValue;
+  const int threads = 128;
+  const long long blocks = (long long)N * Hs + (K * 256 + threads - 1) / threads;
+  if (blocks > 0x7fffffffll) return cudaErrorInvalidValue;
+  launch_pdl(k_stem_s2d, dim3((unsigned)blocks), dim3(threads), shm, s, x, w, xs, wsd, N, H, W, Hs, Ws, K);
+  return counted_launches(1);
+}
+
 __global__ void k_pad_rows(const uint16_t* __restrict__ w, uint16_t* __restrict__ wp, int K, int kin,
                            int kcol) {
   pdl_wait();

@@ -467,6 +467,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
+      // base descriptors (address field 0) and K-step strides in 16-byte units:
+      // a step's descriptor is one add away
+      const uint64_t adesc0 = smem_desc(0, p.a_lbo, p.a_sbo, 2);
+      const uint64_t bdesc0 = smem_desc(0, p.b_lbo, p.b_sbo, 2);
+      const uint32_t ak16 = (uint32_t)p.a_kstep >> 4, bk16 = (uint32_t)p.b_kstep >> 4;
       for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
         int m0, n0, split, kb0, kb1;
         unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
@@ -484,14 +489,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
-          const uint32_t sb = sa + Cfg::A_BYTES;
+          const uint32_t sa16 = smem_u32(smem + stage * Cfg::STAGE_BYTES) >> 4;
+          const uint64_t ab = adesc0 + sa16, bb = bdesc0 + sa16 + (Cfg::A_BYTES >> 4);
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = smem_desc(sa + kk * p.a_kstep, p.a_lbo, p.a_sbo, 2);
-            const uint64_t bd = smem_desc(sb + kk * p.b_kstep, p.b_lbo, p.b_sbo, 2);
-            tc_mma_f16(d_tmem, ad, bd, p.idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
-          }
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            tc_mma_f16(d_tmem, ab + kk * ak16, bb + kk * bk16, p.idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
           tc_commit(smem_u32(&empty[stage]));
           if (++stage == Cfg::STAGES) {
             stage = 0;
@@ -663,27 +665,33 @@ cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, co
 
 
 // ---------------------------------------------------------------------------
-// Halo engine: 3x3 / stride 1 / pad 1 convolution (forward, or data gradient
-// as a convolution of dy with the flipped filter), 64 input channels, 64
-// outputs.  GEMM rows are the pixels of a padded grid whose image rows are ws
-// >= W + 2 columns wide (ws = 64 or 32), so a 128-row tile is 128/ws whole
-// image rows.  One TMA box brings the tile's input rows i0-1 .. i0+128/ws,
-// columns -1 .. ws-2 (zeros outside the image), 128-byte swizzled, one pixel
-// per 128-byte row; tap (dr, ds) is then the 128-row window that starts
-// dr*ws + ds pixels into the box.  The swizzle is a function of the absolute
-// shared-memory address, so a descriptor whose start moves by whole 128-byte
-// rows reads exactly that window (checked on the GPU: rows m + o for offsets
-// o = 1, 2, 3, 8, 9 with base offset 0).  The input is thus read once per
-// tile instead of once per tap.  The nine 64 x 64 weight slices stay in shared
-// memory for the whole launch.  Columns j >= W of the padded grid are
-// computed and then dropped by the 3-D TMA store, which clips at W.
+// Halo engine: stride-1 convolution with 64 outputs read from a padded pixel
+// grid.  GEMM rows are the pixels of a grid whose image rows are ws columns
+// wide (ws = 32, 64 or 128, at least the output width plus the filter width
+// minus one), so a 128-row tile is 128/ws whole output rows.  One TMA box
+// brings the input rows and columns the tile's taps touch (zeros outside the
+// image), one pixel per swizzled row of cb bytes; tap (dr, ds) is then the
+// 128-row window that starts dr*ws + ds pixels into the box.  The swizzle is
+// a function of the absolute shared-memory address, so a descriptor whose
+// start moves by whole rows reads exactly that window (checked on the GPU for
+// 128-byte rows: rows m + o for offsets o = 1, 2, 3, 8, 9 with base offset 0).
+// The input is thus read once per tile instead of once per tap, and the taps'
+// weight slices stay in shared memory for the whole launch.  Two uses:
+//   - 3x3 / stride 1 / pad 1, 64 -> 64 channels (forward, or the data
+//     gradient as a convolution of dy with the flipped filter): cb = 128,
+//     128-byte swizzle, box rows i0-1 .. i0+128/ws, columns -1 .. ws-2;
+//   - the 7x7 / stride 2 / pad 3 stem after a 2x2 space-to-depth of its
+//     three-channel input: a 4x4 / stride 1 / unpadded convolution over 16
+//     channels (12 real), cb = 32, 32-byte swizzle, one K = 16 MMA per tap.
+// Columns j >= Q of the padded grid are computed and then dropped by the 3-D
+// TMA store, which clips at Q.
 // Same roles and bounded waits as k_gemm.
 // ---------------------------------------------------------------------------
 struct HaloCfg {
-  static constexpr int B_TILE = 64 * kBK * 2;       // one tap's 64 x 64 weights
-  static constexpr int B_BYTES = 9 * B_TILE;        // resident
-  static constexpr int A_BOX_MAX = 64 * 4 * 128;    // ws = 64: 4 rows of 64 pixels (ws = 32: 6 x 32)
-  static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's 2-pixel over-read
+  static constexpr int B_BYTES = 9 * 64 * kBK * 2;  // resident: 9 taps x 64 x 64, or 16 x 64 x 16
+  static constexpr int A_BOX_MAX = 64 * 4 * 128;    // ws = 64: 4 rows of 64 pixels (ws = 32: 6 x 32;
+                                                    // the stem: 4 rows of 128 pixels x 32 bytes)
+  static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's over-read
   static constexpr int STAGES = 3;
   static constexpr int TMEM_COLS = 128;
   static constexpr int STAGING_BYTES = kEpiWarps * 4096;  // one 32 x 64 tile per epilogue warp
@@ -691,14 +699,25 @@ struct HaloCfg {
   static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + BAR_BYTES;
 };
 
+// CB = bytes of one input pixel: 128 (3x3, nine taps of four K = 16 steps,
+// 128-byte swizzle) or 32 (the space-to-depth stem, sixteen taps of one step,
+// 32-byte swizzle).  The MMA issue loop is unrolled over taps and steps with
+// descriptors formed by adding 16-byte offsets to two base descriptors (the
+// start-address field is the low 14 bits, and shared-memory addresses stay
+// below 256 KB), so a single thread keeps up with N = 64 MMAs.
+template <int CB>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_halo(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                 const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
   using Cfg = HaloCfg;
+  constexpr int NTAPS = CB == 128 ? 9 : 16;
+  constexpr int KSTEPS = CB / 32;                 // K = 16 steps per tap
+  constexpr uint32_t SWZ = CB == 128 ? 2u : 6u;   // descriptor swizzle code
+  constexpr int B_TILE = 64 * CB;                 // one tap's 64-row weight slice
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* bres = smem;                                   // 9 weight slices
+  uint8_t* bres = smem;                                   // the taps' weight slices
   uint8_t* astages = smem + Cfg::B_BYTES;                 // 1024-aligned stages
   uint8_t* staging = astages + Cfg::STAGES * Cfg::A_STAGE;
   uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
@@ -711,7 +730,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int ws = p.halo_ws, rows = kBM / ws;
-  const uint32_t box_bytes = (uint32_t)((rows + 2) * ws * 128);
+  const uint32_t box_bytes = (uint32_t)(p.halo_box_rows * ws * CB);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < Cfg::STAGES; ++s) {
@@ -744,13 +763,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      // resident weights: the 64 x 64 slice of each of the nine taps
+      // resident weights: the 64-row slice of each tap
       const uint32_t bb = smem_u32(bready);
-      mbar_arrive_expect_tx(bb, Cfg::B_BYTES);
-      for (int t = 0; t < 9; ++t) {
-        const uint32_t dst = smem_u32(bres + t * Cfg::B_TILE);
+      mbar_arrive_expect_tx(bb, (uint32_t)(NTAPS * B_TILE));
+      for (int t = 0; t < NTAPS; ++t) {
+        const uint32_t dst = smem_u32(bres + t * B_TILE);
         if (p.b_mode == LD_TILED_K)
-          tma_load_2d(dst, &mapB, bb, p.tap_w[t] * kBK, 0);
+          tma_load_2d(dst, &mapB, bb, p.tap_w[t] * (CB / 2), 0);
         else
           tma_load_3d(dst, &mapB, bb, 0, p.tap_w[t], 0);
       }
@@ -765,7 +784,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         const uint32_t fb = smem_u32(&full[stage]);
         mbar_arrive_expect_tx(fb, box_bytes);
-        tma_load_4d(smem_u32(astages + stage * Cfg::A_STAGE), &mapA, fb, 0, -1, i0 - 1, n);
+        tma_load_4d(smem_u32(astages + stage * Cfg::A_STAGE), &mapA, fb, 0, p.halo_col0, i0 + p.halo_row0, n);
         ++issued;
         if (++stage == Cfg::STAGES) {
           stage = 0;
@@ -796,7 +815,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      const uint32_t sb0 = smem_u32(bres);
+      // tap windows in 16-byte units, and the two base descriptors
+      uint32_t toff[NTAPS];
+#pragma unroll
+      for (int t = 0; t < NTAPS; ++t) toff[t] = (uint32_t)((p.tap_dr[t] * ws + p.tap_ds[t]) * CB) >> 4;
+      const uint64_t adesc0 = smem_desc(0, 16, 8 * CB, SWZ);
+      const uint64_t bdesc0 = smem_desc(smem_u32(bres), p.b_lbo, p.b_sbo, SWZ);
+      const uint32_t bk16 = (uint32_t)p.b_kstep >> 4;
       for (int u = blockIdx.x; ok && u < total && !*abort_flag; u += gridDim.x) {
         if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim) ||
             !mbar_wait(smem_u32(&full[stage]), phase, lim)) {
@@ -805,18 +830,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 64);
-        const uint32_t sa = smem_u32(astages + stage * Cfg::A_STAGE);
-#pragma unroll 1
-        for (int t = 0; t < 9; ++t) {
-          const uint32_t at = sa + (uint32_t)((p.tap_dr[t] * ws + p.tap_ds[t]) * 128);
-          const uint32_t bt = sb0 + (uint32_t)(t * Cfg::B_TILE);
+        const uint64_t abase = adesc0 + (smem_u32(astages + stage * Cfg::A_STAGE) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
-            const uint64_t ad = smem_desc(at + kk * 32, 16, 1024, 2);
-            const uint64_t bd = smem_desc(bt + kk * p.b_kstep, p.b_lbo, p.b_sbo, 2);
-            tc_mma_f16(d_tmem, ad, bd, p.idesc, (t > 0 || kk > 0) ? 1u : 0u);
-          }
-        }
+        for (int t = 0; t < NTAPS; ++t)
+#pragma unroll
+          for (int kk = 0; kk < KSTEPS; ++kk)
+            tc_mma_f16(d_tmem, abase + toff[t] + kk * 2, bdesc0 + (uint32_t)(t * (B_TILE >> 4)) + kk * bk16,
+                       p.idesc, (t > 0 || kk > 0) ? 1u : 0u);
         tc_commit(smem_u32(&empty[stage]));
         if (++stage == Cfg::STAGES) {
           stage = 0;
@@ -828,8 +848,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
   } else {
-    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1; 32 rows each, which
-    // lie in one image row of the padded grid (ws is a multiple of 32)
+    // epilogue warps 2..9: group (w - 2) / 4 drains accumulator 0 or 1 (the
+    // CTA's even or odd tiles), warp w its TMEM sub-partition w % 4; 32 rows
+    // each, which lie in one image row of the padded grid (ws is a multiple of 32)
     const int e = warp - 2, grp = e >> 2, sub = warp & 3;
     const int acc = grp;
     uint32_t acc_phase = 0;
@@ -869,9 +890,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       __syncwarp();
       if (lane == 0) {
         const int mp = u * kBM + sub * 32;  // first padded-grid row of the warp
-        const int grow = mp / ws;
-        tma_store_3d(&mapC, stg, 0, mp - grow * ws, grow);
-        bulk_commit();
+        const int grow = mp / ws, col = mp - grow * ws;
+        if (col < p.halo_w) {  // a box wholly right of the image has nothing to store
+          tma_store_3d(&mapC, stg, 0, col, grow);
+          bulk_commit();
+        }
       }
       if (p.st_mean) {
         const int mp = u * kBM + sub * 32;
@@ -899,16 +922,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
 cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                              const GemmParams& p, int grid, cudaStream_t s) {
-  static bool attr_set[64] = {false};
+  // the resident weights, the A box and its furthest tap window must fit their buffers
+  const int max_off = [&] {
+    int m = 0;
+    for (int t = 0; t < p.ntaps; ++t) m = max(m, (p.tap_dr[t] * p.halo_ws + p.tap_ds[t]) * p.halo_cb);
+    return m;
+  }();
+  if (p.ntaps != (p.halo_cb == 128 ? 9 : 16) || (p.halo_cb != 128 && p.halo_cb != 32) || p.halo_ws <= 0 ||
+      kBM % p.halo_ws != 0 || p.ntaps * 64 * p.halo_cb > HaloCfg::B_BYTES ||
+      p.halo_box_rows * p.halo_ws * p.halo_cb > HaloCfg::A_BOX_MAX ||
+      max_off + kBM * p.halo_cb > HaloCfg::A_STAGE)
+    return cudaErrorInvalidValue;
+  static bool attr_set[2][64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_halo, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         HaloCfg::SMEM);
+  const int v = p.halo_cb == 128 ? 0 : 1;
+  if (dev < 64 && !attr_set[v][dev]) {
+    cudaError_t e = cudaFuncSetAttribute(v == 0 ? k_gemm_halo<128> : k_gemm_halo<32>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, HaloCfg::SMEM);
     if (e != cudaSuccess) return e;
-    attr_set[dev] = true;
+    attr_set[v][dev] = true;
   }
-  launch_pdl(k_gemm_halo, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
+  if (v == 0)
+    launch_pdl(k_gemm_halo<128>, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
+  else
+    launch_pdl(k_gemm_halo<32>, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
   return counted_launches(1);
 }
 

@@ -108,8 +108,11 @@ struct GemmParams {
   uint32_t b_lbo, b_sbo, b_kstep;
   int* status;            // device status word
   unsigned long long wait_limit_ns;
-  // halo mode (launch_gemm_halo): padded row width, image height and width
-  int halo_ws, halo_h, halo_w;
+  // halo mode (launch_gemm_halo): padded row width, output height and width,
+  // bytes per pixel of the input (128: 64 channels, nine taps; 32: 16
+  // channels, sixteen taps), rows of the A box, its start row / column
+  // relative to the tile's first output row / column 0
+  int halo_ws, halo_h, halo_w, halo_cb, halo_box_rows, halo_row0, halo_col0;
   // BatchNorm forward statistics of the output (OUT_STORE through TMA only;
   // null when off): per epilogue warp a running (mean, variance, count) per
   // output channel over all its rows; the CTA's warps are merged at the end
@@ -139,13 +142,14 @@ cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB
                         cudaStream_t stream);
 int gemm_smem_bytes(int BN);
 
-// Halo engine for 3x3 / stride 1 / pad 1 convolutions with 64 input and 64
-// output channels: A = one 4-D TMA box (64 channels x halo_ws columns x
-// 128/halo_ws + 2 rows) per 128-row tile of the padded pixel grid, taps as
-// row-shifted descriptor windows, the nine 64 x 64 B slices resident; the
-// output leaves through a 3-D map (64, W, N*H) clipped at W.  p.tap_dr/tap_ds
-// are the window offsets (0..2), p.tap_w the weight tap of each of the 9 taps,
-// p.b_mode LD_TILED_K (weights [K][9*64]) or LD_TAP3D_MN (weights (C, 9, K)).
+// Halo engine for stride-1 convolutions with 64 outputs whose input pixel is
+// 128 bytes (64 channels, 3x3 taps) or 32 bytes (16 channels, the stem after
+// space-to-depth, 4x4 taps): A = one 4-D TMA box (channels x halo_ws columns
+// x halo_box_rows rows) per 128-row tile of the padded pixel grid, taps as
+// row-shifted descriptor windows, the taps' 64-row B slices resident; the
+// output leaves through a 3-D map (64, Q, N*P) clipped at Q.  p.ntaps taps,
+// p.tap_dr/tap_ds their window offsets, p.tap_w their weight tap; p.b_mode
+// LD_TILED_K (weights [64][taps*C]) or LD_TAP3D_MN (weights (C, 9, K)).
 cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
                              const GemmParams& p, int grid, cudaStream_t stream);
 
@@ -163,6 +167,10 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
 cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, int W, int P,
                                int Q, int R, int S, int C, int stride, int pad, int kcol,
                                cudaStream_t s);
+// stem space-to-depth: xs = N x Hs x Ws x 16 and the 64 x 256 packed filter wsd
+// of the 4x4 stride-1 form of the 7x7 / stride 2 / pad 3 convolution
+cudaError_t launch_stem_s2d(const uint16_t* x, const uint16_t* w, uint16_t* xs, uint16_t* wsd, int N, int H,
+                            int W, int Hs, int Ws, int K, cudaStream_t s);
 // w[K][kin] -> wpad[K][kcol] (zero padded)
 cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wpad, int K, int kin, int kcol,
                             cudaStream_t s);

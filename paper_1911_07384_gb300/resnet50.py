@@ -107,21 +107,16 @@ class Conv:
     def fwd(self, x, y, with_stats=False):
         if with_stats:
             self.net.call("conv_fwd", self, pf16.conv_fwd_bnstats, self.desc, x, self.w, y, self.stats,
-                          self.ws())
+                          self.net.ws)
         else:
-            self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.ws())
+            self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.net.ws)
 
     def dgrad(self, dy, dx, accumulate=False):
         self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
                       pf16.PF16_ACCUMULATE if accumulate else 0)
 
-    def ws(self):
-        return self.net.stem_ws if self.desc.c == 3 else self.net.ws
-
     def wgrad(self, x, dy):
-        # the stem's patch matrix, gathered by its forward into its own workspace, is still there
-        flags = pf16.PF16_REUSE_PATCHES if self.desc.c == 3 else 0
-        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.ws(), flags)
+        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.net.ws)
 
 
 class BN:
@@ -281,16 +276,10 @@ class ResNet50:
         self.dlogits = e(N, self.classes)
         self.df = e(N, self.cl)
         self.loss = e(1)
-        ws, stem_ws = 0, 0
+        ws = 0
         for c in self.convs:
-            need = max(pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_FWD),
-                       pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD))
-            if c.desc.c == 3:
-                stem_ws = max(stem_ws, need)
-            else:
-                ws = max(ws, need)
-        # the stem keeps its patch matrix from the forward to the weight gradient
-        self.stem_ws = torch.empty(stem_ws, dtype=torch.uint8, device=dev)
+            ws = max(ws, pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_FWD),
+                     pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD))
         for b in self.bns:
             ws = max(ws, pf16.bn_workspace_size(b.desc))
         ws = max(ws, pf16.softmax_xent_workspace_size(N, self.classes))

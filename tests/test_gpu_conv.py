@@ -25,7 +25,12 @@ SHAPES = [
     (2, 14, 14, 64, 256, 1, 1, 1, 0),
     (2, 13, 13, 128, 256, 1, 1, 2, 0),   # strided 1x1 projection, odd size
     (3, 10, 10, 192, 320, 3, 3, 1, 1),   # 3 channel chunks, partial N tile
-    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem (c = 3)
+    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem, space-to-depth halo (rows of 32)
+    (3, 30, 30, 3, 64, 7, 7, 2, 3),      # stem, s2d halo, odd P = 15 (rows of 128)
+    (2, 100, 98, 3, 64, 7, 7, 2, 3),     # stem, s2d halo (rows of 64), H != W
+    (2, 31, 29, 3, 64, 7, 7, 2, 3),      # stem, odd H and W
+    (2, 20, 20, 3, 128, 7, 7, 2, 3),     # stem with 128 outputs: patch GEMM
+    (2, 16, 16, 3, 64, 3, 3, 1, 1),      # c = 3, 3x3: patch GEMM
     (16, 1, 1, 2048, 1000, 1, 1, 1, 0),  # fully connected layer
 ]
 
@@ -99,30 +104,21 @@ def test_conv_wgrad(orc, shape):
     assert rel < 2.0 ** -6, rel
 
 
-def test_stem_wgrad_reuses_forward_patches():
-    """PF16_REUSE_PATCHES: the stem's weight gradient on the patch matrix its
-    forward left in a shared workspace equals the one that gathers again."""
-    shape = (3, 30, 30, 3, 64, 7, 7, 2, 3)
-    x, w, dy, P, Q = inputs(shape, seed_cfg=2)
+def test_stem_full_width_sampled(orc):
+    """The batch-256 stem's row width (224 -> 112 outputs, padded rows of 128)
+    on one image: every output against the oracle."""
+    shape = (1, 224, 224, 3, 64, 7, 7, 2, 3)
+    x, w, dy, P, Q = inputs(shape, seed_cfg=4)
     d = pf16.conv_desc(*shape)
-    ws = workspace(max(pf16.conv_workspace_size(d, pf16.PF16_PASS_FWD),
-                       pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)))
-    tx = dev(x)
-    pf16.conv_fwd(d, tx, dev(w), empty16(d.n * P * Q * d.k), ws)
-    dw = empty16(d.k * d.r * d.s * d.c)
-    pf16.conv_wgrad(d, tx, dev(dy), dw, ws, pf16.PF16_REUSE_PATCHES)
-    assert pf16.sync_status() == 0
-    assert np.array_equal(host(dw), run_wgrad(d, x, dy))
-    # the flag is only for the stem
-    d2 = pf16.conv_desc(2, 14, 14, 64, 64, 1, 1, 1, 0)
-    with pytest.raises(pf16.PF16Error):
-        pf16.conv_wgrad(d2, empty16(2 * 14 * 14 * 64), empty16(2 * 14 * 14 * 64), empty16(64 * 64),
-                        workspace(pf16.conv_workspace_size(d2, pf16.PF16_PASS_WGRAD)),
-                        pf16.PF16_REUSE_PATCHES)
+    y = run_fwd(d, x, w)
+    V, A, _ = orc.conv_fwd(x, w, *shape)
+    rel = assert_conv_close(y, V, A, 147, "fwd")
+    assert rel < 2.0 ** -7, rel
 
 
 @pytest.mark.parametrize("shape", [(2, 9, 9, 64, 128, 3, 3, 1, 1), (2, 10, 10, 64, 64, 1, 1, 2, 0),
-                                   (2, 11, 11, 64, 64, 3, 3, 2, 1), (2, 12, 10, 64, 64, 3, 3, 1, 1)],
+                                   (2, 11, 11, 64, 64, 3, 3, 2, 1), (2, 12, 10, 64, 64, 3, 3, 1, 1),
+                                   (2, 32, 32, 3, 64, 7, 7, 2, 3)],
                          ids=ids)
 def test_accumulate_flag(orc, shape):
     N, H, W, C, K, R, S, st, pd = shape
@@ -132,6 +128,8 @@ def test_accumulate_flag(orc, shape):
     y = run_fwd(d, x, w, pf16.PF16_ACCUMULATE, y0)
     V, A, _ = orc.conv_fwd(x, w, *shape)
     assert_conv_close(y, V, A, C * R * S, "fwd+acc", prev=y0)
+    if C == 3:
+        return  # the stem has no data gradient
     dx0 = syn.normal_f16(78, (N * H * W * C,))
     dx = run_dgrad(d, dy, w, pf16.PF16_ACCUMULATE, dx0)
     V, A, T = orc.conv_dgrad(dy, w, *shape)

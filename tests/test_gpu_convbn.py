@@ -29,7 +29,9 @@ SHAPES = [
     (2, 13, 13, 128, 256, 3, 3, 2, 1),   # strided 3x3, 4 n-chunks in a tile
     (2, 7, 7, 256, 512, 1, 1, 1, 0),     # two n-tiles (BN = 256)
     (3, 7, 7, 512, 1024, 1, 1, 1, 0),    # four n-tiles
-    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem (patch matrix)
+    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem, space-to-depth halo (rows of 32)
+    (1, 30, 30, 3, 64, 7, 7, 2, 3),      # stem, s2d halo (rows of 128, columns 15..127 dropped)
+    (2, 20, 20, 3, 128, 7, 7, 2, 3),     # stem with 128 outputs (patch matrix)
 ]
 
 
