@@ -610,7 +610,7 @@ def count_launches(net):
             phases = d.stride * d.stride if d.r > 1 else 1
             total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
-        total += 1 + (1 if ws else 0) + (1 if stem else 0)  # wgrad (+ split-K reduce, + the stem's patch gather)
+        total += 1 + (1 if ws else 0) + (2 if stem else 0)  # wgrad (+ split-K reduce, + the stem's s2d, scatter)
     total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)  # forward statistics come from the conv
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]

@@ -265,6 +265,28 @@ int stem_s2d_width(const Shape& s, bool accum) {
 }
 size_t stem_s2d_bytes(const Shape& s) { return round_up((size_t)(s.N * (s.P + 3) * (s.Q + 3) * 32), 256); }
 
+// Stem weight gradient on the space-to-depth input (k_stem_wgrad): work units
+// are the N * (P + 1) output rows (padded to 128 columns), accumulated in FP16
+// over chunks of 32 rows (4,096 padded pixels) -- more only beyond 1,024
+// chunks -- then summed by the split-K tree.  Workspace: xs, the chunks'
+// 128 x 128 partials, the reduced 128 x 128 matrix.
+struct StemWgradPlan {
+  bool ok;
+  long long rows;
+  int per_chunk, chunks;
+};
+StemWgradPlan stem_wgrad_plan(const Shape& s) {
+  StemWgradPlan w{false, 0, 0, 0};
+  if (!stem_s2d_width(s, false)) return w;
+  w.rows = s.N * (s.P + 1);
+  w.per_chunk = 32;
+  if (cdiv(w.rows, w.per_chunk) > 1024) w.per_chunk = (int)cdiv(w.rows, 1024);
+  w.chunks = (int)cdiv(w.rows, w.per_chunk);
+  w.ok = w.rows < (1ll << 30);
+  return w;
+}
+size_t stem_wgrad_parts_bytes(const StemWgradPlan& w) { return round_up((size_t)w.chunks * 128 * 128 * 2, 256); }
+
 size_t ws_fwd(const Shape& s) {
   if (s.kind != KIND_STEM) return 0;
   const long long kc = stem_kcol(s);
@@ -274,6 +296,8 @@ size_t ws_fwd(const Shape& s) {
   return std::max(patch, stem_s2d_bytes(s) + (size_t)(s.K * 256 * 2));
 }
 size_t ws_wgrad(const Shape& s) {
+  const StemWgradPlan sw = stem_wgrad_plan(s);
+  if (sw.ok) return stem_s2d_bytes(s) + stem_wgrad_parts_bytes(sw) + 128 * 128 * 2;
   const WgradSplit w = wgrad_split(s);
   size_t b = 0;
   if (w.splits > 1 || s.kind == KIND_STEM) b += round_up((size_t)w.splits * s.K * w.ncols * 2, 256);
@@ -720,6 +744,52 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
   return PF16_OK;
 }
 
+// The stem's weight gradient through k_stem_wgrad (layouts at stem_wgrad_plan).
+static int run_stem_wgrad(const Shape& s, const StemWgradPlan& sw, const uint16_t* x, const uint16_t* dy,
+                          uint16_t* dw, void* work, int* status, int sms, cudaStream_t st) {
+  const long long N = s.N, P = s.P, Q = s.Q, Hs = P + 3, Wsd = Q + 3;
+  uint16_t* xs = static_cast<uint16_t*>(work);
+  uint16_t* parts = xs + stem_s2d_bytes(s) / 2;
+  uint16_t* dws = parts + stem_wgrad_parts_bytes(sw) / 2;
+  if (launch_stem_s2d(x, nullptr, xs, nullptr, (int)N, (int)s.H, (int)s.W, (int)Hs, (int)Wsd, 0, st) !=
+      cudaSuccess)
+    return PF16_ERR_CUDA;
+  CUtensorMap mdy, mxs;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  {
+    cuuint64_t dims[4] = {64, (cuuint64_t)Q, (cuuint64_t)P, (cuuint64_t)N};
+    cuuint64_t strides[3] = {128, (cuuint64_t)(Q * 128), (cuuint64_t)(P * Q * 128)};
+    cuuint32_t box[4] = {64, 128, 2, 1};
+    if (g_encode_tiled(&mdy, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<uint16_t*>(dy), dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  {
+    cuuint64_t dims[4] = {16, (cuuint64_t)Wsd, (cuuint64_t)Hs, (cuuint64_t)N};
+    cuuint64_t strides[3] = {32, (cuuint64_t)(Wsd * 32), (cuuint64_t)(Hs * Wsd * 32)};
+    cuuint32_t box[4] = {16, 128, 4, 1};
+    if (g_encode_tiled(&mxs, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, xs, dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  GemmParams p = base_params(status);
+  p.idesc = idesc_f16(kBM, 64, true, true, false);
+  p.halo_ws = 128;
+  p.halo_h = (int)P;
+  p.halo_w = (int)Q;
+  p.num_kb = (int)sw.rows;
+  p.kb_per_split = sw.per_chunk;
+  p.m_tiles = sw.chunks;
+  p.out = parts;
+  const int grid = sw.chunks < sms ? sw.chunks : sms;
+  if (launch_stem_wgrad(mdy, mxs, p, grid, st) != cudaSuccess) return PF16_ERR_CUDA;
+  if (launch_splitk_reduce(parts, sw.chunks, 128, 128, dws, 128, 128, st) != cudaSuccess) return PF16_ERR_CUDA;
+  if (launch_stem_wgrad_scatter(dws, dw, (int)s.K, st) != cudaSuccess) return PF16_ERR_CUDA;
+  return PF16_OK;
+}
+
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
   Shape s;
@@ -735,6 +805,8 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   if (need && !aligned16(ws)) return PF16_ERR_ALIGN;
   if (!driver_fns()) return PF16_ERR_CUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const StemWgradPlan sw = stem_wgrad_plan(s);
+  if (sw.ok) return run_stem_wgrad(s, sw, x, dy, dw, ws, status, sms, st);
   const WgradSplit wsp = wgrad_split(s);
 
   GemmParams p = base_params(status);

@@ -402,6 +402,27 @@ cudaError_t launch_stem_s2d(const uint16_t* x, const uint16_t* w, uint16_t* xs, 
   return counted_launches(1);
 }
 
+// dws[row][col], row = 64 (tap row even) or 0 (odd) + k, col = (tap row / 2) * 64
+// + (tap column) * 16 + (a*2 + b)*4 + c, for r = 2 * tap row + a, s = 2 * tap
+// column + b (the stem weight gradient's layout) -> dw[k][r][s][c], 7 x 7 x 3
+__global__ void k_stem_wgrad_scatter(const uint16_t* __restrict__ dws, uint16_t* __restrict__ dw, int K) {
+  pdl_wait();
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= K * 147) return;
+  const int k = e / 147, rsc = e - k * 147;
+  const int r = rsc / 21, sc = rsc - r * 21, sx = sc / 3, c = sc - sx * 3;
+  const int tr = r >> 1, tc = sx >> 1;
+  const int row = ((tr & 1) ? 0 : 64) + k;
+  const int col = (tr >> 1) * 64 + tc * 16 + ((r & 1) * 2 + (sx & 1)) * 4 + c;
+  dw[e] = dws[row * 128 + col];
+}
+
+cudaError_t launch_stem_wgrad_scatter(const uint16_t* dws, uint16_t* dw, int K, cudaStream_t s) {
+  if (K != 64) return cudaErrorInvalidValue;
+  launch_pdl(k_stem_wgrad_scatter, dim3((K * 147 + 255) / 256), dim3(256), 0, s, dws, dw, K);
+  return counted_launches(1);
+}
+
 __global__ void k_pad_rows(const uint16_t* __restrict__ w, uint16_t* __restrict__ wp, int K, int kin,
                            int kcol) {
   pdl_wait();

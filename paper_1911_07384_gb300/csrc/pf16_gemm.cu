@@ -950,4 +950,229 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const
   return counted_launches(1);
 }
 
+// ---------------------------------------------------------------------------
+// Stem weight gradient on the space-to-depth input (the stem forward's xs:
+// N x Hs x Ws x 16, Hs = P + 3).  With dy on a padded grid of ws = 128
+// columns per output row (columns >= Q zero), tap (u, v) of the 4x4 form is
+//   dW'[k][u][v][ch] = sum_p dy[p][k] * xs[p + u*ws + v][ch],
+// p over the padded pixels of every output row.  One MMA (M = 128, N = 64,
+// K = 16 pixels, both operands MN-major) yields two tap rows at once:
+//   A = the 64 channels of dy at pixels p - ws (M rows 0..63) and p (rows
+//       64..127): two 128-byte-swizzled M atoms one padded row apart (LBO);
+//   B = xs at p + u*ws + v for v = 0..3: four 16-channel N atoms one pixel
+//       (32 bytes, LBO) apart, 32-byte swizzle.
+// Rows 64..127 then accumulate tap (u, v) over output row i, rows 0..63 tap
+// (u + 1, v) over output row i - 1; u = 0 and u = 2 cover all sixteen taps
+// when i runs over 0..P (dy rows -1 and P read as zeros).  A work unit is
+// one (image, i) row: a stage holds dy rows i - 1, i (2 x 128 x 128 B) and
+// xs rows i .. i + 3 (4 x 128 x 32 B; windows reach at most 3 pixels into
+// row i + 3, and only at padding columns, where dy is zero).  Units are
+// accumulated in FP16 in TMEM over chunks of p.kb_per_split rows (4,096
+// padded pixels at ws = 128), and each chunk's 128 x 128 FP16 partial
+// [(a, k)][(u/2, v, ch)] goes to p.out + chunk * 128 * 128 for the split-K
+// tree.  Same roles and bounded waits as k_gemm_halo.
+// ---------------------------------------------------------------------------
+struct StemWgradCfg {
+  static constexpr int WS = 128;
+  static constexpr int DY_BYTES = 2 * WS * 128;   // dy rows i - 1, i
+  static constexpr int XS_BYTES = 4 * WS * 32;    // xs rows i .. i + 3
+  static constexpr int STAGE = DY_BYTES + XS_BYTES;
+  static constexpr int STAGES = 4;
+  static constexpr int TMEM_COLS = 256;           // two 128-column accumulators
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
+  static constexpr int SMEM = 1024 + STAGES * STAGE + BAR_BYTES;
+};
+constexpr int kStemWgradThreads = 192;
+
+__global__ void __launch_bounds__(kStemWgradThreads, 1)
+    k_stem_wgrad(const __grid_constant__ CUtensorMap mapDy, const __grid_constant__ CUtensorMap mapXs,
+                 const __grid_constant__ GemmParams p) {
+  using Cfg = StemWgradCfg;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + Cfg::STAGES;
+  uint64_t* tfull = bars + 2 * Cfg::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < Cfg::STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&mapDy);
+    tma_prefetch_desc(&mapXs);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  pdl_wait();
+  const uint32_t tmem_base = *tmem_slot;
+  const int rows_total = p.num_kb;      // (P + 1) * N row units
+  const int per_chunk = p.kb_per_split; // row units per accumulator
+  const int chunks = p.m_tiles;
+  const int rows_img = p.halo_h + 1;    // i = 0 .. P
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, issued = 0;
+      for (int c = blockIdx.x; c < chunks && !*abort_flag; c += gridDim.x) {
+        const int g1 = min(rows_total, (c + 1) * per_chunk);
+        for (int g = c * per_chunk; g < g1 && !*abort_flag; ++g) {
+          const int n = g / rows_img, i = g - n * rows_img;
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim)) {
+            record_timeout(p, abort_flag);
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[stage]);
+          const uint32_t dst = smem_u32(smem + stage * Cfg::STAGE);
+          mbar_arrive_expect_tx(fb, (uint32_t)Cfg::STAGE);
+          tma_load_4d(dst, &mapDy, fb, 0, 0, i - 1, n);
+          tma_load_4d(dst + Cfg::DY_BYTES, &mapXs, fb, 0, 0, i, n);
+          ++issued;
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (*abort_flag) {  // let every copy this thread started land before the CTA can exit
+        const uint32_t nn = issued < (uint32_t)Cfg::STAGES ? issued : (uint32_t)Cfg::STAGES;
+        int s = stage;
+        uint32_t ph = phase;
+        for (uint32_t q = 0; q < nn; ++q) {
+          if (--s < 0) {
+            s = Cfg::STAGES - 1;
+            ph ^= 1;
+          }
+          mbar_wait(smem_u32(&full[s]), ph, 1000000000ull);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // A: dy, MN-major 128-byte swizzle, M atoms one padded row (ws * 128 B)
+      // apart, 8-pixel K groups 1 KB apart; B: xs, MN-major 32-byte swizzle,
+      // N atoms one pixel (32 B) apart, 8-pixel K groups 256 B apart
+      const uint64_t adesc0 = smem_desc(0, Cfg::WS * 128, 1024, 2);
+      const uint64_t bdesc0 = smem_desc(0, 32, 256, 6);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int c = blockIdx.x; ok && c < chunks && !*abort_flag; c += gridDim.x) {
+        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim)) {
+          record_timeout(p, abort_flag);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 128);
+        const int g0 = c * per_chunk, g1 = min(rows_total, (c + 1) * per_chunk);
+        for (int g = g0; g < g1; ++g) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, lim)) {
+            record_timeout(p, abort_flag);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa16 = smem_u32(smem + stage * Cfg::STAGE) >> 4;
+          const uint64_t ab = adesc0 + sa16;
+          const uint64_t bb = bdesc0 + sa16 + (Cfg::DY_BYTES >> 4);
+#pragma unroll
+          for (int js = 0; js < Cfg::WS / 16; ++js)
+#pragma unroll
+            for (int uu = 0; uu < 2; ++uu)
+              tc_mma_f16(d_tmem + (uint32_t)(uu * 64), ab + (uint32_t)(js * (2048 >> 4)),
+                         bb + (uint32_t)((uu * 2 * Cfg::WS * 32 + js * 512) >> 4), p.idesc,
+                         (g > g0 || js > 0) ? 1u : 0u);
+          tc_commit(smem_u32(&empty[stage]));
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(&tfull[acc]));
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+    }
+  } else {
+    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1: row = (a, k)
+    const int sub = warp & 3;
+    const int row = sub * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int c = blockIdx.x; c < chunks; c += gridDim.x) {
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) record_timeout(p, abort_flag);
+        break;
+      }
+      tc_fence_after();
+      uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)c * 128 + row) * 128);
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * 128 + half * 64);
+        uint32_t r[64];
+        tmem_ld16(tbase, r);
+        tmem_ld16(tbase + 16, r + 16);
+        tmem_ld16(tbase + 32, r + 32);
+        tmem_ld16(tbase + 48, r + 48);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          dst[half * 8 + j] = make_uint4(pack_lo(r[j * 8 + 0], r[j * 8 + 1]), pack_lo(r[j * 8 + 2], r[j * 8 + 3]),
+                                         pack_lo(r[j * 8 + 4], r[j * 8 + 5]), pack_lo(r[j * 8 + 6], r[j * 8 + 7]));
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+cudaError_t launch_stem_wgrad(const CUtensorMap& mDy, const CUtensorMap& mXs, const GemmParams& p, int grid,
+                              cudaStream_t s) {
+  if (p.halo_ws != StemWgradCfg::WS || p.kb_per_split < 1 || p.m_tiles < 1 || grid < 1) return cudaErrorInvalidValue;
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(k_stem_wgrad, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         StemWgradCfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  launch_pdl(k_stem_wgrad, dim3(grid), dim3(kStemWgradThreads), StemWgradCfg::SMEM, s, mDy, mXs, p);
+  return counted_launches(1);
+}
+
 }  // namespace pf16

@@ -150,6 +150,13 @@ int gemm_smem_bytes(int BN);
 // output leaves through a 3-D map (64, Q, N*P) clipped at Q.  p.ntaps taps,
 // p.tap_dr/tap_ds their window offsets, p.tap_w their weight tap; p.b_mode
 // LD_TILED_K (weights [64][taps*C]) or LD_TAP3D_MN (weights (C, 9, K)).
+// Stem weight gradient on the space-to-depth input: mapDy over dy (64, Q, P, N)
+// with boxes (64, 128, 2, 1), mapXs over xs (16, Q + 3, P + 3, N) with boxes
+// (16, 128, 4, 1); p.num_kb = N * (P + 1) row units, p.kb_per_split units per
+// chunk, p.m_tiles chunks, p.halo_h = P, p.halo_ws = 128, p.out = the chunks'
+// 128 x 128 FP16 partials.
+cudaError_t launch_stem_wgrad(const CUtensorMap& mapDy, const CUtensorMap& mapXs, const GemmParams& p, int grid,
+                              cudaStream_t s);
 cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
                              const GemmParams& p, int grid, cudaStream_t stream);
 
@@ -171,6 +178,9 @@ cudaError_t launch_stem_im2col(const uint16_t* x, uint16_t* col, int N, int H, i
 // of the 4x4 stride-1 form of the 7x7 / stride 2 / pad 3 convolution
 cudaError_t launch_stem_s2d(const uint16_t* x, const uint16_t* w, uint16_t* xs, uint16_t* wsd, int N, int H,
                             int W, int Hs, int Ws, int K, cudaStream_t s);
+// dw[k][r][s][c] (7 x 7 x 3) from the stem weight gradient's reduced 128 x 128
+// [(a, k)][(u/2, v, ch)] matrix
+cudaError_t launch_stem_wgrad_scatter(const uint16_t* dws, uint16_t* dw, int K, cudaStream_t s);
 // w[K][kin] -> wpad[K][kcol] (zero padded)
 cudaError_t launch_pad_rows(const uint16_t* w, uint16_t* wpad, int K, int kin, int kcol,
                             cudaStream_t s);
