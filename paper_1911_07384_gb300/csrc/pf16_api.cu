@@ -396,6 +396,18 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
       return PF16_ERR_CUDA;
     p.tma_store = 1;
   }
+  // Clusters of two CTAs over M-tile pairs share each B tile (multicast), which
+  // halves the B operand's L2 -> SM traffic, the bound of most conv passes.
+  const int pair_cl = (BN >= 128 && p.m_tiles % 2 == 0) ? gemm_pair_clusters(BN) : 0;
+  if (pair_cl > 0) {
+    const long long pair_units = units / 2;
+    int ncl = (int)std::min<long long>(pair_units, std::min(pair_cl, sms / 2));
+    if (p.st_mean) {  // as below, per pair: two slots per cluster
+      ncl = std::min(ncl, kBnStatSlots / 2 * p.n_tiles);
+      ncl -= ncl % p.n_tiles;
+    }
+    if (ncl > 0) return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+  }
   int grid = (int)std::min<long long>(units, sms);
   if (p.st_mean) {
     // fused statistics: every CTA keeps one n-tile (grid a multiple of n_tiles), at most

@@ -130,8 +130,11 @@ struct Cursor {
     }
   }
 
+  // A, and B unless !load_b; MC: B goes to both CTAs of the cluster pair
+  template <bool MC>
   __device__ __forceinline__ void load(const GemmParams& p, const CUtensorMap* ma, const CUtensorMap* mb,
-                                       uint32_t sa, uint32_t sb, uint32_t bar, int m0, int n0) const {
+                                       uint32_t sa, uint32_t sb, uint32_t bar, int m0, int n0,
+                                       bool load_b) const {
     switch (p.a_mode) {
       case LD_TILED_K:
         tma_load_2d(sa, ma, bar, kb * kBK, m0);
@@ -147,24 +150,44 @@ struct Cursor {
       default:
         break;
     }
+    if (!load_b) return;
+    constexpr uint16_t kPair = 0x3;
     switch (p.b_mode) {
       case LD_TILED_K:
-        tma_load_2d(sb, mb, bar, kb * kBK, n0);
+        if (MC)
+          tma_load_2d_mc(sb, mb, bar, kb * kBK, n0, kPair);
+        else
+          tma_load_2d(sb, mb, bar, kb * kBK, n0);
         break;
       case LD_TILED_MN:
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tma_load_2d(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK);
+        for (int j = 0; j < BN / 64; ++j) {
+          if (MC)
+            tma_load_2d_mc(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK, kPair);
+          else
+            tma_load_2d(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK);
+        }
         break;
       case LD_IM2COL_MN: {
         const int bw = b_j * p.gb.step + p.gb.base_w, bh = b_i * p.gb.step + p.gb.base_h;
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j)
-          tma_load_im2col_4d(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
-                             (uint16_t)p.tap_dr[b_tap[j]]);
+        for (int j = 0; j < BN / 64; ++j) {
+          if (MC)
+            tma_load_im2col_4d_mc(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
+                                  (uint16_t)p.tap_dr[b_tap[j]], kPair);
+          else
+            tma_load_im2col_4d(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
+                               (uint16_t)p.tap_dr[b_tap[j]]);
+        }
       } break;
       case LD_TAP3D_MN:
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tma_load_3d(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k);
+        for (int j = 0; j < BN / 64; ++j) {
+          if (MC)
+            tma_load_3d_mc(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k, kPair);
+          else
+            tma_load_3d(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k);
+        }
         break;
       default:
         break;
@@ -172,13 +195,18 @@ struct Cursor {
   }
 };
 
+// Work unit u -> tile origin (m0, n0), split and K-block range.  mt_count M
+// tiles are enumerated; M tile mt is row tile mt * mscale + moff (a cluster
+// pair enumerates tile pairs, mscale = 2, moff = its rank).
 __device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0, int& n0, int& split,
-                                            int& kb0, int& kb1, int BN) {
-  const int per = p.m_tiles * p.n_tiles;
+                                            int& kb0, int& kb1, int BN, int mt_count = -1, int mscale = 1,
+                                            int moff = 0) {
+  if (mt_count < 0) mt_count = p.m_tiles;
+  const int per = mt_count * p.n_tiles;
   split = u / per;
   const int rem = u - split * per;
   const int mt = rem / p.n_tiles;
-  m0 = mt * kBM;
+  m0 = (mt * mscale + moff) * kBM;
   n0 = (rem - mt * p.n_tiles) * BN;
   kb0 = split * p.kb_per_split;
   kb1 = min(p.num_kb, kb0 + p.kb_per_split);
@@ -374,7 +402,15 @@ struct EpiStats {
   }
 };
 
-template <int BN>
+// PAIR: launched in clusters of two CTAs that take the same (n tile, split)
+// units over M tiles 2t and 2t + 1, so they need the same B tiles: the CTA of
+// rank kb mod 2 loads K-block kb's B tile once and multicasts it into both
+// CTAs' stage, halving the B operand's L2 -> SM traffic.  A stage is refilled
+// only after both CTAs' MMAs have read it (each MMA commit arrives on the
+// stage's empty barrier in both CTAs, count 2).  The two CTAs meet at a
+// cluster barrier after set-up and before exit, so neither's shared memory
+// or barriers are written after it has left.
+template <int BN, bool PAIR>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
@@ -395,7 +431,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < Cfg::STAGES; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), 1);
+      mbar_init(smem_u32(&empty[s]), PAIR ? 2 : 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
@@ -414,10 +450,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (PAIR) cluster_sync();  // the partner's barriers are initialised
   // set-up done: wait for the kernel this one depends on
   pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = p.m_tiles * p.n_tiles * p.splits;
+  // work enumeration: a pair walks M-tile pairs, each CTA takes its own tile of the pair
+  const int rank = PAIR ? (int)cluster_ctarank() : 0;
+  const int cid = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int ncl = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  const int mt_count = PAIR ? p.m_tiles / 2 : p.m_tiles;
+  const int mscale = PAIR ? 2 : 1;
+  const int total = mt_count * p.n_tiles * p.splits;
   const uint64_t lim = p.wait_limit_ns;
 
   if (warp == 0) {
@@ -425,9 +468,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0;  // stages loaded so far (for the drain below)
-      for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
+      for (int u = cid; u < total && !*abort_flag; u += ncl) {
         int m0, n0, split, kb0, kb1;
-        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
         Cursor<BN> cur;
         cur.init(p, m0, n0, kb0);
         for (int kb = kb0; kb < kb1; ++kb, cur.advance(p)) {
@@ -438,7 +481,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
-          cur.load(p, &mapA, &mapB, sa, sa + Cfg::A_BYTES, fb, m0, n0);
+          cur.template load<PAIR>(p, &mapA, &mapB, sa, sa + Cfg::A_BYTES, fb, m0, n0,
+                                  !PAIR || (kb & 1) == rank);
           ++issued;
           if (++stage == Cfg::STAGES) {
             stage = 0;
@@ -472,9 +516,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const uint64_t adesc0 = smem_desc(0, p.a_lbo, p.a_sbo, 2);
       const uint64_t bdesc0 = smem_desc(0, p.b_lbo, p.b_sbo, 2);
       const uint32_t ak16 = (uint32_t)p.a_kstep >> 4, bk16 = (uint32_t)p.b_kstep >> 4;
-      for (int u = blockIdx.x; u < total && !*abort_flag; u += gridDim.x) {
+      for (int u = cid; u < total && !*abort_flag; u += ncl) {
         int m0, n0, split, kb0, kb1;
-        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
         if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim)) {
           record_timeout(p, abort_flag);
           break;
@@ -489,12 +533,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t sa16 = smem_u32(smem + stage * Cfg::STAGE_BYTES) >> 4;
+          const uint32_t sa16 = desc_addr16(smem_u32(smem + stage * Cfg::STAGE_BYTES));
           const uint64_t ab = adesc0 + sa16, bb = bdesc0 + sa16 + (Cfg::A_BYTES >> 4);
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
             tc_mma_f16(d_tmem, ab + kk * ak16, bb + kk * bk16, p.idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
-          tc_commit(smem_u32(&empty[stage]));
+          if (PAIR)
+            tc_commit_mc(smem_u32(&empty[stage]), 0x3);  // the stage is free once both CTAs read it
+          else
+            tc_commit(smem_u32(&empty[stage]));
           if (++stage == Cfg::STAGES) {
             stage = 0;
             phase ^= 1;
@@ -516,10 +563,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     EpiStats stats;
     stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
-    for (int u = blockIdx.x + grp * gridDim.x; u < total; u += 2 * gridDim.x) {
+    for (int u = cid + grp * ncl; u < total; u += 2 * ncl) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
-      unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+      unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
       const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
       if (!__all_sync(0xffffffffu, got)) {
         if (lane == 0) record_timeout(p, abort_flag);
@@ -611,15 +658,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     if (p.tma_store && lane == 0) bulk_wait0();
     if (p.st_mean) {
-      // this CTA's tiles all have n-tile blockIdx % n_tiles (the grid is a multiple of n_tiles)
-      const int n0 = (blockIdx.x % p.n_tiles) * BN;
+      // this CTA's tiles all have n-tile cid % n_tiles (the pair count is a multiple of n_tiles);
+      // slot (cid / n_tiles) * mscale + rank
+      const int n0 = (cid % p.n_tiles) * BN;
       const int nch = min(BN, p.N - n0) / 64;
-      stats.write_cta(p, staging, e, blockIdx.x / p.n_tiles, n0, nch, lane, blockIdx.x % p.n_tiles == 0);
-      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = (int)gridDim.x / p.n_tiles;
+      stats.write_cta(p, staging, e, (cid / p.n_tiles) * mscale + rank, n0, nch, lane,
+                      cid % p.n_tiles == 0);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = ncl / p.n_tiles * mscale;
     }
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();  // the partner no longer writes this CTA's stages or barriers
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
@@ -636,31 +686,84 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN>
-static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                               const GemmParams& p, int grid, cudaStream_t s) {
+template <int BN, bool PAIR>
+static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          GemmCfg<BN>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
-  launch_pdl(k_gemm<BN>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
-  return counted_launches(1);
+  return cudaSuccess;
+}
+
+template <int BN>
+static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                               const GemmParams& p, int grid, bool pair, cudaStream_t s) {
+  if (!pair) {
+    cudaError_t e = set_smem_attr<BN, false>();
+    if (e != cudaSuccess) return e;
+    launch_pdl(k_gemm<BN, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
+    return counted_launches(1);
+  }
+  if constexpr (BN >= 128) {
+    if (grid % 2 != 0 || p.m_tiles % 2 != 0) return cudaErrorInvalidValue;
+    cudaError_t e = set_smem_attr<BN, true>();
+    if (e != cudaSuccess) return e;
+    launch_pdl_cluster2(k_gemm<BN, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
+    return counted_launches(1);
+  }
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                        const GemmParams& p, int grid, cudaStream_t s) {
+                        const GemmParams& p, int grid, cudaStream_t s, bool pair) {
   switch (BN) {
-    case 64: return launch_bn_t<64>(mA, mB, mC, p, grid, s);
-    case 128: return launch_bn_t<128>(mA, mB, mC, p, grid, s);
-    case 192: return launch_bn_t<192>(mA, mB, mC, p, grid, s);
-    case 256: return launch_bn_t<256>(mA, mB, mC, p, grid, s);
+    case 64: return launch_bn_t<64>(mA, mB, mC, p, grid, pair, s);
+    case 128: return launch_bn_t<128>(mA, mB, mC, p, grid, pair, s);
+    case 192: return launch_bn_t<192>(mA, mB, mC, p, grid, pair, s);
+    case 256: return launch_bn_t<256>(mA, mB, mC, p, grid, pair, s);
     default: return cudaErrorInvalidValue;
   }
+}
+
+template <int BN>
+static int pair_clusters_t() {
+  if (set_smem_attr<BN, true>() != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 152);
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = GemmCfg<BN>::SMEM;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+int gemm_pair_clusters(int BN) {
+  static int cache[64][4];
+  static bool done[64][4] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const int i = BN == 128 ? 0 : (BN == 192 ? 1 : (BN == 256 ? 2 : -1));
+  if (i < 0 || dev >= 64) return 0;
+  if (!done[dev][i]) {
+    cache[dev][i] = BN == 128 ? pair_clusters_t<128>() : (BN == 192 ? pair_clusters_t<192>() : pair_clusters_t<256>());
+    done[dev][i] = true;
+  }
+  return cache[dev][i];
 }
 
 
@@ -703,8 +806,9 @@ struct HaloCfg {
 // 128-byte swizzle) or 32 (the space-to-depth stem, sixteen taps of one step,
 // 32-byte swizzle).  The MMA issue loop is unrolled over taps and steps with
 // descriptors formed by adding 16-byte offsets to two base descriptors (the
-// start-address field is the low 14 bits, and shared-memory addresses stay
-// below 256 KB), so a single thread keeps up with N = 64 MMAs.
+// start-address field is the low 14 bits; desc_addr16 masks a shared address
+// into it, and a stage plus its tap offsets stays below 256 KB), so a single
+// thread keeps up with N = 64 MMAs.
 template <int CB>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_halo(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
@@ -830,7 +934,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 64);
-        const uint64_t abase = adesc0 + (smem_u32(astages + stage * Cfg::A_STAGE) >> 4);
+        const uint64_t abase = adesc0 + desc_addr16(smem_u32(astages + stage * Cfg::A_STAGE));
 #pragma unroll
         for (int t = 0; t < NTAPS; ++t)
 #pragma unroll
@@ -1093,7 +1197,7 @@ __global__ void __launch_bounds__(kStemWgradThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t sa16 = smem_u32(smem + stage * Cfg::STAGE) >> 4;
+          const uint32_t sa16 = desc_addr16(smem_u32(smem + stage * Cfg::STAGE));
           const uint64_t ab = adesc0 + sa16;
           const uint64_t bb = bdesc0 + sa16 + (Cfg::DY_BYTES >> 4);
 #pragma unroll
