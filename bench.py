@@ -611,7 +611,8 @@ def count_launches(net):
             total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
         total += 1 + (1 if ws else 0) + (2 if stem else 0)  # wgrad (+ split-K reduce, + the stem's s2d, scatter)
-    total += sum(per["bn_fwd"] + per["bn_bwd"] for _ in net.bns)  # forward statistics come from the conv
+    # forward statistics come from the conv; backward ones from the data gradient where fused
+    total += sum(per["bn_fwd"] + per["bn_bwd"] - (1 if getattr(b, "fused_bwd", False) else 0) for b in net.bns)
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]
     return total

@@ -105,6 +105,35 @@ int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint
 int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
+/* Data gradient with the backward statistics of the BatchNorm whose output
+ * gradient it is (Eq. 1-2 differentiated; the backward counterpart of
+ * pf16_conv_fwd_bnstats).  dx, the result, is dL/dy of a BatchNorm described
+ * by `bn`: its input x (n x h x w x c, the conv output its forward normalised),
+ * its ReLU bit mask (as written by pf16_bn_fwd_bwd phase 0; NULL for a
+ * BatchNorm without ReLU) and its saved mean and invstd.  Same arguments and
+ * dx as pf16_conv_dgrad with flags 0; in addition each epilogue warp of the
+ * GEMM reduces, per channel, dy' = dx where the ReLU passed and dy' * xhat,
+ * xhat = rn(rn(x - mean) * invstd), over the 32 rows of each tile it stores:
+ * FP16 halving trees, zero leaves for rows past the tensor, pushed into the
+ * warp's tree of tiles, which is padded with zero leaves to a power of two.
+ * The CTAs' nodes go to `stats` (stats_bytes >= pf16_conv_dgrad_bnstats_size(d),
+ * 16-byte aligned, caller-owned, no initial contents needed);
+ * pf16_bn_fwd_bwd phase 1 takes it through pf16_bn_tensors.conv_stats and
+ * skips its statistics pass over dy and x.  Requires stride 1 (dx rows in
+ * pixel order) and c a multiple of 64 (PF16_ERR_UNSUPPORTED otherwise; the
+ * size function then returns 0); x, mean, invstd 16-byte aligned, relu_mask
+ * 8-byte aligned. */
+typedef struct {
+  const uint16_t* x;         /* the BatchNorm's input, n x h x w x c */
+  const uint8_t* relu_mask;  /* its ReLU decisions (bit mask), or NULL: no ReLU */
+  const uint16_t* mean;      /* its saved mean [c] */
+  const uint16_t* invstd;    /* its saved invstd [c] */
+} pf16_bn_source;
+size_t pf16_conv_dgrad_bnstats_size(const pf16_conv_desc* d);
+int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                            void* ws, size_t ws_bytes, const pf16_bn_source* bn, void* stats,
+                            size_t stats_bytes, void* stream);
+
 /* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*st+r-pad, q*st+s-pad, c].
  * The reduction over n*p*q pixels is split into chunks, each accumulated in
  * FP16 by the tensor core into FP16 partials in the workspace, which are then
@@ -175,11 +204,17 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
  *       moves 1/16 of the bytes.
  * relu_mask is ignored without PF16_BN_RELU (the bit mask is a storage
  * choice of this library, not part of the paper's method).
- * conv_stats (phase 0, optional): when x is the output of a
- * pf16_conv_fwd_bnstats call that filled this 16-byte-aligned buffer (and
- * nothing has written x or the buffer since), the mean and variance are
- * taken from its partial statistics instead of a pass over x; the result is
- * the same BatchNorm up to the FP16 rounding of a different reduction tree.
+ * conv_stats (optional, 16-byte aligned):
+ *   phase 0: when x is the output of a pf16_conv_fwd_bnstats call that filled
+ *       this buffer (and nothing has written x or the buffer since), the mean
+ *       and variance are taken from its partial statistics instead of a pass
+ *       over x;
+ *   phase 1: when dy is the output of a pf16_conv_dgrad_bnstats call that
+ *       filled this buffer for this BatchNorm (same x, mask, mean, invstd),
+ *       the means of dy' and dy'*xhat (and dgamma, dbeta) come from its
+ *       partial trees instead of a pass over dy and x;
+ *   either way the result is the same BatchNorm up to the FP16 rounding of a
+ *   different reduction tree.
  * c must be a multiple of 8 and at most 2048. */
 typedef struct {
   int32_t n, h, w, c;
@@ -192,7 +227,8 @@ typedef struct {
   const uint16_t *x, *gamma, *beta, *residual, *dy, *y_saved;
   uint16_t *y, *mean, *invstd, *dx, *dgamma, *dbeta, *dresidual;
   uint8_t* relu_mask; /* optional ReLU bit mask: written by phase 0, read by phase 1 */
-  const void* conv_stats; /* optional, phase 0: statistics of x from pf16_conv_fwd_bnstats */
+  const void* conv_stats; /* optional: partial statistics from pf16_conv_fwd_bnstats (phase 0)
+                             or pf16_conv_dgrad_bnstats (phase 1) */
 } pf16_bn_tensors;
 
 size_t pf16_bn_workspace_size(const pf16_bn_desc* d);

@@ -373,6 +373,17 @@ GemmParams base_params(int* status) {
   return p;
 }
 
+// Levels of an epilogue warp's padded tile tree (backward statistics): `ctas`
+// CTAs (or CTA pairs) share `units` tiles round robin, and each CTA's two
+// epilogue groups take alternate tiles.
+int tile_tree_levels(long long units, long long ctas) {
+  const long long per_cta = (units + ctas - 1) / ctas;
+  const long long per_group = (per_cta + 1) / 2;
+  int l = 0;
+  while ((1ll << l) < per_group) ++l;
+  return l;
+}
+
 int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int sms,
         cudaStream_t st) {
   p.m_tiles = cdiv(p.M, kBM);
@@ -406,7 +417,11 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
       ncl = std::min(ncl, kBnStatSlots / 2 * p.n_tiles);
       ncl -= ncl % p.n_tiles;
     }
-    if (ncl > 0) return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+    if (ncl > 0) {
+      if (p.bs_x && (p.bs_levels = tile_tree_levels(pair_units, ncl)) >= kMaxTileTreeLevels)
+        return PF16_ERR_UNSUPPORTED;
+      return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+    }
   }
   int grid = (int)std::min<long long>(units, sms);
   if (p.st_mean) {
@@ -414,8 +429,18 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
     // kBnStatSlots / 4 CTAs per n-tile
     grid = std::min(grid, kBnStatSlots * p.n_tiles);
     grid -= grid % p.n_tiles;
+    if (p.bs_x && (p.bs_levels = tile_tree_levels(units, grid)) >= kMaxTileTreeLevels) return PF16_ERR_UNSUPPORTED;
   }
   return launch_gemm(BN, a, b, c, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
+// Point the GEMM's fused statistics at the BatchNorm backward sources.
+void set_bwd_stats(GemmParams& p, const pf16_bn_source* bn) {
+  if (!bn) return;
+  p.bs_x = bn->x;
+  p.bs_mask = bn->relu_mask;
+  p.bs_mean = bn->mean;
+  p.bs_invstd = bn->invstd;
 }
 
 // Point the GEMM's fused statistics at a conv-output statistics buffer of C channels.
@@ -467,9 +492,10 @@ int halo_width(const Shape& s, bool accum) {
 // gradient (dgrad = true: in = dy, weights viewed (C, 9, K), taps flipped)
 // through the halo engine.  in and out are N x H x W x 64.
 int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint16_t* w, uint16_t* out,
-             int* status, int sms, cudaStream_t st, void* stats = nullptr) {
+             int* status, int sms, cudaStream_t st, void* stats = nullptr, const pf16_bn_source* bn = nullptr) {
   GemmParams p = base_params(status);
   set_stats(p, stats, 64);
+  set_bwd_stats(p, bn);
   CUtensorMap ma, mb, mc;
   const long long N = s.N, H = s.H, W = s.W;
   cuuint64_t dims[4] = {64, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
@@ -505,10 +531,12 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
   p.halo_row0 = -1;
   p.halo_col0 = -1;
   p.N = 64;
+  p.ldo = 64;
   p.n_tiles = 1;
   p.m_tiles = (int)(N * H * ws / kBM);
   int grid = p.m_tiles < sms ? p.m_tiles : sms;
   if (stats && grid > kBnStatSlots) grid = kBnStatSlots;
+  if (p.bs_x && (p.bs_levels = tile_tree_levels(p.m_tiles, grid)) >= kMaxTileTreeLevels) return PF16_ERR_UNSUPPORTED;
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
@@ -655,29 +683,41 @@ int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint
   return conv_fwd_impl(d, x, w, y, ws, ws_bytes, 0, stats, stats_bytes, stream);
 }
 
-int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
-                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
-  (void)ws;
-  (void)ws_bytes;
+static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                           uint32_t flags, void* stats, size_t stats_bytes, const pf16_bn_source* bn,
+                           void* stream) {
   Shape s;
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if (s.kind == KIND_STEM) return PF16_ERR_UNSUPPORTED;
   if ((rc = check_common(dy, w, dx)) != PF16_OK) return rc;
   if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  if (stats) {
+    // statistics of a plain output whose rows are pixels in order (stride 1)
+    if (flags != 0) return PF16_ERR_ARG;
+    if (!bn->x || !bn->mean || !bn->invstd) return PF16_ERR_NULL;
+    if (!aligned16(stats) || !aligned16(bn->x) || !aligned16(bn->mean) || !aligned16(bn->invstd) ||
+        (reinterpret_cast<uintptr_t>(bn->relu_mask) & 7u) != 0)
+      return PF16_ERR_ALIGN;
+    if (s.C % 64 != 0 || s.st != 1) return PF16_ERR_UNSUPPORTED;
+    if (stats_bytes < bnstat_bytes(s.C)) return PF16_ERR_WORKSPACE;
+  }
   if (!driver_fns()) return PF16_ERR_CUDA;
   int* status;
   int sms;
   if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const bool accum = (flags & PF16_ACCUMULATE) != 0;
-  if (const int ws = halo_width(s, accum)) return run_halo(s, ws, true, dy, w, dx, status, sms, st);
+  if (const int ws = halo_width(s, accum))
+    return run_halo(s, ws, true, dy, w, dx, status, sms, st, stats, stats ? bn : nullptr);
   const int BN = pick_bn_out(s.C);
   const size_t dx_elems = (size_t)(s.N * s.H * s.W * s.C);
 
   if (s.R == 1 && s.S == 1 && s.pad == 0) {
     // 1x1: dx[n, st*p, st*q, :] = dy[n,p,q,:] . w ; other positions receive nothing
     GemmParams p = base_params(status);
+    set_stats(p, stats, s.C);
+    if (stats) set_bwd_stats(p, bn);
     CUtensorMap ma, mb;
     p.M = (int)(s.N * s.P * s.Q);
     p.N = (int)s.C;
@@ -719,6 +759,8 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
       const int *ar = f.ar, *bs = f.bs, *rr = f.rr, *ss = f.ss;
       const int amin = *std::min_element(ar, ar + nr), bmin = *std::min_element(bs, bs + ns);
       GemmParams p = base_params(status);
+      set_stats(p, stats, s.C);  // stride 1 only: one phase, rows in pixel order
+      if (stats) set_bwd_stats(p, bn);
       CUtensorMap ma, mb;
       p.M = (int)(s.N * gh * gw);
       p.N = (int)s.C;
@@ -754,6 +796,28 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
       if ((rc = run(BN, ma, mb, p, sms, st)) != PF16_OK) return rc;
     }
   return PF16_OK;
+}
+
+int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  return conv_dgrad_impl(d, dy, w, dx, flags, nullptr, 0, nullptr, stream);
+}
+
+size_t pf16_conv_dgrad_bnstats_size(const pf16_conv_desc* d) {
+  Shape s;
+  if (conv_shape(d, &s) != PF16_OK || s.kind == KIND_STEM || s.C % 64 != 0 || s.st != 1) return 0;
+  return bnstat_bytes(s.C);
+}
+
+int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                            void* ws, size_t ws_bytes, const pf16_bn_source* bn, void* stats,
+                            size_t stats_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (!bn || !stats) return PF16_ERR_NULL;
+  return conv_dgrad_impl(d, dy, w, dx, 0, stats, stats_bytes, bn, stream);
 }
 
 // The stem's weight gradient through k_stem_wgrad (layouts at stem_wgrad_plan).
@@ -957,10 +1021,12 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
   if (b.relu && !bits && !t->y_saved) return PF16_ERR_NULL;
   if (b.relu && !bits && !aligned16(t->y_saved)) return PF16_ERR_ALIGN;
   if (t->dresidual && !aligned16(t->dresidual)) return PF16_ERR_ALIGN;
+  if (t->conv_stats && !aligned16(t->conv_stats)) return PF16_ERR_ALIGN;
   if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
   return launch_bn_bwd(b, t->x, t->gamma, t->mean, t->invstd, t->dy,
                        b.relu && !bits ? t->y_saved : nullptr, bits ? t->relu_mask : nullptr, t->dx,
-                       t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws), st) ==
+                       t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws), st,
+                       static_cast<const uint8_t*>(t->conv_stats)) ==
                  cudaSuccess
              ? PF16_OK
              : PF16_ERR_CUDA;

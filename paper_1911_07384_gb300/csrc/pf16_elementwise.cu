@@ -1067,6 +1067,59 @@ __global__ void __launch_bounds__(kFinalThreads)
   }
 }
 
+// Backward statistics from a dgrad statistics buffer (pf16_conv_dgrad_bnstats):
+// the slots hold halving-tree nodes of dy' and dy' * xhat, each over
+// 2^hdr[1] (zero-padded) leaves; a halving tree over the slots padded to a
+// power of two closes the tree over 2^L leaves, then, as k_bn_bwd_final,
+// means x rn(2^L / R) and sums x 2^L exactly.  One CTA per channel group of 8.
+__global__ void __launch_bounds__(kFinalThreads)
+    k_bn_bwd_final_slots(const uint8_t* __restrict__ stats, int C, long long R, uint16_t post_scale,
+                         uint16_t* mm, uint16_t* dgamma, uint16_t* dbeta) {
+  pdl_wait();
+  __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
+  const int tc = C / 8, cg = blockIdx.x, t = threadIdx.x;
+  const int S = reinterpret_cast<const int*>(stats)[0];
+  const int L0 = reinterpret_cast<const int*>(stats)[1];
+  const uint16_t* sd = reinterpret_cast<const uint16_t*>(stats + bnstat_off_mean());
+  const uint16_t* sp = reinterpret_cast<const uint16_t*>(stats + bnstat_off_var(C));
+  int sp2 = 1, ls = 0;
+  while (sp2 < S) {
+    sp2 *= 2;
+    ++ls;
+  }
+  const int nthr = sp2 < kFinalThreads ? sp2 : kFinalThreads;
+  const int seg = sp2 / nthr;
+  if (t < nthr) {
+    Tree4<12, true> t1, t2;
+    for (int i = 0; i < seg; ++i) {
+      const int b = t * seg + i;
+      const bool ok = b < S;
+      t1.push(ok ? __ldg(reinterpret_cast<const uint4*>(sd + (long long)b * C) + cg) : zero4());
+      t2.push(ok ? __ldg(reinterpret_cast<const uint4*>(sp + (long long)b * C) + cg) : zero4());
+    }
+    const int lv = 31 - __clz(seg);
+    s1[t] = t1.finish(lv);
+    s2[t] = t2.finish(lv);
+  }
+  __syncthreads();
+  for (int half = nthr / 2; half >= 1; half /= 2) {
+    if (t < half) {
+      s1[t] = hmerge4(s1[t], s1[t + half]);
+      s2[t] = hmerge4(s2[t], s2[t + half]);
+    }
+    __syncthreads();
+  }
+  if (t == 0) {
+    const int L = L0 + ls;
+    const uint16_t ratio = __half_as_ushort(__float2half_rn((float)(ldexp(1.0, L) / (double)R)));
+    const uint32_t ratio2 = dup2(ratio), ps = dup2(post_scale);
+    reinterpret_cast<uint4*>(mm)[cg] = mul4(s1[0], ratio2);
+    reinterpret_cast<uint4*>(mm)[tc + cg] = mul4(s2[0], ratio2);
+    reinterpret_cast<uint4*>(dbeta)[cg] = mul4(ldexp4(s1[0], L), ps);
+    reinterpret_cast<uint4*>(dgamma)[cg] = mul4(ldexp4(s2[0], L), ps);
+  }
+}
+
 constexpr int kApplyRows = 8;  // rows per thread per CTA in the apply passes
 
 __global__ void __launch_bounds__(256)
@@ -1282,7 +1335,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
                           const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
                           uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
-                          cudaStream_t s) {
+                          cudaStream_t s, const uint8_t* dgrad_stats) {
   static bool attr[3][64] = {{false}};
   BnStatArgs a = bn_args(b, b.bwd, ws);
   a.x = x;
@@ -1300,7 +1353,13 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   const unsigned apply_blocks = (unsigned)((b.R + rows - 1) / rows);
   const unsigned threads = (unsigned)(g.threads + 32);
   cudaError_t e = cudaSuccess;
-  switch (mode) {
+  int launches = 3;
+  if (dgrad_stats) {
+    // statistics from the producing data gradient's epilogue
+    launch_pdl(k_bn_bwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, dgrad_stats, b.C, b.R,
+               b.post_scale, a.mm, dgamma, dbeta);
+    launches = 2;
+  } else switch (mode) {
     case BN_NO_RELU:
       e = stat_smem_attr(k_bn_bwd_stats<BN_NO_RELU>, smem, attr[0]);
       if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_NO_RELU>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
@@ -1315,7 +1374,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
       break;
   }
   if (e != cudaSuccess) return e;
-  launch_pdl(k_bn_bwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a);
+  if (!dgrad_stats) launch_pdl(k_bn_bwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a);
   switch (mode) {
     case BN_NO_RELU:
       launch_pdl(k_bn_bwd_apply<BN_NO_RELU>, dim3(apply_blocks), dim3(g.threads), 0, s, 
@@ -1330,7 +1389,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
           x, gamma, mean, invstd, dy, nullptr, relu_mask, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
       break;
   }
-  return counted_launches(3);
+  return counted_launches(launches);
 }
 
 // ============================================================================

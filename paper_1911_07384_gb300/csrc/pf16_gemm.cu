@@ -245,7 +245,7 @@ __device__ __forceinline__ uint32_t pack_lo(uint32_t a, uint32_t b) { return __b
 // once, after the warp's last tile.  All binary16, one rounding per op.
 // ---------------------------------------------------------------------------
 constexpr int kStChunks = 4;   // 64-column chunks of a tile (BN <= 256)
-constexpr int kStLevels = 12;  // tiles per warp below 2^12
+constexpr int kStLevels = kMaxTileTreeLevels;  // tiles per warp below 2^12
 
 __device__ __forceinline__ uint32_t hmerge2f(uint32_t a, uint32_t b) {  // rn(a/2 + rn(b/2))
   return hfma2_rn(a, 0x38003800u, hmul2_rn(b, 0x38003800u));
@@ -400,7 +400,124 @@ struct EpiStats {
     }
     if (write_count && lane == 0) p.st_cnt[slot] = tot;
   }
+
+  // Backward statistics (GemmParams::bs_x): leaf of chunk c from the staged
+  // gradient tile g and the prefetched inputs of its 32 rows (BwdIn).  Lane l
+  // takes channel pair (2l, 2l+1): dy' = g where the ReLU passed and
+  // dy' * rn(rn(x - mean) * invstd); rows r >= nv are zero leaves.  Each
+  // 32-leaf halving tree is pushed into chunk c's binary counter of halving
+  // nodes (mu: dy', v: dy' xhat).
+  __device__ __forceinline__ void leaf_bwd(int c, uint32_t stg, int lane, int nv, const struct BwdIn& in);
+  // Close the backward counters as if zero leaves padded them to 2^levels,
+  // merge the CTA's 8 epilogue warps by halving (warps 0..7 in a balanced
+  // tree, through `sm` as write_cta) and write the CTA's nodes as `slot`.
+  __device__ __forceinline__ void write_cta_bwd(const GemmParams& p, uint8_t* sm, int e, int slot, int n0,
+                                                int nchunks, int lane, int levels) {
+    uint32_t* node = reinterpret_cast<uint32_t*>(sm);  // [8][kStChunks][32][2]
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
+    for (int c = 0; c < nchunks; ++c) {
+      uint32_t a1 = 0, a2 = 0;
+      bool have = false;
+#pragma unroll 1
+      for (int l = 0; l <= levels && l < kStLevels; ++l) {
+        if (l == levels) {
+          if (!have && (cnt & (1u << l))) {  // exactly 2^levels leaves
+            a1 = this->mu[c][l];
+            a2 = this->v[c][l];
+          }
+        } else if (cnt & (1u << l)) {
+          a1 = hmerge2f(this->mu[c][l], have ? a1 : 0u);
+          a2 = hmerge2f(this->v[c][l], have ? a2 : 0u);
+          have = true;
+        } else if (have) {
+          a1 = hmerge2f(a1, 0u);
+          a2 = hmerge2f(a2, 0u);
+        }
+      }
+      node[((e * kStChunks + c) * 32 + lane) * 2] = a1;
+      node[((e * kStChunks + c) * 32 + lane) * 2 + 1] = a2;
+    }
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
+    if (e != 0) return;
+    for (int c = 0; c < nchunks; ++c) {
+      uint32_t m1[8], m2[8];
+#pragma unroll
+      for (int w = 0; w < 8; ++w) {
+        m1[w] = node[((w * kStChunks + c) * 32 + lane) * 2];
+        m2[w] = node[((w * kStChunks + c) * 32 + lane) * 2 + 1];
+      }
+#pragma unroll
+      for (int h = 1; h < 8; h *= 2)
+#pragma unroll
+        for (int w = 0; w < 8; w += 2 * h) {
+          m1[w] = hmerge2f(m1[w], m1[w + h]);
+          m2[w] = hmerge2f(m2[w], m2[w + h]);
+        }
+      const long long o = (long long)slot * p.N + n0 + c * 64 + 2 * lane;
+      *reinterpret_cast<uint32_t*>(p.st_mean + o) = m1[0];
+      *reinterpret_cast<uint32_t*>(p.st_var + o) = m2[0];
+    }
+  }
 };
+
+// Inputs of one backward leaf, loaded ahead of the tile's accumulator so that
+// their latency overlaps the wait for it: for the warp's 32 rows starting at
+// row0 of [rows][N] (pixels in order) and the 64 columns at col0, lane l
+// holds x of channel pair (2l, 2l+1) for every row, and the 64 ReLU bits of
+// row l (all ones without a mask); plus the pair's mean and invstd.
+struct BwdIn {
+  uint32_t x[32];
+  uint2 m;
+  uint32_t mu2, is2;
+
+  __device__ __forceinline__ void load(const GemmParams& p, long long row0, int col0, int nv, int lane) {
+    const uint16_t* xr = p.bs_x + row0 * p.ldo + col0;
+#pragma unroll
+    for (int r = 0; r < 32; ++r)
+      x[r] = r < nv ? __ldg(reinterpret_cast<const uint32_t*>(xr + r * p.ldo) + lane) : 0u;
+    m = make_uint2(0xFFFFFFFFu, 0xFFFFFFFFu);
+    if (p.bs_mask && lane < nv)
+      m = __ldg(reinterpret_cast<const uint2*>(p.bs_mask + (row0 + lane) * (p.N / 8) + col0 / 8));
+    mu2 = __ldg(reinterpret_cast<const uint32_t*>(p.bs_mean + col0) + lane);
+    is2 = __ldg(reinterpret_cast<const uint32_t*>(p.bs_invstd + col0) + lane);
+  }
+};
+
+__device__ __forceinline__ void EpiStats::leaf_bwd(int c, uint32_t stg, int lane, int nv, const BwdIn& in) {
+  const uint32_t col = (uint32_t)(lane & 3) * 4;
+  uint32_t t1[32], t2[32];
+#pragma unroll
+  for (int r = 0; r < 32; ++r) {
+    uint32_t g;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(g) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
+    // row r's ReLU bits from lane r; this lane's two channels are bits 2l, 2l+1
+    const uint32_t mlo = __shfl_sync(0xffffffffu, in.m.x, r), mhi = __shfl_sync(0xffffffffu, in.m.y, r);
+    const uint32_t b = (lane < 16 ? mlo >> (2 * lane) : mhi >> (2 * lane - 32)) & 3u;
+    const uint32_t mk = ((b & 1u) ? 0x0000FFFFu : 0u) | ((b & 2u) ? 0xFFFF0000u : 0u);
+    const uint32_t d = r < nv ? (g & mk) : 0u;
+    t1[r] = d;
+    t2[r] = r < nv ? hmul2_rn(d, hmul2_rn(hsub2_rn(in.x[r], in.mu2), in.is2)) : 0u;
+  }
+#pragma unroll
+  for (int w = 16; w >= 1; w /= 2)
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      t1[i] = hmerge2f(t1[2 * i], t1[2 * i + 1]);
+      t2[i] = hmerge2f(t2[2 * i], t2[2 * i + 1]);
+    }
+  uint32_t n1 = t1[0], n2 = t2[0];
+#pragma unroll 1
+  for (int l = 0; l < kStLevels; ++l) {
+    if (cnt & (1u << l)) {
+      n1 = hmerge2f(mu[c][l], n1);
+      n2 = hmerge2f(v[c][l], n2);
+    } else {
+      mu[c][l] = n1;
+      v[c][l] = n2;
+      break;
+    }
+  }
+}
 
 // PAIR: launched in clusters of two CTAs that take the same (n tile, split)
 // units over M tiles 2t and 2t + 1, so they need the same B tiles: the CTA of
@@ -410,7 +527,9 @@ struct EpiStats {
 // stage's empty barrier in both CTAs, count 2).  The two CTAs meet at a
 // cluster barrier after set-up and before exit, so neither's shared memory
 // or barriers are written after it has left.
-template <int BN, bool PAIR>
+// BS: the epilogue takes BatchNorm backward statistics (GemmParams::bs_x);
+// a separate instantiation, so that the other GEMMs do not carry its registers.
+template <int BN, bool PAIR, bool BS>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
@@ -563,10 +682,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     EpiStats stats;
     stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
+    const bool bstats = BS && p.st_mean && p.bs_x && p.tma_store;
+    BwdIn bin;
     for (int u = cid + grp * ncl; u < total; u += 2 * ncl) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
       unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+      if (bstats) {  // the first chunk's inputs, loaded while the accumulator is computed
+        const int nv0 = min(32, max(0, p.M - (m0 + sub * 32)));
+        if (nv0 > 0) bin.load(p, (long long)(m0 + sub * 32), n0, nv0, lane);
+      }
       const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
       if (!__all_sync(0xffffffffu, got)) {
         if (lane == 0) record_timeout(p, abort_flag);
@@ -613,7 +738,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
               tma_store_2d(&mapC, stg, n0 + c, m0 + sub * 32);
             bulk_commit();
           }
-          if (p.st_mean && nv > 0 && n0 + c < p.N) stats.leaf(c / 64, stg, lane, nv);
+          if (p.st_mean && nv > 0 && n0 + c < p.N) {
+            if (BS) {
+              stats.leaf_bwd(c / 64, stg, lane, nv, bin);
+              if (c + 64 < BN && n0 + c + 64 < p.N) bin.load(p, (long long)(m0 + sub * 32), n0 + c + 64, nv, lane);
+            } else {
+              stats.leaf(c / 64, stg, lane, nv);
+            }
+          }
         }
         if (p.st_mean && nv > 0) stats.end_tile(nv);
         acc_phase ^= 1;
@@ -662,9 +794,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // slot (cid / n_tiles) * mscale + rank
       const int n0 = (cid % p.n_tiles) * BN;
       const int nch = min(BN, p.N - n0) / 64;
-      stats.write_cta(p, staging, e, (cid / p.n_tiles) * mscale + rank, n0, nch, lane,
-                      cid % p.n_tiles == 0);
-      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = ncl / p.n_tiles * mscale;
+      const int slot = (cid / p.n_tiles) * mscale + rank;
+      if (BS)
+        stats.write_cta_bwd(p, staging, e, slot, n0, nch, lane, p.bs_levels);
+      else
+        stats.write_cta(p, staging, e, slot, n0, nch, lane, cid % p.n_tiles == 0);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) {
+        p.st_hdr[0] = ncl / p.n_tiles * mscale;
+        p.st_hdr[1] = 5 + p.bs_levels + 3;
+      }
     }
   }
   tc_fence_before();
@@ -686,13 +824,13 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN, bool PAIR>
+template <int BN, bool PAIR, bool BS = false>
 static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR, BS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          GemmCfg<BN>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
@@ -703,17 +841,26 @@ static cudaError_t set_smem_attr() {
 template <int BN>
 static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                                const GemmParams& p, int grid, bool pair, cudaStream_t s) {
+  const bool bs = p.bs_x != nullptr;
   if (!pair) {
-    cudaError_t e = set_smem_attr<BN, false>();
+    cudaError_t e = bs ? set_smem_attr<BN, false, true>() : set_smem_attr<BN, false, false>();
     if (e != cudaSuccess) return e;
-    launch_pdl(k_gemm<BN, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
+    if (bs)
+      launch_pdl(k_gemm<BN, false, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
+    else
+      launch_pdl(k_gemm<BN, false, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
     return counted_launches(1);
   }
   if constexpr (BN >= 128) {
     if (grid % 2 != 0 || p.m_tiles % 2 != 0) return cudaErrorInvalidValue;
-    cudaError_t e = set_smem_attr<BN, true>();
+    cudaError_t e = bs ? set_smem_attr<BN, true, true>() : set_smem_attr<BN, true, false>();
     if (e != cudaSuccess) return e;
-    launch_pdl_cluster2(k_gemm<BN, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
+    if (bs)
+      launch_pdl_cluster2(k_gemm<BN, true, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB,
+                          mC, p);
+    else
+      launch_pdl_cluster2(k_gemm<BN, true, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB,
+                          mC, p);
     return counted_launches(1);
   }
   return cudaErrorInvalidValue;
@@ -745,7 +892,7 @@ static int pair_clusters_t() {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -809,7 +956,7 @@ struct HaloCfg {
 // start-address field is the low 14 bits; desc_addr16 masks a shared address
 // into it, and a stage plus its tap offsets stays below 256 KB), so a single
 // thread keeps up with N = 64 MMAs.
-template <int CB>
+template <int CB, bool BS>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_halo(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
                 const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
@@ -961,8 +1108,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t stg = smem_u32(staging) + (uint32_t)(e * 4096);
     EpiStats stats;
     stats.init();
+    BwdIn bin;
     for (int u = blockIdx.x + grp * gridDim.x; u < total; u += 2 * gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      if (BS && p.st_mean) {  // the tile's inputs, loaded while the accumulator is computed
+        const int mp = u * kBM + sub * 32;
+        const int nv0 = min(32, max(0, p.halo_w - mp % ws));
+        // pixel of padded row mp: image row mp / ws, column mp % ws
+        if (nv0 > 0) bin.load(p, (long long)(mp / ws) * p.halo_w + mp % ws, 0, nv0, lane);
+      }
       const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
       if (!__all_sync(0xffffffffu, got)) {
         if (lane == 0) record_timeout(p, abort_flag);
@@ -1004,7 +1158,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int mp = u * kBM + sub * 32;
         const int nv = min(32, max(0, p.halo_w - mp % ws));  // columns j >= W are padding
         if (nv > 0) {
-          stats.leaf(0, stg, lane, nv);
+          if (BS)
+            stats.leaf_bwd(0, stg, lane, nv, bin);
+          else
+            stats.leaf(0, stg, lane, nv);
           stats.end_tile(nv);
         }
       }
@@ -1012,8 +1169,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     if (lane == 0) bulk_wait0();
     if (p.st_mean) {
-      stats.write_cta(p, staging, e, blockIdx.x, 0, 1, lane, true);
-      if (blockIdx.x == 0 && e == 0 && lane == 0) p.st_hdr[0] = (int)gridDim.x;
+      if (BS)
+        stats.write_cta_bwd(p, staging, e, blockIdx.x, 0, 1, lane, p.bs_levels);
+      else
+        stats.write_cta(p, staging, e, blockIdx.x, 0, 1, lane, true);
+      if (blockIdx.x == 0 && e == 0 && lane == 0) {
+        p.st_hdr[0] = (int)gridDim.x;
+        p.st_hdr[1] = 5 + p.bs_levels + 3;
+      }
     }
   }
   tc_fence_before();
@@ -1037,20 +1200,20 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const
       p.halo_box_rows * p.halo_ws * p.halo_cb > HaloCfg::A_BOX_MAX ||
       max_off + kBM * p.halo_cb > HaloCfg::A_STAGE)
     return cudaErrorInvalidValue;
-  static bool attr_set[2][64] = {};
+  // variants: 128-byte pixels, with backward statistics (the 3x3 data gradient) or not; 32-byte pixels
+  static bool attr_set[3][64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
-  const int v = p.halo_cb == 128 ? 0 : 1;
+  const int v = p.halo_cb == 128 ? (p.bs_x ? 1 : 0) : 2;
+  if (v == 2 && p.bs_x) return cudaErrorInvalidValue;
+  void (*const kern[3])(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) = {
+      k_gemm_halo<128, false>, k_gemm_halo<128, true>, k_gemm_halo<32, false>};
   if (dev < 64 && !attr_set[v][dev]) {
-    cudaError_t e = cudaFuncSetAttribute(v == 0 ? k_gemm_halo<128> : k_gemm_halo<32>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, HaloCfg::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(kern[v], cudaFuncAttributeMaxDynamicSharedMemorySize, HaloCfg::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[v][dev] = true;
   }
-  if (v == 0)
-    launch_pdl(k_gemm_halo<128>, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
-  else
-    launch_pdl(k_gemm_halo<32>, dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
+  launch_pdl(kern[v], dim3(grid), dim3(kGemmThreads), HaloCfg::SMEM, s, mA, mB, mC, p);
   return counted_launches(1);
 }
 

@@ -142,12 +142,25 @@ struct GemmParams {
   uint16_t* st_var;       // [kBnStatSlots][N]
   int* st_cnt;            // [kBnStatSlots]
   int* st_hdr;
+  // BatchNorm backward statistics instead (bs_x non-null; same buffer): the
+  // output is the gradient dL/dy of a BatchNorm whose input bs_x ([pixels][N],
+  // row pitch ldo), ReLU bits bs_mask ([pixels][N/8], or null) and saved
+  // bs_mean / bs_invstd are given.  Per slot and channel: the halving-tree
+  // node of dy' (in st_mean) and of dy' * xhat (in st_var), every epilogue
+  // warp's tile trees padded to 2^bs_levels leaves; st_hdr[0] = slots,
+  // st_hdr[1] = tree levels below the slot tree (5 + bs_levels + 3).
+  const uint16_t* bs_x;
+  const uint8_t* bs_mask;
+  const uint16_t* bs_mean;
+  const uint16_t* bs_invstd;
+  int bs_levels;
 };
 
 // Conv-output BatchNorm statistics buffer (pf16_conv_fwd_bnstats): a header of
 // 256 bytes (int slots), then mean and variance [kBnStatSlots][C] binary16 and
 // counts [kBnStatSlots] int32, each section 256-byte aligned.
 constexpr int kBnStatSlots = 256;
+constexpr int kMaxTileTreeLevels = 12;  // an epilogue warp's tile trees hold fewer than 2^12 tiles
 __host__ __device__ inline size_t bnstat_off_mean() { return 256; }
 __host__ __device__ inline size_t bnstat_off_var(long long C) { return 256 + (size_t)kBnStatSlots * C * 2; }
 __host__ __device__ inline size_t bnstat_off_cnt(long long C) {
@@ -241,7 +254,7 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
                           const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
                           uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
-                          cudaStream_t s);
+                          cudaStream_t s, const uint8_t* dgrad_stats = nullptr);
 void bn_plan(int R, int C, BnLaunch* b);
 size_t bn_ws_bytes(const BnLaunch& b);
 

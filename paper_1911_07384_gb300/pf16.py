@@ -34,7 +34,8 @@ EXPORTS = [
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
-    "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats",
+    "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
+    "pf16_conv_dgrad_bnstats",
 ]
 
 
@@ -50,6 +51,11 @@ class ConvDesc(ctypes.Structure):
     def out_hw(self):
         return ((self.h + 2 * self.pad - self.r) // self.stride + 1,
                 (self.w + 2 * self.pad - self.s) // self.stride + 1)
+
+
+class BnSource(ctypes.Structure):
+    """pf16_bn_source: the BatchNorm whose output gradient a data gradient is."""
+    _fields_ = [(n, ctypes.c_void_p) for n in ("x", "relu_mask", "mean", "invstd")]
 
 
 class BnDesc(ctypes.Structure):
@@ -89,6 +95,11 @@ def lib():
             L.pf16_conv_bnstats_size.restype = sz
             L.pf16_conv_fwd_bnstats.argtypes = [cdp, vp, vp, vp, vp, sz, vp, sz, vp]
             L.pf16_conv_fwd_bnstats.restype = I
+            L.pf16_conv_dgrad_bnstats_size.argtypes = [cdp]
+            L.pf16_conv_dgrad_bnstats_size.restype = sz
+            L.pf16_conv_dgrad_bnstats.argtypes = [cdp, vp, vp, vp, vp, sz, ctypes.POINTER(BnSource), vp, sz,
+                                                  vp]
+            L.pf16_conv_dgrad_bnstats.restype = I
             L.pf16_conv_wgrad_noalloc.argtypes = [cdp, vp, vp, vp, u32, vp]
             L.pf16_conv_wgrad_noalloc.restype = I
             L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
@@ -179,6 +190,21 @@ def conv_fwd_bnstats(d, x, w, y, stats, ws=None, stream=None):
 def conv_dgrad(d, dy, w, dx, ws=None, flags=0, stream=None):
     _check(lib().pf16_conv_dgrad(ctypes.byref(d), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws),
                                  _nbytes(ws), flags, _stream(stream)), "pf16_conv_dgrad")
+
+
+def conv_dgrad_bnstats_size(d) -> int:
+    return int(lib().pf16_conv_dgrad_bnstats_size(ctypes.byref(d)))
+
+
+def conv_dgrad_bnstats(d, dy, w, dx, x, relu_mask, mean, invstd, stats, ws=None, stream=None):
+    """Data gradient that also writes the backward statistics of the BatchNorm
+    whose output gradient dx is (input x, ReLU mask or None, saved mean and
+    invstd) into `stats` (conv_dgrad_bnstats_size(d) bytes) for
+    bn_fwd_bwd(phase 1, conv_stats=)."""
+    src = BnSource(_ptr(x), _ptr(relu_mask), _ptr(mean), _ptr(invstd))
+    _check(lib().pf16_conv_dgrad_bnstats(ctypes.byref(d), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws),
+                                         _nbytes(ws), ctypes.byref(src), _ptr(stats), _nbytes(stats),
+                                         _stream(stream)), "pf16_conv_dgrad_bnstats")
 
 
 def conv_wgrad(d, x, dy, dw, ws=None, flags=0, stream=None):

@@ -103,6 +103,9 @@ class Conv:
         # BatchNorm statistics of the output, written by the forward GEMM's epilogue
         size = pf16.conv_bnstats_size(self.desc)
         self.stats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
+        # backward statistics of the BatchNorm whose output gradient the data gradient is
+        size = pf16.conv_dgrad_bnstats_size(self.desc) if self.desc.c != 3 else 0
+        self.dstats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
 
     def fwd(self, x, y, with_stats=False):
         if with_stats:
@@ -111,9 +114,19 @@ class Conv:
         else:
             self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.net.ws)
 
-    def dgrad(self, dy, dx, accumulate=False):
-        self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
-                      pf16.PF16_ACCUMULATE if accumulate else 0)
+    def dgrad(self, dy, dx, accumulate=False, bn=None):
+        """bn: (BN layer, its input x) when dx is that BatchNorm's output gradient and
+        this layer can take its backward statistics (stride 1); see BN.bwd(conv=)."""
+        if bn is not None:
+            layer, x = bn
+            self.net.call("conv_dgrad", self, pf16.conv_dgrad_bnstats, self.desc, dy, self.w, dx, x, layer.mask,
+                          layer.mean, layer.invstd, self.dstats)
+        else:
+            self.net.call("conv_dgrad", self, pf16.conv_dgrad, self.desc, dy, self.w, dx, None,
+                          pf16.PF16_ACCUMULATE if accumulate else 0)
+
+    def fuses_bwd_stats(self):
+        return self.dstats is not None
 
     def wgrad(self, x, dy):
         self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.net.ws)
@@ -148,10 +161,13 @@ class BN:
                       beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd,
                       relu_mask=self.mask, conv_stats=conv.stats if conv is not None else None)
 
-    def bwd(self, x, y_saved, dy, dx, dresidual=None):
+    def bwd(self, x, y_saved, dy, dx, dresidual=None, conv=None):
+        """conv: the layer whose dgrad(bn=(self, x)) produced dy (its statistics are used)."""
         self.net.call("bn_bwd", self, pf16.bn_fwd_bwd, self.desc, 1, self.net.ws, x=x, gamma=self.gamma,
                       mean=self.mean, invstd=self.invstd, dy=dy, relu_mask=self.mask, dx=dx,
-                      dgamma=self.dgamma, dbeta=self.dbeta, dresidual=dresidual)
+                      dgamma=self.dgamma, dbeta=self.dbeta, dresidual=dresidual,
+                      conv_stats=conv.dstats if conv is not None else None)
+        self.fused_bwd = conv is not None
 
 
 class Bottleneck:
@@ -207,11 +223,13 @@ class Bottleneck:
         else:  # identity shortcut: its gradient is the start of dx
             self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=dx)
         self.conv3.wgrad(self.b2, self.da3)
-        self.conv3.dgrad(self.da3, self.db2)
-        self.bn2.bwd(self.a2, self.b2, self.db2, self.da2)
+        # the data gradients also reduce the next BatchNorm's backward statistics
+        self.conv3.dgrad(self.da3, self.db2, bn=(self.bn2, self.a2))
+        self.bn2.bwd(self.a2, self.b2, self.db2, self.da2, conv=self.conv3)
         self.conv2.wgrad(self.b1, self.da2)
-        self.conv2.dgrad(self.da2, self.db1)
-        self.bn1.bwd(self.a1, self.b1, self.db1, self.da1)
+        c2 = self.conv2 if self.conv2.fuses_bwd_stats() else None
+        self.conv2.dgrad(self.da2, self.db1, bn=(self.bn1, self.a1) if c2 else None)
+        self.bn1.bwd(self.a1, self.b1, self.db1, self.da1, conv=c2)
         self.conv1.wgrad(self.x, self.da1)
         if self.proj:
             self.conv1.dgrad(self.da1, dx)

@@ -58,6 +58,23 @@ def test_conv_validation_errors():
     assert L.pf16_conv_dgrad(ctypes.byref(stem), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_UNSUPPORTED
     # stem forward needs its patch workspace
     assert L.pf16_conv_fwd(ctypes.byref(stem), FAKE, FAKE, FAKE, None, 0, 0, None) == pf16.PF16_ERR_WORKSPACE
+    # data gradient with BatchNorm backward statistics
+    src = pf16.BnSource(FAKE, None, FAKE, FAKE)
+    sz = pf16.conv_dgrad_bnstats_size(good)
+    assert sz > 0
+    dg = L.pf16_conv_dgrad_bnstats
+    assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, None, FAKE, sz, None) == pf16.PF16_ERR_NULL
+    assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), None, sz, None) == pf16.PF16_ERR_NULL
+    assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, sz - 1,
+              None) == pf16.PF16_ERR_WORKSPACE
+    assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE_MIS, sz,
+              None) == pf16.PF16_ERR_ALIGN
+    nox = pf16.BnSource(None, None, FAKE, FAKE)
+    assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(nox), FAKE, sz, None) == pf16.PF16_ERR_NULL
+    s2 = pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 2, 1)
+    assert pf16.conv_dgrad_bnstats_size(s2) == 0
+    assert dg(ctypes.byref(s2), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, sz,
+              None) == pf16.PF16_ERR_UNSUPPORTED
 
 
 def test_workspace_sizes_are_host_computable():

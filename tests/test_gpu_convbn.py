@@ -81,3 +81,84 @@ def test_conv_fwd_bnstats_then_bn(orc, shape):
     assert np.all(err <= tol), float(np.max(err / tol))
     assert np.all(np.abs(f64(host(tm)) - mean) <= (L + 8) * U * np.abs(xv).max(0))
     assert np.all(np.abs(f64(host(ti)) - invstd) <= (2 * L + 16) * U * invstd)
+
+
+BWD_SHAPES = [
+    # conv (N, H, W, C, K, R, S, stride, pad) whose data gradient is the BatchNorm's dy; relu
+    ((2, 14, 14, 256, 64, 1, 1, 1, 0), True),    # dense 1x1, 256 channels: paired CTAs, one n-tile
+    ((2, 14, 14, 64, 256, 1, 1, 1, 0), True),    # dense 1x1, 64 channels
+    ((3, 7, 7, 512, 256, 1, 1, 1, 0), False),    # two n-tiles, no ReLU (no mask)
+    ((2, 28, 28, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 32
+    ((2, 56, 56, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 64 (columns 56..63 dropped)
+    ((2, 14, 14, 128, 128, 3, 3, 1, 1), True),   # stride-1 im2col data gradient, paired CTAs
+    ((1, 7, 7, 64, 64, 3, 3, 1, 1), True),       # one partial tile (49 rows)
+]
+
+
+def bwd_ids(c):
+    return ids(c[0]) + ("_relu" if c[1] else "")
+
+
+@pytest.mark.parametrize("case", BWD_SHAPES, ids=bwd_ids)
+def test_conv_dgrad_bnstats_then_bn_bwd(orc, case):
+    """pf16_conv_dgrad_bnstats: dx bit-identical to pf16_conv_dgrad's; the
+    BatchNorm backward from its statistics within the BN backward bound of
+    tests/test_gpu_bn.py against the oracle on the same dy = dx."""
+    shape, relu = case
+    N, H, W, C, K, R, S, st, pd = shape
+    P, Q = (H + 2 * pd - R) // st + 1, (W + 2 * pd - S) // st + 1
+    rows = N * H * W
+    w = syn.he_normal_f16(syn.seed_for(7, "w"), K, R, S, C)
+    dyc = syn.normal_f16(syn.seed_for(7, "dy"), (N, P, Q, K), 0.05)
+    xb = syn.normal_f16(syn.seed_for(7, "x"), (rows, C))     # the BatchNorm's input
+    gamma = f16(1.0 + 0.1 * f64(syn.normal_f16(15, (C,))))
+    beta = f16(0.1 * f64(syn.normal_f16(16, (C,))))
+    s = 0.25
+    bd = pf16.bn_desc(N, H, W, C, EPS, int(f16([s])[0]), pf16.PF16_BN_RELU if relu else 0)
+    bws = workspace(pf16.bn_workspace_size(bd))
+    tx, tg, tb = dev(xb), dev(gamma), dev(beta)
+    ty, tm, ti = empty16(rows * C), empty16(C), empty16(C)
+    tmask = torch.empty(rows * C // 8, dtype=torch.uint8, device="cuda") if relu else None
+    pf16.bn_fwd_bwd(bd, 0, bws, x=tx, gamma=tg, beta=tb, y=ty, mean=tm, invstd=ti, relu_mask=tmask)
+    assert pf16.sync_status() == 0
+
+    d = pf16.conv_desc(*shape)
+    size = pf16.conv_dgrad_bnstats_size(d)
+    assert size > 0
+    stats = torch.empty(size, dtype=torch.uint8, device="cuda")
+    tdyc, tw = dev(dyc), dev(w)
+    dx_ref, dx = empty16(rows * C), empty16(rows * C)
+    pf16.conv_dgrad(d, tdyc, tw, dx_ref)
+    pf16.conv_dgrad_bnstats(d, tdyc, tw, dx, tx, tmask, tm, ti, stats)
+    assert pf16.sync_status() == 0
+    g = host(dx)
+    assert np.array_equal(g, host(dx_ref))  # the statistics do not touch the data gradient
+
+    tdx, tdg, tdb = empty16(rows * C), empty16(C), empty16(C)
+    pf16.bn_fwd_bwd(bd, 1, bws, x=tx, gamma=tg, mean=tm, invstd=ti, dy=dx, y_saved=ty, relu_mask=tmask,
+                    dx=tdx, dgamma=tdg, dbeta=tdb, conv_stats=stats)
+    assert pf16.sync_status() == 0
+    L = int(np.ceil(np.log2(rows)))
+    yb = host(ty)
+    dxo, dgo, dbo, dro = orc.bn_bwd(xb, gamma, g, yb, rows, C, EPS_F, s, relu)
+    _, mean, var, invstd = orc.bn_fwd(xb, gamma, beta, None, rows, C, EPS_F, s, relu)
+    xhat = (f64(xb).reshape(rows, C) - mean) * invstd
+    dyp = np.abs(dro)
+    k = np.abs(s * f64(gamma) * invstd)
+    tol = (4 * L + 8) * U * k * (dyp + dyp.max(0) * (np.abs(xhat) + 1)) + 2.0 ** -24
+    err = np.abs(f64(host(tdx)).reshape(rows, C) - dxo)
+    assert np.all(err <= tol), float(np.max(err / tol))
+    tol_b = (4 * L + 8) * U * s * dyp.sum(0) + 2.0 ** -24
+    tol_g = (4 * L + 8) * U * s * (dyp * (np.abs(xhat) + 1)).sum(0) + 2.0 ** -24
+    assert np.all(np.abs(f64(host(tdb)) - dbo) <= tol_b), float(np.max(np.abs(f64(host(tdb)) - dbo) / tol_b))
+    assert np.all(np.abs(f64(host(tdg)) - dgo) <= tol_g), float(np.max(np.abs(f64(host(tdg)) - dgo) / tol_g))
+
+
+def test_conv_dgrad_bnstats_rejects_strided():
+    d = pf16.conv_desc(2, 14, 14, 64, 64, 3, 3, 2, 1)
+    assert pf16.conv_dgrad_bnstats_size(d) == 0
+    stats = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+    t = empty16(2 * 14 * 14 * 64)
+    with pytest.raises(pf16.PF16Error):
+        pf16.conv_dgrad_bnstats(d, empty16(2 * 7 * 7 * 64), empty16(64 * 9 * 64), t, t, None, empty16(64),
+                                empty16(64), stats)
