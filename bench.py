@@ -565,7 +565,9 @@ def ingest_traffic(csv_path):
         per.setdefault(r[ii], {})[r[mi]] = float(r[vi].replace(",", "")) * scale[r[ui]]
     from paper_1911_07384_gb300.resnet50 import conv_shapes
 
-    step = sum(2 + (0 if c == 3 else (st * st if r > 1 else 1))
+    # per conv: forward + data gradient (one GEMM per stride phase) + weight
+    # gradient; the stem has a forward only (its weight gradient is k_stem_wgrad)
+    step = sum(1 if c == 3 else 2 + (st * st if r > 1 else 1)
                for _, (_, _, _, c, _, r, _, st, _) in conv_shapes(BATCH))
     ids = sorted(per, key=int)[:step]  # the first whole step (the eager warm-up step)
     if len(ids) < step:
@@ -661,8 +663,10 @@ def conv_roofline(net, stream, reps=3):
         Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
         one = 2 * (d.n * d.h * d.w * d.c + d.k * d.r * d.s * d.c + d.n * P * Q * d.k)
         stem = d.c == 3
-        byts += one * (2 if stem else 3)
-        gemms += 2 + (0 if stem else (d.stride * d.stride if d.r > 1 else 1))
+        # the k_gemm launches the stored traffic covers: every pass but the stem's weight
+        # gradient (k_stem_wgrad)
+        byts += one * (1 if stem else 3)
+        gemms += 1 if stem else 2 + (d.stride * d.stride if d.r > 1 else 1)
     out = {"ms": ms, "gflop": gflop, "tflops": gflop / ms, "by_pass": {}, "bytes_per_launch": byts / gemms}
     for k, (t, f) in by_pass.items():
         out["by_pass"][k] = {"ms": t / reps, "tflops": (f / reps) / 1e9 / (t / reps) if t else None}
