@@ -227,7 +227,13 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
                                  uint16_t* out, long long ldo, int cols_out, cudaStream_t s) {
   int sp2 = 1;
   while (sp2 < splits) sp2 *= 2;
-  const int grp = sp2 < 32 ? sp2 : 32;
+  // Split groups per output chunk: only as many as it takes to give the GPU
+  // about 2048 threads per SM, so that a thread sums a long run of splits with
+  // batched loads instead of each CTA paying a shared-memory tree for a few
+  // loads.  Every choice sums the same balanced tree over the padded splits.
+  const long long total_chunks = rows * (cols / 8);
+  int grp = 1;
+  while (grp < sp2 && grp < 256 && total_chunks * grp < 152ll * 2048) grp *= 2;
   const int cl = 256 / grp;
   const long long total = rows * (cols / 8);
   const long long blocks = (total + cl - 1) / cl;
