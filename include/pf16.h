@@ -51,6 +51,9 @@ enum {
 
 /* ----------------------------------------------------------------- flags */
 #define PF16_ACCUMULATE 0x1u  /* conv: out = rn(out + result) instead of out = result */
+#define PF16_F32_ACCUM 0x4u   /* conv: FP32 accumulation in the tensor core, each output rounded once
+                                 to FP16 -- a contrast to the paper's pure-FP16 method (Sec. 1, 2:
+                                 the mixed-precision accumulation it does without), not part of it */
 #define PF16_BN_RELU 0x1u     /* BN: apply ReLU to the output */
 #define PF16_BN_RESIDUAL 0x2u /* BN: add the residual tensor before the ReLU */
 
@@ -78,7 +81,8 @@ size_t pf16_conv_workspace_size(const pf16_conv_desc* d, int pass);
 
 /* Forward: y[n,p,q,k] = sum_{r,s,c} x[n, p*st+r-pad, q*st+s-pad, c] * w[k,r,s,c]
  * (zero outside x).  FP16 products, FP16 accumulation in the tensor core,
- * FP16 result.  flags: PF16_ACCUMULATE. */
+ * FP16 result.  flags: PF16_ACCUMULATE, PF16_F32_ACCUM (the contrast variant:
+ * products accumulated in FP32 inside the tensor core, one rounding to FP16). */
 int pf16_conv_fwd(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
                   void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
@@ -101,6 +105,7 @@ int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint
  * its stride-phase sub-problems, so no zero-insertion work is done.  Every
  * element of dx is written (zeros included) unless PF16_ACCUMULATE, in which
  * case dx = rn(dx + result) and positions no tap reaches are left unchanged.
+ * PF16_F32_ACCUM as for the forward.
  * Not available for c == 3 (the stem needs no input gradient). */
 int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
@@ -137,7 +142,9 @@ int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const u
 /* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*st+r-pad, q*st+s-pad, c].
  * The reduction over n*p*q pixels is split into chunks, each accumulated in
  * FP16 by the tensor core into FP16 partials in the workspace, which are then
- * summed by a balanced pairwise FP16 tree.  flags: 0 (PF16_ERR_ARG otherwise). */
+ * summed by a balanced pairwise FP16 tree.  flags: 0 or PF16_F32_ACCUM (each
+ * chunk accumulated in FP32 and rounded once to its FP16 partial; the tree
+ * stays FP16); PF16_ERR_ARG otherwise. */
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 

@@ -391,7 +391,7 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
   if (p.splits == 1) p.kb_per_split = p.num_kb;
   p.idesc = idesc_f16(kBM, BN, p.a_mode == LD_TILED_MN,
                       p.b_mode == LD_TILED_MN || p.b_mode == LD_IM2COL_MN || p.b_mode == LD_TAP3D_MN,
-                      false);
+                      p.d_f32 != 0);
   const long long units = (long long)p.m_tiles * p.n_tiles * p.splits;
   if (units <= 0 || p.num_kb <= 0) return PF16_OK;
   // Row-major outputs leave through TMA stores of 32-row x 64-column boxes
@@ -492,8 +492,10 @@ int halo_width(const Shape& s, bool accum) {
 // gradient (dgrad = true: in = dy, weights viewed (C, 9, K), taps flipped)
 // through the halo engine.  in and out are N x H x W x 64.
 int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint16_t* w, uint16_t* out,
-             int* status, int sms, cudaStream_t st, void* stats = nullptr, const pf16_bn_source* bn = nullptr) {
+             int* status, int sms, cudaStream_t st, bool f32, void* stats = nullptr,
+             const pf16_bn_source* bn = nullptr) {
   GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
   set_stats(p, stats, 64);
   set_bwd_stats(p, bn);
   CUtensorMap ma, mb, mc;
@@ -522,7 +524,7 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
     set_kmajor(p, false, true);
     if (!map_2d(&mb, w, 9 * 64, 64, 9 * 64, 64, 64)) return PF16_ERR_CUDA;
   }
-  p.idesc = idesc_f16(kBM, 64, false, dgrad, false);
+  p.idesc = idesc_f16(kBM, 64, false, dgrad, f32);
   p.halo_ws = ws;
   p.halo_h = (int)H;
   p.halo_w = (int)W;
@@ -544,7 +546,7 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
 // the workspace, then a 4x4 stride-1 convolution over 16 channels with 32-byte
 // pixel rows (layouts at stem_s2d_width).  y is N x P x Q x 64.
 int run_stem_s2d(const Shape& s, int ws, const uint16_t* x, const uint16_t* w, uint16_t* y, void* work,
-                 int* status, int sms, cudaStream_t st, void* stats) {
+                 int* status, int sms, cudaStream_t st, void* stats, bool f32) {
   const long long N = s.N, P = s.P, Q = s.Q, Hs = P + 3, Wsd = Q + 3;
   uint16_t* xs = static_cast<uint16_t*>(work);
   uint16_t* wsd = xs + stem_s2d_bytes(s) / 2;
@@ -552,6 +554,7 @@ int run_stem_s2d(const Shape& s, int ws, const uint16_t* x, const uint16_t* w, u
     return PF16_ERR_CUDA;
   GemmParams p = base_params(status);
   set_stats(p, stats, 64);
+  p.d_f32 = f32 ? 1 : 0;
   CUtensorMap ma, mb, mc;
   const int rows = kBM / ws;
   cuuint64_t dims[4] = {16, (cuuint64_t)Wsd, (cuuint64_t)Hs, (cuuint64_t)N};
@@ -574,7 +577,7 @@ int run_stem_s2d(const Shape& s, int ws, const uint16_t* x, const uint16_t* w, u
   p.b_lbo = 16;
   p.b_sbo = 256;  // 8 rows of 32 bytes
   p.b_kstep = 32;
-  p.idesc = idesc_f16(kBM, 64, false, false, false);
+  p.idesc = idesc_f16(kBM, 64, false, false, f32);
   p.halo_ws = ws;
   p.halo_h = (int)P;
   p.halo_w = (int)Q;
@@ -597,7 +600,8 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, w, y)) != PF16_OK) return rc;
-  if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  if (flags & ~(PF16_ACCUMULATE | PF16_F32_ACCUM)) return PF16_ERR_ARG;
+  const bool f32 = (flags & PF16_F32_ACCUM) != 0;
   if (stats) {
     if (flags != 0) return PF16_ERR_ARG;  // statistics of a plain (non-accumulating) output only
     if (s.K % 64 != 0) return PF16_ERR_UNSUPPORTED;
@@ -614,6 +618,7 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   cudaStream_t st = static_cast<cudaStream_t>(stream);
 
   GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
   CUtensorMap ma, mb;
   p.M = (int)(s.N * s.P * s.Q);
   p.N = (int)s.K;
@@ -621,9 +626,9 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   p.ldo = s.K;
   p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
   if (const int ws = halo_width(s, (flags & PF16_ACCUMULATE) != 0))
-    return run_halo(s, ws, false, x, w, y, status, sms, st, stats);
+    return run_halo(s, ws, false, x, w, y, status, sms, st, f32, stats);
   if (const int ws_s2d = stem_s2d_width(s, (flags & PF16_ACCUMULATE) != 0))
-    return run_stem_s2d(s, ws_s2d, x, w, y, ws, status, sms, st, stats);
+    return run_stem_s2d(s, ws_s2d, x, w, y, ws, status, sms, st, stats, f32);
   set_stats(p, stats, s.K);
   const int BN = pick_bn_out(s.K);
   p.a_mode = LD_TILED_K;
@@ -691,7 +696,8 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
   if (rc != PF16_OK) return rc;
   if (s.kind == KIND_STEM) return PF16_ERR_UNSUPPORTED;
   if ((rc = check_common(dy, w, dx)) != PF16_OK) return rc;
-  if (flags & ~PF16_ACCUMULATE) return PF16_ERR_ARG;
+  if (flags & ~(PF16_ACCUMULATE | PF16_F32_ACCUM)) return PF16_ERR_ARG;
+  const bool f32 = (flags & PF16_F32_ACCUM) != 0;
   if (stats) {
     // statistics of a plain output whose rows are pixels in order (stride 1)
     if (flags != 0) return PF16_ERR_ARG;
@@ -709,13 +715,14 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const bool accum = (flags & PF16_ACCUMULATE) != 0;
   if (const int ws = halo_width(s, accum))
-    return run_halo(s, ws, true, dy, w, dx, status, sms, st, stats, stats ? bn : nullptr);
+    return run_halo(s, ws, true, dy, w, dx, status, sms, st, f32, stats, stats ? bn : nullptr);
   const int BN = pick_bn_out(s.C);
   const size_t dx_elems = (size_t)(s.N * s.H * s.W * s.C);
 
   if (s.R == 1 && s.S == 1 && s.pad == 0) {
     // 1x1: dx[n, st*p, st*q, :] = dy[n,p,q,:] . w ; other positions receive nothing
     GemmParams p = base_params(status);
+    p.d_f32 = f32 ? 1 : 0;
     set_stats(p, stats, s.C);
     if (stats) set_bwd_stats(p, bn);
     CUtensorMap ma, mb;
@@ -759,6 +766,7 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
       const int *ar = f.ar, *bs = f.bs, *rr = f.rr, *ss = f.ss;
       const int amin = *std::min_element(ar, ar + nr), bmin = *std::min_element(bs, bs + ns);
       GemmParams p = base_params(status);
+      p.d_f32 = f32 ? 1 : 0;
       set_stats(p, stats, s.C);  // stride 1 only: one phase, rows in pixel order
       if (stats) set_bwd_stats(p, bn);
       CUtensorMap ma, mb;
@@ -822,7 +830,7 @@ int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const u
 
 // The stem's weight gradient through k_stem_wgrad (layouts at stem_wgrad_plan).
 static int run_stem_wgrad(const Shape& s, const StemWgradPlan& sw, const uint16_t* x, const uint16_t* dy,
-                          uint16_t* dw, void* work, int* status, int sms, cudaStream_t st) {
+                          uint16_t* dw, void* work, int* status, int sms, cudaStream_t st, bool f32) {
   const long long N = s.N, P = s.P, Q = s.Q, Hs = P + 3, Wsd = Q + 3;
   uint16_t* xs = static_cast<uint16_t*>(work);
   uint16_t* parts = xs + stem_s2d_bytes(s) / 2;
@@ -851,7 +859,8 @@ static int run_stem_wgrad(const Shape& s, const StemWgradPlan& sw, const uint16_
       return PF16_ERR_CUDA;
   }
   GemmParams p = base_params(status);
-  p.idesc = idesc_f16(kBM, 64, true, true, false);
+  p.d_f32 = f32 ? 1 : 0;
+  p.idesc = idesc_f16(kBM, 64, true, true, f32);
   p.halo_ws = 128;
   p.halo_h = (int)P;
   p.halo_w = (int)Q;
@@ -872,7 +881,8 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, dy, dw)) != PF16_OK) return rc;
-  if (flags) return PF16_ERR_ARG;
+  if (flags & ~PF16_F32_ACCUM) return PF16_ERR_ARG;
+  const bool f32 = (flags & PF16_F32_ACCUM) != 0;
   int* status;
   int sms;
   if ((rc = device_consts(&status, &sms)) != PF16_OK) return rc;
@@ -882,10 +892,11 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   if (!driver_fns()) return PF16_ERR_CUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const StemWgradPlan sw = stem_wgrad_plan(s);
-  if (sw.ok) return run_stem_wgrad(s, sw, x, dy, dw, ws, status, sms, st);
+  if (sw.ok) return run_stem_wgrad(s, sw, x, dy, dw, ws, status, sms, st, f32);
   const WgradSplit wsp = wgrad_split(s);
 
   GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
   CUtensorMap ma, mb;
   const long long pixels = s.N * s.P * s.Q;
   p.M = (int)s.K;

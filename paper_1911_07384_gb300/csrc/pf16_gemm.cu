@@ -231,6 +231,12 @@ __device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int spl
 
 // low halves of two 32-bit TMEM words -> one f16x2
 __device__ __forceinline__ uint32_t pack_lo(uint32_t a, uint32_t b) { return __byte_perm(a, b, 0x5410); }
+// FP32 accumulator words -> binary16 (roundTiesToEven) in their low 16 bits, in place
+template <int N>
+__device__ __forceinline__ void f32_to_f16_lo(uint32_t* r) {
+#pragma unroll
+  for (int i = 0; i < N; ++i) r[i] = __half_as_ushort(__float2half_rn(__uint_as_float(r[i])));
+}
 
 
 // ---------------------------------------------------------------------------
@@ -711,6 +717,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tmem_ld16(tbase + c + 32, r + 32);
           tmem_ld16(tbase + c + 48, r + 48);
           tmem_ld_wait();
+          if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
           if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
             tc_fence_before();
             __syncwarp();
@@ -760,6 +767,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         tmem_ld16(tbase + c, r);
         tmem_ld16(tbase + c + 16, r + 16);
         tmem_ld_wait();
+        if (p.d_f32) f32_to_f16_lo<32>(r);  // FP32 accumulator: one rounding to FP16
         if (row_ok) {
 #pragma unroll
           for (int g = 0; g < 4; ++g) {
@@ -1130,6 +1138,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       tmem_ld16(tbase + 32, r + 32);
       tmem_ld16(tbase + 48, r + 48);
       tmem_ld_wait();
+      if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
@@ -1406,6 +1415,7 @@ __global__ void __launch_bounds__(kStemWgradThreads, 1)
         tmem_ld16(tbase + 32, r + 32);
         tmem_ld16(tbase + 48, r + 48);
         tmem_ld_wait();
+        if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
 #pragma unroll
         for (int j = 0; j < 8; ++j)
           dst[half * 8 + j] = make_uint4(pack_lo(r[j * 8 + 0], r[j * 8 + 1]), pack_lo(r[j * 8 + 2], r[j * 8 + 3]),

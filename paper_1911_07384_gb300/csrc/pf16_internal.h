@@ -125,6 +125,7 @@ struct GemmParams {
   int rm_gh, rm_gw, rm_H, rm_W, rm_step, rm_ph, rm_pw;
   // MMA
   uint32_t idesc;
+  int d_f32;              // FP32 accumulator in TMEM (PF16_F32_ACCUM), rounded once to FP16 in the epilogue
   uint32_t a_lbo, a_sbo, a_kstep;  // smem-descriptor strides, bytes per 16-wide k step
   uint32_t b_lbo, b_sbo, b_kstep;
   int* status;            // device status word

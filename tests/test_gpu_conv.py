@@ -10,7 +10,7 @@ import pytest
 
 from paper_1911_07384_gb300 import pf16
 from paper_1911_07384_gb300 import synthetic as syn
-from gpu_util import assert_conv_close, dev, empty16, f64, host, workspace
+from gpu_util import U, assert_conv_close, dev, empty16, f64, host, workspace
 
 pytestmark = pytest.mark.gpu
 
@@ -201,3 +201,46 @@ def test_full_size_sampled(orc, shape):
     V, A, _ = orc.conv_wgrad(x, dy, *shape, idx=idx)
     rel = assert_conv_close(dw[idx], V, A, N * P * Q, "wgrad")
     assert rel < 2.0 ** -5, rel
+
+
+F32_SHAPES = [
+    (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col, reduction 2,304, paired CTAs
+    (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine
+    (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem: space-to-depth halo forward, stem weight gradient
+    (2, 14, 14, 64, 256, 1, 1, 1, 0),    # dense 1x1
+]
+
+
+@pytest.mark.parametrize("shape", F32_SHAPES, ids=ids)
+def test_f32_accumulate_contrast(orc, shape):
+    """PF16_F32_ACCUM: FP32 accumulation inside the tensor core and one
+    rounding to FP16 per output (per partial for the weight gradient).  The
+    forward and the data gradient are then within half an FP16 ulp of the exact
+    value plus an FP32 accumulation term, the weight gradient within the
+    contract bound, and on average none is farther from the exact value than
+    the pure-FP16 result."""
+    N, H, W, C, K, R, S, st, pd = shape
+    x, w, dy, P, Q = inputs(shape, seed_cfg=5)
+    d = pf16.conv_desc(*shape)
+    f32 = pf16.PF16_F32_ACCUM
+
+    def check(g32, g16, V, A, Rn, what):
+        e32 = np.abs(f64(g32).ravel() - V)
+        e16 = np.abs(f64(g16).ravel() - V)
+        bound = U * np.abs(V) + Rn * 2.0 ** -22 * A + 2.0 ** -24
+        assert np.all(e32 <= bound), (what, float(np.max(e32 / bound)))
+        assert e32.mean() <= e16.mean(), (what, e32.mean(), e16.mean())
+
+    V, A, _ = orc.conv_fwd(x, w, *shape)
+    check(run_fwd(d, x, w, f32), run_fwd(d, x, w), V, A, C * R * S, "fwd")
+    if C != 3:
+        V, A, T = orc.conv_dgrad(dy, w, *shape)
+        check(run_dgrad(d, dy, w, f32), run_dgrad(d, dy, w), V, A, np.maximum(T, 1), "dgrad")
+    dw16 = run_wgrad(d, x, dy)
+    dw32 = empty16(d.k * d.r * d.s * d.c)
+    pf16.conv_wgrad(d, dev(x), dev(dy), dw32, workspace(pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)),
+                    f32)
+    assert pf16.sync_status() == 0
+    V, A, _ = orc.conv_wgrad(x, dy, *shape)
+    assert_conv_close(host(dw32), V, A, N * P * Q, "wgrad f32")
+    assert np.abs(f64(host(dw32)).ravel() - V).mean() <= np.abs(f64(dw16).ravel() - V).mean()
