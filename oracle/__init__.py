@@ -80,6 +80,9 @@ def _L():
                                        ctypes.c_double, I, f64p, f64p, f64p, f64p]
             lib.orc_bn_bwd.argtypes = [u16p, u16p, u16p, u16p, ctypes.c_int64, I, ctypes.c_double,
                                        ctypes.c_double, I, f64p, f64p, f64p, f64p]
+            lib.orc_bn_fwd_swap.argtypes = lib.orc_bn_fwd.argtypes
+            lib.orc_bn_bwd_swap.argtypes = [u16p, u16p, u16p, u16p, u16p, ctypes.c_int64, I, ctypes.c_double,
+                                            ctypes.c_double, I, f64p, f64p, f64p, f64p]
             lib.orc_maxpool_fwd.argtypes = [u16p, I, I, I, I, f64p]
             lib.orc_maxpool_bwd.argtypes = [u16p, u16p, I, I, I, I, f64p, f64p]
             lib.orc_avgpool_fwd.argtypes = [u16p, I, I, I, f64p]
@@ -183,6 +186,33 @@ def sgd_update(w, v, g, lr_bits: int, momentum_bits: int, wd_bits: int):
 
 
 # ---------------------------------------------------------------- BatchNorm
+def bn_fwd_swap(x, gamma, beta, residual, R, C, eps, s, relu):
+    """The swap variant (Sec. 4.1): y = gamma*(s*xhat + residual) + beta [, ReLU].
+    Returns y[R,C], mean[C], var[C], invstd[C] (all binary64)."""
+    x, gamma, beta, residual = _u16(x), _u16(gamma), _u16(beta), _u16(residual)
+    y = np.empty(R * C, np.float64)
+    mean, var, invstd = (np.empty(C, np.float64) for _ in range(3))
+    _L().orc_bn_fwd_swap(_p(x, ctypes.c_uint16), _p(gamma, ctypes.c_uint16), _p(beta, ctypes.c_uint16),
+                         _p(residual, ctypes.c_uint16), R, C, float(eps), float(s), int(relu),
+                         _p(y, ctypes.c_double), _p(mean, ctypes.c_double), _p(var, ctypes.c_double),
+                         _p(invstd, ctypes.c_double))
+    return y.reshape(R, C), mean, var, invstd
+
+
+def bn_bwd_swap(x, gamma, dy, y_saved, residual, R, C, eps, s, relu):
+    """Backward of bn_fwd_swap.  Returns dx[R,C], dgamma[C], dbeta[C], dres[R,C] (binary64)."""
+    x, gamma, dy, residual = _u16(x), _u16(gamma), _u16(dy), _u16(residual)
+    y_saved = _u16(y_saved) if y_saved is not None else np.zeros(1, np.uint16)
+    dx = np.empty(R * C, np.float64)
+    dres = np.empty(R * C, np.float64)
+    dg, db = np.empty(C, np.float64), np.empty(C, np.float64)
+    _L().orc_bn_bwd_swap(_p(x, ctypes.c_uint16), _p(gamma, ctypes.c_uint16), _p(dy, ctypes.c_uint16),
+                         _p(y_saved, ctypes.c_uint16), _p(residual, ctypes.c_uint16), R, C, float(eps), float(s),
+                         int(relu), _p(dx, ctypes.c_double), _p(dg, ctypes.c_double), _p(db, ctypes.c_double),
+                         _p(dres, ctypes.c_double))
+    return dx.reshape(R, C), dg, db, dres.reshape(R, C)
+
+
 def bn_fwd(x, gamma, beta, residual, R, C, eps, s, relu):
     """Returns y[R,C], mean[C], var[C], invstd[C] (all binary64)."""
     x, gamma, beta = _u16(x), _u16(gamma), _u16(beta)

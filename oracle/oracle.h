@@ -53,6 +53,16 @@ void orc_bn_bwd(const uint16_t* x, const uint16_t* gamma, const uint16_t* dy,
                 const uint16_t* y_saved, int64_t R, int C, double eps, double s, int relu,
                 double* dx, double* dgamma, double* dbeta, double* dres);
 
+/* The "swap" variant of a residual block's last BatchNorm (Sec. 4.1: the
+ * residual connection and gamma change places): y = gamma * (s * xhat + r) +
+ * beta, then optional ReLU; r is the residual input (required). */
+void orc_bn_fwd_swap(const uint16_t* x, const uint16_t* gamma, const uint16_t* beta,
+                     const uint16_t* residual, int64_t R, int C, double eps, double s, int relu,
+                     double* y, double* mean, double* var, double* invstd);
+void orc_bn_bwd_swap(const uint16_t* x, const uint16_t* gamma, const uint16_t* dy,
+                     const uint16_t* y_saved, const uint16_t* residual, int64_t R, int C, double eps,
+                     double s, int relu, double* dx, double* dgamma, double* dbeta, double* dres);
+
 /* 3x3 stride-2 pad-1 max pooling (padding never wins) and its backward. */
 void orc_maxpool_fwd(const uint16_t* x, int N, int H, int W, int C, double* y);
 void orc_maxpool_bwd(const uint16_t* x, const uint16_t* dy, int N, int H, int W, int C, double* dx,

@@ -263,6 +263,82 @@ void orc_bn_bwd(const uint16_t* x, const uint16_t* gamma, const uint16_t* dy,
   }
 }
 
+/* BatchNorm "swap" (Sec. 4.1: the residual connection and gamma swap places
+ * in a block's last BatchNorm), read as
+ *   u = s * xhat + r,   z = gamma * u + beta,   y = relu ? max(z, 0) : z
+ * with the same batch statistics of x as orc_bn_fwd. */
+void orc_bn_fwd_swap(const uint16_t* x, const uint16_t* gamma, const uint16_t* beta,
+                     const uint16_t* residual, int64_t R, int C, double eps, double s, int relu,
+                     double* y, double* mean, double* var, double* invstd) {
+  const double* lut = orc_f16_lut();
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int c = 0; c < C; ++c) {
+    double sum = 0.0;
+    for (int64_t r = 0; r < R; ++r) sum += lut[x[r * C + c]];
+    const double mu = sum / (double)R;
+    double sq = 0.0;
+    for (int64_t r = 0; r < R; ++r) {
+      const double d = lut[x[r * C + c]] - mu;
+      sq += d * d;
+    }
+    const double va = sq / (double)R;
+    const double is = 1.0 / sqrt(va + eps);
+    mean[c] = mu;
+    var[c] = va;
+    invstd[c] = is;
+    const double g = lut[gamma[c]], b = lut[beta[c]];
+    for (int64_t r = 0; r < R; ++r) {
+      const double xh = (lut[x[r * C + c]] - mu) * is;
+      double z = g * (s * xh + lut[residual[r * C + c]]) + b;
+      if (relu && !(z > 0.0)) z = 0.0;
+      y[r * C + c] = z;
+    }
+  }
+}
+
+/* Its backward, by the chain rule through u and z:
+ *   dz     = dy * [y_saved > 0]          (dz = dy without relu)
+ *   dbeta  = sum dz,   dgamma = sum dz * u = s * sum dz * xhat + sum dz * r
+ *   dres   = gamma * dz                  (gradient of the residual input)
+ *   dx     = s*gamma*invstd * (dz - mean(dz) - xhat * mean(dz * xhat)) */
+void orc_bn_bwd_swap(const uint16_t* x, const uint16_t* gamma, const uint16_t* dy,
+                     const uint16_t* y_saved, const uint16_t* residual, int64_t R, int C, double eps,
+                     double s, int relu, double* dx, double* dgamma, double* dbeta, double* dres) {
+  const double* lut = orc_f16_lut();
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int c = 0; c < C; ++c) {
+    double sum = 0.0;
+    for (int64_t r = 0; r < R; ++r) sum += lut[x[r * C + c]];
+    const double mu = sum / (double)R;
+    double sq = 0.0;
+    for (int64_t r = 0; r < R; ++r) {
+      const double d = lut[x[r * C + c]] - mu;
+      sq += d * d;
+    }
+    const double is = 1.0 / sqrt(sq / (double)R + eps);
+    double s1 = 0.0, s2 = 0.0, s3 = 0.0;
+    for (int64_t r = 0; r < R; ++r) {
+      double d = lut[dy[r * C + c]];
+      if (relu && !(lut[y_saved[r * C + c]] > 0.0)) d = 0.0;
+      const double xh = (lut[x[r * C + c]] - mu) * is;
+      s1 += d;
+      s2 += d * xh;
+      s3 += d * lut[residual[r * C + c]];
+    }
+    const double g = lut[gamma[c]];
+    dbeta[c] = s1;
+    dgamma[c] = s * s2 + s3;
+    const double m1 = s1 / (double)R, m2 = s2 / (double)R;
+    for (int64_t r = 0; r < R; ++r) {
+      double d = lut[dy[r * C + c]];
+      if (relu && !(lut[y_saved[r * C + c]] > 0.0)) d = 0.0;
+      const double xh = (lut[x[r * C + c]] - mu) * is;
+      dx[r * C + c] = s * g * is * (d - m1 - xh * m2);
+      if (dres) dres[r * C + c] = g * d;
+    }
+  }
+}
+
 /* Max pooling, 3x3 window, stride 2, padding 1 (padded cells never win). */
 void orc_maxpool_fwd(const uint16_t* x, int N, int H, int W, int C, double* y) {
   const double* lut = orc_f16_lut();

@@ -6,7 +6,10 @@ invariants (mean(xhat) = 0, var(xhat) = var/(var+eps)), the backward
 invariants (sum dx = 0; sum dx*xhat = gamma*invstd*dgamma*eps/(var+eps), which
 is 0 for eps = 0), and a central finite-difference
 check of the backward against the forward on inputs whose perturbations are
-exact in binary16."""
+exact in binary16.  The swap variant of a block's last BatchNorm (Sec. 4.1,
+gamma * (s * xhat + r) + beta) is pinned by its reduction to the plain one at
+gamma = 1, beta = 0, its closed forms (constant channel, gamma = 0) and the
+same finite-difference check, which also covers the residual gradient."""
 import numpy as np
 import pytest
 
@@ -137,3 +140,80 @@ def test_relu_mask_and_residual_gradient(orc):
     dy_masked = f16(np.where(mask, dyf, 0.0))
     dx_r, dg_r, db_r, _ = orc.bn_bwd(x, g, dy_masked, None, R, C, EPS, 0.25, False)
     assert np.array_equal(dx_m, dx_r) and np.array_equal(dg_m, dg_r) and np.array_equal(db_m, db_r)
+
+
+# ------------------------------------------------------------ swap variant
+def test_swap_with_unit_gamma_zero_beta_is_the_plain_batchnorm(orc):
+    """gamma = 1, beta = 0: gamma*(s*xhat + r) + beta = s*(gamma*xhat + beta) + r, so the
+    swap forward, dx and dres equal the plain ones, and dbeta = plain dbeta / s."""
+    R, C, s = 96, 3, 0.25
+    x = syn.normal_f16(21, (R, C))
+    res = syn.normal_f16(22, (R, C))
+    dy = syn.normal_f16(23, (R, C), 0.1)
+    g, b = f16(np.ones(C)), f16(np.zeros(C))
+    y0, *_ = orc.bn_fwd(x, g, b, res, R, C, EPS, s, True)
+    y1, *_ = orc.bn_fwd_swap(x, g, b, res, R, C, EPS, s, True)
+    assert np.array_equal(y0, y1)
+    ys = f16(y0)
+    dx0, dg0, db0, dr0 = orc.bn_bwd(x, g, dy, ys, R, C, EPS, s, True)
+    dx1, dg1, db1, dr1 = orc.bn_bwd_swap(x, g, dy, ys, res, R, C, EPS, s, True)
+    assert np.array_equal(dx0, dx1) and np.array_equal(dr0, dr1)
+    assert np.allclose(db1, db0 / s, rtol=1e-15, atol=0)
+
+
+def test_swap_constant_channel_and_zero_gamma(orc):
+    """A constant channel has xhat = 0, so y = gamma*r + beta; gamma = 0 gives y = beta
+    whatever x and r are (with the zero-gamma initialisation the block output is beta)."""
+    R, C = 40, 2
+    x = f16(np.tile([1.5, -2.0], (R, 1)))
+    res = syn.normal_f16(24, (R, C))
+    rf = res.view(np.float16).astype(np.float64).reshape(R, C)
+    g, b = f16([2.0, -0.5]), f16([0.25, 1.0])
+    y, *_ = orc.bn_fwd_swap(x, g, b, res, R, C, EPS, 0.25, False)
+    assert np.allclose(y, rf * np.array([2.0, -0.5]) + np.array([0.25, 1.0]), rtol=0, atol=1e-15)
+    x2 = syn.normal_f16(25, (R, C))
+    y2, *_ = orc.bn_fwd_swap(x2, f16([0.0, 0.0]), b, res, R, C, EPS, 0.25, False)
+    assert np.array_equal(y2, np.tile([0.25, 1.0], (R, 1)))
+
+
+@pytest.mark.parametrize("s", [1.0, 0.25])
+def test_swap_backward_matches_finite_differences(orc, s):
+    R, C = 24, 3
+    x = _grid_x(27, R, C)
+    res = _grid_x(28, R, C)
+    gamma, beta = f16([1.0, 0.75, 1.25]), f16([0.5, -0.25, 0.0])
+    u = syn.normal_f16(29, (R, C), 1.0)
+    uf = u.view(np.float16).astype(np.float64)
+
+    def L(xb, gb=gamma, bb=beta, rb=res):
+        y, *_ = orc.bn_fwd_swap(xb, gb, bb, rb, R, C, EPS, s, False)
+        return float(np.sum(y * uf))
+
+    dx, dg, db, dr = orc.bn_bwd_swap(x, gamma, u, None, res, R, C, EPS, s, False)
+    h = 2.0 ** -10
+    xf = x.view(np.float16).astype(np.float64)
+    rf = res.view(np.float16).astype(np.float64)
+    for i in [0, 5, 17, 40, 71]:
+        r, c = divmod(i, C)
+        xp, xm = xf.copy(), xf.copy()
+        xp[r, c] += h
+        xm[r, c] -= h
+        fd = (L(f16(xp)) - L(f16(xm))) / (2 * h)
+        assert abs(fd - dx[r, c]) <= 2e-4 * (np.abs(dx).max() + 1e-30), (i, fd, dx[r, c])
+        rp, rm = rf.copy(), rf.copy()
+        rp[r, c] += h
+        rm[r, c] -= h
+        fdr = (L(x, rb=f16(rp)) - L(x, rb=f16(rm))) / (2 * h)
+        assert abs(fdr - dr[r, c]) <= 1e-9 * (abs(dr[r, c]) + 1), (i, fdr, dr[r, c])
+    gf = gamma.view(np.float16).astype(np.float64)
+    bf = beta.view(np.float16).astype(np.float64)
+    for c in range(C):
+        gp, gm, bp, bm = gf.copy(), gf.copy(), bf.copy(), bf.copy()
+        gp[c] += h
+        gm[c] -= h
+        bp[c] += h
+        bm[c] -= h
+        fdg = (L(x, f16(gp), beta) - L(x, f16(gm), beta)) / (2 * h)
+        fdb = (L(x, gamma, f16(bp)) - L(x, gamma, f16(bm))) / (2 * h)
+        assert abs(fdg - dg[c]) <= 1e-6 * (abs(dg[c]) + 1), (c, fdg, dg[c])
+        assert abs(fdb - db[c]) <= 1e-9 * (abs(db[c]) + 1), (c, fdb, db[c])
