@@ -168,6 +168,8 @@ def main():
     ap.add_argument("--bn", default=None,
                     help="time one BatchNorm pass instead of the step: N,H,W,C (ReLU + residual, s=0.25)")
     ap.add_argument("--bn-pass", default="fwd", choices=["fwd", "bwd"])
+    ap.add_argument("--bn-swap", action="store_true",
+                    help="the BN-swap variant (Sec. 4.1) in every block's last BatchNorm (off in the headline run)")
     ap.add_argument("--layers", action="store_true",
                     help="per-layer CUDA-event times of one eager step (median of 3), one JSON line each")
     ap.add_argument("--ingest-traffic", default=None, metavar="CSV",
@@ -214,7 +216,7 @@ def main():
     from paper_1911_07384_gb300.resnet50 import ResNet50
 
     N = args.batch
-    net = ResNet50(batch=N, seed_cfg=4)
+    net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap)
     imgs = syn.images_f16(syn.seed_for(4, "x", rank), N)
     labs = syn.labels(syn.seed_for(4, "labels", rank), N)
     net.set_batch(imgs, labs)
@@ -303,7 +305,8 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": N * world, "per_gpu_batch": N,
                    "image": "224x224x3 NHWC", "parallelism": f"replicas{world}" if world > 1 else "single",
-                   "l2": "working set (~25 GB of activations per step) far larger than L2; no flush needed"},
+                   "l2": "working set (~25 GB of activations per step) far larger than L2; no flush needed",
+                   **({"bn_swap": True} if args.bn_swap else {})},
         "loss": loss,
         "clocks": clocks.summary(),
         "e2e": e2e,
@@ -614,7 +617,9 @@ def count_launches(net):
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
         total += 1 + (1 if ws else 0) + (2 if stem else 0)  # wgrad (+ split-K reduce, + the stem's s2d, scatter)
     # forward statistics come from the conv; backward ones from the data gradient where fused
-    total += sum(per["bn_fwd"] + per["bn_bwd"] - (1 if getattr(b, "fused_bwd", False) else 0) for b in net.bns)
+    # (the swap variant's backward takes a second statistics pass)
+    total += sum(per["bn_fwd"] + per["bn_bwd"] - (1 if getattr(b, "fused_bwd", False) else 0)
+                 + (1 if b.desc.flags & pf16.PF16_BN_SWAP else 0) for b in net.bns)
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]
     return total

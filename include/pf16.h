@@ -56,6 +56,8 @@ enum {
                                  the mixed-precision accumulation it does without), not part of it */
 #define PF16_BN_RELU 0x1u     /* BN: apply ReLU to the output */
 #define PF16_BN_RESIDUAL 0x2u /* BN: add the residual tensor before the ReLU */
+#define PF16_BN_SWAP 0x4u     /* BN, with PF16_BN_RESIDUAL: the "swap" variant of a block's last
+                                 BatchNorm (Sec. 4.1): y = gamma*(s*xhat + residual) + beta */
 
 /* ------------------------------------------------------------ convolution
  * Convolution of the ResNet-50 layers (Sec. 5.1) in pure FP16 (Sec. 5.2):
@@ -209,6 +211,12 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
  *       non-NULL, dresidual (= dy masked by ReLU, the gradient flowing to the
  *       residual input).  Both sources give bit-identical results; the mask
  *       moves 1/16 of the bytes.
+ *   PF16_BN_SWAP (with PF16_BN_RESIDUAL; Sec. 4.1's switch, off in the
+ *       paper's best runs): the forward is y = gamma * (s*xhat + residual) +
+ *       beta [, ReLU]; the backward also reads residual and gives dbeta =
+ *       sum dy', dgamma = rn(rn(s * sum dy'*xhat) + sum dy'*residual) (a second
+ *       statistics pass) and dresidual = gamma * dy'; dx is unchanged in form.
+ *       conv_stats is not accepted in its phase 1 (PF16_ERR_UNSUPPORTED).
  * relu_mask is ignored without PF16_BN_RELU (the bit mask is a storage
  * choice of this library, not part of the paper's method).
  * conv_stats (optional, 16-byte aligned):

@@ -971,7 +971,8 @@ static int bn_validate(const pf16_bn_desc* d, BnLaunch* b) {
   if (!d) return PF16_ERR_NULL;
   if (d->n <= 0 || d->h <= 0 || d->w <= 0 || d->c <= 0) return PF16_ERR_SHAPE;
   if (d->c % 8 != 0 || d->c > 2048) return PF16_ERR_UNSUPPORTED;
-  if (d->flags & ~(uint32_t)(PF16_BN_RELU | PF16_BN_RESIDUAL)) return PF16_ERR_ARG;
+  if (d->flags & ~(uint32_t)(PF16_BN_RELU | PF16_BN_RESIDUAL | PF16_BN_SWAP)) return PF16_ERR_ARG;
+  if ((d->flags & PF16_BN_SWAP) && !(d->flags & PF16_BN_RESIDUAL)) return PF16_ERR_ARG;
   const long long R = (long long)d->n * d->h * d->w;
   if (R * d->c > (1ll << 34) || R > (1ll << 31) - 1) return PF16_ERR_SHAPE;
   bn_plan((int)R, d->c, b);
@@ -979,6 +980,7 @@ static int bn_validate(const pf16_bn_desc* d, BnLaunch* b) {
   b->post_scale = d->post_scale;
   b->relu = (d->flags & PF16_BN_RELU) ? 1 : 0;
   b->residual = (d->flags & PF16_BN_RESIDUAL) ? 1 : 0;
+  b->swap = (d->flags & PF16_BN_SWAP) ? 1 : 0;
   return PF16_OK;
 }
 
@@ -1033,11 +1035,16 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
   if (b.relu && !bits && !aligned16(t->y_saved)) return PF16_ERR_ALIGN;
   if (t->dresidual && !aligned16(t->dresidual)) return PF16_ERR_ALIGN;
   if (t->conv_stats && !aligned16(t->conv_stats)) return PF16_ERR_ALIGN;
+  if (b.swap) {  // the swap backward reads the residual input, and takes no partial statistics
+    if (!t->residual) return PF16_ERR_NULL;
+    if (!aligned16(t->residual)) return PF16_ERR_ALIGN;
+    if (t->conv_stats) return PF16_ERR_UNSUPPORTED;
+  }
   if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
   return launch_bn_bwd(b, t->x, t->gamma, t->mean, t->invstd, t->dy,
                        b.relu && !bits ? t->y_saved : nullptr, bits ? t->relu_mask : nullptr, t->dx,
                        t->dgamma, t->dbeta, t->dresidual, static_cast<uint16_t*>(ws), st,
-                       static_cast<const uint8_t*>(t->conv_stats)) ==
+                       static_cast<const uint8_t*>(t->conv_stats), b.swap ? t->residual : nullptr) ==
                  cudaSuccess
              ? PF16_OK
              : PF16_ERR_CUDA;

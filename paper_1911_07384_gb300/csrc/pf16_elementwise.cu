@@ -530,6 +530,7 @@ struct BnStatArgs {
   uint16_t* dgamma;
   uint16_t* dbeta;
   uint16_t* mm;         // backward: mean(dy'), mean(dy' xhat) for the apply pass, [2][C]
+  uint16_t* ws4;        // backward, swap variant: per-CTA trees of dy' * residual [blocks][C], else null
 };
 
 __device__ __forceinline__ uint4 tree8(uint4* v) {
@@ -748,7 +749,9 @@ enum BnRelu : int { BN_NO_RELU = 0, BN_RELU_SAVED = 1, BN_RELU_BITS = 2 };
 // Backward statistics, same consumer layout.  The ReLU decisions of the next
 // chunk (bit-mask bytes, or saved-output vectors) are loaded from global
 // memory while the current chunk is reduced.
-template <int RELU>
+// XRAW (the swap variant's second pass, x = the residual input): the second
+// tree sums dy' * x itself instead of dy' * xhat.
+template <int RELU, bool XRAW = false>
 __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats(const BnStatArgs a) {
   pdl_wait();
   extern __shared__ __align__(128) uint8_t stat_smem[];
@@ -765,7 +768,7 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
   const int cg = t % g.tc, rg = t / g.tc;
   const bool active = t < g.tc * g.rpb;
   uint4 mu = zero4(), is = zero4();
-  if (active) {
+  if (active && !XRAW) {
     mu = __ldg(reinterpret_cast<const uint4*>(a.mean_in) + cg);
     is = __ldg(reinterpret_cast<const uint4*>(a.invstd_in) + cg);
   }
@@ -817,7 +820,7 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
       }
       if (RELU == BN_RELU_BITS) dv = and4(dv, bits_mask4(mcur[i]));
       if (RELU == BN_RELU_SAVED) dv = and4(dv, relu_mask4(ycur[i]));
-      const uint4 xh = mul4v(sub4(xv, mu), is);
+      const uint4 xh = XRAW ? xv : mul4v(sub4(xv, mu), is);
       p1[i] = dv;
       p2[i] = okr ? mul4v(dv, xh) : zero4();
     }
@@ -956,40 +959,47 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs
 }
 
 // Backward: halving trees over the per-CTA padded means (zero padding is
-// exact for sums), then means (x rn(2^L/R)) and sums (x 2^L exactly).
+// exact for sums), then means (x rn(2^L/R)) and sums (x 2^L exactly).  Swap
+// variant (a.ws4): dbeta = sum dy' (no post_scale) and dgamma =
+// rn(rn(s * sum dy' xhat) + sum dy' r), the third tree over a.ws4.
 __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs a) {
   pdl_wait();
-  __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
+  __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads], s3[kFinalThreads];
   const int tc = a.C / 8, cg = blockIdx.x, t = threadIdx.x;
   const int nthr = a.blocks_pow2 < kFinalThreads ? a.blocks_pow2 : kFinalThreads;
   const int seg = a.blocks_pow2 / nthr;
+  const bool swap = a.ws4 != nullptr;
   if (t < nthr) {
-    Tree4<12, true> t1, t2;
+    Tree4<12, true> t1, t2, t3;
     for (int i0 = 0; i0 < seg; i0 += 4) {
-      uint4 p[4], q[4];
+      uint4 p[4], q[4], w[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const int b = t * seg + i0 + i;
         const bool ok = (i0 + i < seg) && b < a.blocks;
         p[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws1) + (long long)b * tc + cg) : zero4();
         q[i] = ok ? __ldg(reinterpret_cast<const uint4*>(a.ws2) + (long long)b * tc + cg) : zero4();
+        w[i] = (ok && swap) ? __ldg(reinterpret_cast<const uint4*>(a.ws4) + (long long)b * tc + cg) : zero4();
       }
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         if (i0 + i >= seg) break;
         t1.push(p[i]);
         t2.push(q[i]);
+        if (swap) t3.push(w[i]);
       }
     }
     const int lv = 31 - __clz(seg);
     s1[t] = t1.finish(lv);
     s2[t] = t2.finish(lv);
+    s3[t] = swap ? t3.finish(lv) : zero4();
   }
   __syncthreads();
   for (int half = nthr / 2; half >= 1; half /= 2) {
     if (t < half) {
       s1[t] = hmerge4(s1[t], s1[t + half]);
       s2[t] = hmerge4(s2[t], s2[t + half]);
+      if (swap) s3[t] = hmerge4(s3[t], s3[t + half]);
     }
     __syncthreads();
   }
@@ -997,8 +1007,14 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
     const uint32_t ratio2 = dup2(a.ratio), ps = dup2(a.post_scale);
     reinterpret_cast<uint4*>(a.mm)[cg] = mul4(s1[0], ratio2);
     reinterpret_cast<uint4*>(a.mm)[tc + cg] = mul4(s2[0], ratio2);
-    reinterpret_cast<uint4*>(a.dbeta)[cg] = mul4(ldexp4(s1[0], a.total_levels), ps);
-    reinterpret_cast<uint4*>(a.dgamma)[cg] = mul4(ldexp4(s2[0], a.total_levels), ps);
+    const uint4 sum1 = ldexp4(s1[0], a.total_levels), sum2 = ldexp4(s2[0], a.total_levels);
+    if (swap) {
+      reinterpret_cast<uint4*>(a.dbeta)[cg] = sum1;
+      reinterpret_cast<uint4*>(a.dgamma)[cg] = add4(mul4(sum2, ps), ldexp4(s3[0], a.total_levels));
+    } else {
+      reinterpret_cast<uint4*>(a.dbeta)[cg] = mul4(sum1, ps);
+      reinterpret_cast<uint4*>(a.dgamma)[cg] = mul4(sum2, ps);
+    }
   }
 }
 
@@ -1133,7 +1149,7 @@ __global__ void __launch_bounds__(256)
                const uint16_t* __restrict__ beta, const uint16_t* __restrict__ mean,
                const uint16_t* __restrict__ invstd, const uint16_t* __restrict__ residual,
                uint16_t* __restrict__ y, uint8_t* __restrict__ mask, int R, int C, int rpb,
-               uint16_t post_scale, int relu) {
+               uint16_t post_scale, int relu, int swap) {
   pdl_wait();
   const int tc = C / 8;
   const int t = threadIdx.x;
@@ -1160,8 +1176,13 @@ __global__ void __launch_bounds__(256)
       const long long r = row0 + rg + (long long)(h + i) * rpb;
       if (r >= R) break;
       const uint4 xh = mul4v(sub4(xv[i], mu), is);      // Eq. 1
-      uint4 z = mul4(add4(mul4v(ga, xh), be), ps);      // Eq. 2, then x post_scale
-      if (residual) z = add4(z, rv[i]);
+      uint4 z;
+      if (swap)  // Sec. 4.1: gamma * (s * xhat + residual) + beta
+        z = add4(mul4v(ga, add4(mul4(xh, ps), rv[i])), be);
+      else {
+        z = mul4(add4(mul4v(ga, xh), be), ps);          // Eq. 2, then x post_scale
+        if (residual) z = add4(z, rv[i]);
+      }
       if (relu) {
         uint32_t bits;
         z = relu_bits(z, bits);
@@ -1179,7 +1200,7 @@ __global__ void __launch_bounds__(256)
                    const uint16_t* __restrict__ dy, const uint16_t* __restrict__ y_saved,
                    const uint8_t* __restrict__ mask, const uint16_t* __restrict__ mm,
                    uint16_t* __restrict__ dx, uint16_t* __restrict__ dres, int R, int C, int rpb,
-                   uint16_t post_scale) {
+                   uint16_t post_scale, int swap) {
   pdl_wait();
   const int tc = C / 8;
   const int t = threadIdx.x;
@@ -1218,7 +1239,7 @@ __global__ void __launch_bounds__(256)
       const uint4 tt = sub4(sub4(d, m1), mul4v(xh, m2));  // dy' - mean(dy') - xhat*mean(dy'*xhat)
       const long long off = r * tc + cg;
       reinterpret_cast<uint4*>(dx)[off] = mul4v(k, tt);
-      if (dres) reinterpret_cast<uint4*>(dres)[off] = d;
+      if (dres) reinterpret_cast<uint4*>(dres)[off] = swap ? mul4v(ga, d) : d;  // swap: gamma * dy' 
     }
   }
 }
@@ -1258,7 +1279,8 @@ void bn_plan(int R, int C, BnLaunch* b) {
 // [ws1: blocks*C] [ws2: blocks*C] [mm: 2*C]
 size_t bn_ws_bytes(const BnLaunch& b) {
   const size_t blocks = (size_t)(b.fwd.blocks > b.bwd.blocks ? b.fwd.blocks : b.bwd.blocks);
-  return 256 + 2 * blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) + 256;
+  // [ws1][ws2][mm] (+ the swap variant's second pass: [ws3][ws4])
+  return 256 + (b.swap ? 4 : 2) * blocks * b.C * sizeof(uint16_t) + (size_t)2 * b.C * sizeof(uint16_t) + 256;
 }
 
 static uint16_t f16_bits_host(float f) {
@@ -1320,7 +1342,7 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   const int rows = g.rpb * kApplyRows;
   launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
-      b.post_scale, b.relu);
+      b.post_scale, b.relu, b.swap);
   return counted_launches(3);
 }
 
@@ -1333,16 +1355,35 @@ cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_sta
   const int rows = g.rpb * kApplyRows;
   launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
-      b.post_scale, b.relu);
+      b.post_scale, b.relu, b.swap);
   return counted_launches(2);
+}
+
+// One backward statistics pass of mode RELU (XRAW: the second tree sums dy' * x).
+template <int RELU, bool XRAW>
+static cudaError_t bwd_stats_pass(const BnStatArgs& a, const BnLaunch& b, cudaStream_t s) {
+  static bool attr[64] = {false};
+  const int smem = stat_smem_bytes(2);
+  cudaError_t e = stat_smem_attr(k_bn_bwd_stats<RELU, XRAW>, smem, attr);
+  if (e != cudaSuccess) return e;
+  const BnGeom g = bn_geom(b.C);
+  launch_pdl(k_bn_bwd_stats<RELU, XRAW>, dim3(b.bwd.blocks), dim3((unsigned)(g.threads + 32)), smem, s, a);
+  return cudaSuccess;
+}
+template <bool XRAW>
+static cudaError_t bwd_stats_mode(int mode, const BnStatArgs& a, const BnLaunch& b, cudaStream_t s) {
+  switch (mode) {
+    case BN_NO_RELU: return bwd_stats_pass<BN_NO_RELU, XRAW>(a, b, s);
+    case BN_RELU_SAVED: return bwd_stats_pass<BN_RELU_SAVED, XRAW>(a, b, s);
+    default: return bwd_stats_pass<BN_RELU_BITS, XRAW>(a, b, s);
+  }
 }
 
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
                           const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
                           uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
-                          cudaStream_t s, const uint8_t* dgrad_stats) {
-  static bool attr[3][64] = {{false}};
+                          cudaStream_t s, const uint8_t* dgrad_stats, const uint16_t* residual) {
   BnStatArgs a = bn_args(b, b.bwd, ws);
   a.x = x;
   a.dy = dy;
@@ -1354,10 +1395,8 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   a.dbeta = dbeta;
   const BnGeom g = bn_geom(b.C);
   const int mode = !b.relu ? BN_NO_RELU : (relu_mask ? BN_RELU_BITS : BN_RELU_SAVED);
-  const int smem = stat_smem_bytes(2);
   const int rows = g.rpb * kApplyRows;
   const unsigned apply_blocks = (unsigned)((b.R + rows - 1) / rows);
-  const unsigned threads = (unsigned)(g.threads + 32);
   cudaError_t e = cudaSuccess;
   int launches = 3;
   if (dgrad_stats) {
@@ -1365,34 +1404,33 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
     launch_pdl(k_bn_bwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, dgrad_stats, b.C, b.R,
                b.post_scale, a.mm, dgamma, dbeta);
     launches = 2;
-  } else switch (mode) {
-    case BN_NO_RELU:
-      e = stat_smem_attr(k_bn_bwd_stats<BN_NO_RELU>, smem, attr[0]);
-      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_NO_RELU>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
-      break;
-    case BN_RELU_SAVED:
-      e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_SAVED>, smem, attr[1]);
-      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_RELU_SAVED>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
-      break;
-    default:
-      e = stat_smem_attr(k_bn_bwd_stats<BN_RELU_BITS>, smem, attr[2]);
-      if (e == cudaSuccess) launch_pdl(k_bn_bwd_stats<BN_RELU_BITS>, dim3(b.bwd.blocks), dim3(threads), smem, s, a);
-      break;
+  } else {
+    if ((e = bwd_stats_mode<false>(mode, a, b, s)) != cudaSuccess) return e;
+    if (b.swap) {
+      // the swap variant's dgamma also needs sum dy' * residual: the same pass over
+      // (residual, dy) with the raw second tree, into its own per-CTA buffers
+      BnStatArgs a2 = a;
+      a2.x = residual;
+      a2.ws1 = a.mm + 2 * (size_t)b.C;
+      a2.ws2 = a2.ws1 + (size_t)b.bwd.blocks * b.C;
+      a.ws4 = a2.ws2;
+      if ((e = bwd_stats_mode<true>(mode, a2, b, s)) != cudaSuccess) return e;
+      ++launches;
+    }
+    launch_pdl(k_bn_bwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a);
   }
-  if (e != cudaSuccess) return e;
-  if (!dgrad_stats) launch_pdl(k_bn_bwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a);
   switch (mode) {
     case BN_NO_RELU:
       launch_pdl(k_bn_bwd_apply<BN_NO_RELU>, dim3(apply_blocks), dim3(g.threads), 0, s, 
-          x, gamma, mean, invstd, dy, nullptr, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+          x, gamma, mean, invstd, dy, nullptr, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale, b.swap);
       break;
     case BN_RELU_SAVED:
       launch_pdl(k_bn_bwd_apply<BN_RELU_SAVED>, dim3(apply_blocks), dim3(g.threads), 0, s, 
-          x, gamma, mean, invstd, dy, y_saved, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+          x, gamma, mean, invstd, dy, y_saved, nullptr, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale, b.swap);
       break;
     default:
       launch_pdl(k_bn_bwd_apply<BN_RELU_BITS>, dim3(apply_blocks), dim3(g.threads), 0, s, 
-          x, gamma, mean, invstd, dy, nullptr, relu_mask, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale);
+          x, gamma, mean, invstd, dy, nullptr, relu_mask, a.mm, dx, dres, b.R, b.C, g.rpb, b.post_scale, b.swap);
       break;
   }
   return counted_launches(launches);

@@ -236,6 +236,7 @@ struct BnLaunch {
   int R, C;
   uint16_t eps, post_scale;
   int relu, residual;
+  int swap;               // PF16_BN_SWAP: gamma * (s * xhat + residual) + beta
   int chunk_rows;         // rows per statistics chunk (contiguous in memory)
   BnPlan fwd, bwd;
   int* status;            // device status word (bounded waits record timeouts here)
@@ -255,7 +256,8 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,
                           const uint16_t* y_saved, const uint8_t* relu_mask, uint16_t* dx,
                           uint16_t* dgamma, uint16_t* dbeta, uint16_t* dres, uint16_t* ws,
-                          cudaStream_t s, const uint8_t* dgrad_stats = nullptr);
+                          cudaStream_t s, const uint8_t* dgrad_stats = nullptr,
+                          const uint16_t* residual = nullptr);
 void bn_plan(int R, int C, BnLaunch* b);
 size_t bn_ws_bytes(const BnLaunch& b);
 

@@ -26,6 +26,7 @@ PF16_ACCUMULATE = 0x1
 PF16_F32_ACCUM = 0x4
 PF16_BN_RELU = 0x1
 PF16_BN_RESIDUAL = 0x2
+PF16_BN_SWAP = 0x4
 PF16_PASS_FWD, PF16_PASS_DGRAD, PF16_PASS_WGRAD = 0, 1, 2
 
 EXPORTS = [

@@ -133,9 +133,10 @@ class Conv:
 
 
 class BN:
-    def __init__(self, net, n, h, w, c, post_scale, relu, residual=False, zero_gamma=False):
+    def __init__(self, net, n, h, w, c, post_scale, relu, residual=False, zero_gamma=False, swap=False):
         self.net = net
         flags = (pf16.PF16_BN_RELU if relu else 0) | (pf16.PF16_BN_RESIDUAL if residual else 0)
+        flags |= pf16.PF16_BN_SWAP if swap else 0
         self.desc = pf16.bn_desc(n, h, w, c, EPS, post_scale, flags)
         self.c = c
         self.zero_gamma = zero_gamma
@@ -161,17 +162,19 @@ class BN:
                       beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd,
                       relu_mask=self.mask, conv_stats=conv.stats if conv is not None else None)
 
-    def bwd(self, x, y_saved, dy, dx, dresidual=None, conv=None):
-        """conv: the layer whose dgrad(bn=(self, x)) produced dy (its statistics are used)."""
+    def bwd(self, x, y_saved, dy, dx, dresidual=None, conv=None, residual=None):
+        """conv: the layer whose dgrad(bn=(self, x)) produced dy (its statistics are used);
+        residual: the forward's residual input (read by the swap variant's backward)."""
         self.net.call("bn_bwd", self, pf16.bn_fwd_bwd, self.desc, 1, self.net.ws, x=x, gamma=self.gamma,
                       mean=self.mean, invstd=self.invstd, dy=dy, relu_mask=self.mask, dx=dx,
                       dgamma=self.dgamma, dbeta=self.dbeta, dresidual=dresidual,
-                      conv_stats=conv.dstats if conv is not None else None)
+                      conv_stats=conv.dstats if conv is not None else None,
+                      residual=residual if self.desc.flags & pf16.PF16_BN_SWAP else None)
         self.fused_bwd = conv is not None
 
 
 class Bottleneck:
-    def __init__(self, net, n, h, cin, width, stride, proj):
+    def __init__(self, net, n, h, cin, width, stride, proj, swap=False):
         self.cin, self.width, self.stride = cin, width, stride
         cout = 4 * width
         self.conv1 = Conv(net, n, h, h, cin, width, 1, 1, 1, 0)
@@ -180,7 +183,8 @@ class Bottleneck:
         h2 = self.conv2.P
         self.bn2 = BN(net, n, h2, h2, width, S_BLOCK, relu=True)
         self.conv3 = Conv(net, n, h2, h2, width, cout, 1, 1, 1, 0)
-        self.bn3 = BN(net, n, h2, h2, cout, S_BLOCK, relu=True, residual=True, zero_gamma=True)
+        # swap: Sec. 4.1's variant of the block's last BatchNorm, gamma * (s * xhat + shortcut) + beta
+        self.bn3 = BN(net, n, h2, h2, cout, S_BLOCK, relu=True, residual=True, zero_gamma=True, swap=swap)
         self.proj = proj
         if proj:
             self.convp = Conv(net, n, h, h, cin, cout, 1, 1, stride, 0)
@@ -219,9 +223,9 @@ class Bottleneck:
     def backward(self, dx):
         """self.dy holds dL/dy; writes dL/dx into dx."""
         if self.proj:
-            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=self.dres)
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=self.dres, residual=self.bp)
         else:  # identity shortcut: its gradient is the start of dx
-            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=dx)
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=dx, residual=self.x)
         self.conv3.wgrad(self.b2, self.da3)
         # the data gradients also reduce the next BatchNorm's backward statistics
         self.conv3.dgrad(self.da3, self.db2, bn=(self.bn2, self.a2))
@@ -243,7 +247,7 @@ class Bottleneck:
 class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
-    def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None):
+    def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False):
         self.N, self.image, self.classes, self.device = batch, image, classes, device
         self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
         self.wd, self.nowd = Arena("decayed"), Arena("no-decay")
@@ -258,7 +262,7 @@ class ResNet50:
         self.blocks = []
         for width, nb, stride in STAGES:
             for b in range(nb):
-                blk = Bottleneck(self, N, h, cin, width, stride if b == 0 else 1, proj=(b == 0))
+                blk = Bottleneck(self, N, h, cin, width, stride if b == 0 else 1, proj=(b == 0), swap=bn_swap)
                 self.blocks.append(blk)
                 h, cin = blk.h2, 4 * width
         self.hl, self.cl = h, cin

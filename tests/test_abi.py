@@ -102,6 +102,13 @@ def test_other_validation_errors():
     assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 2, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_ARG
     assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_NULL
     assert L.pf16_bn_fwd_bwd(ctypes.byref(d), 0, ctypes.byref(t), FAKE, 1, None) == pf16.PF16_ERR_WORKSPACE
+    # the swap variant is defined with a residual input only, and needs two more partial buffers
+    ds = pf16.bn_desc(2, 4, 4, 64, 0x00A8, 0x3400, pf16.PF16_BN_SWAP)
+    assert L.pf16_bn_fwd_bwd(ctypes.byref(ds), 0, ctypes.byref(t), FAKE, 1 << 20, None) == pf16.PF16_ERR_ARG
+    assert pf16.bn_workspace_size(ds) == 0
+    dr = pf16.bn_desc(2, 4, 4, 64, 0x00A8, 0x3400, pf16.PF16_BN_RESIDUAL)
+    dsr = pf16.bn_desc(2, 4, 4, 64, 0x00A8, 0x3400, pf16.PF16_BN_RESIDUAL | pf16.PF16_BN_SWAP)
+    assert pf16.bn_workspace_size(dsr) > pf16.bn_workspace_size(dr) > 0
     assert L.pf16_maxpool_fwd(FAKE, FAKE, 1, 8, 8, 12, None) == pf16.PF16_ERR_UNSUPPORTED
     assert L.pf16_maxpool_fwd_argmax(FAKE, FAKE, None, 1, 8, 8, 16, None) == pf16.PF16_ERR_NULL
     assert L.pf16_maxpool_fwd_argmax(FAKE, FAKE, ctypes.c_void_p(0x10004), 1, 8, 8, 16,

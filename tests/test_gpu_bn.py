@@ -119,3 +119,60 @@ def test_bn_constant_channel_and_zero_gamma(orc):
                     invstd=empty16(C))
     y = f64(host(ty)).reshape(R, C)
     assert np.array_equal(y, np.tile(0.25 * f64(beta), (R, 1)))
+
+
+SWAP_CASES = [
+    # N, H, W, C, relu
+    (4, 14, 14, 256, True),
+    (3, 5, 7, 24, False),        # ragged rows, no ReLU
+    (256, 7, 7, 2048, True),     # a stage-4 block's last BatchNorm at batch 256
+]
+
+
+@pytest.mark.parametrize("case", SWAP_CASES, ids=lambda c: "N{}_{}x{}_C{}_relu{}".format(*c))
+def test_bn_swap_fwd_bwd(orc, case):
+    """PF16_BN_SWAP (Sec. 4.1's switch) against the oracle's swap BatchNorm.
+    Forward bound (4L+8) u (|gamma| (s (|xhat|+1) + |r|) + |beta|) + 2^-24; the
+    data gradient has the plain form; dresidual = rn(gamma dy') to one rounding;
+    dbeta = sum dy', dgamma = s sum dy' xhat + sum dy' r within (4L+8) u sum|terms|."""
+    N, H, W, C, relu = case
+    R = N * H * W
+    L = int(np.ceil(np.log2(R)))
+    s = 0.25
+    x = f16(f64(syn.normal_f16(31, (R, C), 2.0)) + 0.5)
+    gamma = f16(1.0 + 0.1 * f64(syn.normal_f16(32, (C,))))
+    beta = f16(0.1 * f64(syn.normal_f16(33, (C,))))
+    resid = syn.normal_f16(34, (R, C))
+    dy = syn.normal_f16(35, (R, C), 0.01)
+    flags = pf16.PF16_BN_RESIDUAL | pf16.PF16_BN_SWAP | (pf16.PF16_BN_RELU if relu else 0)
+    d = pf16.bn_desc(N, H, W, C, EPS, int(f16([s])[0]), flags)
+    ws = workspace(pf16.bn_workspace_size(d))
+    tx, tg, tb, tr = dev(x), dev(gamma), dev(beta), dev(resid)
+    ty, tm, ti = empty16(R * C), empty16(C), empty16(C)
+    tmask = torch.empty(R * C // 8, dtype=torch.uint8, device="cuda") if relu else None
+    pf16.bn_fwd_bwd(d, 0, ws, x=tx, gamma=tg, beta=tb, residual=tr, y=ty, mean=tm, invstd=ti, relu_mask=tmask)
+    assert pf16.sync_status() == 0
+    y = host(ty)
+    yo, mean, var, invstd = orc.bn_fwd_swap(x, gamma, beta, resid, R, C, EPS_F, s, relu)
+    xhat = (f64(x).reshape(R, C) - mean) * invstd
+    gf, bf, rf = f64(gamma), f64(beta), f64(resid).reshape(R, C)
+    tol = (4 * L + 8) * U * (np.abs(gf) * (s * (np.abs(xhat) + 1) + np.abs(rf)) + np.abs(bf)) + 2.0 ** -24
+    err = np.abs(f64(y).reshape(R, C) - yo)
+    assert np.all(err <= tol), float(np.max(err / tol))
+
+    tdx, tdg, tdb, tdr = empty16(R * C), empty16(C), empty16(C), empty16(R * C)
+    pf16.bn_fwd_bwd(d, 1, ws, x=tx, gamma=tg, mean=tm, invstd=ti, dy=dev(dy), y_saved=ty, residual=tr,
+                    relu_mask=tmask, dx=tdx, dgamma=tdg, dbeta=tdb, dresidual=tdr)
+    assert pf16.sync_status() == 0
+    dxo, dgo, dbo, dro = orc.bn_bwd_swap(x, gamma, dy, y, resid, R, C, EPS_F, s, relu)
+    dz = np.abs(dro / np.where(gf == 0, 1, gf))  # |dy'|
+    k = np.abs(s * gf * invstd)
+    tol = (4 * L + 8) * U * k * (dz + dz.max(0) * (np.abs(xhat) + 1)) + 2.0 ** -24
+    e = np.abs(f64(host(tdx)).reshape(R, C) - dxo)
+    assert np.all(e <= tol), float(np.max(e / tol))
+    e = np.abs(f64(host(tdr)).reshape(R, C) - dro)
+    assert np.all(e <= U * np.abs(dro) + 2.0 ** -24), float(np.max(e))
+    tol_b = (4 * L + 8) * U * dz.sum(0) + 2.0 ** -24
+    tol_g = (4 * L + 8) * U * (s * (dz * (np.abs(xhat) + 1)).sum(0) + (dz * np.abs(rf)).sum(0)) + 2.0 ** -24
+    assert np.all(np.abs(f64(host(tdb)) - dbo) <= tol_b), float(np.max(np.abs(f64(host(tdb)) - dbo) / tol_b))
+    assert np.all(np.abs(f64(host(tdg)) - dgo) <= tol_g), float(np.max(np.abs(f64(host(tdg)) - dgo) / tol_g))

@@ -87,3 +87,23 @@ def test_graph_replay_is_deterministic():
     torch.cuda.synchronize()
     assert torch.equal(after_graph, net.wd.w)
     assert not torch.equal(w0, net.wd.w)
+
+
+def test_swap_variant_step():
+    """The BN-swap variant (Sec. 4.1) in every block's last BatchNorm: with the
+    zero-gamma initialisation each block computes ReLU(0 * (s xhat + r) + 0) = 0,
+    so every block output is exactly zero, the logits are the (zero) bias and
+    the first loss is the uniform value; the step then runs and replays."""
+    net = ResNet50(batch=2, image=64, seed_cfg=4, bn_swap=True)
+    net.set_batch(syn.images_f16(syn.seed_for(4, "x"), 2, 64, 64, 3), syn.labels(syn.seed_for(4, "labels"), 2))
+    net.forward()
+    assert pf16.sync_status() == 0
+    for b in net.blocks:
+        assert not torch.any(b.y)
+    net.step()
+    assert pf16.sync_status() == 0
+    loss = float(f64(host(net.loss))[0])
+    assert abs(loss - np.log(1000)) < 2 ** -8 * np.log(1000)
+    net.step()
+    assert pf16.sync_status() == 0
+    assert np.isfinite(float(f64(host(net.loss))[0]))
