@@ -191,19 +191,40 @@ __global__ void __launch_bounds__(256)
     const long long r = chunk / cpr;
     const int cg = (int)(chunk - r * cpr);
     const uint4* src = reinterpret_cast<const uint4*>(parts + r * cols + cg * 8);
-    Tree4<11, false> tree;
-    for (int i0 = 0; i0 < seg; i0 += 4) {
-      uint4 v[4];
+    // seg is a power of two, so the run splits into aligned batches of
+    // nb = min(seg, 16) leaves: each batch is summed as a perfect pairwise
+    // tree with all its loads in flight at once, and the batch sums feed a
+    // register-resident binary counter, which builds the perfect tree above
+    // them.  Together: the perfect pairwise tree over the run's seg leaves.
+    const int nb = seg < 16 ? seg : 16;
+    uint4 st[8];  // st[l]: a finished subtree of 2^l batch sums
+    unsigned cnt = 0;
+    for (int i0 = 0; i0 < seg; i0 += 16) {
+      uint4 v[16];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
+      for (int i = 0; i < 16; ++i) {
         const int sp = g * seg + i0 + i;
-        v[i] = (i0 + i < seg && sp < splits) ? __ldg(src + sp * plane) : zero4();
+        v[i] = (i < nb && sp < splits) ? __ldg(src + sp * plane) : zero4();
       }
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (i0 + i < seg) tree.push(v[i]);
+      for (int w = 1; w < 16; w *= 2)
+#pragma unroll
+        for (int i = 0; i < 16; i += 2 * w)
+          if (i + w < nb) v[i] = add4(v[i], v[i + w]);
+      uint4 b = v[0];
+      bool carry = true;
+#pragma unroll
+      for (int l = 0; l < 8; ++l) {
+        const bool bit = (cnt >> l) & 1u;
+        if (carry && bit) b = add4(st[l], b);
+        if (carry && !bit) { st[l] = b; carry = false; }
+      }
+      ++cnt;
     }
-    acc = tree.finish(ceil_log2(seg));
+    // cnt = seg / nb is a power of two: its one set bit names the full tree
+#pragma unroll
+    for (int l = 0; l < 8; ++l)
+      if (cnt == (1u << l)) acc = st[l];
   }
   sh[t] = acc;
   __syncthreads();
@@ -228,12 +249,13 @@ cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long ro
   int sp2 = 1;
   while (sp2 < splits) sp2 *= 2;
   // Split groups per output chunk: only as many as it takes to give the GPU
-  // about 2048 threads per SM, so that a thread sums a long run of splits with
-  // batched loads instead of each CTA paying a shared-memory tree for a few
-  // loads.  Every choice sums the same balanced tree over the padded splits.
+  // about 512 threads per SM (one wave), each with up to 16 loads in flight,
+  // so that a thread sums a long run of splits instead of each CTA paying a
+  // shared-memory tree for a few loads.  Every choice sums the same balanced
+  // tree over the padded splits.
   const long long total_chunks = rows * (cols / 8);
   int grp = 1;
-  while (grp < sp2 && grp < 256 && total_chunks * grp < 152ll * 2048) grp *= 2;
+  while (grp < sp2 && grp < 256 && total_chunks * grp < 152ll * 512) grp *= 2;
   const int cl = 256 / grp;
   const long long total = rows * (cols / 8);
   const long long blocks = (total + cl - 1) / cl;
