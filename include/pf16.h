@@ -141,6 +141,23 @@ int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const u
                             void* ws, size_t ws_bytes, const pf16_bn_source* bn, void* stats,
                             size_t stats_bytes, void* stream);
 
+/* pf16_conv_dgrad_bnstats plus an addend: dx = rn(result + a), a = add where
+ * add_mask's bit is set (the layout of pf16_bn_desc's relu_mask for a
+ * n x h x w x c tensor) and +0 elsewhere; NULL add_mask: a = add.  The
+ * statistics are those of this dx.  This is the gradient at the input of an
+ * identity-shortcut residual block (Sec. 4.2): the shortcut's share (the
+ * block's output gradient where its final ReLU passed, add and add_mask) plus
+ * the first convolution's data gradient, and it is the output gradient of the
+ * previous block's last BatchNorm (bn).  dx is bit-identical to that
+ * BatchNorm's dresidual followed by pf16_conv_dgrad with PF16_ACCUMULATE;
+ * the residual BatchNorm's backward then needs no dresidual output.
+ * Requires a 1x1 filter with stride 1 and pad 0 and c a multiple of 64
+ * (PF16_ERR_UNSUPPORTED); add is n x h x w x c, 16-byte aligned, and must not
+ * overlap dx (PF16_ERR_ARG); add_mask 8-byte aligned. */
+int pf16_conv_dgrad_bnstats_add(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                                void* ws, size_t ws_bytes, const pf16_bn_source* bn, const uint16_t* add,
+                                const uint8_t* add_mask, void* stats, size_t stats_bytes, void* stream);
+
 /* Weight gradient: dw[k,r,s,c] = sum_{n,p,q} dy[n,p,q,k] * x[n, p*st+r-pad, q*st+s-pad, c].
  * The reduction over n*p*q pixels is split into chunks, each accumulated in
  * FP16 by the tensor core into FP16 partials in the workspace, which are then

@@ -407,6 +407,14 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
       return PF16_ERR_CUDA;
     p.tma_store = 1;
   }
+  // backward statistics: the BatchNorm input (and the addend) enter the
+  // epilogue as TMA tiles of the output's 32 x 64 boxes
+  CUtensorMap mx = c, md = c;
+  if (p.bs_x) {
+    if (!p.tma_store || p.out_mode != OUT_STORE) return PF16_ERR_UNSUPPORTED;
+    if (!map_2d(&mx, p.bs_x, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+    if (p.add_src && !map_2d(&md, p.add_src, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+  }
   // Clusters of two CTAs over M-tile pairs share each B tile (multicast), which
   // halves the B operand's L2 -> SM traffic, the bound of most conv passes.
   const int pair_cl = (BN >= 128 && p.m_tiles % 2 == 0) ? gemm_pair_clusters(BN) : 0;
@@ -420,7 +428,7 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
     if (ncl > 0) {
       if (p.bs_x && (p.bs_levels = tile_tree_levels(pair_units, ncl)) >= kMaxTileTreeLevels)
         return PF16_ERR_UNSUPPORTED;
-      return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+      return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true, &mx, &md) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
     }
   }
   int grid = (int)std::min<long long>(units, sms);
@@ -431,7 +439,7 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
     grid -= grid % p.n_tiles;
     if (p.bs_x && (p.bs_levels = tile_tree_levels(units, grid)) >= kMaxTileTreeLevels) return PF16_ERR_UNSUPPORTED;
   }
-  return launch_gemm(BN, a, b, c, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+  return launch_gemm(BN, a, b, c, p, grid, st, false, &mx, &md) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
 // Point the GEMM's fused statistics at the BatchNorm backward sources.
@@ -690,7 +698,7 @@ int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint
 
 static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
                            uint32_t flags, void* stats, size_t stats_bytes, const pf16_bn_source* bn,
-                           void* stream) {
+                           void* stream, const uint16_t* add = nullptr, const uint8_t* add_mask = nullptr) {
   Shape s;
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
@@ -708,6 +716,15 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
     if (s.C % 64 != 0 || s.st != 1) return PF16_ERR_UNSUPPORTED;
     if (stats_bytes < bnstat_bytes(s.C)) return PF16_ERR_WORKSPACE;
   }
+  if (add) {
+    // the masked addend: a plain 1x1 data gradient (one GEMM, rows in pixel order)
+    if (!stats) return PF16_ERR_ARG;
+    if (s.R != 1 || s.S != 1 || s.pad != 0) return PF16_ERR_UNSUPPORTED;
+    if (!aligned16(add) || (reinterpret_cast<uintptr_t>(add_mask) & 7u) != 0) return PF16_ERR_ALIGN;
+    const size_t bytes = (size_t)(s.N * s.H * s.W * s.C) * 2;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(add), d0 = reinterpret_cast<uintptr_t>(dx);
+    if (a0 < d0 + bytes && d0 < a0 + bytes) return PF16_ERR_ARG;  // read through the read-only path
+  }
   if (!driver_fns()) return PF16_ERR_CUDA;
   int* status;
   int sms;
@@ -716,7 +733,9 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
   const bool accum = (flags & PF16_ACCUMULATE) != 0;
   if (const int ws = halo_width(s, accum))
     return run_halo(s, ws, true, dy, w, dx, status, sms, st, f32, stats, stats ? bn : nullptr);
-  const int BN = pick_bn_out(s.C);
+  // with an addend the TMA-fed epilogue leaves 256-wide tiles two pipeline
+  // stages; reductions of 4+ K-blocks keep three with 128-wide tiles
+  const int BN = (add && s.K >= 4 * kBK) ? std::min(pick_bn_out(s.C), 128) : pick_bn_out(s.C);
   const size_t dx_elems = (size_t)(s.N * s.H * s.W * s.C);
 
   if (s.R == 1 && s.S == 1 && s.pad == 0) {
@@ -725,6 +744,8 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
     p.d_f32 = f32 ? 1 : 0;
     set_stats(p, stats, s.C);
     if (stats) set_bwd_stats(p, bn);
+    p.add_src = add;
+    p.add_mask = add ? add_mask : nullptr;
     CUtensorMap ma, mb;
     p.M = (int)(s.N * s.P * s.Q);
     p.N = (int)s.C;
@@ -826,6 +847,15 @@ int pf16_conv_dgrad_bnstats(const pf16_conv_desc* d, const uint16_t* dy, const u
   (void)ws_bytes;
   if (!bn || !stats) return PF16_ERR_NULL;
   return conv_dgrad_impl(d, dy, w, dx, 0, stats, stats_bytes, bn, stream);
+}
+
+int pf16_conv_dgrad_bnstats_add(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
+                                void* ws, size_t ws_bytes, const pf16_bn_source* bn, const uint16_t* add,
+                                const uint8_t* add_mask, void* stats, size_t stats_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  if (!bn || !stats || !add) return PF16_ERR_NULL;
+  return conv_dgrad_impl(d, dy, w, dx, 0, stats, stats_bytes, bn, stream, add, add_mask);
 }
 
 // The stem's weight gradient through k_stem_wgrad (layouts at stem_wgrad_plan).

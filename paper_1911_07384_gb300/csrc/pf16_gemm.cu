@@ -28,16 +28,22 @@ namespace pf16 {
 constexpr int kEpiWarps = 8;
 constexpr int kGemmThreads = 32 * (2 + kEpiWarps);
 
-template <int BN>
+// TMAE: the TMA-fed backward-statistics epilogue keeps four 32 x 64 tiles per
+// warp (two staging tiles, two BatchNorm-input tiles, filled by TMA a chunk
+// ahead), paid for with pipeline stages; plus two transaction barriers per warp.
+template <int BN, bool TMAE = false>
 struct GemmCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_BYTES = BN * kBK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = BN == 64 ? 8 : (BN == 128 ? 6 : 4);
+  static constexpr int STAGES = TMAE ? (BN == 64 ? 4 : (BN == 128 ? 3 : 2)) : (BN == 64 ? 8 : (BN == 128 ? 6 : 4));
   static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
-  static constexpr int STAGING_BYTES = kEpiWarps * 4096;  // per epilogue warp: one 32 x 64 tile
-  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
+  static constexpr int WARP_BUF = TMAE ? 4 * 4096 : 4096;  // per epilogue warp
+  static constexpr int STAGING_BYTES = kEpiWarps * WARP_BUF;
+  static constexpr int EBARS = TMAE ? 2 * kEpiWarps : 0;
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4 + EBARS) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 static constexpr int kErrTimeout = -7;  // PF16_ERR_TIMEOUT
@@ -414,6 +420,14 @@ struct EpiStats {
   // 32-leaf halving tree is pushed into chunk c's binary counter of halving
   // nodes (mu: dy', v: dy' xhat).
   __device__ __forceinline__ void leaf_bwd(int c, uint32_t stg, int lane, int nv, const struct BwdIn& in);
+  // The same leaf with x read from a 128B-swizzled 32 x 64 tile at xs (laid
+  // out as the staged tile), ReLU bits m of row `lane` and the pair's mean2 /
+  // invstd2.
+  __device__ __forceinline__ void leaf_bwd_tile(int c, uint32_t stg, uint32_t xs, int lane, int nv, uint2 m,
+                                                uint32_t mean2, uint32_t invstd2);
+  template <class XF>
+  __device__ __forceinline__ void leaf_bwd_core(int c, uint32_t stg, int lane, int nv, uint2 m, uint32_t mean2,
+                                                uint32_t invstd2, XF xf);
   // Close the backward counters as if zero leaves padded them to 2^levels,
   // merge the CTA's 8 epilogue warps by halving (warps 0..7 in a balanced
   // tree, through `sm` as write_cta) and write the CTA's nodes as `slot`.
@@ -489,20 +503,23 @@ struct BwdIn {
   }
 };
 
-__device__ __forceinline__ void EpiStats::leaf_bwd(int c, uint32_t stg, int lane, int nv, const BwdIn& in) {
+template <class XF>
+__device__ __forceinline__ void EpiStats::leaf_bwd_core(int c, uint32_t stg, int lane, int nv, uint2 m,
+                                                        uint32_t mean2, uint32_t invstd2, XF xf) {
   const uint32_t col = (uint32_t)(lane & 3) * 4;
   uint32_t t1[32], t2[32];
 #pragma unroll
   for (int r = 0; r < 32; ++r) {
+    const uint32_t off = r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col;
     uint32_t g;
-    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(g) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(g) : "r"(stg + off));
     // row r's ReLU bits from lane r; this lane's two channels are bits 2l, 2l+1
-    const uint32_t mlo = __shfl_sync(0xffffffffu, in.m.x, r), mhi = __shfl_sync(0xffffffffu, in.m.y, r);
+    const uint32_t mlo = __shfl_sync(0xffffffffu, m.x, r), mhi = __shfl_sync(0xffffffffu, m.y, r);
     const uint32_t b = (lane < 16 ? mlo >> (2 * lane) : mhi >> (2 * lane - 32)) & 3u;
     const uint32_t mk = ((b & 1u) ? 0x0000FFFFu : 0u) | ((b & 2u) ? 0xFFFF0000u : 0u);
     const uint32_t d = r < nv ? (g & mk) : 0u;
     t1[r] = d;
-    t2[r] = r < nv ? hmul2_rn(d, hmul2_rn(hsub2_rn(in.x[r], in.mu2), in.is2)) : 0u;
+    t2[r] = r < nv ? hmul2_rn(d, hmul2_rn(hsub2_rn(xf(r, off), mean2), invstd2)) : 0u;
   }
 #pragma unroll
   for (int w = 16; w >= 1; w /= 2)
@@ -525,6 +542,174 @@ __device__ __forceinline__ void EpiStats::leaf_bwd(int c, uint32_t stg, int lane
   }
 }
 
+__device__ __forceinline__ void EpiStats::leaf_bwd(int c, uint32_t stg, int lane, int nv, const BwdIn& in) {
+  leaf_bwd_core(c, stg, lane, nv, in.m, in.mu2, in.is2, [&](int r, uint32_t) { return in.x[r]; });
+}
+
+__device__ __forceinline__ void EpiStats::leaf_bwd_tile(int c, uint32_t stg, uint32_t xs, int lane, int nv, uint2 m,
+                                                        uint32_t mean2, uint32_t invstd2) {
+  leaf_bwd_core(c, stg, lane, nv, m, mean2, invstd2, [&](int, uint32_t off) {
+    uint32_t x;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(xs + off));
+    return x;
+  });
+}
+
+// Register inputs of one 64-column chunk of the backward-statistics epilogue:
+// the ReLU bits of row `lane` (all ones without a mask), the addend's mask
+// bits of row `lane` (ADD; all ones without a mask) and the mean / invstd of
+// channel pair (2 lane, 2 lane + 1).
+struct ChunkIn {
+  uint2 m, am;
+  uint32_t mu2, is2;
+
+  template <bool ADD>
+  __device__ __forceinline__ void load(const GemmParams& p, long long row0, int col0, int lane) {
+    const long long r = row0 + lane;
+    const bool in = r < p.M;
+    const long long mo = r * (p.N / 8) + col0 / 8;
+    m = make_uint2(0xFFFFFFFFu, 0xFFFFFFFFu);
+    if (p.bs_mask && in) m = __ldg(reinterpret_cast<const uint2*>(p.bs_mask + mo));
+    am = make_uint2(0xFFFFFFFFu, 0xFFFFFFFFu);
+    if (ADD && p.add_mask && in) am = __ldg(reinterpret_cast<const uint2*>(p.add_mask + mo));
+    mu2 = __ldg(reinterpret_cast<const uint32_t*>(p.bs_mean + col0) + lane);
+    is2 = __ldg(reinterpret_cast<const uint32_t*>(p.bs_invstd + col0) + lane);
+  }
+};
+
+// Backward-statistics epilogue of one warp (BS, TMA stores): the warp's 32
+// rows of each of its group's tiles (units u0, u0 + ustep, ...), 64 columns
+// (a chunk) at a time.  Chunk q uses buffer b = q & 1 of the warp's four
+// 128B-swizzled 32 x 64 tiles at wbuf: staging tile S[b] (the output; with ADD
+// it first receives the addend) and input tile X[b] (the BatchNorm input x).
+// The TMA loads of chunk q + 1 into buffer b ^ 1 are issued before chunk q is
+// processed, completing on the warp's barrier wbar[b ^ 1]; its register inputs
+// (ChunkIn) are loaded as far ahead.  With ADD the chunk's output is
+// rn(result + addend) where the addend's mask bit is set (rn(result + 0)
+// elsewhere), and the statistics are taken of that sum.
+template <int BN, bool ADD>
+__device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorMap* mapC, const CUtensorMap* mapX,
+                                            const CUtensorMap* mapD, uint8_t* wbuf, uint64_t* wbar,
+                                            uint64_t* tfull, uint64_t* tempty, uint32_t tmem_base, int acc, int sub,
+                                            int lane, int u0, int ustep, int total, int mt_count, int mscale,
+                                            int rank, uint64_t lim, volatile int* abort_flag, EpiStats& stats) {
+  if (u0 >= total) return;
+  const uint32_t S0 = smem_u32(wbuf), X0 = S0 + 2 * 4096;
+  const uint32_t B0 = smem_u32(wbar);
+  const uint32_t tx = ADD ? 2 * 4096 : 4096;
+  // lane 0: the chunk index whose loads are in flight in each buffer (-1: none)
+  int pend[2] = {-1, -1};
+  auto issue = [&](int b, int row0, int col0, int q) {
+    mbar_arrive_expect_tx(B0 + 8 * b, tx);
+    tma_load_2d(X0 + b * 4096, mapX, B0 + 8 * b, col0, row0);
+    if (ADD) tma_load_2d(S0 + b * 4096, mapD, B0 + 8 * b, col0, row0);
+    pend[b] = q;
+  };
+  int u = u0, m0, n0, split, kb0, kb1;
+  unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+  int c = 0;
+  if (lane == 0) issue(0, m0 + sub * 32, n0, 0);
+  ChunkIn cur, nxt;
+  cur.load<ADD>(p, (long long)(m0 + sub * 32), n0, lane);
+  uint32_t acc_phase = 0, tbase = 0;
+  int nv = 0;
+  for (int q = 0;; ++q) {
+    if (c == 0) {  // a new tile: wait for its accumulator
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      const bool got = mbar_wait(smem_u32(&tfull[acc]), acc_phase, lim);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) record_timeout(p, abort_flag);
+        break;
+      }
+      tc_fence_after();
+      tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * BN);
+      nv = min(32, max(0, p.M - (m0 + sub * 32)));
+    }
+    const int b = q & 1;
+    // the next chunk: this tile's next 64 columns, else the group's next tile
+    int u2 = u, c2 = c + 64, m2 = m0, n2 = n0;
+    const bool last = c2 >= BN || n0 + c2 >= p.N;  // the tile's last chunk
+    if (last) {
+      u2 = u + ustep;
+      c2 = 0;
+      if (u2 < total) unit_decode(p, u2, m2, n2, split, kb0, kb1, BN, mt_count, mscale, rank);
+    }
+    const bool more = u2 < total;
+    if (more) {
+      __syncwarp();  // every lane is done reading buffer b ^ 1 (chunk q - 1)
+      if (lane == 0) {
+        bulk_wait_read0();         // chunk q - 1's store has read S[b ^ 1]
+        fence_proxy_async_smem();  // the warp's reads of X[b ^ 1] before the copy's writes
+        issue(b ^ 1, m2 + sub * 32, n2 + c2, q + 1);
+      }
+      nxt.load<ADD>(p, (long long)(m2 + sub * 32), n2 + c2, lane);
+    }
+    uint32_t r[64];
+    tmem_ld16(tbase + c, r);
+    tmem_ld16(tbase + c + 16, r + 16);
+    tmem_ld16(tbase + c + 32, r + 32);
+    tmem_ld16(tbase + c + 48, r + 48);
+    tmem_ld_wait();
+    if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
+    if (last) {  // accumulator fully read: hand TMEM back
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+    }
+    const bool ok = mbar_wait(B0 + 8 * b, (uint32_t)(q >> 1) & 1u, lim);
+    if (!__all_sync(0xffffffffu, ok)) {
+      if (lane == 0) record_timeout(p, abort_flag);
+      break;
+    }
+    if (lane == 0) pend[b] = -1;
+    const uint32_t S = S0 + b * 4096, X = X0 + b * 4096;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      uint4 v;
+      v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
+      v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
+      v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
+      v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
+      const uint32_t addr = S + lane * 128 + ((j ^ (lane & 7)) << 4);
+      if (ADD) {
+        uint4 a;
+        ld_shared_v4(addr, a);
+        const uint32_t bits = ((j < 4 ? cur.am.x : cur.am.y) >> (8 * (j & 3))) & 0xFFu;
+        uint32_t mk[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mk[k] = (((bits >> (2 * k)) & 1u) ? 0x0000FFFFu : 0u) | (((bits >> (2 * k + 1)) & 1u) ? 0xFFFF0000u : 0u);
+        v.x = hadd2_rn(v.x, a.x & mk[0]);
+        v.y = hadd2_rn(v.y, a.y & mk[1]);
+        v.z = hadd2_rn(v.z, a.z & mk[2]);
+        v.w = hadd2_rn(v.w, a.w & mk[3]);
+      }
+      st_shared_v4(addr, v);
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(mapC, S, n0 + c, m0 + sub * 32);
+      bulk_commit();
+    }
+    if (p.st_mean && nv > 0) stats.leaf_bwd_tile(c / 64, S, X, lane, nv, cur.m, cur.mu2, cur.is2);
+    if (last) {
+      if (p.st_mean && nv > 0) stats.end_tile(nv);
+      acc_phase ^= 1;
+    }
+    if (!more) break;
+    cur = nxt;
+    u = u2;
+    c = c2;
+    m0 = m2;
+    n0 = n2;
+  }
+  // after an abort: let the loads still in flight land before shared memory is released
+  if (lane == 0)
+    for (int b = 0; b < 2; ++b)
+      if (pend[b] >= 0) mbar_wait(B0 + 8 * b, (uint32_t)(pend[b] >> 1) & 1u, 1000000000ull);
+}
+
 // PAIR: launched in clusters of two CTAs that take the same (n tile, split)
 // units over M tiles 2t and 2t + 1, so they need the same B tiles: the CTA of
 // rank kb mod 2 loads K-block kb's B tile once and multicasts it into both
@@ -533,13 +718,21 @@ __device__ __forceinline__ void EpiStats::leaf_bwd(int c, uint32_t stg, int lane
 // stage's empty barrier in both CTAs, count 2).  The two CTAs meet at a
 // cluster barrier after set-up and before exit, so neither's shared memory
 // or barriers are written after it has left.
-// BS: the epilogue takes BatchNorm backward statistics (GemmParams::bs_x);
-// a separate instantiation, so that the other GEMMs do not carry its registers.
-template <int BN, bool PAIR, bool BS>
+// EPI: the epilogue's kind, each a separate instantiation so that the others
+// do not carry its registers or give up its pipeline stages --
+//   EPI_PLAIN: stores (forward statistics optional);
+//   EPI_BS: BatchNorm backward statistics (GemmParams::bs_x), inputs loaded
+//     into registers (for long reductions, which need every pipeline stage);
+//   EPI_BS_TMA: the same statistics from TMA-fed tiles (epilogue_bs; for short
+//     reductions, whose epilogue is the bound);
+//   EPI_BS_ADD: EPI_BS_TMA plus the addend (GemmParams::add_src).
+template <int BN, bool PAIR, int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-           const __grid_constant__ CUtensorMap mapC, const __grid_constant__ GemmParams p) {
-  using Cfg = GemmCfg<BN>;
+           const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapX,
+           const __grid_constant__ CUtensorMap mapD, const __grid_constant__ GemmParams p) {
+  constexpr bool BS = EPI != EPI_PLAIN, TMAE = EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, ADD = EPI == EPI_BS_ADD;
+  using Cfg = GemmCfg<BN, TMAE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -549,7 +742,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint64_t* empty = bars + Cfg::STAGES;
   uint64_t* tfull = bars + 2 * Cfg::STAGES;
   uint64_t* tempty = tfull + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  uint64_t* ebar = tempty + 2;  // TMAE: per epilogue warp, one transaction barrier per input buffer
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ebar + Cfg::EBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -562,11 +756,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(smem_u32(&tfull[a]), 1);
       mbar_init(smem_u32(&tempty[a]), 4);
     }
+    for (int b = 0; b < Cfg::EBARS; ++b) mbar_init(smem_u32(&ebar[b]), 1);
     *abort_flag = 0;
     fence_mbar_init();
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapB);
     if (p.tma_store) tma_prefetch_desc(&mapC);
+    if (TMAE) tma_prefetch_desc(&mapX);
+    if (ADD) tma_prefetch_desc(&mapD);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
@@ -684,13 +881,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int row = sub * 32 + lane;
     const int acc = grp;
     uint32_t acc_phase = 0;
-    const uint32_t stg = smem_u32(staging) + (uint32_t)(e * 4096);
+    const uint32_t stg = smem_u32(staging) + (uint32_t)(e * Cfg::WARP_BUF);
     EpiStats stats;
     stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
+    if constexpr (TMAE)  // (the host launches these only with TMA stores of rows in pixel order)
+      epilogue_bs<BN, ADD>(p, &mapC, &mapX, &mapD, staging + e * Cfg::WARP_BUF, ebar + 2 * e, tfull, tempty,
+                           tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, mt_count, mscale, rank, lim,
+                           abort_flag, stats);
     const bool bstats = BS && p.st_mean && p.bs_x && p.tma_store;
     BwdIn bin;
-    for (int u = cid + grp * ncl; u < total; u += 2 * ncl) {
+    for (int u = cid + grp * ncl; u < total && !TMAE; u += 2 * ncl) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
       unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
@@ -832,55 +1033,72 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN, bool PAIR, bool BS = false>
+template <int BN, bool PAIR, int EPI = EPI_PLAIN>
 static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR, BS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         GemmCfg<BN>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
   return cudaSuccess;
 }
 
+template <int BN, bool PAIR, int EPI>
+static cudaError_t launch_variant(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                                  const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
+                                  cudaStream_t s) {
+  cudaError_t e = set_smem_attr<BN, PAIR, EPI>();
+  if (e != cudaSuccess) return e;
+  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM;
+  if (PAIR)
+    launch_pdl_cluster2(k_gemm<BN, PAIR, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
+  else
+    launch_pdl(k_gemm<BN, PAIR, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
+  return counted_launches(1);
+}
+
+template <int BN, bool PAIR>
+static cudaError_t launch_epi(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
+                              const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
+                              int epi, cudaStream_t s) {
+  switch (epi) {
+    case EPI_PLAIN: return launch_variant<BN, PAIR, EPI_PLAIN>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS: return launch_variant<BN, PAIR, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS_TMA: return launch_variant<BN, PAIR, EPI_BS_TMA>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS_ADD: return launch_variant<BN, PAIR, EPI_BS_ADD>(mA, mB, mC, mX, mD, p, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 template <int BN>
 static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                               const GemmParams& p, int grid, bool pair, cudaStream_t s) {
-  const bool bs = p.bs_x != nullptr;
-  if (!pair) {
-    cudaError_t e = bs ? set_smem_attr<BN, false, true>() : set_smem_attr<BN, false, false>();
-    if (e != cudaSuccess) return e;
-    if (bs)
-      launch_pdl(k_gemm<BN, false, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
-    else
-      launch_pdl(k_gemm<BN, false, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB, mC, p);
-    return counted_launches(1);
-  }
+                               const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
+                               bool pair, cudaStream_t s) {
+  const int epi = gemm_epilogue(p);
+  if (epi != EPI_PLAIN && (!p.tma_store || p.out_mode != OUT_STORE)) return cudaErrorInvalidValue;
+  if (!pair) return launch_epi<BN, false>(mA, mB, mC, mX, mD, p, grid, epi, s);
   if constexpr (BN >= 128) {
     if (grid % 2 != 0 || p.m_tiles % 2 != 0) return cudaErrorInvalidValue;
-    cudaError_t e = bs ? set_smem_attr<BN, true, true>() : set_smem_attr<BN, true, false>();
-    if (e != cudaSuccess) return e;
-    if (bs)
-      launch_pdl_cluster2(k_gemm<BN, true, true>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB,
-                          mC, p);
-    else
-      launch_pdl_cluster2(k_gemm<BN, true, false>, dim3(grid), dim3(kGemmThreads), GemmCfg<BN>::SMEM, s, mA, mB,
-                          mC, p);
-    return counted_launches(1);
+    return launch_epi<BN, true>(mA, mB, mC, mX, mD, p, grid, epi, s);
   }
   return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                        const GemmParams& p, int grid, cudaStream_t s, bool pair) {
+                        const GemmParams& p, int grid, cudaStream_t s, bool pair, const CUtensorMap* mX,
+                        const CUtensorMap* mD) {
+  // the BatchNorm-input and addend maps (unused without backward statistics)
+  const CUtensorMap& x = mX ? *mX : mC;
+  const CUtensorMap& d = mD ? *mD : x;
   switch (BN) {
-    case 64: return launch_bn_t<64>(mA, mB, mC, p, grid, pair, s);
-    case 128: return launch_bn_t<128>(mA, mB, mC, p, grid, pair, s);
-    case 192: return launch_bn_t<192>(mA, mB, mC, p, grid, pair, s);
-    case 256: return launch_bn_t<256>(mA, mB, mC, p, grid, pair, s);
+    case 64: return launch_bn_t<64>(mA, mB, mC, x, d, p, grid, pair, s);
+    case 128: return launch_bn_t<128>(mA, mB, mC, x, d, p, grid, pair, s);
+    case 192: return launch_bn_t<192>(mA, mB, mC, x, d, p, grid, pair, s);
+    case 256: return launch_bn_t<256>(mA, mB, mC, x, d, p, grid, pair, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -900,7 +1118,7 @@ static int pair_clusters_t() {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true, false>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true, EPI_PLAIN>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }

@@ -155,6 +155,12 @@ struct GemmParams {
   const uint16_t* bs_mean;
   const uint16_t* bs_invstd;
   int bs_levels;
+  // With the backward statistics only: an addend of the output, out =
+  // rn(result + add_src) where add_mask's bit ([pixels][N/8], as bs_mask) is
+  // set and out = rn(result + 0) elsewhere; add_src [pixels][N], pitch ldo.
+  // The statistics are taken of that sum.  Null: no addend.
+  const uint16_t* add_src;
+  const uint8_t* add_mask;
 };
 
 // Conv-output BatchNorm statistics buffer (pf16_conv_fwd_bnstats): a header of
@@ -174,9 +180,25 @@ __host__ __device__ inline size_t bnstat_bytes(long long C) {
 // Launch the engine (BN in {64, 128, 192, 256}).  pair: clusters of two CTAs
 // sharing each B tile by multicast (BN >= 128, p.m_tiles and grid even; the
 // grid then counts CTAs, two per tile pair).  Returns a cudaError_t.
+// Epilogue kinds of the conv GEMM (k_gemm's EPI).  The backward statistics
+// take the TMA-fed epilogue for short reductions (at most kTmaEpiMaxKb
+// K-blocks per tile: there the epilogue's traffic is the bound) and always
+// with an addend; else their inputs go through registers, which leaves the
+// main loop all of its pipeline stages.
+enum GemmEpi : int { EPI_PLAIN = 0, EPI_BS = 1, EPI_BS_TMA = 2, EPI_BS_ADD = 3 };
+constexpr int kTmaEpiMaxKb = 8;
+inline int gemm_epilogue(const GemmParams& p) {
+  if (!p.bs_x) return EPI_PLAIN;
+  if (p.add_src) return EPI_BS_ADD;
+  return p.kb_per_split <= kTmaEpiMaxKb ? EPI_BS_TMA : EPI_BS;
+}
+
+// mapX / mapD: 128B-swizzled 32 x 64 boxes over bs_x and add_src ([M][N],
+// pitch ldo), needed with the backward statistics (and the addend).
 cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const CUtensorMap& mapC, const GemmParams& p, int grid,
-                        cudaStream_t stream, bool pair = false);
+                        cudaStream_t stream, bool pair = false, const CUtensorMap* mapX = nullptr,
+                        const CUtensorMap* mapD = nullptr);
 int gemm_smem_bytes(int BN);
 // Clusters of two GEMM CTAs (tile width BN) that can be resident at once (0: none).
 int gemm_pair_clusters(int BN);

@@ -37,7 +37,7 @@ EXPORTS = [
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
     "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
-    "pf16_conv_dgrad_bnstats",
+    "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add",
 ]
 
 
@@ -102,6 +102,9 @@ def lib():
             L.pf16_conv_dgrad_bnstats.argtypes = [cdp, vp, vp, vp, vp, sz, ctypes.POINTER(BnSource), vp, sz,
                                                   vp]
             L.pf16_conv_dgrad_bnstats.restype = I
+            L.pf16_conv_dgrad_bnstats_add.argtypes = [cdp, vp, vp, vp, vp, sz, ctypes.POINTER(BnSource), vp, vp,
+                                                      vp, sz, vp]
+            L.pf16_conv_dgrad_bnstats_add.restype = I
             L.pf16_conv_wgrad_noalloc.argtypes = [cdp, vp, vp, vp, u32, vp]
             L.pf16_conv_wgrad_noalloc.restype = I
             L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
@@ -207,6 +210,17 @@ def conv_dgrad_bnstats(d, dy, w, dx, x, relu_mask, mean, invstd, stats, ws=None,
     _check(lib().pf16_conv_dgrad_bnstats(ctypes.byref(d), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws),
                                          _nbytes(ws), ctypes.byref(src), _ptr(stats), _nbytes(stats),
                                          _stream(stream)), "pf16_conv_dgrad_bnstats")
+
+
+def conv_dgrad_bnstats_add(d, dy, w, dx, x, relu_mask, mean, invstd, add, add_mask, stats, ws=None,
+                           stream=None):
+    """conv_dgrad_bnstats with dx = rn(data gradient + add where add_mask's bit
+    is set); add_mask None: the whole of add."""
+    src = BnSource(_ptr(x), _ptr(relu_mask), _ptr(mean), _ptr(invstd))
+    _check(lib().pf16_conv_dgrad_bnstats_add(ctypes.byref(d), _ptr(dy), _ptr(w), _ptr(dx), _ptr(ws),
+                                             _nbytes(ws), ctypes.byref(src), _ptr(add), _ptr(add_mask),
+                                             _ptr(stats), _nbytes(stats), _stream(stream)),
+           "pf16_conv_dgrad_bnstats_add")
 
 
 def conv_wgrad(d, x, dy, dw, ws=None, flags=0, stream=None):

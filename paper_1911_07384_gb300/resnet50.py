@@ -114,10 +114,16 @@ class Conv:
         else:
             self.net.call("conv_fwd", self, pf16.conv_fwd, self.desc, x, self.w, y, self.net.ws)
 
-    def dgrad(self, dy, dx, accumulate=False, bn=None):
+    def dgrad(self, dy, dx, accumulate=False, bn=None, add=None):
         """bn: (BN layer, its input x) when dx is that BatchNorm's output gradient and
-        this layer can take its backward statistics (stride 1); see BN.bwd(conv=)."""
-        if bn is not None:
+        this layer can take its backward statistics (stride 1); see BN.bwd(conv=).
+        add (with bn, 1x1 only): (tensor, bit mask) added to the data gradient where
+        the mask's bit is set -- an identity shortcut's share of dx."""
+        if bn is not None and add is not None:
+            layer, x = bn
+            self.net.call("conv_dgrad", self, pf16.conv_dgrad_bnstats_add, self.desc, dy, self.w, dx, x,
+                          layer.mask, layer.mean, layer.invstd, add[0], add[1], self.dstats)
+        elif bn is not None:
             layer, x = bn
             self.net.call("conv_dgrad", self, pf16.conv_dgrad_bnstats, self.desc, dy, self.w, dx, x, layer.mask,
                           layer.mean, layer.invstd, self.dstats)
@@ -137,6 +143,7 @@ class BN:
         self.net = net
         flags = (pf16.PF16_BN_RELU if relu else 0) | (pf16.PF16_BN_RESIDUAL if residual else 0)
         flags |= pf16.PF16_BN_SWAP if swap else 0
+        self.swap = swap
         self.desc = pf16.bn_desc(n, h, w, c, EPS, post_scale, flags)
         self.c = c
         self.zero_gamma = zero_gamma
@@ -190,6 +197,9 @@ class Bottleneck:
             self.convp = Conv(net, n, h, h, cin, cout, 1, 1, stride, 0)
             self.bnp = BN(net, n, h2, h2, cout, S_BLOCK, relu=False)
         self.h, self.h2, self.n, self.cout = h, h2, n, cout
+        # the layer whose data gradient carries bn3's backward statistics (the
+        # next block's conv1, set by that block's backward), or None
+        self.bn3_stats_conv = None
 
     def allocate(self, dev):
         n, h, h2, w, c = self.n, self.h, self.h2, self.width, self.cout
@@ -220,12 +230,25 @@ class Bottleneck:
             self.bn3.fwd(self.a3, self.y, residual=x, conv=self.conv3)
         return self.y
 
-    def backward(self, dx):
-        """self.dy holds dL/dy; writes dL/dx into dx."""
+    def fuses_prev(self, prev):
+        """Whether this block's first data gradient can produce the whole of
+        dL/dx (shortcut share added in its epilogue) and, with it, the backward
+        statistics of prev's last BatchNorm (prev: the block whose output is
+        this block's input)."""
+        return (not self.proj and self.conv1.fuses_bwd_stats() and prev.bn3.mask is not None
+                and self.bn3.mask is not None and not prev.bn3.swap and not self.bn3.swap)
+
+    def backward(self, dx, prev=None):
+        """self.dy holds dL/dy; writes dL/dx into dx.  prev: the block whose
+        output is this block's input, or None."""
+        fuse = prev is not None and self.fuses_prev(prev)
+        bn3_conv = self.bn3_stats_conv
         if self.proj:
-            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=self.dres, residual=self.bp)
-        else:  # identity shortcut: its gradient is the start of dx
-            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=dx, residual=self.x)
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=self.dres, residual=self.bp,
+                         conv=bn3_conv)
+        else:  # identity shortcut: its gradient (dy where the ReLU passed) is the start of dx
+            self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=None if fuse else dx, residual=self.x,
+                         conv=bn3_conv)
         self.conv3.wgrad(self.b2, self.da3)
         # the data gradients also reduce the next BatchNorm's backward statistics
         self.conv3.dgrad(self.da3, self.db2, bn=(self.bn2, self.a2))
@@ -240,8 +263,15 @@ class Bottleneck:
             self.bnp.bwd(self.ap, None, self.dres, self.dap)
             self.convp.wgrad(self.x, self.dap)
             self.convp.dgrad(self.dap, dx, accumulate=True)
+        elif fuse:
+            # dx = shortcut share + data gradient in one epilogue, which also
+            # reduces prev.bn3's backward statistics
+            self.conv1.dgrad(self.da1, dx, bn=(prev.bn3, prev.a3), add=(self.dy, self.bn3.mask))
+            prev.bn3_stats_conv = self.conv1
         else:
             self.conv1.dgrad(self.da1, dx, accumulate=True)
+            if prev is not None:
+                prev.bn3_stats_conv = None
 
 
 class ResNet50:
@@ -353,7 +383,7 @@ class ResNet50:
                   self.cl)
         for i in range(len(self.blocks) - 1, -1, -1):
             dx = self.blocks[i - 1].dy if i > 0 else self.dp0
-            self.blocks[i].backward(dx)
+            self.blocks[i].backward(dx, self.blocks[i - 1] if i > 0 else None)
         self.call("maxpool_bwd", None, pf16.maxpool_bwd_argmax, self.pool_arg, self.dp0, self.db0, self.N,
                   self.h0, self.h0, 64)
         self.bn0.bwd(self.a0, self.b0, self.db0, self.da0)

@@ -75,6 +75,23 @@ def test_conv_validation_errors():
     assert pf16.conv_dgrad_bnstats_size(s2) == 0
     assert dg(ctypes.byref(s2), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, sz,
               None) == pf16.PF16_ERR_UNSUPPORTED
+    # ... plus a masked addend: 1x1 stride 1 only, no overlap with dx
+    da = L.pf16_conv_dgrad_bnstats_add
+    one = pf16.conv_desc(2, 8, 8, 256, 64, 1, 1, 1, 0)
+    sz1 = pf16.conv_dgrad_bnstats_size(one)
+    far = ctypes.c_void_p(0x1000000)  # past dx's 2*8*8*256*2 bytes at FAKE
+    assert da(ctypes.byref(one), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), None, None, FAKE, sz1,
+              None) == pf16.PF16_ERR_NULL
+    assert da(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), far, None, FAKE, sz,
+              None) == pf16.PF16_ERR_UNSUPPORTED  # 3x3
+    assert da(ctypes.byref(one), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, None, FAKE, sz1,
+              None) == pf16.PF16_ERR_ARG  # add is dx
+    assert da(ctypes.byref(one), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), ctypes.c_void_p(0x10100), None,
+              FAKE, sz1, None) == pf16.PF16_ERR_ARG  # add overlaps dx
+    assert da(ctypes.byref(one), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), ctypes.c_void_p(0x1000008), None,
+              FAKE, sz1, None) == pf16.PF16_ERR_ALIGN
+    assert da(ctypes.byref(one), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), far, ctypes.c_void_p(0x2000004),
+              FAKE, sz1, None) == pf16.PF16_ERR_ALIGN  # mask not 8-byte aligned
 
 
 def test_workspace_sizes_are_host_computable():

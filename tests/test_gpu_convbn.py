@@ -92,6 +92,8 @@ BWD_SHAPES = [
     ((2, 56, 56, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 64 (columns 56..63 dropped)
     ((2, 14, 14, 128, 128, 3, 3, 1, 1), True),   # stride-1 im2col data gradient, paired CTAs
     ((1, 7, 7, 64, 64, 3, 3, 1, 1), True),       # one partial tile (49 rows)
+    ((2, 7, 7, 256, 1024, 1, 1, 1, 0), True),    # long reduction (16 K-blocks): register-fed epilogue
+    ((4, 14, 14, 256, 128, 1, 1, 1, 0), True),   # short reduction, many tiles per CTA: TMA-fed epilogue
 ]
 
 
@@ -133,7 +135,15 @@ def test_conv_dgrad_bnstats_then_bn_bwd(orc, case):
     assert pf16.sync_status() == 0
     g = host(dx)
     assert np.array_equal(g, host(dx_ref))  # the statistics do not touch the data gradient
+    check_bn_bwd_from_stats(orc, bd, bws, tx, tg, tm, ti, ty, tmask, dx, stats, xb, gamma, beta, N * H * W, C,
+                            s, relu)
 
+
+def check_bn_bwd_from_stats(orc, bd, bws, tx, tg, tm, ti, ty, tmask, dx, stats, xb, gamma, beta, rows, C, s,
+                            relu):
+    """The BatchNorm backward (phase 1) from the fused statistics in `stats`
+    against the oracle's on the same dy = dx."""
+    g = host(dx)
     tdx, tdg, tdb = empty16(rows * C), empty16(C), empty16(C)
     pf16.bn_fwd_bwd(bd, 1, bws, x=tx, gamma=tg, mean=tm, invstd=ti, dy=dx, y_saved=ty, relu_mask=tmask,
                     dx=tdx, dgamma=tdg, dbeta=tdb, conv_stats=stats)
@@ -162,3 +172,57 @@ def test_conv_dgrad_bnstats_rejects_strided():
     with pytest.raises(pf16.PF16Error):
         pf16.conv_dgrad_bnstats(d, empty16(2 * 7 * 7 * 64), empty16(64 * 9 * 64), t, t, None, empty16(64),
                                 empty16(64), stats)
+
+
+ADD_SHAPES = [
+    # 1x1 stride-1 data gradients whose dx also takes a masked addend
+    (2, 14, 14, 256, 64, 1, 1, 1, 0),    # paired CTAs, one n-tile of 256
+    (3, 7, 7, 512, 128, 1, 1, 1, 0),     # two n-tiles, 147 rows (a partial M tile)
+    (1, 7, 7, 64, 64, 1, 1, 1, 0),       # 64-wide tile, one partial M tile
+]
+
+
+@pytest.mark.parametrize("shape", ADD_SHAPES, ids=ids)
+@pytest.mark.parametrize("masked", [True, False], ids=["mask", "nomask"])
+def test_conv_dgrad_bnstats_add(orc, shape, masked):
+    """pf16_conv_dgrad_bnstats_add: dx bit-identical to the masked addend
+    followed by pf16_conv_dgrad with PF16_ACCUMULATE (Sec. 4.2's identity
+    shortcut: dresidual plus the first convolution's data gradient); the
+    BatchNorm backward from its statistics within the bound of the test
+    above."""
+    N, H, W, C, K, R, S, st, pd = shape
+    rows = N * H * W
+    w = syn.he_normal_f16(syn.seed_for(9, "w"), K, R, S, C)
+    dyc = syn.normal_f16(syn.seed_for(9, "dy"), (N, H, W, K), 0.05)
+    add = syn.normal_f16(syn.seed_for(9, 6), (rows, C), 0.05)
+    gate = syn.normal_f16(syn.seed_for(9, 7), (rows, C))     # the addend's ReLU decisions
+    on = f64(gate).reshape(rows, C) > 0
+    add_mask = np.packbits(on, axis=1, bitorder="little").reshape(-1)
+    xb = syn.normal_f16(syn.seed_for(9, "x"), (rows, C))
+    gamma = f16(1.0 + 0.1 * f64(syn.normal_f16(17, (C,))))
+    beta = f16(0.1 * f64(syn.normal_f16(18, (C,))))
+    s = 0.25
+    bd = pf16.bn_desc(N, H, W, C, EPS, int(f16([s])[0]), pf16.PF16_BN_RELU)
+    bws = workspace(pf16.bn_workspace_size(bd))
+    tx, tg, tb = dev(xb), dev(gamma), dev(beta)
+    ty, tm, ti = empty16(rows * C), empty16(C), empty16(C)
+    tmask = torch.empty(rows * C // 8, dtype=torch.uint8, device="cuda")
+    pf16.bn_fwd_bwd(bd, 0, bws, x=tx, gamma=tg, beta=tb, y=ty, mean=tm, invstd=ti, relu_mask=tmask)
+    assert pf16.sync_status() == 0
+
+    d = pf16.conv_desc(*shape)
+    stats = torch.empty(pf16.conv_dgrad_bnstats_size(d), dtype=torch.uint8, device="cuda")
+    tdyc, tw, tadd = dev(dyc), dev(w), dev(add)
+    tam = torch.from_numpy(add_mask).to("cuda") if masked else None
+    # the two-call path: the masked addend (exact), then the accumulating data gradient
+    a_eff = add.reshape(rows, C).copy()
+    if masked:
+        a_eff[~on] = 0
+    dx_ref = dev(a_eff.reshape(-1))
+    pf16.conv_dgrad(d, tdyc, tw, dx_ref, None, pf16.PF16_ACCUMULATE)
+    dx = empty16(rows * C)
+    pf16.conv_dgrad_bnstats_add(d, tdyc, tw, dx, tx, tmask, tm, ti, tadd, tam, stats)
+    assert pf16.sync_status() == 0
+    assert np.array_equal(host(dx), host(dx_ref))
+    check_bn_bwd_from_stats(orc, bd, bws, tx, tg, tm, ti, ty, tmask, dx, stats, xb, gamma, beta, rows, C, s,
+                            True)
