@@ -297,36 +297,40 @@ struct EpiStats {
 
   // leaf of chunk c from the staged tile (row r at stg + r*128, 128B-swizzled)
   __device__ __forceinline__ void leaf(int c, uint32_t stg, int lane, int nv) {
+    if (nv == 32)  // a full leaf (every tile but a tensor's last): no row tests
+      leaf_impl<true>(c, stg, lane, nv);
+    else
+      leaf_impl<false>(c, stg, lane, nv);
+  }
+  template <bool FULL>
+  __device__ __forceinline__ void leaf_impl(int c, uint32_t stg, int lane, int nv) {
     const uint32_t col = (uint32_t)(lane & 3) * 4;
-    uint32_t t[32];
+    uint32_t x[32], t[32];  // the 32 rows' channel pair, read once
 #pragma unroll
     for (int r = 0; r < 32; ++r) {
-      uint32_t x;
-      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
-      t[r] = r < nv ? x : 0u;
+      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x[r]) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
+      t[r] = (FULL || r < nv) ? x[r] : 0u;
     }
 #pragma unroll
     for (int w = 16; w >= 1; w /= 2)
 #pragma unroll
       for (int i = 0; i < w; ++i) t[i] = hmerge2f(t[2 * i], t[2 * i + 1]);
     uint32_t mu = t[0], sc = 0;
-    if (nv < 32) {
+    if (!FULL && nv < 32) {
       sc = dup2h(__half_as_ushort(__float2half_rn(32.0f / (float)nv)));
       mu = hmul2_rn(mu, sc);
     }
 #pragma unroll
     for (int r = 0; r < 32; ++r) {
-      uint32_t x;
-      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(stg + r * 128 + ((((uint32_t)lane >> 2) ^ (r & 7)) << 4) + col));
-      const uint32_t e = hsub2_rn(x, mu);
-      t[r] = r < nv ? hmul2_rn(e, e) : 0u;
+      const uint32_t e = hsub2_rn(x[r], mu);
+      t[r] = (FULL || r < nv) ? hmul2_rn(e, e) : 0u;
     }
 #pragma unroll
     for (int w = 16; w >= 1; w /= 2)
 #pragma unroll
       for (int i = 0; i < w; ++i) t[i] = hmerge2f(t[2 * i], t[2 * i + 1]);
     uint32_t var = t[0];
-    if (nv < 32) var = hmul2_rn(var, sc);
+    if (!FULL && nv < 32) var = hmul2_rn(var, sc);
     // push into chunk c's stack (counts are updated by end_tile)
     int nn = nv;
 #pragma unroll 1
@@ -428,6 +432,9 @@ struct EpiStats {
   template <class XF>
   __device__ __forceinline__ void leaf_bwd_core(int c, uint32_t stg, int lane, int nv, uint2 m, uint32_t mean2,
                                                 uint32_t invstd2, XF xf);
+  template <bool FULL, class XF>
+  __device__ __forceinline__ void leaf_bwd_impl(int c, uint32_t stg, int lane, int nv, uint2 m, uint32_t mean2,
+                                                uint32_t invstd2, XF xf);
   // Close the backward counters as if zero leaves padded them to 2^levels,
   // merge the CTA's 8 epilogue warps by halving (warps 0..7 in a balanced
   // tree, through `sm` as write_cta) and write the CTA's nodes as `slot`.
@@ -506,6 +513,15 @@ struct BwdIn {
 template <class XF>
 __device__ __forceinline__ void EpiStats::leaf_bwd_core(int c, uint32_t stg, int lane, int nv, uint2 m,
                                                         uint32_t mean2, uint32_t invstd2, XF xf) {
+  if (nv == 32)  // a full leaf: no row tests
+    leaf_bwd_impl<true>(c, stg, lane, nv, m, mean2, invstd2, xf);
+  else
+    leaf_bwd_impl<false>(c, stg, lane, nv, m, mean2, invstd2, xf);
+}
+
+template <bool FULL, class XF>
+__device__ __forceinline__ void EpiStats::leaf_bwd_impl(int c, uint32_t stg, int lane, int nv, uint2 m,
+                                                        uint32_t mean2, uint32_t invstd2, XF xf) {
   const uint32_t col = (uint32_t)(lane & 3) * 4;
   uint32_t t1[32], t2[32];
 #pragma unroll
@@ -517,9 +533,9 @@ __device__ __forceinline__ void EpiStats::leaf_bwd_core(int c, uint32_t stg, int
     const uint32_t mlo = __shfl_sync(0xffffffffu, m.x, r), mhi = __shfl_sync(0xffffffffu, m.y, r);
     const uint32_t b = (lane < 16 ? mlo >> (2 * lane) : mhi >> (2 * lane - 32)) & 3u;
     const uint32_t mk = ((b & 1u) ? 0x0000FFFFu : 0u) | ((b & 2u) ? 0xFFFF0000u : 0u);
-    const uint32_t d = r < nv ? (g & mk) : 0u;
+    const uint32_t d = (FULL || r < nv) ? (g & mk) : 0u;
     t1[r] = d;
-    t2[r] = r < nv ? hmul2_rn(d, hmul2_rn(hsub2_rn(xf(r, off), mean2), invstd2)) : 0u;
+    t2[r] = (FULL || r < nv) ? hmul2_rn(d, hmul2_rn(hsub2_rn(xf(r, off), mean2), invstd2)) : 0u;
   }
 #pragma unroll
   for (int w = 16; w >= 1; w /= 2)
