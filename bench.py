@@ -177,6 +177,9 @@ def main():
     ap.add_argument("--sweep", default=None, choices=["cfg2", "cfg3"],
                     help="per-layer conv lines: cfg2 = every distinct ResNet-50 conv at N=64, "
                          "cfg3 = the N=256 pure-GEMM 1x1 layers")
+    ap.add_argument("--tc-rate", action="store_true",
+                    help="the library's MMA-only probe: kind::f16 tcgen05 TFLOP/s for N = 64..256, f16 and f32 "
+                         "accumulators, one or two accumulator chains; one JSON line each")
     args = ap.parse_args()
     rank, world, local = dist_env()
     if args.ingest_traffic:
@@ -191,6 +194,8 @@ def main():
         return run_sweep(args)
     if args.layers:
         return run_layers(args)
+    if args.tc_rate:
+        return run_tc_rate()
     if args.bn:
         print(json.dumps(time_bn(tuple(int(v) for v in args.bn.split(",")), args.bn_pass, args.steps,
                                  args.warmup)), flush=True)
@@ -324,6 +329,28 @@ def main():
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+    return 0
+
+
+def run_tc_rate():
+    """pf16_tc_rate over tile widths, accumulator types and chain counts, against
+    the measured bf16 cuBLAS peaks the rooflines use."""
+    import torch
+
+    from paper_1911_07384_gb300 import pf16
+
+    torch.cuda.init()
+    pk = peaks()
+    for n in (64, 128, 192, 256):
+        for f32 in (False, True):
+            for chains in (1, 2):
+                tf = pf16.tc_rate(n, f32_accum=f32, chains=chains, reps=20000)
+                print(json.dumps({"probe": "tcgen05.mma kind::f16 M=128", "n": n, "accumulator": "f32" if f32 else "f16",
+                                  "chains": chains, "tflops": tf,
+                                  "of_bf16_burst": tf / pk["bf16_tflops"], "peak_src": pk["src"]}),
+                      flush=True)
+    if pf16.sync_status() != 0:
+        raise RuntimeError("device status after the rate probe")
     return 0
 
 

@@ -322,6 +322,22 @@ int pf16_device_arch(void);
  * the paper). */
 uint64_t pf16_kernel_launches(void);
 
+/* ------------------------------------------------------------ diagnostics
+ * Tensor-core rate probe: the 16-bit dense rate of the instruction the
+ * convolutions issue, measured by the library's own MMA-only kernel (the
+ * conv rooflines are quoted against a cuBLAS bf16 GEMM; this is the check
+ * that FP16 accumulation runs at that rate; not part of the paper's method).
+ * One CTA per SM issues reps x 4 tcgen05.mma kind::f16 (M = 128, N = n,
+ * K = 16; f16 operands resident in shared memory; f16 accumulator, or f32
+ * with f32_accum = 1) into one TMEM accumulator (chains = 1: each MMA adds
+ * onto the previous one, as along a GEMM's K loop) or two in turn
+ * (chains = 2).  After a warm-up launch, times one launch with CUDA events on
+ * `stream` and writes 2*128*n*16 flop per MMA / time, in TFLOP/s, to *tflops.
+ * Synchronous (waits for the stream).  n in {64, 128, 192, 256}, f32_accum
+ * and chains as above, 1 <= reps <= 2^20 (PF16_ERR_ARG otherwise); tflops
+ * non-NULL.  A bounded wait that expires is reported by pf16_sync_status. */
+int pf16_tc_rate(int32_t n, int32_t f32_accum, int32_t chains, int32_t reps, double* tflops, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpf16.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
-SOURCES = ["pf16_api.cu", "pf16_gemm.cu", "pf16_elementwise.cu", "pf16_noalloc.cu"]
+SOURCES = ["pf16_api.cu", "pf16_gemm.cu", "pf16_elementwise.cu", "pf16_noalloc.cu", "pf16_probe.cu"]
 HEADERS = ["pf16_internal.h", "pf16_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v",

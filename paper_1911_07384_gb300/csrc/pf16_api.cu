@@ -1193,6 +1193,38 @@ int pf16_sync_status(void* stream) {
   return v;
 }
 
+int pf16_tc_rate(int32_t n, int32_t f32_accum, int32_t chains, int32_t reps, double* tflops, void* stream) {
+  if (!tflops) return PF16_ERR_NULL;
+  if ((n != 64 && n != 128 && n != 192 && n != 256) || (f32_accum != 0 && f32_accum != 1) ||
+      (chains != 1 && chains != 2) || reps < 1 || reps > (1 << 20))
+    return PF16_ERR_ARG;
+  int* status;
+  int sms;
+  int rc = device_consts(&status, &sms);
+  if (rc != PF16_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const uint32_t idesc = idesc_f16(kBM, n, false, false, f32_accum != 0);
+  cudaEvent_t e0, e1;
+  if (cudaEventCreate(&e0) != cudaSuccess) return PF16_ERR_CUDA;
+  if (cudaEventCreate(&e1) != cudaSuccess) {
+    cudaEventDestroy(e0);
+    return PF16_ERR_CUDA;
+  }
+  const unsigned long long wait_ns = 4000000000ull;
+  float ms = 0.f;
+  bool ok = launch_tc_rate(idesc, n, chains, reps / 4 + 1, sms, status, wait_ns, st) == cudaSuccess &&  // warm-up
+            cudaEventRecord(e0, st) == cudaSuccess &&
+            launch_tc_rate(idesc, n, chains, reps, sms, status, wait_ns, st) == cudaSuccess &&
+            cudaEventRecord(e1, st) == cudaSuccess && cudaEventSynchronize(e1) == cudaSuccess &&
+            cudaEventElapsedTime(&ms, e0, e1) == cudaSuccess;
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  if (!ok || ms <= 0.f) return PF16_ERR_CUDA;
+  const double flop = (double)sms * reps * 4.0 * 2.0 * kBM * n * 16.0;
+  *tflops = flop / ((double)ms * 1e-3) / 1e12;
+  return PF16_OK;
+}
+
 const char* pf16_status_string(int status) {
   switch (status) {
     case PF16_OK: return "ok";

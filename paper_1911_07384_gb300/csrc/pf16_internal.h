@@ -193,6 +193,11 @@ inline int gemm_epilogue(const GemmParams& p) {
   return p.kb_per_split <= kTmaEpiMaxKb ? EPI_BS_TMA : EPI_BS;
 }
 
+// The tensor-core rate probe (pf16_tc_rate): reps x 4 kind::f16 MMAs of
+// M = 128, N = n per CTA, grid CTAs (one per SM).
+cudaError_t launch_tc_rate(uint32_t idesc, int n, int chains, int reps, int grid, int* status,
+                           unsigned long long wait_ns, cudaStream_t s);
+
 // mapX / mapD: 128B-swizzled 32 x 64 boxes over bs_x and add_src ([M][N],
 // pitch ldo), needed with the backward statistics (and the addend).
 cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,

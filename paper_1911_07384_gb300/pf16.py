@@ -37,7 +37,7 @@ EXPORTS = [
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
     "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
-    "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add",
+    "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add", "pf16_tc_rate",
 ]
 
 
@@ -131,6 +131,8 @@ def lib():
             L.pf16_sync_status.restype = I
             L.pf16_status_string.argtypes = [I]
             L.pf16_status_string.restype = ctypes.c_char_p
+            L.pf16_tc_rate.argtypes = [i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), vp]
+            L.pf16_tc_rate.restype = I
             L.pf16_device_arch.argtypes = []
             L.pf16_device_arch.restype = I
             L.pf16_kernel_launches.argtypes = []
@@ -309,3 +311,12 @@ def kernel_launches() -> int:
 
 def loaded_path() -> str:
     return os.path.abspath(_build.LIB)
+
+
+def tc_rate(n, f32_accum=False, chains=1, reps=20000, stream=None) -> float:
+    """TFLOP/s of the library's MMA-only probe (pf16_tc_rate): kind::f16
+    tcgen05 MMAs of M = 128, N = n from shared memory, on every SM."""
+    out = ctypes.c_double(0.0)
+    _check(lib().pf16_tc_rate(int(n), 1 if f32_accum else 0, int(chains), int(reps), ctypes.byref(out),
+                              _stream(stream)), "pf16_tc_rate")
+    return out.value

@@ -94,6 +94,15 @@ def test_conv_validation_errors():
               FAKE, sz1, None) == pf16.PF16_ERR_ALIGN  # mask not 8-byte aligned
 
 
+def test_tc_rate_validation_errors():
+    L = pf16.lib()
+    out = ctypes.c_double(0.0)
+    assert L.pf16_tc_rate(256, 0, 1, 100, None, None) == pf16.PF16_ERR_NULL
+    for n, f32, chains, reps in [(96, 0, 1, 100), (256, 2, 1, 100), (256, 0, 3, 100), (256, 0, 1, 0),
+                                 (64, 0, 1, (1 << 20) + 1)]:
+        assert L.pf16_tc_rate(n, f32, chains, reps, ctypes.byref(out), None) == pf16.PF16_ERR_ARG
+
+
 def test_workspace_sizes_are_host_computable():
     cfg3 = pf16.conv_desc(256, 56, 56, 256, 64, 1, 1, 1, 0)
     assert pf16.conv_workspace_size(cfg3, pf16.PF16_PASS_FWD) == 0
