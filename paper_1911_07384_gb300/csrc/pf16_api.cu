@@ -287,6 +287,29 @@ StemWgradPlan stem_wgrad_plan(const Shape& s) {
 }
 size_t stem_wgrad_parts_bytes(const StemWgradPlan& w) { return round_up((size_t)w.chunks * 128 * 128 * 2, 256); }
 
+// The 3x3 / stride 1 / pad 1 weight gradient with 64 input and 64 output
+// channels on padded rows of 64 pixels (W + 2 <= 64): units of two output
+// rows, at most 32 units (4,096 padded pixels) per FP16 accumulation and at
+// most 1,024 chunks for the split-K tree.
+struct Wgrad3Plan {
+  bool ok;
+  long long units;
+  int per_chunk, chunks;
+};
+Wgrad3Plan wgrad3_plan(const Shape& s) {
+  Wgrad3Plan w{false, 0, 0, 0};
+  if (s.kind != KIND_GENERIC || s.R != 3 || s.S != 3 || s.st != 1 || s.pad != 1 || s.C != 64 || s.K != 64 ||
+      s.W + 2 > 64)
+    return w;
+  w.units = s.N * ((s.P + 2) / 2);
+  w.per_chunk = 32;
+  if (cdiv(w.units, w.per_chunk) > 1024) w.per_chunk = (int)cdiv(w.units, 1024);
+  w.chunks = (int)cdiv(w.units, w.per_chunk);
+  w.ok = w.units < (1ll << 30);
+  return w;
+}
+size_t wgrad3_parts_bytes(const Wgrad3Plan& w) { return round_up((size_t)w.chunks * 64 * 576 * 2, 256); }
+
 size_t ws_fwd(const Shape& s) {
   if (s.kind != KIND_STEM) return 0;
   const long long kc = stem_kcol(s);
@@ -298,6 +321,8 @@ size_t ws_fwd(const Shape& s) {
 size_t ws_wgrad(const Shape& s) {
   const StemWgradPlan sw = stem_wgrad_plan(s);
   if (sw.ok) return stem_s2d_bytes(s) + stem_wgrad_parts_bytes(sw) + 128 * 128 * 2;
+  const Wgrad3Plan w3 = wgrad3_plan(s);
+  if (w3.ok) return wgrad3_parts_bytes(w3);
   const WgradSplit w = wgrad_split(s);
   size_t b = 0;
   if (w.splits > 1 || s.kind == KIND_STEM) b += round_up((size_t)w.splits * s.K * w.ncols * 2, 256);
@@ -905,6 +930,48 @@ static int run_stem_wgrad(const Shape& s, const StemWgradPlan& sw, const uint16_
   return PF16_OK;
 }
 
+// The 3x3, 64 -> 64 weight gradient through k_wgrad3x3_halo (layouts at
+// wgrad3_plan), then the split-K tree straight into dw.
+static int run_wgrad3x3(const Shape& s, const Wgrad3Plan& w3, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
+                        void* work, int* status, int sms, cudaStream_t st, bool f32) {
+  const long long N = s.N, H = s.H, W = s.W, P = s.P, Q = s.Q;
+  uint16_t* parts = static_cast<uint16_t*>(work);
+  CUtensorMap mdy, mx;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  {
+    cuuint64_t dims[4] = {64, (cuuint64_t)Q, (cuuint64_t)P, (cuuint64_t)N};
+    cuuint64_t strides[3] = {128, (cuuint64_t)(Q * 128), (cuuint64_t)(P * Q * 128)};
+    cuuint32_t box[4] = {64, 64, 3, 1};
+    if (g_encode_tiled(&mdy, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<uint16_t*>(dy), dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  {
+    cuuint64_t dims[4] = {64, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t strides[3] = {128, (cuuint64_t)(W * 128), (cuuint64_t)(H * W * 128)};
+    cuuint32_t box[4] = {64, 64, 4, 1};
+    if (g_encode_tiled(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<uint16_t*>(x), dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
+  p.idesc = idesc_f16(kBM, 192, true, true, f32);
+  p.halo_ws = 64;
+  p.halo_h = (int)P;
+  p.halo_w = (int)Q;
+  p.num_kb = (int)w3.units;
+  p.kb_per_split = w3.per_chunk;
+  p.m_tiles = w3.chunks;
+  p.out = parts;
+  const int grid = w3.chunks < sms ? w3.chunks : sms;
+  if (launch_wgrad3x3_halo(mdy, mx, p, grid, st) != cudaSuccess) return PF16_ERR_CUDA;
+  if (launch_splitk_reduce(parts, w3.chunks, 64, 576, dw, 576, 576, st) != cudaSuccess) return PF16_ERR_CUDA;
+  return PF16_OK;
+}
+
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
   Shape s;
@@ -923,6 +990,8 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const StemWgradPlan sw = stem_wgrad_plan(s);
   if (sw.ok) return run_stem_wgrad(s, sw, x, dy, dw, ws, status, sms, st, f32);
+  const Wgrad3Plan w3 = wgrad3_plan(s);
+  if (w3.ok) return run_wgrad3x3(s, w3, x, dy, dw, ws, status, sms, st, f32);
   const WgradSplit wsp = wgrad_split(s);
 
   GemmParams p = base_params(status);

@@ -1686,4 +1686,238 @@ cudaError_t launch_stem_wgrad(const CUtensorMap& mDy, const CUtensorMap& mXs, co
   return counted_launches(1);
 }
 
+// ---------------------------------------------------------------------------
+// Weight gradient of the 3x3 / stride 1 / pad 1 convolution with 64 input and
+// 64 output channels (the 56x56 layers of ResNet-50), on padded rows of
+// ws = 64 pixels (W + 2 <= ws).  Output pixel (i, j) is padded pixel p = i*ws + j
+// of dy (zero at j >= W); the input grid holds x[i][j' - 1] at column j'
+// (zero outside the image), so that
+//   dW[k][r][s][c] = sum_p dy[p][k] * xp[p + (r - 1)*ws + s][c].
+// One MMA (M = 128, N = 192, K = 16 pixels, both operands MN-major, 128-byte
+// swizzle) covers three filter columns and two filter rows:
+//   A = the 64 channels of dy at pixels p - ws (M rows 0..63) and p (rows
+//       64..127): two M atoms one padded row apart (LBO = ws * 128 B);
+//   B = the input at p + u*ws + s - ws for s = 0, 1, 2: three 64-channel N
+//       atoms one pixel apart (LBO = 128 B; the 128-byte swizzle is a function
+//       of the absolute address, so a window may start at any row).
+// For output row i, u = 0 accumulates filter row 0 in M rows 64..127 (dy row i
+// against input row i - 1) and filter row 1 in rows 0..63 (dy row i - 1 against
+// input row i - 1); u = 1 accumulates filter row 2 in rows 0..63 (the same
+// product for rows 64..127, filter row 1 again, is discarded).  Summing over
+// i = 0 .. P (dy rows -1 and P read as zeros) covers every term once.  A unit
+// is two output rows (i0, i0 + 1) of one image: a stage holds dy rows
+// i0 - 1 .. i0 + 1 (3 x 64 x 128 B) and input rows i0 - 1 .. i0 + 2
+// (4 x 64 x 128 B; a window reaches past its row only at columns where dy is
+// zero).  Units are accumulated in FP16 in TMEM (two 192-column accumulators,
+// u = 0 and 1) over chunks of p.kb_per_split units (4,096 padded pixels), and
+// each chunk's 64 x 576 partial [k][(r, s, c)] goes to p.out + chunk * 64 * 576
+// for the split-K tree, laid out as the weight gradient itself.  Roles and
+// bounded waits as k_stem_wgrad; the accumulators are single-buffered (2 x 192
+// of the 512 columns), so a chunk's MMAs wait for the previous chunk's drain.
+// ---------------------------------------------------------------------------
+struct Wgrad3Cfg {
+  static constexpr int WS = 64;
+  static constexpr int DY_BYTES = 3 * WS * 128;  // dy rows i0 - 1 .. i0 + 1
+  static constexpr int X_BYTES = 4 * WS * 128;   // input rows i0 - 1 .. i0 + 2
+  static constexpr int STAGE = DY_BYTES + X_BYTES;
+  static constexpr int STAGES = 3;
+  static constexpr int TMEM_COLS = 512;          // accumulators u = 0, 1 at columns 0 and 192
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 2) + 16;
+  static constexpr int SMEM = 1024 + STAGES * STAGE + BAR_BYTES;
+};
+constexpr int kWgrad3Threads = 192;
+
+__global__ void __launch_bounds__(kWgrad3Threads, 1)
+    k_wgrad3x3_halo(const __grid_constant__ CUtensorMap mapDy, const __grid_constant__ CUtensorMap mapX,
+                    const __grid_constant__ GemmParams p) {
+  using Cfg = Wgrad3Cfg;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + Cfg::STAGES;
+  uint64_t* tfull = bars + 2 * Cfg::STAGES;
+  uint64_t* tempty = tfull + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < Cfg::STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    mbar_init(smem_u32(tfull), 1);
+    mbar_init(smem_u32(tempty), 4);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&mapDy);
+    tma_prefetch_desc(&mapX);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  pdl_wait();
+  const uint32_t tmem_base = *tmem_slot;
+  const int units = p.num_kb;            // N * ceil((P + 1) / 2) two-row units
+  const int per_chunk = p.kb_per_split;  // units per accumulation
+  const int chunks = p.m_tiles;
+  const int upi = (p.halo_h + 2) / 2;    // units per image: output rows i = 0 .. P in pairs
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, issued = 0;
+      for (int c = blockIdx.x; c < chunks && !*abort_flag; c += gridDim.x) {
+        const int g1 = min(units, (c + 1) * per_chunk);
+        for (int g = c * per_chunk; g < g1 && !*abort_flag; ++g) {
+          const int n = g / upi, i0 = 2 * (g - n * upi);
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim)) {
+            record_timeout(p, abort_flag);
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[stage]);
+          const uint32_t dst = smem_u32(smem + stage * Cfg::STAGE);
+          mbar_arrive_expect_tx(fb, (uint32_t)Cfg::STAGE);
+          tma_load_4d(dst, &mapDy, fb, 0, 0, i0 - 1, n);
+          tma_load_4d(dst + Cfg::DY_BYTES, &mapX, fb, 0, -1, i0 - 1, n);
+          ++issued;
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (*abort_flag) {  // let every copy this thread started land before the CTA can exit
+        const uint32_t nn = issued < (uint32_t)Cfg::STAGES ? issued : (uint32_t)Cfg::STAGES;
+        int s = stage;
+        uint32_t ph = phase;
+        for (uint32_t q = 0; q < nn; ++q) {
+          if (--s < 0) {
+            s = Cfg::STAGES - 1;
+            ph ^= 1;
+          }
+          mbar_wait(smem_u32(&full[s]), ph, 1000000000ull);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // A: dy, MN-major 128-byte swizzle, M atoms one padded row apart, 8-pixel
+      // K groups 1 KB apart; B: the input, three N atoms one pixel apart
+      const uint64_t adesc0 = smem_desc(0, Cfg::WS * 128, 1024, 2);
+      const uint64_t bdesc0 = smem_desc(0, 128, 1024, 2);
+      int stage = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true;
+      for (int c = blockIdx.x; ok && c < chunks && !*abort_flag; c += gridDim.x) {
+        if (!mbar_wait(smem_u32(tempty), acc_phase ^ 1, lim)) {
+          record_timeout(p, abort_flag);
+          break;
+        }
+        tc_fence_after();
+        const int g0 = c * per_chunk, g1 = min(units, (c + 1) * per_chunk);
+        for (int g = g0; g < g1; ++g) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, lim)) {
+            record_timeout(p, abort_flag);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa16 = desc_addr16(smem_u32(smem + stage * Cfg::STAGE));
+          const uint64_t ab = adesc0 + sa16;
+          const uint64_t bb = bdesc0 + sa16 + (Cfg::DY_BYTES >> 4);
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int js = 0; js < Cfg::WS / 16; ++js)
+#pragma unroll
+              for (int u = 0; u < 2; ++u)
+                tc_mma_f16(tmem_base + (uint32_t)(u * 192), ab + (uint32_t)((h * Cfg::WS * 128 + js * 2048) >> 4),
+                           bb + (uint32_t)(((h + u) * Cfg::WS * 128 + js * 2048) >> 4), p.idesc,
+                           (g > g0 || h > 0 || js > 0) ? 1u : 0u);
+          tc_commit(smem_u32(&empty[stage]));
+          if (++stage == Cfg::STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(tfull));
+        acc_phase ^= 1;
+      }
+    }
+  } else {
+    // epilogue warps 2..5 -> TMEM sub-partitions 2, 3, 0, 1.  Row m < 64: k = m,
+    // filter rows 1 (u = 0) and 2 (u = 1); m >= 64: k = m - 64, filter row 0 (u = 0).
+    const int sub = warp & 3;
+    const int m = sub * 32 + lane;
+    const int k = m & 63;
+    uint32_t acc_phase = 0;
+    for (int c = blockIdx.x; c < chunks; c += gridDim.x) {
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      const bool got = mbar_wait(smem_u32(tfull), acc_phase, lim);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) record_timeout(p, abort_flag);
+        break;
+      }
+      tc_fence_after();
+      uint16_t* prow = p.out + ((size_t)c * 64 + k) * 576;
+#pragma unroll 1
+      for (int u = 0; u < 2; ++u) {
+        if (u == 1 && m >= 64) continue;  // warp-uniform: sub-partitions 2, 3 hold rows 64..127
+        const int r = u == 0 ? (m < 64 ? 1 : 0) : 2;
+        uint4* dst = reinterpret_cast<uint4*>(prow + r * 192);
+#pragma unroll 1
+        for (int cc = 0; cc < 192; cc += 64) {
+          const uint32_t tb = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(u * 192 + cc);
+          uint32_t v[64];
+          tmem_ld16(tb, v);
+          tmem_ld16(tb + 16, v + 16);
+          tmem_ld16(tb + 32, v + 32);
+          tmem_ld16(tb + 48, v + 48);
+          tmem_ld_wait();
+          if (p.d_f32) f32_to_f16_lo<64>(v);  // FP32 accumulator: one rounding to FP16
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            dst[cc / 8 + j] = make_uint4(pack_lo(v[j * 8 + 0], v[j * 8 + 1]), pack_lo(v[j * 8 + 2], v[j * 8 + 3]),
+                                         pack_lo(v[j * 8 + 4], v[j * 8 + 5]), pack_lo(v[j * 8 + 6], v[j * 8 + 7]));
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(tempty));
+      acc_phase ^= 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+  }
+}
+
+cudaError_t launch_wgrad3x3_halo(const CUtensorMap& mDy, const CUtensorMap& mX, const GemmParams& p, int grid,
+                                 cudaStream_t s) {
+  if (p.kb_per_split < 1 || p.m_tiles < 1 || grid < 1 || p.halo_h < 1) return cudaErrorInvalidValue;
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !attr_set[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(k_wgrad3x3_halo, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Wgrad3Cfg::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  launch_pdl(k_wgrad3x3_halo, dim3(grid), dim3(kWgrad3Threads), Wgrad3Cfg::SMEM, s, mDy, mX, p);
+  return counted_launches(1);
+}
+
 }  // namespace pf16

@@ -221,6 +221,11 @@ int gemm_pair_clusters(int BN);
 // (16, 128, 4, 1); p.num_kb = N * (P + 1) row units, p.kb_per_split units per
 // chunk, p.m_tiles chunks, p.halo_h = P, p.halo_ws = 128, p.out = the chunks'
 // 128 x 128 FP16 partials.
+// The 3x3 / stride 1 / pad 1, 64 -> 64 channel weight gradient on padded rows
+// of 64 pixels (k_wgrad3x3_halo): p.num_kb two-row units, p.kb_per_split per
+// chunk, p.m_tiles chunks, p.halo_h = P; partials [chunk][64][576] at p.out.
+cudaError_t launch_wgrad3x3_halo(const CUtensorMap& mDy, const CUtensorMap& mX, const GemmParams& p, int grid,
+                                 cudaStream_t s);
 cudaError_t launch_stem_wgrad(const CUtensorMap& mapDy, const CUtensorMap& mapXs, const GemmParams& p, int grid,
                               cudaStream_t s);
 cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,

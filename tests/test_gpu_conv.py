@@ -160,10 +160,12 @@ def test_delta_kernel_bit_exact(orc, r0, s0, st):
     assert np.array_equal(f64(dx), V)
 
 
-def test_delta_gradient_wgrad_bit_exact(orc):
+@pytest.mark.parametrize("shape", [(2, 8, 8, 64, 128, 3, 3, 1, 1),    # im2col GEMM
+                                   (2, 9, 12, 64, 64, 3, 3, 1, 1)],  # halo weight gradient, odd P
+                         ids=ids)
+def test_delta_gradient_wgrad_bit_exact(orc, shape):
     """dy nonzero (= 1) at a single pixel per channel: every dw element is one
     product x * 1, exact in FP16."""
-    shape = (2, 8, 8, 64, 128, 3, 3, 1, 1)
     N, H, W, C, K, R, S, st, pd = shape
     x, _, _, P, Q = inputs(shape, seed_cfg=3)
     dyf = np.zeros((N, P, Q, K), np.float16)
@@ -177,13 +179,14 @@ def test_delta_gradient_wgrad_bit_exact(orc):
 
 
 CFG3 = [(256, 56, 56, 256, 64, 1, 1, 1, 0), (256, 28, 28, 512, 128, 1, 1, 1, 0),
-        (256, 14, 14, 1024, 256, 1, 1, 1, 0), (256, 7, 7, 512, 2048, 1, 1, 1, 0)]
+        (256, 14, 14, 1024, 256, 1, 1, 1, 0), (256, 7, 7, 512, 2048, 1, 1, 1, 0),
+        (256, 56, 56, 64, 64, 3, 3, 1, 1)]  # the 3x3 64-channel layer: halo engines, 802,816-pixel weight gradient
 
 
 @pytest.mark.parametrize("shape", CFG3, ids=ids)
 def test_full_size_sampled(orc, shape):
-    """The N=256 pure-GEMM 1x1 layers at full size, checked on sampled outputs
-    (wgrad reductions of up to 802,816 pixels)."""
+    """The N=256 pure-GEMM 1x1 layers and the 56x56 3x3 64-channel layer at
+    full size, checked on sampled outputs (wgrad reductions of 802,816 pixels)."""
     N, H, W, C, K, R, S, st, pd = shape
     x, w, dy, P, Q = inputs(shape, seed_cfg=3)
     d = pf16.conv_desc(*shape)
