@@ -302,7 +302,10 @@ Wgrad3Plan wgrad3_plan(const Shape& s) {
       s.W + 2 > 64)
     return w;
   w.units = s.N * ((s.P + 2) / 2);
-  w.per_chunk = 32;
+  // as many rounds of 152 chunks (GB300's SM count) as 32-unit chunks need,
+  // the units spread evenly over them
+  const long long rounds = cdiv(w.units, 32ll * 152);
+  w.per_chunk = (int)cdiv(w.units, rounds * 152);
   if (cdiv(w.units, w.per_chunk) > 1024) w.per_chunk = (int)cdiv(w.units, 1024);
   w.chunks = (int)cdiv(w.units, w.per_chunk);
   w.ok = w.units < (1ll << 30);

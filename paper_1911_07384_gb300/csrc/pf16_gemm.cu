@@ -1720,10 +1720,11 @@ struct Wgrad3Cfg {
   static constexpr int DY_BYTES = 3 * WS * 128;  // dy rows i0 - 1 .. i0 + 1
   static constexpr int X_BYTES = 4 * WS * 128;   // input rows i0 - 1 .. i0 + 2
   static constexpr int STAGE = DY_BYTES + X_BYTES;
-  static constexpr int STAGES = 3;
+  static constexpr int STAGES = 4;
   static constexpr int TMEM_COLS = 512;          // accumulators u = 0, 1 at columns 0 and 192
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 2) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE + BAR_BYTES;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 constexpr int kWgrad3Threads = 192;
 
