@@ -270,19 +270,51 @@ def main():
     loss = float(np.uint16(net.loss.cpu().numpy().view(np.uint16)[0]).view(np.float16))
     value = world * N * args.steps / (ms_max / 1e3)
 
-    # ---------------- end to end through host buffers (pinned), copies in the timed region
+    # ---------------- end to end through host buffers (pinned), copies in the timed region.
+    # Two input buffers, as a prefetching loader keeps them: step i reads buffer i % 2,
+    # whose host-to-device copy ran on a copy stream while step i - 1 computed; a copy
+    # into a buffer waits for the step that last read it.  Every step's copies and its
+    # loss read-back lie between the two events.
+    x_bufs, l_bufs = [net.x, torch.empty_like(net.x)], [net.labels, torch.empty_like(net.labels)]
+    net.x, net.labels = x_bufs[1], l_bufs[1]
+    graph_b = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph_b, stream=stream):
+        net.step()
+    net.x, net.labels = x_bufs[0], l_bufs[0]
+    graphs = [graph, graph_b]
     h_img = torch.from_numpy(imgs.reshape(-1).view(np.int16)).pin_memory()
     h_lab = torch.from_numpy(labs.astype(np.int32)).pin_memory()
     h_loss = torch.empty(1, dtype=torch.int16).pin_memory()
+    copy_stream = torch.cuda.Stream()
+    done = [torch.cuda.Event(), torch.cuda.Event()]
+    ready = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def load(b, after=None):
+        with torch.cuda.stream(copy_stream):
+            if after is not None:
+                copy_stream.wait_event(after)
+            x_bufs[b].copy_(h_img, non_blocking=True)
+            l_bufs[b].copy_(h_lab, non_blocking=True)
+            ready[b].record(copy_stream)
+
+    for b in (0, 1):  # warm both graphs on their own buffers
+        load(b)
+        stream.wait_event(ready[b])
+        graphs[b].replay()
+    torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         e0.record(stream)
-        for _ in range(args.steps):
-            net.x.copy_(h_img, non_blocking=True)
-            net.labels.copy_(h_lab, non_blocking=True)
-            graph.replay()
+        load(0, after=e0)
+        for i in range(args.steps):
+            b = i % 2
+            if i + 1 < args.steps:
+                load(1 - b, after=done[1 - b] if i >= 1 else e0)
+            stream.wait_event(ready[b])
+            graphs[b].replay()
+            done[b].record(stream)
             h_loss.copy_(net.loss, non_blocking=True)
         e1.record(stream)
     torch.cuda.synchronize()
@@ -563,6 +595,15 @@ TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_resnet50_b256_step_traffic
 GEMM_SOURCES = ["pf16_gemm.cu", "pf16_api.cu", "pf16_internal.h", "pf16_ptx.cuh"]
 
 
+def wgrad_is_gemm(h, w, c, k, r, s, st, pad):
+    """Whether a layer's weight gradient runs as k_gemm launches: not the stem's
+    (k_stem_wgrad) nor the 3x3 64-channel layers' on padded rows of 64
+    (k_wgrad3x3_halo)."""
+    if c == 3:
+        return False
+    return not (r == 3 and s == 3 and st == 1 and pad == 1 and c == 64 and k == 64 and w + 2 <= 64)
+
+
 def gemm_source_digest():
     """sha256 over the conv GEMM kernel and the code that plans its launches."""
     import hashlib
@@ -596,9 +637,9 @@ def ingest_traffic(csv_path):
     from paper_1911_07384_gb300.resnet50 import conv_shapes
 
     # per conv: forward + data gradient (one GEMM per stride phase) + weight
-    # gradient; the stem has a forward only (its weight gradient is k_stem_wgrad)
-    step = sum(1 if c == 3 else 2 + (st * st if r > 1 else 1)
-               for _, (_, _, _, c, _, r, _, st, _) in conv_shapes(BATCH))
+    # gradient where it is a k_gemm launch; the stem has no data gradient
+    step = sum(1 + (0 if c == 3 else (st * st if r > 1 else 1)) + (1 if wgrad_is_gemm(h, w, c, k, r, s, st, pd) else 0)
+               for _, (_, h, w, c, k, r, s, st, pd) in conv_shapes(BATCH))
     ids = sorted(per, key=int)[:step]  # the first whole step (the eager warm-up step)
     if len(ids) < step:
         raise SystemExit(f"{csv_path}: {len(ids)} k_gemm launches, one step has {step}")
@@ -695,10 +736,11 @@ def conv_roofline(net, stream, reps=3):
         Q = (d.w + 2 * d.pad - d.s) // d.stride + 1
         one = 2 * (d.n * d.h * d.w * d.c + d.k * d.r * d.s * d.c + d.n * P * Q * d.k)
         stem = d.c == 3
-        # the k_gemm launches the stored traffic covers: every pass but the stem's weight
-        # gradient (k_stem_wgrad)
-        byts += one * (1 if stem else 3)
-        gemms += 1 if stem else 2 + (d.stride * d.stride if d.r > 1 else 1)
+        # the k_gemm launches the stored traffic covers: every pass but the weight
+        # gradients of other kernels (k_stem_wgrad, k_wgrad3x3_halo)
+        wg = wgrad_is_gemm(d.h, d.w, d.c, d.k, d.r, d.s, d.stride, d.pad)
+        byts += one * ((1 if stem else 2) + (1 if wg else 0))
+        gemms += 1 + (0 if stem else (d.stride * d.stride if d.r > 1 else 1)) + (1 if wg else 0)
     out = {"ms": ms, "gflop": gflop, "tflops": gflop / ms, "by_pass": {}, "bytes_per_launch": byts / gemms}
     for k, (t, f) in by_pass.items():
         out["by_pass"][k] = {"ms": t / reps, "tflops": (f / reps) / 1e9 / (t / reps) if t else None}
