@@ -221,7 +221,7 @@ def main():
     from paper_1911_07384_gb300.resnet50 import ResNet50
 
     N = args.batch
-    net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap)
+    net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap, wgrad_branch=True)
     imgs = syn.images_f16(syn.seed_for(4, "x", rank), N)
     labs = syn.labels(syn.seed_for(4, "labels", rank), N)
     net.set_batch(imgs, labs)
@@ -712,6 +712,7 @@ def conv_roofline(net, stream, reps=3):
 
     totals = []
     by_pass = {"conv_fwd": [0.0, 0.0], "conv_dgrad": [0.0, 0.0], "conv_wgrad": [0.0, 0.0]}
+    side, net.side = net.side, None  # per-call events need every call on `stream`, in program order
     for _ in range(reps):
         recs.clear()
         net.hook = hook
@@ -726,6 +727,7 @@ def conv_roofline(net, stream, reps=3):
             by_pass[kind][0] += t
             by_pass[kind][1] += layer.flops
         totals.append(ms)
+    net.side = side
     ms = float(np.median(totals))
     gflop = net.conv_flops() / 1e9
     # algorithmic bytes of a pass: |x| + |w| + |y| in FP16, each touched once

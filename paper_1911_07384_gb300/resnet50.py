@@ -135,7 +135,15 @@ class Conv:
         return self.dstats is not None
 
     def wgrad(self, x, dy):
-        self.net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, self.net.ws)
+        net = self.net
+        if net.side is None:
+            net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, net.ws)
+            return
+        # only the update reads the weight gradient: it runs on a branch of its own
+        # (with its own workspace), off the chain of data gradients and BatchNorms
+        net.side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(net.side):
+            net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, net.ws_w)
 
 
 class BN:
@@ -277,9 +285,15 @@ class Bottleneck:
 class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
-    def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False):
+    def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False,
+                 wgrad_branch=False):
+        """wgrad_branch: issue the weight gradients on a second stream that joins
+        before the update (in a captured step graph: a parallel branch), so that
+        they fill the gaps of the data-gradient chain; off, every call runs on the
+        current stream in program order (what per-call timing needs)."""
         self.N, self.image, self.classes, self.device = batch, image, classes, device
         self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
+        self.side = torch.cuda.Stream(device=device) if wgrad_branch else None
         self.wd, self.nowd = Arena("decayed"), Arena("no-decay")
         self.convs, self.bns = [], []
         N = batch
@@ -336,6 +350,9 @@ class ResNet50:
             ws = max(ws, pf16.bn_workspace_size(b.desc))
         ws = max(ws, pf16.softmax_xent_workspace_size(N, self.classes))
         self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
+        # the weight gradients' own scratch when they run on the side branch
+        wsw = max(pf16.conv_workspace_size(c.desc, pf16.PF16_PASS_WGRAD) for c in self.convs)
+        self.ws_w = torch.empty(max(wsw, 256), dtype=torch.uint8, device=dev) if self.side is not None else None
 
     def _init_params(self):
         """He-normal conv / FC weights (std sqrt(2 / fan_in)), FC bias 0, BN gamma
@@ -390,6 +407,8 @@ class ResNet50:
         self.stem.wgrad(self.x, self.da0)
 
     def update(self):
+        if self.side is not None:  # every weight gradient is in before the update reads it
+            torch.cuda.current_stream().wait_stream(self.side)
         self.call("sgd", None, pf16.sgd_update, self.wd.w, self.wd.v, self.wd.g, LR, MOMENTUM, WD)
         self.call("sgd", None, pf16.sgd_update, self.nowd.w, self.nowd.v, self.nowd.g, LR, MOMENTUM, 0)
 

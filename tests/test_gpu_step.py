@@ -107,3 +107,22 @@ def test_swap_variant_step():
     net.step()
     assert pf16.sync_status() == 0
     assert np.isfinite(float(f64(host(net.loss))[0]))
+
+
+def test_weight_gradient_branch_is_bit_identical():
+    """Weight gradients on a side branch that joins before the update (the
+    captured step graph of bench.py) give the same bits as program order: two
+    steps, every weight, momentum and loss compared exactly."""
+    results = []
+    for branch in (False, True):
+        net = ResNet50(batch=2, image=64, seed_cfg=4, wgrad_branch=branch)
+        net.set_batch(syn.images_f16(syn.seed_for(4, "x"), 2, 64, 64, 3), syn.labels(syn.seed_for(4, "labels"), 2))
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            net.step()
+            net.step()
+        torch.cuda.synchronize()
+        assert pf16.sync_status(stream) == 0
+        results.append([t.clone() for t in (net.wd.w, net.wd.v, net.nowd.w, net.nowd.v, net.loss)])
+    for a, b in zip(*results):
+        assert torch.equal(a, b)
