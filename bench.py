@@ -106,6 +106,24 @@ def dist_env():
             int(os.environ.get("LOCAL_RANK", 0)))
 
 
+def max_over_ranks(v, dist, device):
+    """The largest of every rank's v: a replica job ends with its slowest rank
+    (dist None: one process)."""
+    if dist is None:
+        return float(v)
+    import torch
+
+    t = torch.tensor([float(v)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world, per_rank_batch, steps, ms):
+    """Images per second of the whole job: every rank's images over the slowest
+    rank's time (weak scaling: each rank trains its own batch)."""
+    return world * per_rank_batch * steps / (ms / 1e3)
+
+
 # --------------------------------------------------------------------------- CPU oracle
 def oracle_step_time(batch=1, image=224, reps=1):
     """Time the oracle's ResNet-50 training step (binary64 C loops, OpenMP) on
@@ -262,13 +280,9 @@ def main():
     rc = pf16.sync_status(stream)
     if rc != 0:
         raise RuntimeError(f"device status {rc} after timed steps")
-    ms_max = ms
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_max = float(t.item())
+    ms_max = max_over_ranks(ms, dist, "cuda")
     loss = float(np.uint16(net.loss.cpu().numpy().view(np.uint16)[0]).view(np.float16))
-    value = world * N * args.steps / (ms_max / 1e3)
+    value = job_throughput(world, N, args.steps, ms_max)
 
     # ---------------- end to end through host buffers (pinned), copies in the timed region.
     # Two input buffers, as a prefetching loader keeps them: step i reads buffer i % 2,
@@ -318,12 +332,8 @@ def main():
             h_loss.copy_(net.loss, non_blocking=True)
         e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": world * N * args.steps / (e2e_ms / 1e3), "unit": UNIT,
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+    e2e = {"value": job_throughput(world, N, args.steps, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": int(h_img.numel() * 2 + h_lab.numel() * 4), "d2h_bytes_per_step": 2}
 
     # ---------------- dominant kernel (the tcgen05 conv GEMM): per-call CUDA events
