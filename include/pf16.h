@@ -322,6 +322,23 @@ int pf16_device_arch(void);
  * the paper). */
 uint64_t pf16_kernel_launches(void);
 
+/* Stream-ordered bounded wait on a device flag: enqueues one single-thread
+ * kernel that polls the 32-bit word *flag (device memory, or mapped pinned
+ * host memory; acquire loads at system scope) until it equals `value`, for at
+ * most timeout_ns nanoseconds of GPU global-timer time.  If the time runs out
+ * the kernel records PF16_ERR_TIMEOUT in the device status word (read and
+ * cleared by pf16_sync_status) and returns: work queued after it on the
+ * stream still runs and the CUDA context stays usable.  This is the failure
+ * detection of the library's bounded device-side waits in its smallest form:
+ * a producer that never signals (a host thread, a copy on another stream, a
+ * peer rank that died) turns into a status code instead of a hung GPU.  No
+ * counterpart in the paper.  flag non-NULL (PF16_ERR_NULL) and 4-byte
+ * aligned (PF16_ERR_ALIGN); timeout_ns <= 10^10, i.e. 10 s (PF16_ERR_ARG).
+ * The flag must be set by something that does not wait on this stream: a
+ * kernel that sets it queued behind this one on the same stream never runs
+ * in time. */
+int pf16_wait_flag(const uint32_t* flag, uint32_t value, uint64_t timeout_ns, void* stream);
+
 /* ------------------------------------------------------------ diagnostics
  * Tensor-core rate probe: the 16-bit dense rate of the instruction the
  * convolutions issue, measured by the library's own MMA-only kernel (the

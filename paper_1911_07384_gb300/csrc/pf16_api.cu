@@ -1265,6 +1265,19 @@ int pf16_sync_status(void* stream) {
   return v;
 }
 
+int pf16_wait_flag(const uint32_t* flag, uint32_t value, uint64_t timeout_ns, void* stream) {
+  if (!flag) return PF16_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(flag) & 3u) != 0) return PF16_ERR_ALIGN;
+  if (timeout_ns > 10000000000ull) return PF16_ERR_ARG;
+  int* status;
+  int sms;
+  int rc = device_consts(&status, &sms);
+  if (rc != PF16_OK) return rc;
+  return launch_wait_flag(flag, value, timeout_ns, status, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
 int pf16_tc_rate(int32_t n, int32_t f32_accum, int32_t chains, int32_t reps, double* tflops, void* stream) {
   if (!tflops) return PF16_ERR_NULL;
   if ((n != 64 && n != 128 && n != 192 && n != 256) || (f32_accum != 0 && f32_accum != 1) ||

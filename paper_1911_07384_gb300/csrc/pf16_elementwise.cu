@@ -1893,4 +1893,31 @@ cudaError_t launch_softmax_xent(const uint16_t* logits, const uint16_t* bias,
   return counted_launches(2);
 }
 
+// ============================================================================
+// Bounded wait on a device flag: one thread polls *flag (acquire, system
+// scope, so a host write through mapped pinned memory is seen as well) until
+// it holds `value`, or until limit_ns of %globaltimer time have passed; then it
+// records PF16_ERR_TIMEOUT in the status word (the first error stays) and
+// returns, so the stream moves on and the context stays usable.
+// ============================================================================
+__global__ void k_wait_flag(const uint32_t* flag, uint32_t value, unsigned long long limit_ns, int* status) {
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    uint32_t v;
+    asm volatile("ld.acquire.sys.global.u32 %0, [%1];" : "=r"(v) : "l"(flag) : "memory");
+    if (v == value) return;
+    if (globaltimer_ns() - t0 > limit_ns) {
+      atomicCAS(status, 0, -7);  // PF16_ERR_TIMEOUT
+      return;
+    }
+    __nanosleep(256);
+  }
+}
+
+cudaError_t launch_wait_flag(const uint32_t* flag, uint32_t value, unsigned long long limit_ns, int* status,
+                             cudaStream_t s) {
+  k_wait_flag<<<1, 1, 0, s>>>(flag, value, limit_ns, status);
+  return counted_launches(1);
+}
+
 }  // namespace pf16

@@ -237,6 +237,10 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, c
 // ---------------------------------------------------------------------------
 cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
                        uint16_t mom, uint16_t wd, cudaStream_t s);
+// one thread waits (bounded by limit_ns) for *flag == value; expiry records
+// PF16_ERR_TIMEOUT in *status.  A plain launch: it starts after its predecessor.
+cudaError_t launch_wait_flag(const uint32_t* flag, uint32_t value, unsigned long long limit_ns, int* status,
+                             cudaStream_t s);
 // sum of `splits` FP16 partial matrices [splits][rows][cols] by a balanced
 // pairwise tree; the result row r goes to out + r*ldo (only cols_out columns).
 cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long rows, int cols,

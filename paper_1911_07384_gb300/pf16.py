@@ -37,7 +37,7 @@ EXPORTS = [
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
     "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
-    "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add", "pf16_tc_rate",
+    "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add", "pf16_tc_rate", "pf16_wait_flag",
 ]
 
 
@@ -133,6 +133,8 @@ def lib():
             L.pf16_status_string.restype = ctypes.c_char_p
             L.pf16_tc_rate.argtypes = [i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double), vp]
             L.pf16_tc_rate.restype = I
+            L.pf16_wait_flag.argtypes = [vp, ctypes.c_uint32, ctypes.c_uint64, vp]
+            L.pf16_wait_flag.restype = I
             L.pf16_device_arch.argtypes = []
             L.pf16_device_arch.restype = I
             L.pf16_kernel_launches.argtypes = []
@@ -320,3 +322,11 @@ def tc_rate(n, f32_accum=False, chains=1, reps=20000, stream=None) -> float:
     _check(lib().pf16_tc_rate(int(n), 1 if f32_accum else 0, int(chains), int(reps), ctypes.byref(out),
                               _stream(stream)), "pf16_tc_rate")
     return out.value
+
+
+def wait_flag(flag, value, timeout_ns, stream=None):
+    """Enqueue a bounded wait until the int32 device word `flag` equals `value`
+    (pf16_wait_flag); an expired wait shows up in sync_status() as
+    PF16_ERR_TIMEOUT."""
+    _check(lib().pf16_wait_flag(_ptr(flag), int(value) & 0xFFFFFFFF, int(timeout_ns), _stream(stream)),
+           "pf16_wait_flag")

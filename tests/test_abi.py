@@ -144,3 +144,10 @@ def test_other_validation_errors():
     assert L.pf16_avgpool_fwd(FAKE, None, 1, 49, 64, None) == pf16.PF16_ERR_NULL
     assert L.pf16_softmax_xent(FAKE, None, FAKE, 4, 5000, FAKE, FAKE, None, FAKE, 1 << 20,
                                None) == pf16.PF16_ERR_UNSUPPORTED
+
+
+def test_wait_flag_validation_errors():
+    L = pf16.lib()
+    assert L.pf16_wait_flag(None, 1, 1000, None) == pf16.PF16_ERR_NULL
+    assert L.pf16_wait_flag(FAKE_MIS, 1, 1000, None) == pf16.PF16_ERR_ALIGN
+    assert L.pf16_wait_flag(FAKE, 1, 10_000_000_001, None) == pf16.PF16_ERR_ARG
