@@ -186,6 +186,9 @@ def main():
     ap.add_argument("--bn", default=None,
                     help="time one BatchNorm pass instead of the step: N,H,W,C (ReLU + residual, s=0.25)")
     ap.add_argument("--bn-pass", default="fwd", choices=["fwd", "bwd"])
+    ap.add_argument("--nvtx", action="store_true",
+                    help="name every library call of the step with an NVTX range (pf16:<kind>:<shape>) for "
+                         "profilers; host-side only, the replayed step graph is unchanged")
     ap.add_argument("--bn-swap", action="store_true",
                     help="the BN-swap variant (Sec. 4.1) in every block's last BatchNorm (off in the headline run)")
     ap.add_argument("--layers", action="store_true",
@@ -240,6 +243,10 @@ def main():
 
     N = args.batch
     net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap, wgrad_branch=True)
+    if args.nvtx:
+        from paper_1911_07384_gb300.resnet50 import nvtx_hook
+
+        net.hook = nvtx_hook
     imgs = syn.images_f16(syn.seed_for(4, "x", rank), N)
     labs = syn.labels(syn.seed_for(4, "labels", rank), N)
     net.set_batch(imgs, labs)

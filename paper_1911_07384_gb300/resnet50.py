@@ -282,6 +282,27 @@ class Bottleneck:
                 prev.bn3_stats_conv = None
 
 
+def layer_label(layer):
+    """Shape label of a Conv or BN layer ("n,h,w,c[,k,r,s,stride,pad]"), "-" for none."""
+    d = getattr(layer, "desc", None)
+    if d is None:
+        return "-" if layer is None else str(layer)
+    keep = ("n", "h", "w", "c", "k", "r", "s", "stride", "pad")
+    return ",".join(str(getattr(d, f[0])) for f in d._fields_ if f[0] in keep)
+
+
+def nvtx_hook(kind, layer, fn, *args, **kw):
+    """Instrumentation hook (ResNet50(hook=nvtx_hook)): wraps each library call
+    in an NVTX range "pf16:<kind>:<layer>", so that profilers can attribute
+    kernels to calls (e.g. ncu --nvtx --nvtx-include "pf16:bn_bwd*/").  The
+    ranges are host-side only; a step captured into a CUDA graph carries none."""
+    torch.cuda.nvtx.range_push(f"pf16:{kind}:{layer_label(layer)}")
+    try:
+        return fn(*args, **kw)
+    finally:
+        torch.cuda.nvtx.range_pop()
+
+
 class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
