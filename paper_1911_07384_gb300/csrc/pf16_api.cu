@@ -402,7 +402,7 @@ GemmParams base_params(int* status) {
 }
 
 // Levels of an epilogue warp's padded tile tree (backward statistics): `ctas`
-// CTAs (or CTA pairs) share `units` tiles round robin, and each CTA's two
+// CTAs share `units` tiles round robin, and each CTA's two
 // epilogue groups take alternate tiles.
 int tile_tree_levels(long long units, long long ctas) {
   const long long per_cta = (units + ctas - 1) / ctas;
@@ -443,31 +443,15 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
     if (!map_2d(&mx, p.bs_x, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
     if (p.add_src && !map_2d(&md, p.add_src, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
   }
-  // Clusters of two CTAs over M-tile pairs share each B tile (multicast), which
-  // halves the B operand's L2 -> SM traffic, the bound of most conv passes.
-  const int pair_cl = (BN >= 128 && p.m_tiles % 2 == 0) ? gemm_pair_clusters(BN) : 0;
-  if (pair_cl > 0) {
-    const long long pair_units = units / 2;
-    int ncl = (int)std::min<long long>(pair_units, std::min(pair_cl, sms / 2));
-    if (p.st_mean) {  // as below, per pair: two slots per cluster
-      ncl = std::min(ncl, kBnStatSlots / 2 * p.n_tiles);
-      ncl -= ncl % p.n_tiles;
-    }
-    if (ncl > 0) {
-      if (p.bs_x && (p.bs_levels = tile_tree_levels(pair_units, ncl)) >= kMaxTileTreeLevels)
-        return PF16_ERR_UNSUPPORTED;
-      return launch_gemm(BN, a, b, c, p, 2 * ncl, st, true, &mx, &md) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
-    }
-  }
   int grid = (int)std::min<long long>(units, sms);
   if (p.st_mean) {
     // fused statistics: every CTA keeps one n-tile (grid a multiple of n_tiles), at most
-    // kBnStatSlots / 4 CTAs per n-tile
+    // kBnStatSlots CTAs (one statistics slot each) per n-tile
     grid = std::min(grid, kBnStatSlots * p.n_tiles);
     grid -= grid % p.n_tiles;
     if (p.bs_x && (p.bs_levels = tile_tree_levels(units, grid)) >= kMaxTileTreeLevels) return PF16_ERR_UNSUPPORTED;
   }
-  return launch_gemm(BN, a, b, c, p, grid, st, false, &mx, &md) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+  return launch_gemm(BN, a, b, c, p, grid, st, &mx, &md) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
 // Point the GEMM's fused statistics at the BatchNorm backward sources.

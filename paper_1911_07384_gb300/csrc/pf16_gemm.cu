@@ -3,7 +3,7 @@
 // FP16 accumulation in tensor memory, FP16 results -- no FP32 anywhere
 // (paper Sec. 5.2: all arithmetic and storage in FP16).
 //
-// One persistent CTA per SM, 6 warps:
+// One persistent CTA per SM, 10 warps:
 //   warp 0    TMA producer: one elected lane streams 64-wide K-blocks of A
 //             and B into a ring of shared-memory stages (mbarrier full/empty).
 //   warp 1    allocates tensor memory; one lane issues tcgen05.mma
@@ -11,8 +11,11 @@
 //             stage back to the producer and each finished tile to the
 //             epilogue.  Two TMEM accumulators alternate so the epilogue of
 //             tile i overlaps the MMAs of tile i + 1.
-//   warps 2-5 epilogue: tcgen05.ld of one accumulator row per thread, pack to
-//             FP16, store (or FP16-accumulate, or write a split-K partial).
+//   warps 2-9 epilogue, two groups of four: group g drains accumulator g (the
+//             CTA's even or odd tiles), warp w its TMEM sub-partition w % 4;
+//             tcgen05.ld of one accumulator row per thread, pack to FP16,
+//             stage in shared memory and store by TMA (or FP16-accumulate, or
+//             write a split-K partial), with the fused BatchNorm statistics.
 // Every mbarrier wait is bounded; on expiry the CTA records PF16_ERR_TIMEOUT
 // and all roles leave their loops, so the kernel always terminates.
 #include <cstdio>
@@ -136,11 +139,9 @@ struct Cursor {
     }
   }
 
-  // A, and B unless !load_b; MC: B goes to both CTAs of the cluster pair
-  template <bool MC>
+  // the K-block's A and B boxes into stage (sa, sb), completing on bar
   __device__ __forceinline__ void load(const GemmParams& p, const CUtensorMap* ma, const CUtensorMap* mb,
-                                       uint32_t sa, uint32_t sb, uint32_t bar, int m0, int n0,
-                                       bool load_b) const {
+                                       uint32_t sa, uint32_t sb, uint32_t bar, int m0, int n0) const {
     switch (p.a_mode) {
       case LD_TILED_K:
         tma_load_2d(sa, ma, bar, kb * kBK, m0);
@@ -156,43 +157,28 @@ struct Cursor {
       default:
         break;
     }
-    if (!load_b) return;
-    constexpr uint16_t kPair = 0x3;
     switch (p.b_mode) {
       case LD_TILED_K:
-        if (MC)
-          tma_load_2d_mc(sb, mb, bar, kb * kBK, n0, kPair);
-        else
-          tma_load_2d(sb, mb, bar, kb * kBK, n0);
+        tma_load_2d(sb, mb, bar, kb * kBK, n0);
         break;
       case LD_TILED_MN:
 #pragma unroll
         for (int j = 0; j < BN / 64; ++j) {
-          if (MC)
-            tma_load_2d_mc(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK, kPair);
-          else
-            tma_load_2d(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK);
+          tma_load_2d(sb + j * 8192, mb, bar, n0 + 64 * j, kb * kBK);
         }
         break;
       case LD_IM2COL_MN: {
         const int bw = b_j * p.gb.step + p.gb.base_w, bh = b_i * p.gb.step + p.gb.base_h;
 #pragma unroll
         for (int j = 0; j < BN / 64; ++j) {
-          if (MC)
-            tma_load_im2col_4d_mc(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
-                                  (uint16_t)p.tap_dr[b_tap[j]], kPair);
-          else
-            tma_load_im2col_4d(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
-                               (uint16_t)p.tap_dr[b_tap[j]]);
+          tma_load_im2col_4d(sb + j * 8192, mb, bar, b_c[j], bw, bh, b_n, (uint16_t)p.tap_ds[b_tap[j]],
+                             (uint16_t)p.tap_dr[b_tap[j]]);
         }
       } break;
       case LD_TAP3D_MN:
 #pragma unroll
         for (int j = 0; j < BN / 64; ++j) {
-          if (MC)
-            tma_load_3d_mc(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k, kPair);
-          else
-            tma_load_3d(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k);
+          tma_load_3d(sb + j * 8192, mb, bar, n0 + 64 * j, p.tap_w[b_t], b_k);
         }
         break;
       default:
@@ -201,18 +187,15 @@ struct Cursor {
   }
 };
 
-// Work unit u -> tile origin (m0, n0), split and K-block range.  mt_count M
-// tiles are enumerated; M tile mt is row tile mt * mscale + moff (a cluster
-// pair enumerates tile pairs, mscale = 2, moff = its rank).
+// Work unit u -> tile origin (m0, n0), split and K-block range (n tiles
+// fastest, then M tiles, then splits).
 __device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0, int& n0, int& split,
-                                            int& kb0, int& kb1, int BN, int mt_count = -1, int mscale = 1,
-                                            int moff = 0) {
-  if (mt_count < 0) mt_count = p.m_tiles;
-  const int per = mt_count * p.n_tiles;
+                                            int& kb0, int& kb1, int BN) {
+  const int per = p.m_tiles * p.n_tiles;
   split = u / per;
   const int rem = u - split * per;
   const int mt = rem / p.n_tiles;
-  m0 = (mt * mscale + moff) * kBM;
+  m0 = mt * kBM;
   n0 = (rem - mt * p.n_tiles) * BN;
   kb0 = split * p.kb_per_split;
   kb1 = min(p.num_kb, kb0 + p.kb_per_split);
@@ -607,8 +590,8 @@ template <int BN, bool ADD>
 __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorMap* mapC, const CUtensorMap* mapX,
                                             const CUtensorMap* mapD, uint8_t* wbuf, uint64_t* wbar,
                                             uint64_t* tfull, uint64_t* tempty, uint32_t tmem_base, int acc, int sub,
-                                            int lane, int u0, int ustep, int total, int mt_count, int mscale,
-                                            int rank, uint64_t lim, volatile int* abort_flag, EpiStats& stats) {
+                                            int lane, int u0, int ustep, int total, uint64_t lim,
+                                            volatile int* abort_flag, EpiStats& stats) {
   if (u0 >= total) return;
   const uint32_t S0 = smem_u32(wbuf), X0 = S0 + 2 * 4096;
   const uint32_t B0 = smem_u32(wbar);
@@ -622,7 +605,7 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
     pend[b] = q;
   };
   int u = u0, m0, n0, split, kb0, kb1;
-  unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+  unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
   int c = 0;
   if (lane == 0) issue(0, m0 + sub * 32, n0, 0);
   ChunkIn cur, nxt;
@@ -648,7 +631,7 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
     if (last) {
       u2 = u + ustep;
       c2 = 0;
-      if (u2 < total) unit_decode(p, u2, m2, n2, split, kb0, kb1, BN, mt_count, mscale, rank);
+      if (u2 < total) unit_decode(p, u2, m2, n2, split, kb0, kb1, BN);
     }
     const bool more = u2 < total;
     if (more) {
@@ -726,14 +709,6 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
       if (pend[b] >= 0) mbar_wait(B0 + 8 * b, (uint32_t)(pend[b] >> 1) & 1u, 1000000000ull);
 }
 
-// PAIR: launched in clusters of two CTAs that take the same (n tile, split)
-// units over M tiles 2t and 2t + 1, so they need the same B tiles: the CTA of
-// rank kb mod 2 loads K-block kb's B tile once and multicasts it into both
-// CTAs' stage, halving the B operand's L2 -> SM traffic.  A stage is refilled
-// only after both CTAs' MMAs have read it (each MMA commit arrives on the
-// stage's empty barrier in both CTAs, count 2).  The two CTAs meet at a
-// cluster barrier after set-up and before exit, so neither's shared memory
-// or barriers are written after it has left.
 // EPI: the epilogue's kind, each a separate instantiation so that the others
 // do not carry its registers or give up its pipeline stages --
 //   EPI_PLAIN: stores (forward statistics optional);
@@ -742,7 +717,7 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
 //   EPI_BS_TMA: the same statistics from TMA-fed tiles (epilogue_bs; for short
 //     reductions, whose epilogue is the bound);
 //   EPI_BS_ADD: EPI_BS_TMA plus the addend (GemmParams::add_src).
-template <int BN, bool PAIR, int EPI>
+template <int BN, int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapX,
@@ -766,7 +741,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < Cfg::STAGES; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), PAIR ? 2 : 1);
+      mbar_init(smem_u32(&empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
@@ -788,17 +763,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (PAIR) cluster_sync();  // the partner's barriers are initialised
   // set-up done: wait for the kernel this one depends on
   pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
-  // work enumeration: a pair walks M-tile pairs, each CTA takes its own tile of the pair
-  const int rank = PAIR ? (int)cluster_ctarank() : 0;
-  const int cid = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
-  const int ncl = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
-  const int mt_count = PAIR ? p.m_tiles / 2 : p.m_tiles;
-  const int mscale = PAIR ? 2 : 1;
-  const int total = mt_count * p.n_tiles * p.splits;
+  // work enumeration: CTA cid takes units cid, cid + ncl, ...
+  const int cid = (int)blockIdx.x;
+  const int ncl = (int)gridDim.x;
+  const int total = p.m_tiles * p.n_tiles * p.splits;
   const uint64_t lim = p.wait_limit_ns;
 
   if (warp == 0) {
@@ -808,7 +779,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       uint32_t issued = 0;  // stages loaded so far (for the drain below)
       for (int u = cid; u < total && !*abort_flag; u += ncl) {
         int m0, n0, split, kb0, kb1;
-        unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
         Cursor<BN> cur;
         cur.init(p, m0, n0, kb0);
         for (int kb = kb0; kb < kb1; ++kb, cur.advance(p)) {
@@ -819,8 +790,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
-          cur.template load<PAIR>(p, &mapA, &mapB, sa, sa + Cfg::A_BYTES, fb, m0, n0,
-                                  !PAIR || (kb & 1) == rank);
+          cur.load(p, &mapA, &mapB, sa, sa + Cfg::A_BYTES, fb, m0, n0);
           ++issued;
           if (++stage == Cfg::STAGES) {
             stage = 0;
@@ -856,7 +826,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const uint32_t ak16 = (uint32_t)p.a_kstep >> 4, bk16 = (uint32_t)p.b_kstep >> 4;
       for (int u = cid; u < total && !*abort_flag; u += ncl) {
         int m0, n0, split, kb0, kb1;
-        unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+        unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
         if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1, lim)) {
           record_timeout(p, abort_flag);
           break;
@@ -876,10 +846,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
             tc_mma_f16(d_tmem, ab + kk * ak16, bb + kk * bk16, p.idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
-          if (PAIR)
-            tc_commit_mc(smem_u32(&empty[stage]), 0x3);  // the stage is free once both CTAs read it
-          else
-            tc_commit(smem_u32(&empty[stage]));
+          tc_commit(smem_u32(&empty[stage]));
           if (++stage == Cfg::STAGES) {
             stage = 0;
             phase ^= 1;
@@ -903,14 +870,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
     if constexpr (TMAE)  // (the host launches these only with TMA stores of rows in pixel order)
       epilogue_bs<BN, ADD>(p, &mapC, &mapX, &mapD, staging + e * Cfg::WARP_BUF, ebar + 2 * e, tfull, tempty,
-                           tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, mt_count, mscale, rank, lim,
-                           abort_flag, stats);
+                           tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, lim, abort_flag, stats);
     const bool bstats = BS && p.st_mean && p.bs_x && p.tma_store;
     BwdIn bin;
     for (int u = cid + grp * ncl; u < total && !TMAE; u += 2 * ncl) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
-      unit_decode(p, u, m0, n0, split, kb0, kb1, BN, mt_count, mscale, rank);
+      unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
       if (bstats) {  // the first chunk's inputs, loaded while the accumulator is computed
         const int nv0 = min(32, max(0, p.M - (m0 + sub * 32)));
         if (nv0 > 0) bin.load(p, (long long)(m0 + sub * 32), n0, nv0, lane);
@@ -1015,24 +981,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     if (p.tma_store && lane == 0) bulk_wait0();
     if (p.st_mean) {
-      // this CTA's tiles all have n-tile cid % n_tiles (the pair count is a multiple of n_tiles);
-      // slot (cid / n_tiles) * mscale + rank
+      // this CTA's tiles all have n-tile cid % n_tiles (the grid is a multiple of n_tiles);
+      // slot cid / n_tiles
       const int n0 = (cid % p.n_tiles) * BN;
       const int nch = min(BN, p.N - n0) / 64;
-      const int slot = (cid / p.n_tiles) * mscale + rank;
+      const int slot = cid / p.n_tiles;
       if (BS)
         stats.write_cta_bwd(p, staging, e, slot, n0, nch, lane, p.bs_levels);
       else
         stats.write_cta(p, staging, e, slot, n0, nch, lane, cid % p.n_tiles == 0);
       if (blockIdx.x == 0 && e == 0 && lane == 0) {
-        p.st_hdr[0] = ncl / p.n_tiles * mscale;
+        p.st_hdr[0] = ncl / p.n_tiles;
         p.st_hdr[1] = 5 + p.bs_levels + 3;
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (PAIR) cluster_sync();  // the partner no longer writes this CTA's stages or barriers
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
@@ -1049,13 +1014,13 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN, bool PAIR, int EPI = EPI_PLAIN>
+template <int BN, int EPI = EPI_PLAIN>
 static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, PAIR, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
@@ -1063,96 +1028,45 @@ static cudaError_t set_smem_attr() {
   return cudaSuccess;
 }
 
-template <int BN, bool PAIR, int EPI>
+template <int BN, int EPI>
 static cudaError_t launch_variant(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                                   const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
                                   cudaStream_t s) {
-  cudaError_t e = set_smem_attr<BN, PAIR, EPI>();
+  cudaError_t e = set_smem_attr<BN, EPI>();
   if (e != cudaSuccess) return e;
   constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM;
-  if (PAIR)
-    launch_pdl_cluster2(k_gemm<BN, PAIR, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
-  else
-    launch_pdl(k_gemm<BN, PAIR, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
+  launch_pdl(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
   return counted_launches(1);
-}
-
-template <int BN, bool PAIR>
-static cudaError_t launch_epi(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                              const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
-                              int epi, cudaStream_t s) {
-  switch (epi) {
-    case EPI_PLAIN: return launch_variant<BN, PAIR, EPI_PLAIN>(mA, mB, mC, mX, mD, p, grid, s);
-    case EPI_BS: return launch_variant<BN, PAIR, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);
-    case EPI_BS_TMA: return launch_variant<BN, PAIR, EPI_BS_TMA>(mA, mB, mC, mX, mD, p, grid, s);
-    case EPI_BS_ADD: return launch_variant<BN, PAIR, EPI_BS_ADD>(mA, mB, mC, mX, mD, p, grid, s);
-    default: return cudaErrorInvalidValue;
-  }
 }
 
 template <int BN>
 static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                                const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
-                               bool pair, cudaStream_t s) {
+                               cudaStream_t s) {
   const int epi = gemm_epilogue(p);
   if (epi != EPI_PLAIN && (!p.tma_store || p.out_mode != OUT_STORE)) return cudaErrorInvalidValue;
-  if (!pair) return launch_epi<BN, false>(mA, mB, mC, mX, mD, p, grid, epi, s);
-  if constexpr (BN >= 128) {
-    if (grid % 2 != 0 || p.m_tiles % 2 != 0) return cudaErrorInvalidValue;
-    return launch_epi<BN, true>(mA, mB, mC, mX, mD, p, grid, epi, s);
+  switch (epi) {
+    case EPI_PLAIN: return launch_variant<BN, EPI_PLAIN>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS: return launch_variant<BN, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS_TMA: return launch_variant<BN, EPI_BS_TMA>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS_ADD: return launch_variant<BN, EPI_BS_ADD>(mA, mB, mC, mX, mD, p, grid, s);
+    default: return cudaErrorInvalidValue;
   }
-  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
-                        const GemmParams& p, int grid, cudaStream_t s, bool pair, const CUtensorMap* mX,
+                        const GemmParams& p, int grid, cudaStream_t s, const CUtensorMap* mX,
                         const CUtensorMap* mD) {
   // the BatchNorm-input and addend maps (unused without backward statistics)
   const CUtensorMap& x = mX ? *mX : mC;
   const CUtensorMap& d = mD ? *mD : x;
   switch (BN) {
-    case 64: return launch_bn_t<64>(mA, mB, mC, x, d, p, grid, pair, s);
-    case 128: return launch_bn_t<128>(mA, mB, mC, x, d, p, grid, pair, s);
-    case 192: return launch_bn_t<192>(mA, mB, mC, x, d, p, grid, pair, s);
-    case 256: return launch_bn_t<256>(mA, mB, mC, x, d, p, grid, pair, s);
+    case 64: return launch_bn_t<64>(mA, mB, mC, x, d, p, grid, s);
+    case 128: return launch_bn_t<128>(mA, mB, mC, x, d, p, grid, s);
+    case 192: return launch_bn_t<192>(mA, mB, mC, x, d, p, grid, s);
+    case 256: return launch_bn_t<256>(mA, mB, mC, x, d, p, grid, s);
     default: return cudaErrorInvalidValue;
   }
-}
-
-template <int BN>
-static int pair_clusters_t() {
-  if (set_smem_attr<BN, true>() != cudaSuccess) return 0;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2 * 152);
-  cfg.blockDim = dim3(kGemmThreads);
-  cfg.dynamicSmemBytes = GemmCfg<BN>::SMEM;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k_gemm<BN, true, EPI_PLAIN>, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  return n;
-}
-
-int gemm_pair_clusters(int BN) {
-  static int cache[64][4];
-  static bool done[64][4] = {};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  const int i = BN == 128 ? 0 : (BN == 192 ? 1 : (BN == 256 ? 2 : -1));
-  if (i < 0 || dev >= 64) return 0;
-  if (!done[dev][i]) {
-    cache[dev][i] = BN == 128 ? pair_clusters_t<128>() : (BN == 192 ? pair_clusters_t<192>() : pair_clusters_t<256>());
-    done[dev][i] = true;
-  }
-  return cache[dev][i];
 }
 
 

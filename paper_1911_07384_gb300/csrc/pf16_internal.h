@@ -31,27 +31,6 @@ inline cudaError_t launch_pdl(void (*kernel)(K...), dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
 }
 
-// The same with a cluster of two CTAs along x (gridDim.x even).
-template <typename... K, typename... A>
-inline cudaError_t launch_pdl_cluster2(void (*kernel)(K...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
-                                       A&&... args) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = 2;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
-}
-
 // Status of the n launches just made; they are counted when they succeeded.
 inline cudaError_t counted_launches(int n) {
   const cudaError_t e = cudaGetLastError();
@@ -177,9 +156,6 @@ __host__ __device__ inline size_t bnstat_bytes(long long C) {
   return bnstat_off_cnt(C) + (size_t)kBnStatSlots * 4;
 }
 
-// Launch the engine (BN in {64, 128, 192, 256}).  pair: clusters of two CTAs
-// sharing each B tile by multicast (BN >= 128, p.m_tiles and grid even; the
-// grid then counts CTAs, two per tile pair).  Returns a cudaError_t.
 // Epilogue kinds of the conv GEMM (k_gemm's EPI).  The backward statistics
 // take the TMA-fed epilogue for short reductions (at most kTmaEpiMaxKb
 // K-blocks per tile: there the epilogue's traffic is the bound) and always
@@ -200,13 +176,13 @@ cudaError_t launch_tc_rate(uint32_t idesc, int n, int chains, int reps, int grid
 
 // mapX / mapD: 128B-swizzled 32 x 64 boxes over bs_x and add_src ([M][N],
 // pitch ldo), needed with the backward statistics (and the addend).
+// Launch the engine (BN in {64, 128, 192, 256}) on `grid` persistent CTAs.
+// Returns a cudaError_t.
 cudaError_t launch_gemm(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const CUtensorMap& mapC, const GemmParams& p, int grid,
-                        cudaStream_t stream, bool pair = false, const CUtensorMap* mapX = nullptr,
+                        cudaStream_t stream, const CUtensorMap* mapX = nullptr,
                         const CUtensorMap* mapD = nullptr);
 int gemm_smem_bytes(int BN);
-// Clusters of two GEMM CTAs (tile width BN) that can be resident at once (0: none).
-int gemm_pair_clusters(int BN);
 
 // Halo engine for stride-1 convolutions with 64 outputs whose input pixel is
 // 128 bytes (64 channels, 3x3 taps) or 32 bytes (16 channels, the stem after

@@ -116,47 +116,6 @@ __device__ __forceinline__ void tma_load_im2col_4d(uint32_t dst, const CUtensorM
       : "memory");
 }
 
-// Multicast forms: the box lands at the same shared-memory offset in every CTA
-// of the cluster named in ctamask, each signalling its own mbarrier at `bar`'s
-// offset.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* m, uint32_t bar, int x, int y,
-                                               uint16_t ctamask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(x), "r"(y), "h"(ctamask)
-      : "memory");
-}
-__device__ __forceinline__ void tma_load_3d_mc(uint32_t dst, const CUtensorMap* m, uint32_t bar, int x, int y,
-                                               int z, uint16_t ctamask) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(x), "r"(y), "r"(z), "h"(ctamask)
-      : "memory");
-}
-__device__ __forceinline__ void tma_load_im2col_4d_mc(uint32_t dst, const CUtensorMap* m, uint32_t bar, int c,
-                                                      int w, int h, int n, uint16_t ow, uint16_t oh,
-                                                      uint16_t ctamask) {
-  asm volatile(
-      "cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4, %5, %6}], [%2], {%7, %8}, %9;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c), "r"(w), "r"(h), "r"(n), "h"(ow), "h"(oh),
-      "h"(ctamask)
-      : "memory");
-}
-
-// Cluster: this CTA's rank, and a full barrier of all threads of all its CTAs
-// (release / acquire: shared-memory writes before it are visible after it).
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
 // TMA stores from shared memory (bulk async-group completion).
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, uint32_t src, int x, int y) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
@@ -247,14 +206,6 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
                    bar)
                : "memory");
 }
-// The same arrival on the mbarrier at `bar`'s offset in every CTA of ctamask.
-__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t ctamask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-          bar),
-      "h"(ctamask)
-      : "memory");
-}
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -272,10 +223,8 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* r) {
 // Shared-memory matrix descriptor for tcgen05.mma (sm_100 family, version 1).
 // swz: 0 = no swizzle, 2 = 128-byte swizzle.
 // The start-address field of a descriptor (bits 0-13, 16-byte units) for a
-// shared address.  In a cluster launch a CTA's shared addresses carry its
-// cluster rank above bit 23 (rank 1's window starts at 16 MB), so the address
-// must be masked before it is added to a base descriptor: unmasked, the rank
-// bit lands in the leading-byte-offset field.
+// shared address, masked to its 14 bits so that it can be added to a base
+// descriptor without touching the leading-byte-offset field.
 __device__ __forceinline__ uint32_t desc_addr16(uint32_t saddr) { return (saddr >> 4) & 0x3FFFu; }
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo,
                                               uint32_t swz) {

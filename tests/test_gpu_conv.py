@@ -207,7 +207,7 @@ def test_full_size_sampled(orc, shape):
 
 
 F32_SHAPES = [
-    (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col, reduction 2,304, paired CTAs
+    (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col, reduction 2,304, 256-wide N tiles
     (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine
     (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem: space-to-depth halo forward, stem weight gradient
     (2, 14, 14, 64, 256, 1, 1, 1, 0),    # dense 1x1

@@ -85,12 +85,12 @@ def test_conv_fwd_bnstats_then_bn(orc, shape):
 
 BWD_SHAPES = [
     # conv (N, H, W, C, K, R, S, stride, pad) whose data gradient is the BatchNorm's dy; relu
-    ((2, 14, 14, 256, 64, 1, 1, 1, 0), True),    # dense 1x1, 256 channels: paired CTAs, one n-tile
+    ((2, 14, 14, 256, 64, 1, 1, 1, 0), True),    # dense 1x1, 256 channels: one 256-wide n-tile
     ((2, 14, 14, 64, 256, 1, 1, 1, 0), True),    # dense 1x1, 64 channels
     ((3, 7, 7, 512, 256, 1, 1, 1, 0), False),    # two n-tiles, no ReLU (no mask)
     ((2, 28, 28, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 32
     ((2, 56, 56, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 64 (columns 56..63 dropped)
-    ((2, 14, 14, 128, 128, 3, 3, 1, 1), True),   # stride-1 im2col data gradient, paired CTAs
+    ((2, 14, 14, 128, 128, 3, 3, 1, 1), True),   # stride-1 im2col data gradient, 128-wide n-tile
     ((1, 7, 7, 64, 64, 3, 3, 1, 1), True),       # one partial tile (49 rows)
     ((2, 7, 7, 256, 1024, 1, 1, 1, 0), True),    # long reduction (16 K-blocks): register-fed epilogue
     ((4, 14, 14, 256, 128, 1, 1, 1, 0), True),   # short reduction, many tiles per CTA: TMA-fed epilogue
@@ -176,7 +176,7 @@ def test_conv_dgrad_bnstats_rejects_strided():
 
 ADD_SHAPES = [
     # 1x1 stride-1 data gradients whose dx also takes a masked addend
-    (2, 14, 14, 256, 64, 1, 1, 1, 0),    # paired CTAs, one n-tile of 256
+    (2, 14, 14, 256, 64, 1, 1, 1, 0),    # one n-tile of 256
     (3, 7, 7, 512, 128, 1, 1, 1, 0),     # two n-tiles, 147 rows (a partial M tile)
     (1, 7, 7, 64, 64, 1, 1, 1, 0),       # 64-wide tile, one partial M tile
 ]

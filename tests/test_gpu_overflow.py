@@ -13,7 +13,7 @@ from gpu_util import dev, empty16, f64, host, workspace
 pytestmark = pytest.mark.gpu
 
 SHAPES = [(1, 8, 8, 64, 64, 3, 3, 1, 1),     # halo engine
-          (1, 8, 8, 128, 128, 3, 3, 1, 1),   # im2col GEMM, paired CTAs
+          (1, 8, 8, 128, 128, 3, 3, 1, 1),   # im2col GEMM, 128-wide N tile
           (2, 7, 7, 256, 64, 1, 1, 1, 0)]    # dense 1x1
 
 BIG = np.float16(64.0).view(np.uint16)      # products 4096; >= 64 terms per output here
