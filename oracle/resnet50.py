@@ -100,7 +100,11 @@ class OracleResNet50:
         return f64_to_f16(dx.ravel()), f64_to_f16(dg), f64_to_f16(db), f64_to_f16(dres.ravel())
 
     # ------------------------------------------------------------------ step
-    def step(self, images, labels):
+    def forward(self, images, labels):
+        """Forward pass and loss.  Returns (loss, cache); cache holds every
+        layer's binary16 output (per block: x, a1, b1, a2, b2, a3, ap, bp, y),
+        the stem's (a0, b0, p0), the pooled features f, the logits and the
+        loss gradients (dlogits and dbias, binary64 before storage)."""
         N = self.N
         act = {}
         a0 = self._cf("stem", images)
@@ -120,18 +124,29 @@ class OracleResNet50:
             else:
                 ap, bp = None, x
             y = self._bf(nm + "n3", a3, residual=bp)
-            act[nm] = (x, a1, b1, a2, b2, a3, ap, y)
+            act[nm] = (x, a1, b1, a2, b2, a3, ap, bp, y)
             h = y
         f = f64_to_f16(avgpool_fwd(h, N, self.hl * self.hl, self.cl))
         logits = self._cf("fc", f)
         loss, dl, db = softmax_xent(logits, self.bias, labels, N, self.classes)
-        dl, gbias = f64_to_f16(dl), f64_to_f16(db)
-        grads = {}
-        grads["fc"], df = self._cb("fc", f, dl)
+        cache = dict(images=images, a0=a0, b0=b0, p0=p0, act=act, f=f, logits=logits, dlogits=dl, dbias=db)
+        return loss, cache
+
+    def backward(self, cache):
+        """Backward pass through the cached forward.  Returns (grads, bgrads,
+        gbias): binary16 gradients of every conv / FC weight (by conv name),
+        of every BatchNorm gamma and beta (by BN name + "g" / "b") and of the FC
+        bias.  Also records in the cache each block's output gradient
+        (cache["dy"][name]) and the max-pool output's (cache["dp0"])."""
+        N, act = self.N, cache["act"]
+        dl, gbias = f64_to_f16(cache["dlogits"]), f64_to_f16(cache["dbias"])
+        grads, bgrads = {}, {}
+        grads["fc"], df = self._cb("fc", cache["f"], dl)
         dy = f64_to_f16(avgpool_bwd(df, N, self.hl * self.hl, self.cl))
-        bgrads = {}
+        cache["dy"] = dys = {}  # each block's output gradient, as the block received it
         for nm, hh, h2, cin, width, proj in reversed(self.blocks):
-            x, a1, b1, a2, b2, a3, ap, y = act[nm]
+            x, a1, b1, a2, b2, a3, ap, bp, y = act[nm]
+            dys[nm] = dy
             da3, bgrads[nm + "n3g"], bgrads[nm + "n3b"], dres = self._bb(nm + "n3", a3, y, dy)
             grads[nm + "c3"], db2 = self._cb(nm + "c3", b2, da3)
             da2, bgrads[nm + "n2g"], bgrads[nm + "n2b"], _ = self._bb(nm + "n2", a2, b2, db2)
@@ -144,9 +159,16 @@ class OracleResNet50:
                 dy = f64_to_f16(f16_to_f64(dx1) + f16_to_f64(dxp))
             else:
                 dy = f64_to_f16(f16_to_f64(dx1) + f16_to_f64(dres))
+        cache["dp0"] = dy  # the gradient with respect to the max-pool output
+        b0 = cache["b0"]
         db0 = f64_to_f16(maxpool_bwd(b0, dy, N, self.h0, self.h0, 64)[0])
-        da0, bgrads["bn0g"], bgrads["bn0b"], _ = self._bb("bn0", a0, b0, db0)
-        grads["stem"], _ = self._cb("stem", images, da0, need_dx=False)
+        da0, bgrads["bn0g"], bgrads["bn0b"], _ = self._bb("bn0", cache["a0"], b0, db0)
+        grads["stem"], _ = self._cb("stem", cache["images"], da0, need_dx=False)
+        return grads, bgrads, gbias
+
+    def update(self, grads, bgrads, gbias):
+        """The pure-FP16 SGD step on every parameter: weight decay on conv / FC
+        weights and the FC bias, none on BatchNorm parameters (Sec. 5.1)."""
         for name, g in grads.items():
             c = self.convs[name]
             c[1], c[2] = sgd_update(c[1], c[2], g, LR, MOMENTUM, WD)
@@ -154,4 +176,16 @@ class OracleResNet50:
         for name, st in self.bns.items():
             st[1], st[3] = sgd_update(st[1], st[3], bgrads[name + "g"], LR, MOMENTUM, 0)
             st[2], st[4] = sgd_update(st[2], st[4], bgrads[name + "b"], LR, MOMENTUM, 0)
+
+    def step(self, images, labels):
+        """One training step (forward, backward, update); returns the loss."""
+        loss, cache = self.forward(images, labels)
+        self.update(*self.backward(cache))
         return loss
+
+    def param_counts(self):
+        """(decayed, not decayed) parameter counts: conv / FC weights and the FC
+        bias; BatchNorm gamma and beta."""
+        wd = sum(c[1].size for c in self.convs.values()) + self.bias.size
+        nowd = sum(2 * st[0] for st in self.bns.values())
+        return wd, nowd
