@@ -121,7 +121,7 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
  * dx as pf16_conv_dgrad with flags 0; in addition each epilogue warp of the
  * GEMM reduces, per channel, dy' = dx where the ReLU passed and dy' * xhat,
  * xhat = rn(rn(x - mean) * invstd), over the 32 rows of each tile it stores:
- * FP16 halving trees, zero leaves for rows past the tensor, pushed into the
+ * FP16 pairwise sums, zero leaves for rows past the tensor, pushed into the
  * warp's tree of tiles, which is padded with zero leaves to a power of two.
  * The CTAs' nodes go to `stats` (stats_bytes >= pf16_conv_dgrad_bnstats_size(d),
  * 16-byte aligned, caller-owned, no initial contents needed);
@@ -204,17 +204,46 @@ int pf16_conv_wgrad_noalloc(const pf16_conv_desc* d, const uint16_t* x, const ui
 int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
                     uint16_t momentum, uint16_t wd, uint32_t flags, void* stream);
 
+/* ------------------------------------------------- data-parallel exchange
+ * The combining step of the fixed-order FP16 gradient all-reduce of
+ * data-parallel training (Sec. 5.1: ResNet-50 on 8 to 128 GPUs, each with
+ * its own batch and its own BatchNorm statistics, their gradients averaged
+ * before every SGD step; Sec. 5.2: that average is taken in FP16 too).
+ * `planes` holds `world` gradient planes of n binary16 values, plane r at
+ * planes + r * plane_stride (elements) -- the same slice of every rank's
+ * gradient, in rank order.  Per element i:
+ *   out[i] = rn(T(i) * scale),  T(i) = the perfect pairwise tree over the
+ *   leaves planes[0][i], ..., planes[world-1][i], padded with +0 leaves to
+ *   the next power of two, each node rn(left + right)
+ * with scale normally rn(1/world) (binary16 bits; the multiply is skipped
+ * when scale is 0x3C00 = 1).  The sum comes before the scaling so that small
+ * gradients keep their low bits (a scale of 1/128 first would push them 7
+ * binades toward underflow); it overflows only where the sum of the world's
+ * gradients exceeds 65,504.  The order depends only on world and i, so every
+ * rank that combines the same planes gets the same bits, whatever the
+ * launch configuration.
+ * n and plane_stride are multiples of 8, plane_stride >= n, 1 <= world <=
+ * 1024; out may be planes itself (plane 0 is overwritten only after every
+ * plane of an element was read) and must not overlap the other planes.
+ * n == 0 launches nothing.  Errors: PF16_ERR_NULL, PF16_ERR_ALIGN (16-byte
+ * alignment), PF16_ERR_SHAPE. */
+int pf16_allreduce_combine(const uint16_t* planes, int32_t world, size_t n, size_t plane_stride,
+                           uint16_t scale, uint16_t* out, void* stream);
+
 /* ------------------------------------------------------------- BatchNorm
  * BatchNorm with batch statistics over the n*h*w rows of each of c channels
  * (Eq. 1, Eq. 2), each output then multiplied by post_scale (0x3400 = 0.25
  * inside residual blocks, 0x3C00 = 1 for the stem, Sec. 4.2), optionally
  * plus a residual tensor and followed by ReLU (flags).  All arithmetic FP16,
- * and no partial result can overflow unless the data do: the forward mean
- * and biased variance are balanced pairwise trees of (mean, mean squared
- * deviation) nodes merged by the parallel-variance rule with exact counts
- * (equal counts: mean node rn(a/2 + rn(b/2)), one fused multiply-add); the
- * backward means of dy' and dy'*xhat are "halving" trees of the same node
- * over zero-padded power-of-two leaves, scaled once by the padding ratio.
+ * and no forward partial result can overflow unless the data do: the
+ * forward mean and biased variance are balanced pairwise trees of (mean, mean
+ * squared deviation) nodes merged by the parallel-variance rule with exact
+ * counts (equal counts: mean node rn(a/2 + rn(b/2)), one fused multiply-add).
+ * The backward sums of dy' and dy'*xhat are pairwise trees of rn(a + b) over
+ * zero-padded power-of-two leaves -- gradients are small, and a halving node
+ * would drop the low bits of subnormal partial means -- giving dbeta =
+ * rn(s * sum dy') and dgamma = rn(s * sum dy'*xhat), and the means
+ * rn(rn(sum * rn(2^L/R)) * 2^-L), L = ceil(log2 R).
  * The tree shapes depend only on n*h*w and c.
  *   phase 0 (forward, training):  reads x, gamma, beta[, residual];
  *       writes y, mean, invstd (per channel, saved for the backward).

@@ -49,13 +49,15 @@ __host__ __device__ __forceinline__ int ceil_log2(long long v) {
   return l;
 }
 
-// x * 2^e for e >= 0 by exact power-of-two steps (each exact unless it overflows)
-__device__ __forceinline__ uint4 ldexp4(uint4 v, int e) {
+// x * 2^-e for e >= 0 by power-of-two steps: exact while the result is
+// normal; a subnormal result is rounded (at most twice, once per step below
+// 2^-14)
+__device__ __forceinline__ uint4 ldexp_down4(uint4 v, int e) {
   while (e > 14) {
-    v = mul4(v, dup2(0x7400));  // 2^14
+    v = mul4(v, dup2(0x0400));  // 2^-14
     e -= 14;
   }
-  const uint16_t pe = (uint16_t)((e + 15) << 10);  // 2^e, 0 <= e <= 14
+  const uint16_t pe = (uint16_t)((15 - e) << 10);  // 2^-e, 0 <= e <= 14
   return mul4(v, dup2(pe));
 }
 
@@ -488,14 +490,16 @@ cudaError_t launch_fill_zero(uint16_t* p, size_t n, cudaStream_t s) {
 //             read once), merged over the thread's chunks and then over the
 //             CTA's row groups by the count-aware pairwise parallel-variance
 //             rule;
-//   backward: the padded halving-tree means of dy' and dy' * xhat over the 8
-//             rows, a halving tree over the thread's chunks, then over the
-//             CTA's row groups (zero padded to powers of two throughout).
+//   backward: the pairwise sums of dy' and dy' * xhat over the 8 rows, a
+//             pairwise tree over the thread's chunks, then over the CTA's row
+//             groups (zero padded to powers of two throughout).
 // A second small kernel (one CTA per channel group) combines the per-CTA
 // results over a balanced tree: forward by the parallel-variance rule (exact
-// counts), backward by halving trees scaled once by rn(leaves / R) for the
-// means and by 2^L (exact power-of-two steps) for the sums behind dgamma and
-// dbeta.  Then one elementwise pass applies.  With ReLU the forward can also
+// counts), backward by pairwise sum trees: dgamma and dbeta are the sums x
+// post_scale, the means rn(rn(sum * rn(2^L/R)) * 2^-L).  (Sums, not halving
+// means: gradients are small, and halving a subnormal partial mean drops its
+// low bits -- in the last stage of the batch-256 step that lost the whole of
+// dbeta.)  Then one elementwise pass applies.  With ReLU the forward can also
 // store the ReLU decisions as a bit mask, which the backward then reads in
 // place of the saved output (1/16 of its bytes).
 // ============================================================================
@@ -538,9 +542,10 @@ struct BnStatArgs {
   const uint8_t* mask_in;     // backward, ReLU from the bit mask
   const uint16_t* mean_in;    // backward: saved mean
   const uint16_t* invstd_in;  // backward: saved invstd
-  int R, C, blocks, blocks_pow2, total_levels;
+  int R, C, blocks, blocks_pow2;
+  int mean_levels;      // backward: ceil(log2 R); mean = (sum * ratio) * 2^-mean_levels
   int chunk_levels;     // the CTA's per-thread chunk trees are padded to 2^chunk_levels
-  uint16_t ratio;       // rn(leaves / R), leaves = 2^total_levels
+  uint16_t ratio;       // backward: rn(2^mean_levels / R), in [1, 2)
   uint16_t eps, post_scale;
   int* status;          // device status word
   unsigned long long wait_limit_ns;
@@ -560,6 +565,14 @@ __device__ __forceinline__ uint4 tree8(uint4* v) {
   for (int w = 4; w >= 1; w /= 2)
 #pragma unroll
     for (int i = 0; i < w; ++i) v[i] = hmerge4(v[2 * i], v[2 * i + 1]);
+  return v[0];
+}
+// the pairwise sum of 8 rows (backward statistics)
+__device__ __forceinline__ uint4 sum8(uint4* v) {
+#pragma unroll
+  for (int w = 4; w >= 1; w /= 2)
+#pragma unroll
+    for (int i = 0; i < w; ++i) v[i] = add4(v[2 * i], v[2 * i + 1]);
   return v[0];
 }
 
@@ -848,12 +861,12 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
     }
     __syncwarp();
     if ((t & 31) == 0) mbar_arrive(bars + 8 * (kStatStages + s));
-    uint4 n1 = tree8(p1), n2 = tree8(p2);
+    uint4 n1 = sum8(p1), n2 = sum8(p2);
 #pragma unroll 1
     for (int l = 0; l < kStatLevels; ++l) {
       if (cnt & (1u << l)) {
-        n1 = hmerge4(st1[l], n1);
-        n2 = hmerge4(st2[l], n2);
+        n1 = add4(st1[l], n1);
+        n2 = add4(st2[l], n2);
       } else {
         st1[l] = n1;
         st2[l] = n2;
@@ -870,12 +883,12 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
   for (int l = 0; l < kStatLevels; ++l) {
     if (l < a.chunk_levels) {
       if (cnt & (1u << l)) {
-        acc1 = hmerge4(st1[l], have ? acc1 : zero4());
-        acc2 = hmerge4(st2[l], have ? acc2 : zero4());
+        acc1 = add4(st1[l], have ? acc1 : zero4());
+        acc2 = add4(st2[l], have ? acc2 : zero4());
         have = true;
       } else if (have) {
-        acc1 = hmerge4(acc1, zero4());
-        acc2 = hmerge4(acc2, zero4());
+        acc1 = add4(acc1, zero4());
+        acc2 = add4(acc2, zero4());
       }
     } else if (l == a.chunk_levels && (cnt & (1u << l))) {
       acc1 = st1[l];
@@ -888,8 +901,8 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
   for (int half = g.rpb / 2; half >= 1; half /= 2) {
     if (active && rg < half) {
       const int o = (rg + half) * g.tc + cg;
-      s1[t] = hmerge4(s1[t], s1[o]);
-      s2[t] = hmerge4(s2[t], s2[o]);
+      s1[t] = add4(s1[t], s1[o]);
+      s2[t] = add4(s2[t], s2[o]);
     }
     consumers_sync(ncons);
   }
@@ -980,10 +993,11 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_fwd_final(const BnStatArgs
   }
 }
 
-// Backward: halving trees over the per-CTA padded means (zero padding is
-// exact for sums), then means (x rn(2^L/R)) and sums (x 2^L exactly).  Swap
-// variant (a.ws4): dbeta = sum dy' (no post_scale) and dgamma =
-// rn(rn(s * sum dy' xhat) + sum dy' r), the third tree over a.ws4.
+// Backward: pairwise sum trees over the per-CTA sums (zero padding is exact),
+// then the sums scaled by post_scale (dbeta, dgamma) and the means
+// rn(rn(sum * rn(2^L/R)) * 2^-L), L = ceil(log2 R).  Swap variant (a.ws4):
+// dbeta = sum dy' (no post_scale) and dgamma = rn(rn(s * sum dy' xhat) +
+// sum dy' r), the third tree over a.ws4.
 __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs a) {
   pdl_wait();
   __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads], s3[kFinalThreads];
@@ -992,7 +1006,7 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
   const int seg = a.blocks_pow2 / nthr;
   const bool swap = a.ws4 != nullptr;
   if (t < nthr) {
-    Tree4<12, true> t1, t2, t3;
+    Tree4<12, false> t1, t2, t3;
     for (int i0 = 0; i0 < seg; i0 += 4) {
       uint4 p[4], q[4], w[4];
 #pragma unroll
@@ -1019,20 +1033,20 @@ __global__ void __launch_bounds__(kFinalThreads) k_bn_bwd_final(const BnStatArgs
   __syncthreads();
   for (int half = nthr / 2; half >= 1; half /= 2) {
     if (t < half) {
-      s1[t] = hmerge4(s1[t], s1[t + half]);
-      s2[t] = hmerge4(s2[t], s2[t + half]);
-      if (swap) s3[t] = hmerge4(s3[t], s3[t + half]);
+      s1[t] = add4(s1[t], s1[t + half]);
+      s2[t] = add4(s2[t], s2[t + half]);
+      if (swap) s3[t] = add4(s3[t], s3[t + half]);
     }
     __syncthreads();
   }
   if (t == 0) {
     const uint32_t ratio2 = dup2(a.ratio), ps = dup2(a.post_scale);
-    reinterpret_cast<uint4*>(a.mm)[cg] = mul4(s1[0], ratio2);
-    reinterpret_cast<uint4*>(a.mm)[tc + cg] = mul4(s2[0], ratio2);
-    const uint4 sum1 = ldexp4(s1[0], a.total_levels), sum2 = ldexp4(s2[0], a.total_levels);
+    reinterpret_cast<uint4*>(a.mm)[cg] = ldexp_down4(mul4(s1[0], ratio2), a.mean_levels);
+    reinterpret_cast<uint4*>(a.mm)[tc + cg] = ldexp_down4(mul4(s2[0], ratio2), a.mean_levels);
+    const uint4 sum1 = s1[0], sum2 = s2[0];
     if (swap) {
       reinterpret_cast<uint4*>(a.dbeta)[cg] = sum1;
-      reinterpret_cast<uint4*>(a.dgamma)[cg] = add4(mul4(sum2, ps), ldexp4(s3[0], a.total_levels));
+      reinterpret_cast<uint4*>(a.dgamma)[cg] = add4(mul4(sum2, ps), s3[0]);
     } else {
       reinterpret_cast<uint4*>(a.dbeta)[cg] = mul4(sum1, ps);
       reinterpret_cast<uint4*>(a.dgamma)[cg] = mul4(sum2, ps);
@@ -1112,29 +1126,26 @@ __global__ void __launch_bounds__(kFinalThreads)
 }
 
 // Backward statistics from a dgrad statistics buffer (pf16_conv_dgrad_bnstats):
-// the slots hold halving-tree nodes of dy' and dy' * xhat, each over
-// 2^hdr[1] (zero-padded) leaves; a halving tree over the slots padded to a
-// power of two closes the tree over 2^L leaves, then, as k_bn_bwd_final,
-// means x rn(2^L / R) and sums x 2^L exactly.  One CTA per channel group of 8.
+// the slots hold pairwise sums of dy' and dy' * xhat; a pairwise tree over
+// the slots (padded to a power of two with zeros) closes the sums, then, as
+// k_bn_bwd_final, dbeta / dgamma = rn(sum * post_scale) and the means
+// rn(rn(sum * rn(2^L/R)) * 2^-L), L = ceil(log2 R).  One CTA per channel
+// group of 8.
 __global__ void __launch_bounds__(kFinalThreads)
-    k_bn_bwd_final_slots(const uint8_t* __restrict__ stats, int C, long long R, uint16_t post_scale,
-                         uint16_t* mm, uint16_t* dgamma, uint16_t* dbeta) {
+    k_bn_bwd_final_slots(const uint8_t* __restrict__ stats, int C, int mean_levels, uint16_t ratio,
+                         uint16_t post_scale, uint16_t* mm, uint16_t* dgamma, uint16_t* dbeta) {
   pdl_wait();
   __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
   const int tc = C / 8, cg = blockIdx.x, t = threadIdx.x;
   const int S = reinterpret_cast<const int*>(stats)[0];
-  const int L0 = reinterpret_cast<const int*>(stats)[1];
   const uint16_t* sd = reinterpret_cast<const uint16_t*>(stats + bnstat_off_mean());
   const uint16_t* sp = reinterpret_cast<const uint16_t*>(stats + bnstat_off_var(C));
-  int sp2 = 1, ls = 0;
-  while (sp2 < S) {
-    sp2 *= 2;
-    ++ls;
-  }
+  int sp2 = 1;
+  while (sp2 < S) sp2 *= 2;
   const int nthr = sp2 < kFinalThreads ? sp2 : kFinalThreads;
   const int seg = sp2 / nthr;
   if (t < nthr) {
-    Tree4<12, true> t1, t2;
+    Tree4<12, false> t1, t2;
     for (int i = 0; i < seg; ++i) {
       const int b = t * seg + i;
       const bool ok = b < S;
@@ -1148,19 +1159,17 @@ __global__ void __launch_bounds__(kFinalThreads)
   __syncthreads();
   for (int half = nthr / 2; half >= 1; half /= 2) {
     if (t < half) {
-      s1[t] = hmerge4(s1[t], s1[t + half]);
-      s2[t] = hmerge4(s2[t], s2[t + half]);
+      s1[t] = add4(s1[t], s1[t + half]);
+      s2[t] = add4(s2[t], s2[t + half]);
     }
     __syncthreads();
   }
   if (t == 0) {
-    const int L = L0 + ls;
-    const uint16_t ratio = __half_as_ushort(__float2half_rn((float)(ldexp(1.0, L) / (double)R)));
     const uint32_t ratio2 = dup2(ratio), ps = dup2(post_scale);
-    reinterpret_cast<uint4*>(mm)[cg] = mul4(s1[0], ratio2);
-    reinterpret_cast<uint4*>(mm)[tc + cg] = mul4(s2[0], ratio2);
-    reinterpret_cast<uint4*>(dbeta)[cg] = mul4(ldexp4(s1[0], L), ps);
-    reinterpret_cast<uint4*>(dgamma)[cg] = mul4(ldexp4(s2[0], L), ps);
+    reinterpret_cast<uint4*>(mm)[cg] = ldexp_down4(mul4(s1[0], ratio2), mean_levels);
+    reinterpret_cast<uint4*>(mm)[tc + cg] = ldexp_down4(mul4(s2[0], ratio2), mean_levels);
+    reinterpret_cast<uint4*>(dbeta)[cg] = mul4(s1[0], ps);
+    reinterpret_cast<uint4*>(dgamma)[cg] = mul4(s2[0], ps);
   }
 }
 
@@ -1318,10 +1327,9 @@ static BnStatArgs bn_args(const BnLaunch& b, const BnPlan& p, uint16_t* ws) {
   a.blocks = p.blocks;
   a.blocks_pow2 = p.blocks_pow2;
   a.chunk_levels = ceil_log2(p.chunks_per_cta);
-  // leaves of the backward trees: 8 rows x 2^chunk_levels chunks x rpb row groups x CTAs
-  const long long leaves = ((long long)b.chunk_rows << a.chunk_levels) * p.blocks_pow2;
-  a.total_levels = ceil_log2(leaves);
-  a.ratio = f16_bits_host((float)((double)leaves / (double)b.R));
+  // backward means: sum * rn(2^L / R) * 2^-L, L = ceil(log2 R)
+  a.mean_levels = ceil_log2(b.R);
+  a.ratio = f16_bits_host((float)(ldexp(1.0, a.mean_levels) / (double)b.R));
   a.eps = b.eps;
   a.post_scale = b.post_scale;
   a.status = b.status;
@@ -1423,8 +1431,8 @@ cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   int launches = 3;
   if (dgrad_stats) {
     // statistics from the producing data gradient's epilogue
-    launch_pdl(k_bn_bwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, dgrad_stats, b.C, b.R,
-               b.post_scale, a.mm, dgamma, dbeta);
+    launch_pdl(k_bn_bwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, dgrad_stats, b.C, a.mean_levels,
+               a.ratio, b.post_scale, a.mm, dgamma, dbeta);
     launches = 2;
   } else {
     if ((e = bwd_stats_mode<false>(mode, a, b, s)) != cudaSuccess) return e;

@@ -404,8 +404,8 @@ struct EpiStats {
   // gradient tile g and the prefetched inputs of its 32 rows (BwdIn).  Lane l
   // takes channel pair (2l, 2l+1): dy' = g where the ReLU passed and
   // dy' * rn(rn(x - mean) * invstd); rows r >= nv are zero leaves.  Each
-  // 32-leaf halving tree is pushed into chunk c's binary counter of halving
-  // nodes (mu: dy', v: dy' xhat).
+  // 32-leaf pairwise sum is pushed into chunk c's binary counter of sum nodes
+  // (mu: dy', v: dy' xhat).
   __device__ __forceinline__ void leaf_bwd(int c, uint32_t stg, int lane, int nv, const struct BwdIn& in);
   // The same leaf with x read from a 128B-swizzled 32 x 64 tile at xs (laid
   // out as the staged tile), ReLU bits m of row `lane` and the pair's mean2 /
@@ -419,8 +419,8 @@ struct EpiStats {
   __device__ __forceinline__ void leaf_bwd_impl(int c, uint32_t stg, int lane, int nv, uint2 m, uint32_t mean2,
                                                 uint32_t invstd2, XF xf);
   // Close the backward counters as if zero leaves padded them to 2^levels,
-  // merge the CTA's 8 epilogue warps by halving (warps 0..7 in a balanced
-  // tree, through `sm` as write_cta) and write the CTA's nodes as `slot`.
+  // add the CTA's 8 epilogue warps' sums (warps 0..7 in a balanced tree,
+  // through `sm` as write_cta) and write the CTA's sums as `slot`.
   __device__ __forceinline__ void write_cta_bwd(const GemmParams& p, uint8_t* sm, int e, int slot, int n0,
                                                 int nchunks, int lane, int levels) {
     uint32_t* node = reinterpret_cast<uint32_t*>(sm);  // [8][kStChunks][32][2]
@@ -436,12 +436,12 @@ struct EpiStats {
             a2 = this->v[c][l];
           }
         } else if (cnt & (1u << l)) {
-          a1 = hmerge2f(this->mu[c][l], have ? a1 : 0u);
-          a2 = hmerge2f(this->v[c][l], have ? a2 : 0u);
+          a1 = hadd2_rn(this->mu[c][l], have ? a1 : 0u);
+          a2 = hadd2_rn(this->v[c][l], have ? a2 : 0u);
           have = true;
         } else if (have) {
-          a1 = hmerge2f(a1, 0u);
-          a2 = hmerge2f(a2, 0u);
+          a1 = hadd2_rn(a1, 0u);
+          a2 = hadd2_rn(a2, 0u);
         }
       }
       node[((e * kStChunks + c) * 32 + lane) * 2] = a1;
@@ -460,8 +460,8 @@ struct EpiStats {
       for (int h = 1; h < 8; h *= 2)
 #pragma unroll
         for (int w = 0; w < 8; w += 2 * h) {
-          m1[w] = hmerge2f(m1[w], m1[w + h]);
-          m2[w] = hmerge2f(m2[w], m2[w + h]);
+          m1[w] = hadd2_rn(m1[w], m1[w + h]);
+          m2[w] = hadd2_rn(m2[w], m2[w + h]);
         }
       const long long o = (long long)slot * p.N + n0 + c * 64 + 2 * lane;
       *reinterpret_cast<uint32_t*>(p.st_mean + o) = m1[0];
@@ -524,15 +524,15 @@ __device__ __forceinline__ void EpiStats::leaf_bwd_impl(int c, uint32_t stg, int
   for (int w = 16; w >= 1; w /= 2)
 #pragma unroll
     for (int i = 0; i < w; ++i) {
-      t1[i] = hmerge2f(t1[2 * i], t1[2 * i + 1]);
-      t2[i] = hmerge2f(t2[2 * i], t2[2 * i + 1]);
+      t1[i] = hadd2_rn(t1[2 * i], t1[2 * i + 1]);
+      t2[i] = hadd2_rn(t2[2 * i], t2[2 * i + 1]);
     }
   uint32_t n1 = t1[0], n2 = t2[0];
 #pragma unroll 1
   for (int l = 0; l < kStLevels; ++l) {
     if (cnt & (1u << l)) {
-      n1 = hmerge2f(mu[c][l], n1);
-      n2 = hmerge2f(v[c][l], n2);
+      n1 = hadd2_rn(mu[c][l], n1);
+      n2 = hadd2_rn(v[c][l], n2);
     } else {
       mu[c][l] = n1;
       v[c][l] = n2;

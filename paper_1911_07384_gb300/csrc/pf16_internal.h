@@ -125,10 +125,10 @@ struct GemmParams {
   // BatchNorm backward statistics instead (bs_x non-null; same buffer): the
   // output is the gradient dL/dy of a BatchNorm whose input bs_x ([pixels][N],
   // row pitch ldo), ReLU bits bs_mask ([pixels][N/8], or null) and saved
-  // bs_mean / bs_invstd are given.  Per slot and channel: the halving-tree
-  // node of dy' (in st_mean) and of dy' * xhat (in st_var), every epilogue
-  // warp's tile trees padded to 2^bs_levels leaves; st_hdr[0] = slots,
-  // st_hdr[1] = tree levels below the slot tree (5 + bs_levels + 3).
+  // bs_mean / bs_invstd are given.  Per slot and channel: the pairwise sum
+  // of dy' (in st_mean) and of dy' * xhat (in st_var), every epilogue warp's
+  // tile trees padded with zeros to 2^bs_levels leaves; st_hdr[0] = slots,
+  // st_hdr[1] = tree levels below the slot tree (5 + bs_levels + 3; informational).
   const uint16_t* bs_x;
   const uint8_t* bs_mask;
   const uint16_t* bs_mean;
