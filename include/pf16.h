@@ -183,6 +183,8 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
  *    buffer is far larger.  Every other ResNet-50 layer at batch 256 fits.
  *  - The first call on each device looks up the array's device address (with
  *    that device current); make that first call before any stream capture.
+ *    The address is kept for the life of the process: after cudaDeviceReset
+ *    on a device this entry point must not be called on that device again.
  *  - All calls share the one array, which keeps the last call's contents
  *    (no call depends on them).  Calls that can overlap on the GPU -- on
  *    different streams, or on one device from several threads -- race on it;

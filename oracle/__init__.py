@@ -17,6 +17,7 @@ Paper passages followed (arXiv 1911.07384):
   * Eq. 1, Eq. 2 and the x0.25 scaling of Sec. 4.2        -> bn_fwd, bn_bwd
   * Sec. 5.1 (rest of the ResNet-50 training step)        -> maxpool, avgpool,
                                                              softmax_xent
+  * Sec. 5.1 / 5.2 (data-parallel gradient average, FP16)  -> allreduce_combine
 """
 from __future__ import annotations
 
@@ -76,6 +77,8 @@ def _L():
                 getattr(lib, nm).argtypes = conv_args
             lib.orc_sgd_update.argtypes = [u16p, u16p, u16p, ctypes.c_int64, ctypes.c_uint16,
                                            ctypes.c_uint16, ctypes.c_uint16]
+            lib.orc_allreduce_combine.argtypes = [u16p, I, ctypes.c_int64, ctypes.c_int64, ctypes.c_uint16,
+                                                  u16p]
             lib.orc_bn_fwd.argtypes = [u16p, u16p, u16p, u16p, ctypes.c_int64, I, ctypes.c_double,
                                        ctypes.c_double, I, f64p, f64p, f64p, f64p]
             lib.orc_bn_bwd.argtypes = [u16p, u16p, u16p, u16p, ctypes.c_int64, I, ctypes.c_double,
@@ -183,6 +186,18 @@ def sgd_update(w, v, g, lr_bits: int, momentum_bits: int, wd_bits: int):
     _L().orc_sgd_update(_p(w, ctypes.c_uint16), _p(v, ctypes.c_uint16), _p(g, ctypes.c_uint16),
                         w.size, lr_bits, momentum_bits, wd_bits)
     return w, v
+
+
+# ---------------------------------------------------------------- data-parallel exchange
+def allreduce_combine(planes, scale_bits: int):
+    """planes: [world][n] binary16 bits, one plane per rank in rank order.
+    Returns the n binary16 bits of the fixed-order FP16 average (Sec. 5.1,
+    5.2): a pairwise tree of additions over the ranks, then x scale."""
+    planes = _u16(planes)
+    world, n = planes.shape
+    out = np.empty(n, np.uint16)
+    _L().orc_allreduce_combine(_p(planes, ctypes.c_uint16), world, n, n, scale_bits, _p(out, ctypes.c_uint16))
+    return out
 
 
 # ---------------------------------------------------------------- BatchNorm

@@ -45,6 +45,12 @@ void orc_conv_wgrad(const uint16_t* x, const uint16_t* dy, int N, int H, int W, 
 void orc_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, int64_t n, uint16_t lr,
                     uint16_t momentum, uint16_t wd);
 
+/* Data-parallel gradient average: per element, a pairwise tree of binary16
+ * additions over the world's planes in rank order (+0 leaves up to a power of
+ * two), then one multiplication by scale (skipped when scale is 1).  Bit-exact. */
+void orc_allreduce_combine(const uint16_t* planes, int world, int64_t n, int64_t plane_stride,
+                           uint16_t scale, uint16_t* out);
+
 /* BatchNorm over R rows of C channels (training mode, batch statistics). */
 void orc_bn_fwd(const uint16_t* x, const uint16_t* gamma, const uint16_t* beta,
                 const uint16_t* residual, int64_t R, int C, double eps, double s, int relu,

@@ -15,6 +15,8 @@
  *  - SGD with momentum and coupled weight decay (the PyTorch ImageNet recipe
  *    the paper adopts, Sec. 5.1) in pure FP16 with no master copy (Sec. 5.2):
  *    each op one binary16 rounding, bit-exact.
+ *  - The FP16 gradient average of data-parallel training (Sec. 5.1, 5.2) in a
+ *    fixed summation order, bit-exact.
  *  - BatchNorm with batch statistics (Eq. 1, Eq. 2) followed by the x0.25
  *    output scaling inside residual blocks (Sec. 4.2), residual add and ReLU.
  *  - Max pooling, global average pooling and softmax cross-entropy, the rest
@@ -180,6 +182,30 @@ void orc_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, int64_t n, uint
     const uint16_t vi = orc_h_add(orc_h_mul(momentum, v[i]), gi);
     w[i] = orc_h_sub(w[i], orc_h_mul(lr, vi));
     v[i] = vi;
+  }
+}
+
+/* The combining step of data-parallel training's gradient exchange (Sec. 5.1:
+ * each of `world` GPUs computes the gradient of its own batch; they are
+ * averaged before the SGD step, in FP16 like everything else, Sec. 5.2).
+ * The reading taken here: the world's gradients are summed first, by a
+ * pairwise tree over the ranks in rank order -- at each level, neighbours
+ * (0,1), (2,3), ... are added, one binary16 rounding per addition, the rank
+ * count padded with +0 leaves up to a power of two -- and the sum is then
+ * multiplied by `scale` (normally rn(1/world)), unless scale is 1.  Out of
+ * place or in place on plane 0. */
+void orc_allreduce_combine(const uint16_t* planes, int world, int64_t n, int64_t plane_stride,
+                           uint16_t scale, uint16_t* out) {
+  int leaves = 1;
+  while (leaves < world) leaves *= 2;
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < n; ++i) {
+    uint16_t* t = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)leaves);
+    for (int r = 0; r < leaves; ++r) t[r] = r < world ? planes[(int64_t)r * plane_stride + i] : 0x0000;
+    for (int width = leaves; width > 1; width /= 2)
+      for (int k = 0; k < width / 2; ++k) t[k] = orc_h_add(t[2 * k], t[2 * k + 1]);
+    out[i] = scale == 0x3C00 ? t[0] : orc_h_mul(t[0], scale);
+    free(t);
   }
 }
 

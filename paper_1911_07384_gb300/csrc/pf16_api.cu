@@ -1053,6 +1053,24 @@ int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint1
              : PF16_ERR_CUDA;
 }
 
+int pf16_allreduce_combine(const uint16_t* planes, int32_t world, size_t n, size_t plane_stride,
+                           uint16_t scale, uint16_t* out, void* stream) {
+  if (world < 1 || world > 1024 || n % 8 != 0 || plane_stride % 8 != 0 || plane_stride < n)
+    return PF16_ERR_SHAPE;
+  if ((size_t)world * plane_stride > ((size_t)1 << 40)) return PF16_ERR_SHAPE;
+  if (n == 0) return PF16_OK;
+  if (!planes || !out) return PF16_ERR_NULL;
+  if (!aligned16(planes) || !aligned16(out)) return PF16_ERR_ALIGN;
+  // out is plane 0 or lies clear of every plane
+  const uintptr_t o = reinterpret_cast<uintptr_t>(out), b = reinterpret_cast<uintptr_t>(planes);
+  const uintptr_t e = b + ((size_t)(world - 1) * plane_stride + n) * 2;
+  if (o != b && o + n * 2 > b && o < e) return PF16_ERR_SHAPE;
+  return launch_dp_combine(planes, world, n, plane_stride, scale, out, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
 static int bn_validate(const pf16_bn_desc* d, BnLaunch* b) {
   if (!d) return PF16_ERR_NULL;
   if (d->n <= 0 || d->h <= 0 || d->w <= 0 || d->c <= 0) return PF16_ERR_SHAPE;

@@ -167,6 +167,74 @@ cudaError_t launch_sgd(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, ui
 }
 
 // ============================================================================
+// Data-parallel gradient exchange, combining step: out = rn(T * scale), T the
+// perfect pairwise FP16 tree over `world` planes in plane order (padded with
+// +0 leaves to a power of two).  Each thread owns one 8-element chunk: its
+// leaves are loaded in aligned batches of up to 16 (all loads of a batch in
+// flight), each batch summed as a perfect tree, and the batch sums merged by
+// a register-resident binary counter -- together the perfect tree over the
+// padded leaves.  Every load of a chunk precedes its store, so out may be
+// plane 0.
+// ============================================================================
+__global__ void __launch_bounds__(256)
+    k_dp_combine(const uint16_t* __restrict__ planes, int world, int world_pow2, long long nvec,
+                 long long pstride_vec, uint32_t scale2, int do_scale, uint16_t* out) {
+  pdl_wait();
+  const uint4* P = reinterpret_cast<const uint4*>(planes);
+  uint4* O = reinterpret_cast<uint4*>(out);
+  const int nb = world_pow2 < 16 ? world_pow2 : 16;
+  const long long step = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += step) {
+    uint4 st[7];  // st[l]: a finished subtree of 2^l batch sums (1024 / 16 = 2^6 batches at most)
+    unsigned cnt = 0;
+    for (int j0 = 0; j0 < world_pow2; j0 += 16) {
+      uint4 v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int r = j0 + j;
+        v[j] = (j < nb && r < world) ? P[(long long)r * pstride_vec + i] : zero4();
+      }
+#pragma unroll
+      for (int w = 1; w < 16; w *= 2)
+#pragma unroll
+        for (int j = 0; j < 16; j += 2 * w)
+          if (j + w < nb) v[j] = add4(v[j], v[j + w]);
+      uint4 b = v[0];
+      bool carry = true;
+#pragma unroll
+      for (int l = 0; l < 7; ++l) {
+        const bool bit = (cnt >> l) & 1u;
+        if (carry && bit) b = add4(st[l], b);
+        if (carry && !bit) {
+          st[l] = b;
+          carry = false;
+        }
+      }
+      ++cnt;
+    }
+    uint4 acc = zero4();
+#pragma unroll
+    for (int l = 0; l < 7; ++l)
+      if (cnt == (1u << l)) acc = st[l];
+    O[i] = do_scale ? mul4(acc, scale2) : acc;
+  }
+}
+
+cudaError_t launch_dp_combine(const uint16_t* planes, int world, size_t n, size_t plane_stride, uint16_t scale,
+                              uint16_t* out, cudaStream_t s) {
+  int w2 = 1;
+  while (w2 < world) w2 *= 2;
+  const long long nvec = (long long)(n / 8);
+  long long blocks = (nvec + 255) / 256;
+  if (blocks > 152ll * 8) blocks = 152ll * 8;
+  if (blocks < 1) blocks = 1;
+  const uint32_t scale2 = (uint32_t)scale | ((uint32_t)scale << 16);
+  launch_pdl(k_dp_combine, dim3((unsigned)blocks), dim3(256), 0, s, planes, world, w2, nvec,
+             (long long)(plane_stride / 8), scale2, scale != 0x3C00 ? 1 : 0, out);
+  return counted_launches(1);
+}
+
+// ============================================================================
 // Split-K weight-gradient reduction: out = balanced pairwise FP16 tree over
 // the `splits` partial matrices.
 // ============================================================================

@@ -219,6 +219,10 @@ cudaError_t launch_wait_flag(const uint32_t* flag, uint32_t value, unsigned long
                              cudaStream_t s);
 // sum of `splits` FP16 partial matrices [splits][rows][cols] by a balanced
 // pairwise tree; the result row r goes to out + r*ldo (only cols_out columns).
+// Data-parallel exchange, combining step (pf16_allreduce_combine): n and
+// plane_stride multiples of 8, 1 <= world <= 1024.
+cudaError_t launch_dp_combine(const uint16_t* planes, int world, size_t n, size_t plane_stride, uint16_t scale,
+                              uint16_t* out, cudaStream_t s);
 cudaError_t launch_splitk_reduce(const uint16_t* parts, int splits, long long rows, int cols,
                                  uint16_t* out, long long ldo, int cols_out, cudaStream_t s);
 // stem patches: col[m][j] = x[n, 2p+r-3, 2q+s-3, c] for j = (r*7+s)*3+c < 147, 0 up to kcol.

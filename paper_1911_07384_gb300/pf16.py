@@ -31,7 +31,7 @@ PF16_PASS_FWD, PF16_PASS_DGRAD, PF16_PASS_WGRAD = 0, 1, 2
 
 EXPORTS = [
     "pf16_conv_workspace_size", "pf16_conv_fwd", "pf16_conv_dgrad", "pf16_conv_wgrad",
-    "pf16_sgd_update", "pf16_bn_workspace_size", "pf16_bn_fwd_bwd", "pf16_maxpool_fwd",
+    "pf16_sgd_update", "pf16_allreduce_combine", "pf16_bn_workspace_size", "pf16_bn_fwd_bwd", "pf16_maxpool_fwd",
     "pf16_maxpool_bwd", "pf16_avgpool_fwd", "pf16_avgpool_bwd",
     "pf16_softmax_xent_workspace_size", "pf16_softmax_xent", "pf16_sync_status",
     "pf16_status_string", "pf16_device_arch", "pf16_conv_wgrad_noalloc",
@@ -109,6 +109,8 @@ def lib():
             L.pf16_conv_wgrad_noalloc.restype = I
             L.pf16_sgd_update.argtypes = [vp, vp, vp, sz, u16, u16, u16, u32, vp]
             L.pf16_sgd_update.restype = I
+            L.pf16_allreduce_combine.argtypes = [vp, i32, sz, sz, u16, vp, vp]
+            L.pf16_allreduce_combine.restype = I
             L.pf16_bn_workspace_size.argtypes = [ctypes.POINTER(BnDesc)]
             L.pf16_bn_workspace_size.restype = sz
             L.pf16_bn_fwd_bwd.argtypes = [ctypes.POINTER(BnDesc), I, ctypes.POINTER(BnTensors), vp,
@@ -245,6 +247,13 @@ WGRAD_NOALLOC_SCRATCH_BYTES = 32 << 20
 def sgd_update(w, v, g, lr_bits, momentum_bits, wd_bits, flags=0, stream=None):
     _check(lib().pf16_sgd_update(_ptr(w), _ptr(v), _ptr(g), w.numel(), lr_bits, momentum_bits,
                                  wd_bits, flags, _stream(stream)), "pf16_sgd_update")
+
+
+def allreduce_combine(planes, world, n, plane_stride, scale_bits, out, stream=None):
+    """planes: a device tensor holding `world` planes of n binary16 values,
+    plane r at element offset r * plane_stride; out: n values (may be planes)."""
+    _check(lib().pf16_allreduce_combine(_ptr(planes), world, n, plane_stride, scale_bits, _ptr(out),
+                                        _stream(stream)), "pf16_allreduce_combine")
 
 
 def bn_desc(n, h, w, c, eps_bits=0x00A8, post_scale_bits=0x3400, flags=0) -> BnDesc:

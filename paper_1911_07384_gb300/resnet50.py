@@ -307,13 +307,18 @@ class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
     def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False,
-                 wgrad_branch=False):
+                 wgrad_branch=False, exchange=None):
         """wgrad_branch: issue the weight gradients on a second stream that joins
         before the update (in a captured step graph: a parallel branch), so that
         they fill the gaps of the data-gradient chain; off, every call runs on the
-        current stream in program order (what per-call timing needs)."""
+        current stream in program order (what per-call timing needs).
+        exchange: data-parallel training (Sec. 5.1): a callable applied, before
+        the update, to each flat gradient arena (decayed, then not decayed) to
+        average it over the ranks in place, e.g. functools.partial(
+        dp.allreduce_mean_, group=g); None on one GPU."""
         self.N, self.image, self.classes, self.device = batch, image, classes, device
         self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
+        self.exchange = exchange
         self.side = torch.cuda.Stream(device=device) if wgrad_branch else None
         self.wd, self.nowd = Arena("decayed"), Arena("no-decay")
         self.convs, self.bns = [], []
@@ -430,6 +435,9 @@ class ResNet50:
     def update(self):
         if self.side is not None:  # every weight gradient is in before the update reads it
             torch.cuda.current_stream().wait_stream(self.side)
+        if self.exchange is not None:  # the ranks' gradients averaged, in a fixed FP16 order
+            self.call("exchange", None, self.exchange, self.wd.g)
+            self.call("exchange", None, self.exchange, self.nowd.g)
         self.call("sgd", None, pf16.sgd_update, self.wd.w, self.wd.v, self.wd.g, LR, MOMENTUM, WD)
         self.call("sgd", None, pf16.sgd_update, self.nowd.w, self.nowd.v, self.nowd.g, LR, MOMENTUM, 0)
 
