@@ -29,6 +29,7 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   __shared__ uint64_t bar;
   __shared__ uint32_t tslot;
+  __shared__ int drained;  // the MMAs are known complete: their TMEM may be released
   const int warp = threadIdx.x >> 5;
   const int words = (kBM * 64 * 2 + n * 64 * 2) / 16;
   for (int i = threadIdx.x; i < words; i += blockDim.x)
@@ -57,14 +58,17 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
         tc_mma_f16(d, a0 + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), idesc, (it >= chains || kk > 0) ? 1u : 0u);
     }
     tc_commit(smem_u32(&bar));
+    drained = 1;
     if (!mbar_wait(smem_u32(&bar), 0, wait_ns)) {
       atomicCAS(status, 0, -7);  // PF16_ERR_TIMEOUT
-      mbar_wait(smem_u32(&bar), 0, 1000000000ull);
+      // a second bounded wait; if the MMAs still have not completed, their
+      // TMEM is left allocated rather than released under them
+      drained = mbar_wait(smem_u32(&bar), 0, 1000000000ull) ? 1 : 0;
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 0 && drained) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
