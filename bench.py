@@ -189,6 +189,8 @@ def main():
     ap.add_argument("--nvtx", action="store_true",
                     help="name every library call of the step with an NVTX range (pf16:<kind>:<shape>) for "
                          "profilers; host-side only, the replayed step graph is unchanged")
+    ap.add_argument("--bn-in-operand", action="store_true",
+                    help="apply each block's second BatchNorm in its last conv's operand path (off by default)")
     ap.add_argument("--bn-swap", action="store_true",
                     help="the BN-swap variant (Sec. 4.1) in every block's last BatchNorm (off in the headline run)")
     ap.add_argument("--layers", action="store_true",
@@ -242,7 +244,7 @@ def main():
     from paper_1911_07384_gb300.resnet50 import ResNet50
 
     N = args.batch
-    net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap, wgrad_branch=True)
+    net = ResNet50(batch=N, seed_cfg=4, bn_swap=args.bn_swap, wgrad_branch=True, bn_in_operand=args.bn_in_operand)
     if args.nvtx:
         from paper_1911_07384_gb300.resnet50 import nvtx_hook
 
@@ -347,9 +349,14 @@ def main():
     conv = conv_roofline(net, stream, reps=3)
     pk = peaks()
     peak = pk["bf16_tflops_sustained"]  # FP16 and BF16 share the dense tensor rate
+    kr = kernel_roofline(pk)
+    # the aggregate over every conv call of the step; its per-launch DRAM traffic
+    # is not measured (a whole-step capture is not made); the single dominant
+    # launch class with its captured traffic is roofline_kernel
     roof = {"bound": "tensor", "achieved": conv["tflops"], "peak": peak, "unit": "TFLOP/s",
-            "frac": conv["tflops"] / peak, "traffic": gemm_traffic(),
+            "frac": conv["tflops"] / peak, "traffic": None,
             "algorithmic_bytes_per_launch": conv["bytes_per_launch"],
+            "frac_of_f16_mma_probe": conv["tflops"] / kr["peak_f16_mma_probe"],
             "kernel": "k_gemm (all conv passes of the step, split-K reduce included)",
             "peak_src": f"{pk['src']} bf16 dense sustained"}
 
@@ -360,12 +367,14 @@ def main():
         "config": {"workload": WORKLOAD, "global_batch": N * world, "per_gpu_batch": N,
                    "image": "224x224x3 NHWC", "parallelism": f"replicas{world}" if world > 1 else "single",
                    "l2": "working set (~25 GB of activations per step) far larger than L2; no flush needed",
-                   **({"bn_swap": True} if args.bn_swap else {})},
+                   **({"bn_swap": True} if args.bn_swap else {}),
+                   **({"bn_in_operand": True} if args.bn_in_operand else {})},
         "loss": loss,
         "clocks": clocks.summary(),
         "e2e": e2e,
         "gpu_launches": launches * args.steps,
         "roofline": roof,
+        "roofline_kernel": kr,
         "conv": {"tflops": conv["tflops"], "ms_per_step": conv["ms"], "gflop_per_step": conv["gflop"],
                  "frac_of_dense_peak": conv["tflops"] / pk["bf16_tflops"], "by_pass": conv["by_pass"]},
     }
@@ -416,7 +425,7 @@ def run_layers(args):
     from paper_1911_07384_gb300 import synthetic as syn
     from paper_1911_07384_gb300.resnet50 import ResNet50
 
-    net = ResNet50(batch=args.batch, seed_cfg=4)
+    net = ResNet50(batch=args.batch, seed_cfg=4, bn_in_operand=args.bn_in_operand)
     net.set_batch(syn.images_f16(syn.seed_for(4, "x", 0), args.batch),
                   syn.labels(syn.seed_for(4, "labels", 0), args.batch))
     stream = torch.cuda.Stream()
@@ -628,7 +637,13 @@ def time_bn(shape, bn_pass, steps, warmup):
             "frac_of_hbm": byts / ms / 1e6 / pk["hbm_gbs"], "algorithmic_bytes": byts}
 
 
-TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_resnet50_b256_step_traffic.json")
+# The dominant launch class of the step, k_gemm<256> (BN = 256, plain epilogue),
+# on one of its layers: the 14x14, 256 -> 256, 3x3 forward at batch 256 (five
+# calls per step; 59.2 GFLOP per launch).  Its DRAM traffic comes from one
+# ncu capture of that single launch (bench.py --conv ... under ncu -c 1).
+KERNEL_LAYER = (256, 14, 14, 256, 256, 3, 3, 1, 1)
+KERNEL_NAME = "k_gemm<256> (plain epilogue), 14x14 256->256 3x3 forward, batch 256"
+TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_256_conv_14x14_256_3x3_fwd_b256_traffic.json")
 GEMM_SOURCES = ["pf16_gemm.cu", "pf16_api.cu", "pf16_internal.h", "pf16_ptx.cuh"]
 
 
@@ -653,9 +668,10 @@ def gemm_source_digest():
 
 
 def ingest_traffic(csv_path):
-    """Per-launch DRAM traffic of k_gemm from an ncu CSV of one bench step
-    (metrics gpu__time_duration.sum, dram__bytes_read.sum, dram__bytes_write.sum),
-    stored with the digest of the sources it was measured on."""
+    """DRAM traffic of the one k_gemm launch in an ncu CSV (metrics
+    gpu__time_duration.sum, dram__bytes_read.sum, dram__bytes_write.sum) of
+    `bench.py --conv <KERNEL_LAYER> --pass fwd`, stored with the digest of the
+    sources it was measured on."""
     import csv as _csv
 
     with open(csv_path) as f:
@@ -671,22 +687,15 @@ def ingest_traffic(csv_path):
         if len(r) <= vi or "k_gemm" not in r[ki]:
             continue
         per.setdefault(r[ii], {})[r[mi]] = float(r[vi].replace(",", "")) * scale[r[ui]]
-    from paper_1911_07384_gb300.resnet50 import conv_shapes
-
-    # per conv: forward + data gradient (one GEMM per stride phase) + weight
-    # gradient where it is a k_gemm launch; the stem has no data gradient
-    step = sum(1 + (0 if c == 3 else (st * st if r > 1 else 1)) + (1 if wgrad_is_gemm(h, w, c, k, r, s, st, pd) else 0)
-               for _, (_, h, w, c, k, r, s, st, pd) in conv_shapes(BATCH))
-    ids = sorted(per, key=int)[:step]  # the first whole step (the eager warm-up step)
-    if len(ids) < step:
-        raise SystemExit(f"{csv_path}: {len(ids)} k_gemm launches, one step has {step}")
-    per = {i: per[i] for i in ids}
-    n = len(per)
-    rd = sum(v["dram__bytes_read.sum"] for v in per.values())
-    wr = sum(v["dram__bytes_write.sum"] for v in per.values())
-    ns = sum(v["gpu__time_duration.sum"] for v in per.values())
-    out = {"kernel": "k_gemm", "workload": WORKLOAD, "launches": n, "dram_read_bytes": rd,
-           "dram_write_bytes": wr, "time_ns": ns, "traffic_per_launch": (rd + wr) / n,
+    if len(per) != 1:
+        raise SystemExit(f"{csv_path}: {len(per)} k_gemm launches, expected the one captured launch")
+    v = next(iter(per.values()))
+    rd, wr = v["dram__bytes_read.sum"], v["dram__bytes_write.sum"]
+    N, H, W, C, K, R, S, st, pd = KERNEL_LAYER
+    P, Q = (H + 2 * pd - R) // st + 1, (W + 2 * pd - S) // st + 1
+    out = {"kernel": KERNEL_NAME, "layer": list(KERNEL_LAYER), "dram_read_bytes": rd, "dram_write_bytes": wr,
+           "traffic_per_launch": rd + wr, "ncu_time_ns": v.get("gpu__time_duration.sum"),
+           "algorithmic_bytes": 2 * (N * H * W * C + K * R * S * C + N * P * Q * K),
            "source_sha256": gemm_source_digest()}
     with open(TRAFFIC_JSON, "w") as f:
         json.dump(out, f, indent=1)
@@ -696,13 +705,30 @@ def ingest_traffic(csv_path):
 
 
 def gemm_traffic():
-    """Stored per-launch DRAM bytes of k_gemm, or None once the sources changed."""
+    """Stored DRAM bytes of the one-launch capture, or None once the sources changed."""
     try:
         with open(TRAFFIC_JSON) as f:
             t = json.load(f)
     except (OSError, ValueError):
         return None
     return t["traffic_per_launch"] if t.get("source_sha256") == gemm_source_digest() else None
+
+
+def kernel_roofline(pk, reps=10):
+    """The dominant launch class on its representative layer, timed alone with
+    CUDA events (L2 flushed between launches), against the measured sustained
+    16-bit peak and against the FP16 MMA rate the library's probe measures on
+    this GPU (kind::f16, N = 256)."""
+    from paper_1911_07384_gb300 import pf16
+
+    r = time_conv(KERNEL_LAYER, "fwd", reps, 3)
+    mma = pf16.tc_rate(256, reps=20000)
+    return {"bound": "tensor", "kernel": KERNEL_NAME, "achieved": r["tflops"],
+            "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": r["tflops"] / pk["bf16_tflops_sustained"],
+            "peak_f16_mma_probe": mma, "frac_of_f16_mma_probe": r["tflops"] / mma,
+            "ms_per_launch": r["ms"], "gflop_per_launch": r["tflops"] * r["ms"],
+            "traffic": gemm_traffic(), "algorithmic_bytes": r["gbs"] * r["ms"] * 1e6,
+            "peak_src": f"{pk['src']} bf16 dense sustained; f16 MMA probe measured in this run"}
 
 
 def count_launches(net):
@@ -723,7 +749,9 @@ def count_launches(net):
         total += 1 + (1 if ws else 0) + (2 if stem else 0)  # wgrad (+ split-K reduce, + the stem's s2d, scatter)
     # forward statistics come from the conv; backward ones from the data gradient where fused
     # (the swap variant's backward takes a second statistics pass)
+    # (a BatchNorm applied in the next conv's operand path launches no apply pass)
     total += sum(per["bn_fwd"] + per["bn_bwd"] - (1 if getattr(b, "fused_bwd", False) else 0)
+                 - (1 if getattr(b, "fused_apply", False) else 0)
                  + (1 if b.desc.flags & pf16.PF16_BN_SWAP else 0) for b in net.bns)
     total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]

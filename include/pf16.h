@@ -167,6 +167,43 @@ int pf16_conv_dgrad_bnstats_add(const pf16_conv_desc* d, const uint16_t* dy, con
 int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                     void* ws, size_t ws_bytes, uint32_t flags, void* stream);
 
+/* ----------------------------------------- BatchNorm in the operand path
+ * A conv whose input is the output of a BatchNorm (Eq. 1, Eq. 2, x post_scale
+ * of Sec. 4.2, optional ReLU) can take the BatchNorm's INPUT x and apply it
+ * to each operand tile in shared memory, between the tile's arrival and the
+ * tensor core's read -- the same FP16 op sequence as pf16_bn_fwd_bwd's apply
+ * (xhat = rn(rn(x - mean) * invstd); z = rn(rn(rn(gamma * xhat) + beta) *
+ * post_scale); ReLU), so the conv sees bit for bit the operand it would read
+ * from the stored BatchNorm output, and its result is bit-identical to
+ * pf16_bn_fwd_bwd phase 0 followed by the plain call.  The BatchNorm output
+ * is then never written: phase 0 runs with y = NULL (statistics only) and the
+ * convs that read the output take the input instead.
+ * mean, invstd: the BatchNorm's saved statistics (phase 0); gamma, beta: its
+ * parameters; all [c], 16-byte aligned.  flags: PF16_BN_RELU or 0. */
+typedef struct {
+  const uint16_t* mean;
+  const uint16_t* invstd;
+  const uint16_t* gamma;
+  const uint16_t* beta;
+  uint16_t post_scale;  /* binary16 bits */
+  uint32_t flags;       /* PF16_BN_RELU or 0 */
+  uint8_t* relu_mask;   /* pf16_conv_fwd_bnin only, optional (needs PF16_BN_RELU): the ReLU decisions,
+                           written in pf16_bn_fwd_bwd's bit-mask layout (any alignment) */
+} pf16_bn_operand;
+
+/* Forward conv of x' = BN(x) (x: the BatchNorm's input, n x h x w x c):
+ * y as pf16_conv_fwd of x', and, with a non-NULL stats buffer, the
+ * statistics of y as pf16_conv_fwd_bnstats.  Covers the dense 1x1 / stride 1
+ * / pad 0 layers (a bottleneck's last conv); other shapes return
+ * PF16_ERR_UNSUPPORTED.  No workspace. */
+int pf16_conv_fwd_bnin(const pf16_conv_desc* d, const uint16_t* x, const pf16_bn_operand* bn, const uint16_t* w,
+                       uint16_t* y, void* stats, size_t stats_bytes, void* stream);
+/* Weight gradient of the same layer from x' = BN(x): dw as pf16_conv_wgrad
+ * of x' (flags 0; the same workspace).  bn->relu_mask must be NULL.  Same
+ * shape coverage as pf16_conv_fwd_bnin. */
+int pf16_conv_wgrad_bnin(const pf16_conv_desc* d, const uint16_t* x, const pf16_bn_operand* bn, const uint16_t* dy,
+                         uint16_t* dw, void* ws, size_t ws_bytes, void* stream);
+
 /* Weight gradient without any caller workspace (the paper has no counterpart:
  * this is a convenience of the library).  Same arguments, result and error
  * codes as pf16_conv_wgrad, minus ws / ws_bytes.  It is meant for callers that
@@ -249,6 +286,9 @@ int pf16_allreduce_combine(const uint16_t* planes, int32_t world, size_t n, size
  * The tree shapes depend only on n*h*w and c.
  *   phase 0 (forward, training):  reads x, gamma, beta[, residual];
  *       writes y, mean, invstd (per channel, saved for the backward).
+ *       y may be NULL: then only mean and invstd are computed (relu_mask
+ *       must be NULL too), for a conv that applies this BatchNorm in its
+ *       operand path (pf16_conv_fwd_bnin).
  *       With PF16_BN_RELU and a non-NULL relu_mask it also writes the ReLU
  *       decisions: n*h*w*c/8 bytes, bit j of byte [row*(c/8) + g] set iff
  *       output channel 8g+j of that row is > 0 (so y > 0).  Any alignment.

@@ -613,13 +613,38 @@ int run_stem_s2d(const Shape& s, int ws, const uint16_t* x, const uint16_t* w, u
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
+// BatchNorm in the operand path: validate `bn` for an input of C channels
+// and point the GEMM's transform at it (xf_operand 1: A, 2: B).
+static int set_bn_operand(GemmParams& p, const pf16_bn_operand* bn, long long C, long long rows, int operand,
+                          bool allow_mask) {
+  if (!bn->mean || !bn->invstd || !bn->gamma || !bn->beta) return PF16_ERR_NULL;
+  if (!aligned16(bn->mean) || !aligned16(bn->invstd) || !aligned16(bn->gamma) || !aligned16(bn->beta))
+    return PF16_ERR_ALIGN;
+  if (bn->flags & ~(uint32_t)PF16_BN_RELU) return PF16_ERR_ARG;
+  if (bn->relu_mask && (!allow_mask || !(bn->flags & PF16_BN_RELU))) return PF16_ERR_ARG;
+  if (C % 8 != 0) return PF16_ERR_UNSUPPORTED;
+  p.xf_operand = operand;
+  p.xf_relu = (bn->flags & PF16_BN_RELU) ? 1 : 0;
+  p.xf_scale = bn->post_scale;
+  p.xf_C = (int)C;
+  p.xf_rows = rows;
+  p.xf_mean = bn->mean;
+  p.xf_invstd = bn->invstd;
+  p.xf_gamma = bn->gamma;
+  p.xf_beta = bn->beta;
+  p.xf_mask = bn->relu_mask;
+  return PF16_OK;
+}
+
 static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* w, uint16_t* y,
                          void* ws, size_t ws_bytes, uint32_t flags, void* stats, size_t stats_bytes,
-                         void* stream) {
+                         void* stream, const pf16_bn_operand* bn = nullptr) {
   Shape s;
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, w, y)) != PF16_OK) return rc;
+  const bool dense = s.kind == KIND_GENERIC && s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0;
+  if (bn && (!dense || flags != 0)) return PF16_ERR_UNSUPPORTED;
   if (flags & ~(PF16_ACCUMULATE | PF16_F32_ACCUM)) return PF16_ERR_ARG;
   const bool f32 = (flags & PF16_F32_ACCUM) != 0;
   if (stats) {
@@ -645,7 +670,8 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   p.out = y;
   p.ldo = s.K;
   p.out_mode = (flags & PF16_ACCUMULATE) ? OUT_ACCUM : OUT_STORE;
-  if (const int ws = halo_width(s, (flags & PF16_ACCUMULATE) != 0))
+  if (bn && (rc = set_bn_operand(p, bn, s.C, (long long)p.M, 1, true)) != PF16_OK) return rc;
+  if (const int ws = bn ? 0 : halo_width(s, (flags & PF16_ACCUMULATE) != 0))
     return run_halo(s, ws, false, x, w, y, status, sms, st, f32, stats);
   if (const int ws_s2d = stem_s2d_width(s, (flags & PF16_ACCUMULATE) != 0))
     return run_stem_s2d(s, ws_s2d, x, w, y, ws, status, sms, st, stats, f32);
@@ -667,7 +693,6 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
       return PF16_ERR_CUDA;
     p.num_kb = cdiv(kc, kBK);
   } else {
-    const bool dense = s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0;
     if (dense) {
       if (!map_2d(&ma, x, s.C, s.N * s.H * s.W, s.C, 64, kBM)) return PF16_ERR_CUDA;
     } else {
@@ -706,6 +731,12 @@ int pf16_conv_fwd_bnstats(const pf16_conv_desc* d, const uint16_t* x, const uint
                           void* ws, size_t ws_bytes, void* stats, size_t stats_bytes, void* stream) {
   if (!stats) return PF16_ERR_NULL;
   return conv_fwd_impl(d, x, w, y, ws, ws_bytes, 0, stats, stats_bytes, stream);
+}
+
+int pf16_conv_fwd_bnin(const pf16_conv_desc* d, const uint16_t* x, const pf16_bn_operand* bn, const uint16_t* w,
+                       uint16_t* y, void* stats, size_t stats_bytes, void* stream) {
+  if (!bn) return PF16_ERR_NULL;
+  return conv_fwd_impl(d, x, w, y, nullptr, 0, 0, stats, stats_bytes, stream, bn);
 }
 
 static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t* w, uint16_t* dx,
@@ -959,13 +990,16 @@ static int run_wgrad3x3(const Shape& s, const Wgrad3Plan& w3, const uint16_t* x,
   return PF16_OK;
 }
 
-int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
-                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+static int conv_wgrad_impl(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
+                           void* ws, size_t ws_bytes, uint32_t flags, void* stream,
+                           const pf16_bn_operand* bn = nullptr) {
   Shape s;
   int rc = conv_shape(d, &s);
   if (rc != PF16_OK) return rc;
   if ((rc = check_common(x, dy, dw)) != PF16_OK) return rc;
   if (flags & ~PF16_F32_ACCUM) return PF16_ERR_ARG;
+  const bool dense = s.kind == KIND_GENERIC && s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0;
+  if (bn && (!dense || flags != 0)) return PF16_ERR_UNSUPPORTED;
   const bool f32 = (flags & PF16_F32_ACCUM) != 0;
   int* status;
   int sms;
@@ -1008,6 +1042,7 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
   } else if (s.R == 1 && s.S == 1 && s.st == 1 && s.pad == 0) {
     p.b_mode = LD_TILED_MN;
     if (!map_2d(&mb, x, s.C, pixels, s.C, 64, 64)) return PF16_ERR_CUDA;
+    if (bn && (rc = set_bn_operand(p, bn, s.C, pixels, 2, false)) != PF16_OK) return rc;
   } else {
     p.b_mode = LD_IM2COL_MN;
     p.gb = PixGrid{(int)s.P, (int)s.Q, (int)s.st, (int)-s.pad, (int)-s.pad};
@@ -1040,6 +1075,17 @@ int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* 
       return PF16_ERR_CUDA;
   }
   return PF16_OK;
+}
+
+int pf16_conv_wgrad(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
+                    void* ws, size_t ws_bytes, uint32_t flags, void* stream) {
+  return conv_wgrad_impl(d, x, dy, dw, ws, ws_bytes, flags, stream);
+}
+
+int pf16_conv_wgrad_bnin(const pf16_conv_desc* d, const uint16_t* x, const pf16_bn_operand* bn, const uint16_t* dy,
+                         uint16_t* dw, void* ws, size_t ws_bytes, void* stream) {
+  if (!bn) return PF16_ERR_NULL;
+  return conv_wgrad_impl(d, x, dy, dw, ws, ws_bytes, 0, stream, bn);
 }
 
 int pf16_sgd_update(uint16_t* w, uint16_t* v, const uint16_t* g, size_t n, uint16_t lr,
@@ -1107,13 +1153,24 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int sms = 0;
   if (phase == 0) {
-    const void* req[] = {t->x, t->gamma, t->beta, t->y, t->mean, t->invstd};
+    // y == NULL: the statistics only (mean, invstd), for a consumer that
+    // applies the BatchNorm in its operand path
+    const void* req[] = {t->x, t->mean, t->invstd};
     for (const void* p : req) {
       if (!p) return PF16_ERR_NULL;
       if (!aligned16(p)) return PF16_ERR_ALIGN;
     }
-    if (b.residual && !t->residual) return PF16_ERR_NULL;
-    if (b.residual && !aligned16(t->residual)) return PF16_ERR_ALIGN;
+    if (t->y) {
+      const void* req2[] = {t->gamma, t->beta, t->y};
+      for (const void* p : req2) {
+        if (!p) return PF16_ERR_NULL;
+        if (!aligned16(p)) return PF16_ERR_ALIGN;
+      }
+      if (b.residual && !t->residual) return PF16_ERR_NULL;
+      if (b.residual && !aligned16(t->residual)) return PF16_ERR_ALIGN;
+    } else if (t->relu_mask) {
+      return PF16_ERR_ARG;  // the decisions come from the apply
+    }
     if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
     if (t->conv_stats) {
       if (!aligned16(t->conv_stats)) return PF16_ERR_ALIGN;

@@ -61,11 +61,6 @@ __device__ __forceinline__ uint4 ldexp_down4(uint4 v, int e) {
   return mul4(v, dup2(pe));
 }
 
-// per-lane all-ones where the binary16 lane is > 0 and not NaN: as an unsigned
-// 16-bit code h, 1 <= h <= 0x7C00, i.e. (h - 1) < 0x7C00 -- two SIMD ops
-__device__ __forceinline__ uint32_t relu_mask2(uint32_t y) {
-  return __vcmpltu2(__vsub2(y, 0x00010001u), 0x7C007C00u);
-}
 
 // Balanced pairwise tree over a stream of leaves, built as a binary counter:
 // after 2^k pushes it holds exactly the perfect tree of those leaves; finish()
@@ -1437,6 +1432,7 @@ cudaError_t launch_bn_fwd(const BnLaunch& b, const uint16_t* x, const uint16_t* 
   const BnGeom g = bn_geom(b.C);
   launch_pdl(k_bn_fwd_stats, dim3(b.fwd.blocks), dim3(g.threads + 32), stat_smem_bytes(1), s, a);
   launch_pdl(k_bn_fwd_final, dim3(b.C / 8), dim3(kFinalThreads), 0, s, a, (long long)b.chunk_rows);
+  if (!y) return counted_launches(2);  // statistics only
   const int rows = g.rpb * kApplyRows;
   launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 
       x, gamma, beta, mean, invstd, residual, y, b.relu ? relu_mask : nullptr, b.R, b.C, g.rpb,
@@ -1449,6 +1445,7 @@ cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_sta
                                       const uint16_t* residual, uint16_t* y, uint8_t* relu_mask,
                                       uint16_t* mean, uint16_t* invstd, cudaStream_t s) {
   launch_pdl(k_bn_fwd_final_slots, dim3(b.C / 8), dim3(kFinalThreads), 0, s, conv_stats, b.C, b.eps, mean, invstd);
+  if (!y) return counted_launches(1);  // statistics only
   const BnGeom g = bn_geom(b.C);
   const int rows = g.rpb * kApplyRows;
   launch_pdl(k_bn_apply, dim3((unsigned)((b.R + rows - 1) / rows)), dim3(g.threads), 0, s, 

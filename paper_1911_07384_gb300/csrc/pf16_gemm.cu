@@ -30,11 +30,15 @@ namespace pf16 {
 // (its odd tiles), so two tiles drain at once.
 constexpr int kEpiWarps = 8;
 constexpr int kGemmThreads = 32 * (2 + kEpiWarps);
+// XF (BatchNorm in the operand path): eight transform warps after the epilogue's
+constexpr int kXfWarp0 = 2 + kEpiWarps;
+constexpr int kXfWarps = 8;
+constexpr int kGemmThreadsXf = kGemmThreads + 32 * kXfWarps;
 
 // TMAE: the TMA-fed backward-statistics epilogue keeps four 32 x 64 tiles per
 // warp (two staging tiles, two BatchNorm-input tiles, filled by TMA a chunk
 // ahead), paid for with pipeline stages; plus two transaction barriers per warp.
-template <int BN, bool TMAE = false>
+template <int BN, bool TMAE = false, bool XF = false>
 struct GemmCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_BYTES = BN * kBK * 2;
@@ -44,7 +48,7 @@ struct GemmCfg {
   static constexpr int WARP_BUF = TMAE ? 4 * 4096 : 4096;  // per epilogue warp
   static constexpr int STAGING_BYTES = kEpiWarps * WARP_BUF;
   static constexpr int EBARS = TMAE ? 2 * kEpiWarps : 0;
-  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4 + EBARS) + 16;
+  static constexpr int BAR_BYTES = 8 * ((XF ? 3 : 2) * STAGES + 4 + EBARS) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
@@ -709,6 +713,87 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
       if (pend[b] >= 0) mbar_wait(B0 + 8 * b, (uint32_t)(pend[b] >> 1) & 1u, 1000000000ull);
 }
 
+// ---------------------------------------------------------------------------
+// BatchNorm in the operand path (GemmParams::xf_*).  An operand stage is
+// made of 128-byte rows -- one pixel's 64 channels, 128B-swizzled: channel
+// chunk g of row r sits in 16-byte slot g ^ (r & 7) -- and is replaced in
+// place by the BatchNorm's output, with the apply pass's op sequence.  Each
+// transform thread owns one slot column of rows congruent mod 8 (so a single
+// channel chunk and one set of per-channel parameters), loads all its rows
+// before computing and stores after, and holds the parameters in registers,
+// loaded ahead of use.
+//   A (K-major, 128 pixel rows, the 64 channels of K-block kb): thread t takes
+//     slot t & 7 of rows t / 8 + 32 i (4 rows).
+//   B (MN-major, BN / 64 atoms of 64 pixel rows, atom j = channels n0 + 64 j):
+//     tpa = 256 / 2^ceil(log2(BN / 64)) threads per atom; thread t takes atom
+//     t / tpa, slot t & 7 of rows (t % tpa) / 8 + (tpa / 8) i.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t xf_pair(uint32_t x, uint32_t mu, uint32_t is, uint32_t ga, uint32_t be,
+                                            uint32_t ps) {
+  const uint32_t xh = hmul2_rn(hsub2_rn(x, mu), is);  // Eq. 1
+  return hmul2_rn(hadd2_rn(hmul2_rn(ga, xh), be), ps);  // Eq. 2, then x post_scale (Sec. 4.2)
+}
+// bit 15 of each 16-bit lane set where the lane is > 0 and not NaN: magnitude
+// m = h & 0x7FFF non-zero (m + 0x7FFF carries into bit 15), at most 0x7C00
+// (m + 0x3FF does not), sign clear.  No carry crosses a lane.
+__device__ __forceinline__ uint32_t pos15(uint32_t h) {
+  const uint32_t m = h & 0x7FFF7FFFu;
+  return (m + 0x7FFF7FFFu) & ~((m + 0x03FF03FFu) | h) & 0x80008000u;
+}
+
+struct XfParams {
+  uint4 mu, is, ga, be;
+  __device__ __forceinline__ void load(const GemmParams& p, int c) {
+    if (c < p.xf_C) {
+      mu = __ldg(reinterpret_cast<const uint4*>(p.xf_mean + c));
+      is = __ldg(reinterpret_cast<const uint4*>(p.xf_invstd + c));
+      ga = __ldg(reinterpret_cast<const uint4*>(p.xf_gamma + c));
+      be = __ldg(reinterpret_cast<const uint4*>(p.xf_beta + c));
+    }
+  }
+};
+
+// Transform `n` rows (row i at smem address a0 + i * astep, pixel pix0 + i *
+// pstep) of one slot column holding channels c .. c + 7.
+template <int MAXR>
+__device__ __forceinline__ void xf_rows(const GemmParams& p, const XfParams& q, uint32_t a0, uint32_t astep, int n,
+                                        long long pix0, long long pstep, int c, uint8_t* mask_out) {
+  const bool cok = c < p.xf_C;
+  const uint32_t ps = (uint32_t)p.xf_scale | ((uint32_t)p.xf_scale << 16);
+  uint4 v[MAXR];
+#pragma unroll
+  for (int i = 0; i < MAXR; ++i)
+    if (i < n) ld_shared_v4(a0 + (uint32_t)i * astep, v[i]);
+  const long long cpr = p.xf_C / 8;  // mask bytes per pixel row
+#pragma unroll
+  for (int i = 0; i < MAXR; ++i) {
+    if (i >= n) break;
+    const long long pix = pix0 + (long long)i * pstep;
+    uint4 z = make_uint4(0, 0, 0, 0);
+    if (cok && pix < p.xf_rows) {
+      z.x = xf_pair(v[i].x, q.mu.x, q.is.x, q.ga.x, q.be.x, ps);
+      z.y = xf_pair(v[i].y, q.mu.y, q.is.y, q.ga.y, q.be.y, ps);
+      z.z = xf_pair(v[i].z, q.mu.z, q.is.z, q.ga.z, q.be.z, ps);
+      z.w = xf_pair(v[i].w, q.mu.w, q.is.w, q.ga.w, q.be.w, ps);
+      if (p.xf_relu) {
+        const uint32_t k0 = pos15(z.x), k1 = pos15(z.y), k2 = pos15(z.z), k3 = pos15(z.w);
+        z = make_uint4(z.x & ((k0 >> 15) * 0xFFFFu), z.y & ((k1 >> 15) * 0xFFFFu), z.z & ((k2 >> 15) * 0xFFFFu),
+                       z.w & ((k3 >> 15) * 0xFFFFu));
+        if (mask_out) {
+          // lane 2k's decision (bit 15 of word k) -> bit 2k, lane 2k+1's (bit 31) -> bit 2k+1
+          const uint32_t b = (k0 >> 15 & 1u) | (k0 >> 30 & 2u) | (k1 >> 13 & 4u) | (k1 >> 28 & 8u) |
+                             (k2 >> 11 & 16u) | (k2 >> 26 & 32u) | (k3 >> 9 & 64u) | (k3 >> 24 & 128u);
+          mask_out[pix * cpr + c / 8] = (uint8_t)b;
+        }
+      }
+    }
+    v[i] = z;
+  }
+#pragma unroll
+  for (int i = 0; i < MAXR; ++i)
+    if (i < n) st_shared_v4(a0 + (uint32_t)i * astep, v[i]);
+}
+
 // EPI: the epilogue's kind, each a separate instantiation so that the others
 // do not carry its registers or give up its pipeline stages --
 //   EPI_PLAIN: stores (forward statistics optional);
@@ -717,13 +802,16 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
 //   EPI_BS_TMA: the same statistics from TMA-fed tiles (epilogue_bs; for short
 //     reductions, whose epilogue is the bound);
 //   EPI_BS_ADD: EPI_BS_TMA plus the addend (GemmParams::add_src).
-template <int BN, int EPI>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// XF (with EPI_PLAIN): BatchNorm in the operand path (GemmParams::xf_*):
+// eight more warps transform each stage between the TMA's arrival (full) and
+// the MMAs (xready), see xf_rows.
+template <int BN, int EPI, bool XF = false>
+__global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapX,
            const __grid_constant__ CUtensorMap mapD, const __grid_constant__ GemmParams p) {
   constexpr bool BS = EPI != EPI_PLAIN, TMAE = EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, ADD = EPI == EPI_BS_ADD;
-  using Cfg = GemmCfg<BN, TMAE>;
+  using Cfg = GemmCfg<BN, TMAE, XF>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -734,7 +822,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint64_t* tfull = bars + 2 * Cfg::STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* ebar = tempty + 2;  // TMAE: per epilogue warp, one transaction barrier per input buffer
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ebar + Cfg::EBARS);
+  uint64_t* xready = ebar + Cfg::EBARS;  // XF: the stage has been transformed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xready + (XF ? Cfg::STAGES : 0));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -748,6 +837,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(smem_u32(&tempty[a]), 4);
     }
     for (int b = 0; b < Cfg::EBARS; ++b) mbar_init(smem_u32(&ebar[b]), 1);
+    if (XF)
+      for (int s = 0; s < Cfg::STAGES; ++s) mbar_init(smem_u32(&xready[s]), kXfWarps);
     *abort_flag = 0;
     fence_mbar_init();
     tma_prefetch_desc(&mapA);
@@ -835,7 +926,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(smem_u32(&full[stage]), phase, lim)) {
+          if (!mbar_wait(smem_u32(XF ? &xready[stage] : &full[stage]), phase, lim)) {
             record_timeout(p, abort_flag);
             ok = false;
             break;
@@ -857,6 +948,71 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
       }
+    }
+  } else if (XF && warp >= kXfWarp0) {
+    // transform warps: each stage, once the TMA has landed, into the BatchNorm's output
+    const int xt = threadIdx.x - 32 * kXfWarp0;  // 0 .. 255
+    const int slot = xt & 7;
+    // B: atoms of this stage, threads per atom (a power of two), this thread's atom and rows
+    constexpr int kAtoms = BN / 64;
+    constexpr int kTpa = kAtoms == 1 ? 256 : (kAtoms == 2 ? 128 : 64);
+    const int bj = xt / kTpa, btt = xt % kTpa, brow0 = btt >> 3;
+    const bool bact = bj < kAtoms;
+    const int arow0 = xt >> 3;  // A: rows arow0 + 32 i
+    const int ag = slot ^ (arow0 & 7), bg = slot ^ (brow0 & 7);
+    int stage = 0;
+    uint32_t phase = 0;
+    XfParams q;
+    bool have_next = false;  // A: q already holds the parameters of the next K-block
+    for (int u = cid; u < total; u += ncl) {
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+      int m0, n0, split, kb0, kb1;
+      unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
+      if (p.xf_operand == 2) {
+        q.load(p, n0 + 64 * bj + 8 * bg);  // constant over the unit's K-blocks
+      } else if (!have_next) {
+        q.load(p, kb0 * kBK + 8 * ag);
+      }
+      bool ok = true;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const bool got = mbar_wait(smem_u32(&full[stage]), phase, lim);
+        if (!__all_sync(0xffffffffu, got)) {
+          if (lane == 0) record_timeout(p, abort_flag);
+          ok = false;
+          break;
+        }
+        const uint32_t sa = smem_u32(smem + stage * Cfg::STAGE_BYTES);
+        if (p.xf_operand == 1) {
+          const XfParams cur = q;
+          // the next K-block's parameters, in flight while this one is transformed
+          int nkb = kb + 1;
+          if (nkb >= kb1) {
+            int u2 = u + ncl, mm, nn, ss, k0, k1;
+            nkb = -1;
+            if (u2 < total) {
+              unit_decode(p, u2, mm, nn, ss, k0, k1, BN);
+              nkb = k0;
+            }
+          }
+          have_next = nkb >= 0;
+          if (have_next) q.load(p, nkb * kBK + 8 * ag);
+          const uint32_t a0 = sa + (uint32_t)arow0 * 128u + (uint32_t)slot * 16u;
+          xf_rows<kBM / 32>(p, cur, a0, 32u * 128u, kBM / 32, (long long)m0 + arow0, 32, kb * kBK + 8 * ag,
+                            (p.xf_mask != nullptr && n0 == 0) ? p.xf_mask : nullptr);
+        } else if (bact) {
+          const uint32_t a0 = sa + Cfg::A_BYTES + (uint32_t)bj * 8192u + (uint32_t)brow0 * 128u + (uint32_t)slot * 16u;
+          xf_rows<512 / kTpa>(p, q, a0, (uint32_t)(kTpa / 8) * 128u, 512 / kTpa, (long long)kb * kBK + brow0,
+                              kTpa / 8, n0 + 64 * bj + 8 * bg, nullptr);
+        }
+        fence_proxy_async_smem();  // the transformed tile, before the tensor core reads it
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&xready[stage]));
+        if (++stage == Cfg::STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      if (!ok) break;
     }
   } else {
     // epilogue warps 2..9 -> TMEM sub-partitions 2, 3, 0, 1; group grp drains accumulator grp
@@ -1014,28 +1170,29 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN, int EPI = EPI_PLAIN>
+template <int BN, int EPI = EPI_PLAIN, bool XF = false>
 static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI, XF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
   return cudaSuccess;
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, bool XF = false>
 static cudaError_t launch_variant(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                                   const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
                                   cudaStream_t s) {
-  cudaError_t e = set_smem_attr<BN, EPI>();
+  cudaError_t e = set_smem_attr<BN, EPI, XF>();
   if (e != cudaSuccess) return e;
-  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD>::SMEM;
-  launch_pdl(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, mA, mB, mC, mX, mD, p);
+  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF>::SMEM;
+  launch_pdl(k_gemm<BN, EPI, XF>, dim3(grid), dim3(XF ? kGemmThreadsXf : kGemmThreads), smem, s, mA, mB, mC, mX,
+             mD, p);
   return counted_launches(1);
 }
 
@@ -1045,6 +1202,10 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
                                cudaStream_t s) {
   const int epi = gemm_epilogue(p);
   if (epi != EPI_PLAIN && (!p.tma_store || p.out_mode != OUT_STORE)) return cudaErrorInvalidValue;
+  if (p.xf_operand) {
+    if (epi != EPI_PLAIN) return cudaErrorInvalidValue;
+    return launch_variant<BN, EPI_PLAIN, true>(mA, mB, mC, mX, mD, p, grid, s);
+  }
   switch (epi) {
     case EPI_PLAIN: return launch_variant<BN, EPI_PLAIN>(mA, mB, mC, mX, mD, p, grid, s);
     case EPI_BS: return launch_variant<BN, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);

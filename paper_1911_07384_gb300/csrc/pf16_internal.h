@@ -140,6 +140,27 @@ struct GemmParams {
   // The statistics are taken of that sum.  Null: no addend.
   const uint16_t* add_src;
   const uint8_t* add_mask;
+  // BatchNorm applied in the operand path (xf_operand != 0; k_gemm's XF
+  // variant): the operand's tiles hold a BatchNorm's input x, and before the
+  // MMAs read a stage four transform warps replace each element of pixel row
+  // r, channel c by the BatchNorm's output -- rn(rn(rn(gamma * rn(rn(x - mean)
+  // * invstd)) + beta) * xf_scale), then ReLU when xf_relu -- the op sequence
+  // of pf16_bn_fwd_bwd's apply, so the operand is bit-identical to the
+  // BatchNorm's stored output.  Rows past xf_rows and channels past xf_C are
+  // zero.  xf_operand 1: A (K-major, 128 pixel rows, the 64 channels of
+  // K-block kb); 2: B (MN-major 64-pixel x 64-channel atoms of K-block kb,
+  // channels n0 + 64 j).  With xf_mask (A only) the CTAs of n-tile 0 also
+  // write the ReLU decisions in pf16_bn_fwd_bwd's bit-mask layout.
+  int xf_operand;
+  int xf_relu;
+  uint16_t xf_scale;
+  int xf_C;
+  long long xf_rows;
+  const uint16_t* xf_mean;
+  const uint16_t* xf_invstd;
+  const uint16_t* xf_gamma;
+  const uint16_t* xf_beta;
+  uint8_t* xf_mask;
 };
 
 // Conv-output BatchNorm statistics buffer (pf16_conv_fwd_bnstats): a header of

@@ -242,6 +242,11 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool a_mn, bool b
 // Exact binary16 arithmetic: one IEEE roundTiesToEven rounding per op, never
 // contracted into an FMA, subnormals kept (no .ftz).
 // ----------------------------------------------------------------------------
+// per-lane all-ones where the binary16 lane is > 0 and not NaN: as an unsigned
+// 16-bit code h, 1 <= h <= 0x7C00, i.e. (h - 1) < 0x7C00 -- two SIMD ops
+__device__ __forceinline__ uint32_t relu_mask2(uint32_t y) {
+  return __vcmpltu2(__vsub2(y, 0x00010001u), 0x7C007C00u);
+}
 __device__ __forceinline__ uint32_t hadd2_rn(uint32_t a, uint32_t b) {
   uint32_t d;
   asm("add.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));

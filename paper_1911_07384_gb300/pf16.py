@@ -38,6 +38,7 @@ EXPORTS = [
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
     "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
     "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add", "pf16_tc_rate", "pf16_wait_flag",
+    "pf16_conv_fwd_bnin", "pf16_conv_wgrad_bnin",
 ]
 
 
@@ -58,6 +59,13 @@ class ConvDesc(ctypes.Structure):
 class BnSource(ctypes.Structure):
     """pf16_bn_source: the BatchNorm whose output gradient a data gradient is."""
     _fields_ = [(n, ctypes.c_void_p) for n in ("x", "relu_mask", "mean", "invstd")]
+
+
+class BnOperand(ctypes.Structure):
+    """pf16_bn_operand: a BatchNorm applied in a conv's operand path."""
+    _fields_ = [("mean", ctypes.c_void_p), ("invstd", ctypes.c_void_p), ("gamma", ctypes.c_void_p),
+                ("beta", ctypes.c_void_p), ("post_scale", ctypes.c_uint16), ("flags", ctypes.c_uint32),
+                ("relu_mask", ctypes.c_void_p)]
 
 
 class BnDesc(ctypes.Structure):
@@ -96,6 +104,11 @@ def lib():
             L.pf16_conv_bnstats_size.argtypes = [cdp]
             L.pf16_conv_bnstats_size.restype = sz
             L.pf16_conv_fwd_bnstats.argtypes = [cdp, vp, vp, vp, vp, sz, vp, sz, vp]
+            bop = ctypes.POINTER(BnOperand)
+            L.pf16_conv_fwd_bnin.argtypes = [cdp, vp, bop, vp, vp, vp, sz, vp]
+            L.pf16_conv_fwd_bnin.restype = I
+            L.pf16_conv_wgrad_bnin.argtypes = [cdp, vp, bop, vp, vp, vp, sz, vp]
+            L.pf16_conv_wgrad_bnin.restype = I
             L.pf16_conv_fwd_bnstats.restype = I
             L.pf16_conv_dgrad_bnstats_size.argtypes = [cdp]
             L.pf16_conv_dgrad_bnstats_size.restype = sz
@@ -196,6 +209,25 @@ def conv_fwd_bnstats(d, x, w, y, stats, ws=None, stream=None):
     (a device buffer of conv_bnstats_size(d) bytes) for bn_fwd_bwd(conv_stats=)."""
     _check(lib().pf16_conv_fwd_bnstats(ctypes.byref(d), _ptr(x), _ptr(w), _ptr(y), _ptr(ws), _nbytes(ws),
                                        _ptr(stats), _nbytes(stats), _stream(stream)), "pf16_conv_fwd_bnstats")
+
+
+def bn_operand(mean, invstd, gamma, beta, post_scale_bits, relu, relu_mask=None) -> BnOperand:
+    return BnOperand(_ptr(mean), _ptr(invstd), _ptr(gamma), _ptr(beta), post_scale_bits,
+                     PF16_BN_RELU if relu else 0, _ptr(relu_mask))
+
+
+def conv_fwd_bnin(d, x, bn: BnOperand, w, y, stats=None, stream=None):
+    """Forward conv of BN(x): x is the BatchNorm's input; the BatchNorm is
+    applied to each operand tile (and its ReLU decisions written to
+    bn.relu_mask when given); optional statistics of y as conv_fwd_bnstats."""
+    _check(lib().pf16_conv_fwd_bnin(ctypes.byref(d), _ptr(x), ctypes.byref(bn), _ptr(w), _ptr(y), _ptr(stats),
+                                    _nbytes(stats), _stream(stream)), "pf16_conv_fwd_bnin")
+
+
+def conv_wgrad_bnin(d, x, bn: BnOperand, dy, dw, ws=None, stream=None):
+    """Weight gradient with input BN(x), applied in the operand path."""
+    _check(lib().pf16_conv_wgrad_bnin(ctypes.byref(d), _ptr(x), ctypes.byref(bn), _ptr(dy), _ptr(dw), _ptr(ws),
+                                      _nbytes(ws), _stream(stream)), "pf16_conv_wgrad_bnin")
 
 
 def conv_dgrad(d, dy, w, dx, ws=None, flags=0, stream=None):

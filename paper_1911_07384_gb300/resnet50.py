@@ -107,8 +107,13 @@ class Conv:
         size = pf16.conv_dgrad_bnstats_size(self.desc) if self.desc.c != 3 else 0
         self.dstats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
 
-    def fwd(self, x, y, with_stats=False):
-        if with_stats:
+    def fwd(self, x, y, with_stats=False, bn_in=None):
+        """bn_in: the BN layer whose input x is; this conv applies it in its
+        operand path (pf16_conv_fwd_bnin) and writes its ReLU mask."""
+        if bn_in is not None:
+            self.net.call("conv_fwd", self, pf16.conv_fwd_bnin, self.desc, x, bn_in.operand(with_mask=True), self.w,
+                          y, self.stats if with_stats else None)
+        elif with_stats:
             self.net.call("conv_fwd", self, pf16.conv_fwd_bnstats, self.desc, x, self.w, y, self.stats,
                           self.net.ws)
         else:
@@ -134,16 +139,24 @@ class Conv:
     def fuses_bwd_stats(self):
         return self.dstats is not None
 
-    def wgrad(self, x, dy):
+    def wgrad(self, x, dy, bn_in=None):
+        """bn_in: as in fwd -- x is that BatchNorm's input."""
         net = self.net
+
+        def call(ws):
+            if bn_in is not None:
+                net.call("conv_wgrad", self, pf16.conv_wgrad_bnin, self.desc, x, bn_in.operand(), dy, self.gw, ws)
+            else:
+                net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, ws)
+
         if net.side is None:
-            net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, net.ws)
+            call(net.ws)
             return
         # only the update reads the weight gradient: it runs on a branch of its own
         # (with its own workspace), off the chain of data gradients and BatchNorms
         net.side.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(net.side):
-            net.call("conv_wgrad", self, pf16.conv_wgrad, self.desc, x, dy, self.gw, net.ws_w)
+            call(net.ws_w)
 
 
 class BN:
@@ -155,6 +168,9 @@ class BN:
         self.desc = pf16.bn_desc(n, h, w, c, EPS, post_scale, flags)
         self.c = c
         self.zero_gamma = zero_gamma
+        self.post_scale = post_scale
+        self.relu = relu
+        self.fused_apply = False  # applied in the next conv's operand path (the output is never stored)
         self.g_off = net.nowd.add(c)
         self.b_off = net.nowd.add(c)
         self.elems = n * h * w * c
@@ -172,10 +188,18 @@ class BN:
         self.mask = torch.empty(self.elems // 8, dtype=torch.uint8, device=device) if relu else None
 
     def fwd(self, x, y, residual=None, conv=None):
-        """conv: the layer whose fwd(with_stats=True) produced x (its statistics are used)."""
+        """conv: the layer whose fwd(with_stats=True) produced x (its statistics are used).
+        y None: statistics only (mean, invstd), for a conv that applies this
+        BatchNorm in its operand path and writes the ReLU mask."""
         self.net.call("bn_fwd", self, pf16.bn_fwd_bwd, self.desc, 0, self.net.ws, x=x, gamma=self.gamma,
                       beta=self.beta, residual=residual, y=y, mean=self.mean, invstd=self.invstd,
-                      relu_mask=self.mask, conv_stats=conv.stats if conv is not None else None)
+                      relu_mask=self.mask if y is not None else None,
+                      conv_stats=conv.stats if conv is not None else None)
+
+    def operand(self, with_mask=False):
+        """This BatchNorm as a conv's operand transform (pf16_bn_operand)."""
+        return pf16.bn_operand(self.mean, self.invstd, self.gamma, self.beta, self.post_scale, self.relu,
+                               self.mask if with_mask else None)
 
     def bwd(self, x, y_saved, dy, dx, dresidual=None, conv=None, residual=None):
         """conv: the layer whose dgrad(bn=(self, x)) produced dy (its statistics are used);
@@ -191,6 +215,7 @@ class BN:
 class Bottleneck:
     def __init__(self, net, n, h, cin, width, stride, proj, swap=False):
         self.cin, self.width, self.stride = cin, width, stride
+        self.net = net
         cout = 4 * width
         self.conv1 = Conv(net, n, h, h, cin, width, 1, 1, 1, 0)
         self.bn1 = BN(net, n, h, h, width, S_BLOCK, relu=True)
@@ -208,12 +233,17 @@ class Bottleneck:
         # the layer whose data gradient carries bn3's backward statistics (the
         # next block's conv1, set by that block's backward), or None
         self.bn3_stats_conv = None
+        # bn2 applied in conv3's operand path (forward and weight gradient): its
+        # output b2 is never stored
+        self.fuse_bn2 = net.bn_in_operand
+        self.bn2.fused_apply = self.fuse_bn2
 
     def allocate(self, dev):
         n, h, h2, w, c = self.n, self.h, self.h2, self.width, self.cout
         e = lambda *s: torch.empty(int(np.prod(s)), dtype=torch.int16, device=dev)
         self.a1, self.b1 = e(n, h, h, w), e(n, h, h, w)
-        self.a2, self.b2 = e(n, h2, h2, w), e(n, h2, h2, w)
+        self.a2 = e(n, h2, h2, w)
+        self.b2 = None if self.fuse_bn2 else e(n, h2, h2, w)
         self.a3, self.y = e(n, h2, h2, c), e(n, h2, h2, c)
         self.dy = e(n, h2, h2, c)  # gradient w.r.t. y (written by the next block)
         self.da3 = e(n, h2, h2, c)
@@ -228,8 +258,12 @@ class Bottleneck:
         self.conv1.fwd(x, self.a1, with_stats=True)
         self.bn1.fwd(self.a1, self.b1, conv=self.conv1)
         self.conv2.fwd(self.b1, self.a2, with_stats=True)
-        self.bn2.fwd(self.a2, self.b2, conv=self.conv2)
-        self.conv3.fwd(self.b2, self.a3, with_stats=True)
+        if self.fuse_bn2:  # bn2's statistics only; conv3 applies it to its operand
+            self.bn2.fwd(self.a2, None, conv=self.conv2)
+            self.conv3.fwd(self.a2, self.a3, with_stats=True, bn_in=self.bn2)
+        else:
+            self.bn2.fwd(self.a2, self.b2, conv=self.conv2)
+            self.conv3.fwd(self.b2, self.a3, with_stats=True)
         if self.proj:
             self.convp.fwd(x, self.ap, with_stats=True)
             self.bnp.fwd(self.ap, self.bp, conv=self.convp)
@@ -257,7 +291,10 @@ class Bottleneck:
         else:  # identity shortcut: its gradient (dy where the ReLU passed) is the start of dx
             self.bn3.bwd(self.a3, self.y, self.dy, self.da3, dresidual=None if fuse else dx, residual=self.x,
                          conv=bn3_conv)
-        self.conv3.wgrad(self.b2, self.da3)
+        if self.fuse_bn2:
+            self.conv3.wgrad(self.a2, self.da3, bn_in=self.bn2)
+        else:
+            self.conv3.wgrad(self.b2, self.da3)
         # the data gradients also reduce the next BatchNorm's backward statistics
         self.conv3.dgrad(self.da3, self.db2, bn=(self.bn2, self.a2))
         self.bn2.bwd(self.a2, self.b2, self.db2, self.da2, conv=self.conv3)
@@ -307,7 +344,7 @@ class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
     def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False,
-                 wgrad_branch=False, exchange=None):
+                 wgrad_branch=False, exchange=None, bn_in_operand=False):
         """wgrad_branch: issue the weight gradients on a second stream that joins
         before the update (in a captured step graph: a parallel branch), so that
         they fill the gaps of the data-gradient chain; off, every call runs on the
@@ -315,10 +352,17 @@ class ResNet50:
         exchange: data-parallel training (Sec. 5.1): a callable applied, before
         the update, to each flat gradient arena (decayed, then not decayed) to
         average it over the ranks in place, e.g. functools.partial(
-        dp.allreduce_mean_, group=g); None on one GPU."""
+        dp.allreduce_mean_, group=g); None on one GPU.
+        bn_in_operand: each block's second BatchNorm is applied in its last
+        conv's operand path (bit-identical results, its output never stored);
+        off by default: on GB300 the conv's transform costs more than the
+        apply pass it replaces (the 1x1 convs re-transform each operand tile
+        once per tile of the other GEMM dimension, and their epilogues already
+        fill the SM's issue slots)."""
         self.N, self.image, self.classes, self.device = batch, image, classes, device
         self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
         self.exchange = exchange
+        self.bn_in_operand = bn_in_operand
         self.side = torch.cuda.Stream(device=device) if wgrad_branch else None
         self.wd, self.nowd = Arena("decayed"), Arena("no-decay")
         self.convs, self.bns = [], []

@@ -126,3 +126,24 @@ def test_weight_gradient_branch_is_bit_identical():
         results.append([t.clone() for t in (net.wd.w, net.wd.v, net.nowd.w, net.nowd.v, net.loss)])
     for a, b in zip(*results):
         assert torch.equal(a, b)
+
+
+def test_bn_in_operand_path_step_is_bit_identical():
+    """Each block's second BatchNorm applied in its last conv's operand path
+    against the same BatchNorm stored and read back (the default): two steps
+    at batch 4 on 64 x 64 and one at batch 8 on 96 x 96 (a ragged last tile in
+    stage 4), every weight, momentum and loss compared exactly."""
+    for batch, image, steps in ((4, 64, 2), (8, 96, 1)):
+        results = []
+        for fused in (False, True):
+            net = ResNet50(batch=batch, image=image, seed_cfg=4, bn_in_operand=fused)
+            net.set_batch(syn.images_f16(syn.seed_for(4, "x"), batch, image, image, 3),
+                          syn.labels(syn.seed_for(4, "labels"), batch))
+            for _ in range(steps):
+                net.step()
+            torch.cuda.synchronize()
+            assert pf16.sync_status() == 0
+            assert all(b.fuse_bn2 == fused and (b.b2 is None) == fused for b in net.blocks)
+            results.append([t.clone() for t in (net.wd.w, net.wd.v, net.nowd.w, net.nowd.v, net.loss)])
+        for a, b in zip(*results):
+            assert torch.equal(a, b)

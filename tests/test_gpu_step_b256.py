@@ -20,7 +20,9 @@ are compared element by element under that layer's bound --
   tests/test_gpu_glue.py.
 
 The weights are the initial ones: no update runs, so the arenas still hold
-the weights every call used."""
+the weights every call used.  Where the step applies a BatchNorm inside the
+next conv's operand path (each block's second), the conv is checked against
+the oracle on that BatchNorm's output, stored afterwards by the apply pass."""
 import zlib
 
 import numpy as np
@@ -55,6 +57,18 @@ def step():
     net.forward()
     net.backward()
     torch.cuda.synchronize()
+    assert pf16.sync_status() == 0
+    # A block's second BatchNorm is applied in its last conv's operand path and
+    # never stored; store it now (the apply pass, bit-identical to the operand
+    # transform: tests/test_gpu_bnin.py) so that the checks below can read it.
+    # Its ReLU mask, written by the conv, must come out the same.
+    for b in net.blocks:
+        if b.fuse_bn2:
+            mask = b.bn2.mask.clone()
+            b.b2 = torch.empty_like(b.a2)
+            b.bn2.fwd(b.a2, b.b2, conv=b.conv2)
+            torch.cuda.synchronize()
+            assert torch.equal(mask, b.bn2.mask)
     assert pf16.sync_status() == 0
     yield net
     del net
