@@ -45,6 +45,17 @@ def peaks():
     return p
 
 
+def preload(stream, ms):
+    """Keep `stream` busy for about `ms` milliseconds (a one-thread spin
+    kernel), so that the host enqueues the calls timed after it before the GPU
+    reaches their first event: the events then bracket device time only, not
+    the host's argument marshalling and tensor-map encoding of an idle stream."""
+    import torch
+
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(ms * 2.2e6))  # SM clock cycles (at most ~2.1 GHz)
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle samples every 200 ms while running."""
 
@@ -81,7 +92,7 @@ class ClockSampler:
                 self.proc.kill()
 
     def summary(self):
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for ln in self.lines:
             f = [x.strip() for x in ln.split(",")]
@@ -92,13 +103,17 @@ class ClockSampler:
                 mx.append(float(f[2]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(f[3]))
+            except ValueError:
+                pass
             for nm, v in zip(names, f[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(nm)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
         return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), **({"power_w": float(np.median(pw)), "power_w_max": float(max(pw))} if pw else {})}
 
 
 def dist_env():
@@ -414,7 +429,8 @@ def run_tc_rate():
 
 def run_layers(args):
     """Every library call of one training step timed with CUDA events on the
-    launching stream (eager, median of 3 steps), aggregated per (call, shape).
+    launching stream (eager, median of 3 steps; the stream is pre-loaded so that
+    each pair of events brackets device time only), aggregated per (call, shape).
     Convs report TFLOP/s; BatchNorm reports GB/s of its minimum bytes (forward
     x, y, residual, ReLU mask; backward x, dy, dx, residual gradient, mask)."""
     import collections
@@ -445,10 +461,15 @@ def run_layers(args):
     for _ in range(3):
         recs.clear()
         net.hook = hook
+        preload(stream, 300)
+        h0 = time.perf_counter()
         with torch.cuda.stream(stream):
             net.step()
+        host_ms = 1e3 * (time.perf_counter() - h0)
         net.hook = None
         torch.cuda.synchronize()
+        if host_ms > 250:
+            raise RuntimeError(f"the step's host enqueue ({host_ms:.0f} ms) outlasted the stream pre-load")
         runs.append([(k, l, e0.elapsed_time(e1)) for k, l, e0, e1 in recs])
     if pf16.sync_status(stream) != 0:
         raise RuntimeError("device status error")
@@ -564,6 +585,7 @@ def time_conv(shape, conv_pass, steps, warmup):
     for _ in range(steps):
         if flush is not None:
             flush.fill_(1)
+        preload(s, 2)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(s)
         fn()
@@ -622,6 +644,7 @@ def time_bn(shape, bn_pass, steps, warmup):
     times = []
     s = torch.cuda.current_stream()
     for _ in range(steps):
+        preload(s, 2)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(s)
         fn()
@@ -760,7 +783,8 @@ def count_launches(net):
 
 def conv_roofline(net, stream, reps=3):
     """Eager steps with CUDA events around every conv call on the launching
-    stream: algorithmic conv FLOPs / summed conv-call time."""
+    stream (the stream pre-loaded, so that the events time the device only):
+    algorithmic conv FLOPs / summed conv-call time."""
     import torch
 
     recs = []
@@ -781,10 +805,15 @@ def conv_roofline(net, stream, reps=3):
     for _ in range(reps):
         recs.clear()
         net.hook = hook
+        preload(stream, 300)
+        h0 = time.perf_counter()
         with torch.cuda.stream(stream):
             net.step()
+        host_ms = 1e3 * (time.perf_counter() - h0)
         net.hook = None
         torch.cuda.synchronize()
+        if host_ms > 250:
+            raise RuntimeError(f"the step's host enqueue ({host_ms:.0f} ms) outlasted the stream pre-load")
         ms = 0.0
         for kind, layer, e0, e1 in recs:
             t = e0.elapsed_time(e1)

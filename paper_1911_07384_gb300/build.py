@@ -17,8 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libpf16.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
-SOURCES = ["pf16_api.cu", "pf16_gemm.cu", "pf16_elementwise.cu", "pf16_noalloc.cu", "pf16_probe.cu"]
-HEADERS = ["pf16_internal.h", "pf16_ptx.cuh"]
+SOURCES = ["pf16_api.cu", "pf16_gemm.cu", "pf16_halo.cu", "pf16_elementwise.cu", "pf16_noalloc.cu", "pf16_probe.cu"]
+HEADERS = ["pf16_internal.h", "pf16_ptx.cuh", "pf16_epi.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v",
          "--expt-relaxed-constexpr", "-I", INCLUDE]

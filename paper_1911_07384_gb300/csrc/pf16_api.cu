@@ -562,6 +562,99 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
   return launch_gemm_halo(ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
 }
 
+// Layout of the wide halo engine (pf16_halo.cu) for a 3x3 / stride 1 / pad 1
+// layer with cin input and cout output channels (cout 128 or 256, cin a
+// multiple of 64), or ipr = 0 where it does not apply: one image per padded
+// row of ws = 32 or 64 columns (at least W + 2; the tile's 128 / ws rows must
+// divide H), or four images of wi = 16 columns side by side (W <= 14, two rows
+// per tile dividing H, N a multiple of 4), whichever wastes fewer padding
+// columns, and only when at least three quarters of the columns are pixels.
+struct WidePlan {
+  int ipr, wi, ws;
+};
+WidePlan halo_wide_plan(const Shape& s, long long cin, long long cout, bool accum) {
+  WidePlan best{0, 0, 0};
+  if (accum || s.kind != KIND_GENERIC || s.R != 3 || s.S != 3 || s.st != 1 || s.pad != 1) return best;
+  if (cin % 64 != 0 || (cout != 128 && cout != 256)) return best;
+  double eff = 0.0;
+  for (int ws : {32, 64})
+    if (s.W + 2 <= ws && s.H % (kBM / ws) == 0 && (double)s.W / ws > eff) {
+      eff = (double)s.W / ws;
+      best = WidePlan{1, ws, ws};
+    }
+  if (s.W + 2 <= 16 && s.H % 2 == 0 && s.N % 4 == 0 && (double)s.W / 16 > eff) {
+    eff = (double)s.W / 16;
+    best = WidePlan{4, 16, 64};
+  }
+  if (eff < 0.75) best = WidePlan{0, 0, 0};
+  return best;
+}
+
+// 3x3 stride-1 forward through the wide halo engine: in = x [N,H,W,C],
+// weights [K][9*C], out = y [N,H,W,K].  (The data gradients keep the im2col
+// GEMM: with their fused backward statistics, which every 3x3 data gradient of
+// the training step takes, the wide engine measured no faster -- 28x28, 128
+// channels: 103 against 95 us at batch 256 -- its MMAs then sharing the SM
+// with the epilogue's loads and trees; and the plain call must give the same
+// bits as the one with statistics.)
+int run_halo_wide(const Shape& s, const WidePlan& wp, const uint16_t* in, const uint16_t* w, uint16_t* out,
+                  int* status, int sms, cudaStream_t st, bool f32, void* stats = nullptr) {
+  const long long cin = s.C, cout = s.K;
+  const long long N = s.N, H = s.H, W = s.W;
+  const int rpt = kBM / wp.ws;
+  GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
+  set_stats(p, stats, cout);
+  CUtensorMap ma, mb, mc;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  {
+    const cuuint64_t pix = (cuuint64_t)cin * 2, row = (cuuint64_t)W * pix, img = (cuuint64_t)H * row;
+    const bool one = wp.ipr == 1;
+    cuuint64_t dims[4] = {(cuuint64_t)cin, (cuuint64_t)W, (cuuint64_t)(one ? H : N), (cuuint64_t)(one ? N : H)};
+    cuuint64_t strides[3] = {pix, one ? row : img, one ? img : row};
+    cuuint32_t box[4] = {64, (cuuint32_t)wp.wi, (cuuint32_t)(one ? rpt + 2 : wp.ipr), (cuuint32_t)(one ? 1 : rpt + 2)};
+    if (g_encode_tiled(&ma, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<uint16_t*>(in), dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  {
+    const cuuint64_t pix = (cuuint64_t)cout * 2, row = (cuuint64_t)W * pix, img = (cuuint64_t)H * row;
+    const bool one = wp.ipr == 1;
+    cuuint64_t dims[4] = {(cuuint64_t)cout, (cuuint64_t)W, (cuuint64_t)(one ? H : N), (cuuint64_t)(one ? N : H)};
+    cuuint64_t strides[3] = {pix, one ? row : img, one ? img : row};
+    cuuint32_t box[4] = {64, (cuuint32_t)(one ? 32 : 16), (cuuint32_t)(one ? 1 : 2), 1};
+    if (g_encode_tiled(&mc, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, out, dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  p.ntaps = 9;
+  for (int t = 0; t < 9; ++t) {
+    p.tap_dr[t] = (int8_t)(t / 3);
+    p.tap_ds[t] = (int8_t)(t % 3);
+    p.tap_w[t] = (int8_t)t;
+  }
+  p.b_mode = LD_TILED_K;
+  set_kmajor(p, false, true);
+  if (!map_2d(&mb, w, 9 * cin, cout, 9 * cin, 64, (uint32_t)cout)) return PF16_ERR_CUDA;
+  p.idesc = idesc_f16(kBM, (int)cout, false, false, f32);
+  p.halo_ws = wp.ws;
+  p.halo_ipr = wp.ipr;
+  p.halo_wi = wp.wi;
+  p.halo_h = (int)H;
+  p.halo_w = (int)W;
+  p.halo_box_rows = rpt + 2;
+  p.halo_chunks = (int)(cin / 64);
+  p.N = (int)cout;
+  p.ldo = cout;
+  p.n_tiles = 1;
+  p.m_tiles = (int)((N / wp.ipr) * (H / rpt));
+  int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  if (stats && grid > kBnStatSlots) grid = kBnStatSlots;
+  return launch_gemm_halo_wide((int)cout, ma, mb, mc, p, grid, st) == cudaSuccess ? PF16_OK : PF16_ERR_CUDA;
+}
+
 // The stem through the halo engine: space-to-depth of x and the filter into
 // the workspace, then a 4x4 stride-1 convolution over 16 channels with 32-byte
 // pixel rows (layouts at stem_s2d_width).  y is N x P x Q x 64.
@@ -673,6 +766,10 @@ static int conv_fwd_impl(const pf16_conv_desc* d, const uint16_t* x, const uint1
   if (bn && (rc = set_bn_operand(p, bn, s.C, (long long)p.M, 1, true)) != PF16_OK) return rc;
   if (const int ws = bn ? 0 : halo_width(s, (flags & PF16_ACCUMULATE) != 0))
     return run_halo(s, ws, false, x, w, y, status, sms, st, f32, stats);
+  if (!bn) {
+    const WidePlan wp = halo_wide_plan(s, s.C, s.K, (flags & PF16_ACCUMULATE) != 0);
+    if (wp.ipr) return run_halo_wide(s, wp, x, w, y, status, sms, st, f32, stats);
+  }
   if (const int ws_s2d = stem_s2d_width(s, (flags & PF16_ACCUMULATE) != 0))
     return run_stem_s2d(s, ws_s2d, x, w, y, ws, status, sms, st, stats, f32);
   set_stats(p, stats, s.K);

@@ -114,6 +114,10 @@ struct GemmParams {
   // channels, sixteen taps), rows of the A box, its start row / column
   // relative to the tile's first output row / column 0
   int halo_ws, halo_h, halo_w, halo_cb, halo_box_rows, halo_row0, halo_col0;
+  // wide halo engine (launch_gemm_halo_wide): images side by side in one
+  // padded row (1, or 4 for narrow images), padded columns per image, and
+  // 64-channel chunks of the input
+  int halo_ipr, halo_wi, halo_chunks;
   // BatchNorm forward statistics of the output (OUT_STORE through TMA only;
   // null when off): per epilogue warp a running (mean, variance, count) per
   // output channel over all its rows; the CTA's warps are merged at the end
@@ -227,6 +231,18 @@ cudaError_t launch_stem_wgrad(const CUtensorMap& mapDy, const CUtensorMap& mapXs
                               cudaStream_t s);
 cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
                              const GemmParams& p, int grid, cudaStream_t stream);
+// Wide halo engine (pf16_halo.cu): 3x3 / stride 1 / pad 1 forward convolutions with
+// BN = 128 or 256 output channels (one N tile) over p.halo_chunks 64-channel
+// input chunks.  mapA: 4-D tiled map over the input, dims (c, w, h, n) with
+// boxes (64, halo_ws, halo_box_rows, 1) when halo_ipr = 1, or (c, w, n, h)
+// with boxes (64, 16, 4, halo_box_rows) when four images of halo_wi = 16
+// columns share a padded row; mapB: weights [BN][9 * Cin] (LD_TILED_K, boxes
+// 64 x BN); mapC:
+// 4-D map over the output, (c, w, h, n) with boxes (64, 32, 1, 1) or
+// (c, w, n, h) with boxes (64, 16, 2, 1).  p.m_tiles tiles of 128 padded-grid
+// rows; forward statistics (optional) as k_gemm's plain epilogue.
+cudaError_t launch_gemm_halo_wide(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
+                                  const GemmParams& p, int grid, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------
 // Memory-bound kernels (pf16_elementwise.cu).  All return cudaError_t of the

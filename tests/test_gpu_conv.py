@@ -32,6 +32,10 @@ SHAPES = [
     (2, 20, 20, 3, 128, 7, 7, 2, 3),     # stem with 128 outputs: patch GEMM
     (2, 16, 16, 3, 64, 3, 3, 1, 1),      # c = 3, 3x3: patch GEMM
     (16, 1, 1, 2048, 1000, 1, 1, 1, 0),  # fully connected layer
+    (2, 28, 28, 128, 128, 3, 3, 1, 1),   # wide halo forward, one image per padded row of 32
+    (4, 14, 14, 256, 256, 3, 3, 1, 1),   # wide halo forward, four images per padded row of 64
+    (4, 12, 12, 128, 256, 3, 3, 1, 1),   # wide halo forward, four images, W = 12, C != K
+    (2, 12, 24, 192, 128, 3, 3, 1, 1),   # wide halo forward, W = 24 of 32, three input chunks
 ]
 
 
@@ -160,6 +164,29 @@ def test_delta_kernel_bit_exact(orc, r0, s0, st):
     assert np.array_equal(f64(dx), V)
 
 
+@pytest.mark.parametrize("shape", [(4, 12, 12, 128, 128, 3, 3, 1, 1),   # wide halo, four images per padded row
+                                   (2, 8, 28, 256, 256, 3, 3, 1, 1)],   # wide halo, one image per padded row
+                         ids=ids)
+@pytest.mark.parametrize("tap", [0, 4, 8])
+def test_delta_kernel_wide_halo_bit_exact(orc, shape, tap):
+    """The delta kernel through the wide halo engine: each tap window of the
+    input box is an exact shift (and so is the data gradient)."""
+    N, H, W, C, K, R, S, st, pd = shape
+    x, _, _, P, Q = inputs(shape, seed_cfg=2)
+    w = np.zeros((K, 3, 3, C), np.float16)
+    for k in range(K):
+        w[k, tap // 3, tap % 3, k % C] = 1.0
+    w = w.view(np.uint16)
+    d = pf16.conv_desc(*shape)
+    y = run_fwd(d, x, w)
+    V, _, _ = orc.conv_fwd(x, w, *shape)
+    assert np.array_equal(f64(y), V)
+    dy = syn.normal_f16(9, (N, P, Q, K))
+    dx = run_dgrad(d, dy, w)
+    V, _, _ = orc.conv_dgrad(dy, w, *shape)
+    assert np.array_equal(f64(dx), V)
+
+
 @pytest.mark.parametrize("shape", [(2, 8, 8, 64, 128, 3, 3, 1, 1),    # im2col GEMM
                                    (2, 9, 12, 64, 64, 3, 3, 1, 1)],  # halo weight gradient, odd P
                          ids=ids)
@@ -208,6 +235,7 @@ def test_full_size_sampled(orc, shape):
 
 F32_SHAPES = [
     (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col, reduction 2,304, 256-wide N tiles
+    (4, 14, 14, 256, 256, 3, 3, 1, 1),   # wide halo engine, four images per padded row
     (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine
     (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem: space-to-depth halo forward, stem weight gradient
     (2, 14, 14, 64, 256, 1, 1, 1, 0),    # dense 1x1

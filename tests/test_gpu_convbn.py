@@ -29,6 +29,8 @@ SHAPES = [
     (2, 13, 13, 128, 256, 3, 3, 2, 1),   # strided 3x3, 4 n-chunks in a tile
     (2, 7, 7, 256, 512, 1, 1, 1, 0),     # two n-tiles (BN = 256)
     (3, 7, 7, 512, 1024, 1, 1, 1, 0),    # four n-tiles
+    (2, 28, 28, 128, 128, 3, 3, 1, 1),   # wide halo engine, one image per padded row of 32
+    (4, 14, 14, 256, 256, 3, 3, 1, 1),   # wide halo engine, four images per padded row (non-prefix rows)
     (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem, space-to-depth halo (rows of 32)
     (1, 30, 30, 3, 64, 7, 7, 2, 3),      # stem, s2d halo (rows of 128, columns 15..127 dropped)
     (2, 20, 20, 3, 128, 7, 7, 2, 3),     # stem with 128 outputs (patch matrix)
@@ -91,6 +93,7 @@ BWD_SHAPES = [
     ((2, 28, 28, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 32
     ((2, 56, 56, 64, 64, 3, 3, 1, 1), True),     # halo engine, padded rows of 64 (columns 56..63 dropped)
     ((2, 14, 14, 128, 128, 3, 3, 1, 1), True),   # stride-1 im2col data gradient, 128-wide n-tile
+    ((2, 28, 28, 128, 128, 3, 3, 1, 1), True),   # the shape whose forward takes the wide halo engine
     ((1, 7, 7, 64, 64, 3, 3, 1, 1), True),       # one partial tile (49 rows)
     ((2, 7, 7, 256, 1024, 1, 1, 1, 0), True),    # long reduction (16 K-blocks): register-fed epilogue
     ((4, 14, 14, 256, 128, 1, 1, 1, 0), True),   # short reduction, many tiles per CTA: TMA-fed epilogue
