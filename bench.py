@@ -198,6 +198,9 @@ def main():
     ap.add_argument("--conv", default=None,
                     help="time one conv pass instead of the step: N,H,W,C,K,R,S,stride,pad")
     ap.add_argument("--pass", dest="conv_pass", default="fwd", choices=["fwd", "dgrad", "wgrad"])
+    ap.add_argument("--stats", action="store_true",
+                    help="with --conv --pass fwd: the forward that also reduces the BatchNorm statistics of its "
+                         "output (pf16_conv_fwd_bnstats, as the training step calls it)")
     ap.add_argument("--bn", default=None,
                     help="time one BatchNorm pass instead of the step: N,H,W,C (ReLU + residual, s=0.25)")
     ap.add_argument("--bn-pass", default="fwd", choices=["fwd", "bwd"])
@@ -225,8 +228,8 @@ def main():
     if args.impl == "reference":
         return run_reference(args, rank, world)
     if args.conv:
-        print(json.dumps(time_conv(tuple(int(v) for v in args.conv.split(",")), args.conv_pass,
-                                   args.steps, args.warmup)), flush=True)
+        print(json.dumps(time_conv(tuple(int(v) for v in args.conv.split(",")), args.conv_pass, stats=args.stats,
+                                   steps=args.steps, warmup=args.warmup)), flush=True)
         return 0
     if args.sweep:
         return run_sweep(args)
@@ -365,15 +368,16 @@ def main():
     pk = peaks()
     peak = pk["bf16_tflops_sustained"]  # FP16 and BF16 share the dense tensor rate
     kr = kernel_roofline(pk)
+    mma = pf16.tc_rate(256, reps=20000)  # the FP16 kind::f16 MMA rate of this GPU (the library's probe)
     # the aggregate over every conv call of the step; its per-launch DRAM traffic
     # is not measured (a whole-step capture is not made); the single dominant
     # launch class with its captured traffic is roofline_kernel
     roof = {"bound": "tensor", "achieved": conv["tflops"], "peak": peak, "unit": "TFLOP/s",
             "frac": conv["tflops"] / peak, "traffic": None,
             "algorithmic_bytes_per_launch": conv["bytes_per_launch"],
-            "frac_of_f16_mma_probe": conv["tflops"] / kr["peak_f16_mma_probe"],
+            "peak_f16_mma_probe": mma, "frac_of_f16_mma_probe": conv["tflops"] / mma,
             "kernel": "k_gemm (all conv passes of the step, split-K reduce included)",
-            "peak_src": f"{pk['src']} bf16 dense sustained"}
+            "peak_src": f"{pk['src']} bf16 dense sustained; f16 MMA probe measured in this run"}
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -548,10 +552,12 @@ def run_sweep(args):
     return 0
 
 
-def time_conv(shape, conv_pass, steps, warmup):
+def time_conv(shape, conv_pass, steps, warmup, stats=False):
     """One convolution pass on synthetic N(0,1) inputs, He weights, dy ~ N(0, 0.01^2):
     `steps` launches timed with CUDA events on the launching stream; when the
-    operands fit in L2 a 256 MiB buffer is rewritten between launches."""
+    operands fit in L2 a 256 MiB buffer is rewritten between launches.  stats:
+    the forward also reduces the BatchNorm statistics of its output, as the
+    training step's forwards do."""
     import torch
 
     from paper_1911_07384_gb300 import pf16
@@ -574,7 +580,8 @@ def time_conv(shape, conv_pass, steps, warmup):
     io_bytes = 2 * (x.numel() + w.numel() + (y.numel() if conv_pass != "dgrad" else dy.numel()))
     if io_bytes < 2 * 135 * 2 ** 20:
         flush = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device="cuda")
-    fn = {"fwd": lambda: pf16.conv_fwd(d, x, w, y, ws),
+    st = torch.empty(pf16.conv_bnstats_size(d), dtype=torch.uint8, device="cuda") if stats else None
+    fn = {"fwd": (lambda: pf16.conv_fwd_bnstats(d, x, w, y, st, ws)) if stats else (lambda: pf16.conv_fwd(d, x, w, y, ws)),
           "dgrad": lambda: pf16.conv_dgrad(d, dy, w, dx),
           "wgrad": lambda: pf16.conv_wgrad(d, x, dy, dw, ws)}[conv_pass]
     for _ in range(max(warmup, 3)):
@@ -603,7 +610,7 @@ def time_conv(shape, conv_pass, steps, warmup):
     gbs = byts / ms / 1e6
     attainable = min(pk["bf16_tflops"], byts and flops / byts * pk["hbm_gbs"] / 1e3)
     del x, w, dy, y, dx, dw, ws, flush
-    return {"metric": "conv pass TFLOP/s", "conv": list(shape), "pass": conv_pass, "ms": ms,
+    return {"metric": "conv pass TFLOP/s", "conv": list(shape), "pass": conv_pass, "bn_stats": bool(stats), "ms": ms,
             "ms_best": float(np.min(times)), "tflops": tf, "gbs": gbs,
             "frac_of_dense_peak": tf / pk["bf16_tflops"],
             "frac_of_attainable": tf / attainable, "arith_intensity": flops / byts,
@@ -660,14 +667,16 @@ def time_bn(shape, bn_pass, steps, warmup):
             "frac_of_hbm": byts / ms / 1e6 / pk["hbm_gbs"], "algorithmic_bytes": byts}
 
 
-# The dominant launch class of the step, k_gemm<256> (BN = 256, plain epilogue),
-# on one of its layers: the 14x14, 256 -> 256, 3x3 forward at batch 256 (five
-# calls per step; 59.2 GFLOP per launch).  Its DRAM traffic comes from one
-# ncu capture of that single launch (bench.py --conv ... under ncu -c 1).
-KERNEL_LAYER = (256, 14, 14, 256, 256, 3, 3, 1, 1)
-KERNEL_NAME = "k_gemm<256> (plain epilogue), 14x14 256->256 3x3 forward, batch 256"
-TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_256_conv_14x14_256_3x3_fwd_b256_traffic.json")
-GEMM_SOURCES = ["pf16_gemm.cu", "pf16_api.cu", "pf16_internal.h", "pf16_ptx.cuh"]
+# The dominant launch class of the step, k_gemm<256> (BN = 256, plain epilogue;
+# a quarter of the step's kernel time in the ncu launch list), on its largest
+# call: the 56x56, 64 -> 256 1x1 forward with the fused BatchNorm statistics
+# (four calls per step, 26.3 GFLOP and 514 MB of |x|+|w|+|y| per launch; AI 51
+# flop/B, so HBM-bound).  Its DRAM traffic comes from one ncu capture of that
+# single launch (bench.py --conv ... --stats under ncu -c 1).
+KERNEL_LAYER = (256, 56, 56, 64, 256, 1, 1, 1, 0)
+KERNEL_NAME = "k_gemm<256> (plain epilogue, forward statistics), 56x56 64->256 1x1 forward, batch 256"
+TRAFFIC_JSON = os.path.join(ROOT, "profiles", "k_gemm_256_conv_56x56_64to256_fwd_stats_b256_traffic.json")
+GEMM_SOURCES = ["pf16_gemm.cu", "pf16_epi.cuh", "pf16_api.cu", "pf16_internal.h", "pf16_ptx.cuh"]
 
 
 def wgrad_is_gemm(h, w, c, k, r, s, st, pad):
@@ -693,8 +702,8 @@ def gemm_source_digest():
 def ingest_traffic(csv_path):
     """DRAM traffic of the one k_gemm launch in an ncu CSV (metrics
     gpu__time_duration.sum, dram__bytes_read.sum, dram__bytes_write.sum) of
-    `bench.py --conv <KERNEL_LAYER> --pass fwd`, stored with the digest of the
-    sources it was measured on."""
+    `bench.py --conv <KERNEL_LAYER> --pass fwd --stats`, stored with the digest
+    of the sources it was measured on."""
     import csv as _csv
 
     with open(csv_path) as f:
@@ -738,20 +747,17 @@ def gemm_traffic():
 
 
 def kernel_roofline(pk, reps=10):
-    """The dominant launch class on its representative layer, timed alone with
-    CUDA events (L2 flushed between launches), against the measured sustained
-    16-bit peak and against the FP16 MMA rate the library's probe measures on
-    this GPU (kind::f16, N = 256)."""
-    from paper_1911_07384_gb300 import pf16
-
-    r = time_conv(KERNEL_LAYER, "fwd", reps, 3)
-    mma = pf16.tc_rate(256, reps=20000)
-    return {"bound": "tensor", "kernel": KERNEL_NAME, "achieved": r["tflops"],
-            "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": r["tflops"] / pk["bf16_tflops_sustained"],
-            "peak_f16_mma_probe": mma, "frac_of_f16_mma_probe": r["tflops"] / mma,
-            "ms_per_launch": r["ms"], "gflop_per_launch": r["tflops"] * r["ms"],
-            "traffic": gemm_traffic(), "algorithmic_bytes": r["gbs"] * r["ms"] * 1e6,
-            "peak_src": f"{pk['src']} bf16 dense sustained; f16 MMA probe measured in this run"}
+    """The dominant launch class on its largest call of the step, timed alone
+    with CUDA events on a pre-loaded stream (its operands are larger than L2):
+    algorithmic bytes |x|+|w|+|y| per launch over the launch time, against the
+    measured copy bandwidth (the layer is HBM-bound); the tensor rate beside
+    it for context."""
+    r = time_conv(KERNEL_LAYER, "fwd", reps, 3, stats=True)
+    byts = r["gbs"] * r["ms"] * 1e6
+    return {"bound": "hbm", "kernel": KERNEL_NAME, "achieved": r["gbs"], "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": r["gbs"] / pk["hbm_gbs"], "traffic": gemm_traffic(), "algorithmic_bytes": byts,
+            "ms_per_launch": r["ms"], "tflops": r["tflops"], "gflop_per_launch": r["tflops"] * r["ms"],
+            "peak_src": f"{pk['src']} HBM copy"}
 
 
 def count_launches(net):
