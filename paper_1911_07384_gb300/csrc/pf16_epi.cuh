@@ -13,6 +13,11 @@ namespace pf16 {
 // (its odd tiles), so two tiles drain at once.
 constexpr int kEpiWarps = 8;
 constexpr int kGemmThreads = 32 * (2 + kEpiWarps);
+// The wide epilogue of k_gemm (WE, plain epilogue of short reductions): 16
+// warps, two per TMEM sub-partition and accumulator, each draining one column
+// half of the tile.
+constexpr int kEpiWarpsWide = 16;
+constexpr int kGemmThreadsWide = 32 * (2 + kEpiWarpsWide);
 // XF (BatchNorm in the operand path): eight transform warps after the epilogue's
 constexpr int kXfWarp0 = 2 + kEpiWarps;
 constexpr int kXfWarps = 8;
@@ -166,14 +171,18 @@ struct EpiStats {
   // Close the stacks, merge the CTA's 8 epilogue warps (a balanced tree over
   // warps 0..7, in shared memory `sm`, >= 8.3 KB, free of pending TMA reads)
   // and write the CTA's node as `slot` for chunks c < nchunks.  Called by all
-  // 8 epilogue warps; uses named barrier 1.
+  // ew epilogue warps; uses named barrier 1.  With the wide epilogue (ew = 16)
+  // warps 8h .. 8h + 7 hold the chunks of column half h (cph chunks each), and
+  // chunk c is merged over the eight warps of its half, in the same tree.
   __device__ __forceinline__ void write_cta(const GemmParams& p, uint8_t* sm, int e, int slot, int n0,
-                                            int nchunks, int lane, bool write_count) {
-    uint32_t* node = reinterpret_cast<uint32_t*>(sm);              // [8][kStChunks][32][2]
-    int* ncnt = reinterpret_cast<int*>(sm + 8 * kStChunks * 32 * 8);  // [8]
-    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
+                                            int nchunks, int lane, bool write_count, int ew = kEpiWarps,
+                                            int cph = kStChunks) {
+    uint32_t* node = reinterpret_cast<uint32_t*>(sm);                // [ew][kStChunks][32][2]
+    int* ncnt = reinterpret_cast<int*>(sm + ew * kStChunks * 32 * 8);  // [ew]
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * ew) : "memory");
     int total = 0;
     for (int c = 0; c < nchunks; ++c) {
+      if (ew > 8 && c / cph != (e >> 3)) continue;  // a chunk of the other column half
       uint32_t am = 0, av = 0;
       int an = 0;
 #pragma unroll 1
@@ -191,17 +200,18 @@ struct EpiStats {
       total = an;
     }
     if (lane == 0) ncnt[e] = total;
-    asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps) : "memory");
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * ew) : "memory");
     if (e != 0) return;
     int tot = 0;
     for (int c = 0; c < nchunks; ++c) {
       uint32_t m[8], vv[8];
       int nn[8];
+      const int w0 = ew > 8 ? 8 * (c / cph) : 0;
 #pragma unroll
       for (int w = 0; w < 8; ++w) {
-        m[w] = node[((w * kStChunks + c) * 32 + lane) * 2];
-        vv[w] = node[((w * kStChunks + c) * 32 + lane) * 2 + 1];
-        nn[w] = ncnt[w];
+        m[w] = node[(((w0 + w) * kStChunks + c) * 32 + lane) * 2];
+        vv[w] = node[(((w0 + w) * kStChunks + c) * 32 + lane) * 2 + 1];
+        nn[w] = ncnt[w0 + w];
       }
 #pragma unroll
       for (int h = 1; h < 8; h *= 2)

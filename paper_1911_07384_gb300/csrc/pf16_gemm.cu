@@ -30,15 +30,20 @@ namespace pf16 {
 // TMAE: the TMA-fed backward-statistics epilogue keeps four 32 x 64 tiles per
 // warp (two staging tiles, two BatchNorm-input tiles, filled by TMA a chunk
 // ahead), paid for with pipeline stages; plus two transaction barriers per warp.
-template <int BN, bool TMAE = false, bool XF = false>
+// WE: the wide epilogue (16 warps, 4 KB of staging each), paid for with
+// pipeline stages -- it serves short reductions, whose few K-blocks per tile
+// need few stages.
+template <int BN, bool TMAE = false, bool XF = false, bool WE = false>
 struct GemmCfg {
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_BYTES = BN * kBK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = TMAE ? (BN == 64 ? 4 : (BN == 128 ? 3 : 2)) : (BN == 64 ? 8 : (BN == 128 ? 6 : 4));
+  static constexpr int STAGES = WE ? (BN == 128 ? 5 : 3)
+                                   : TMAE ? (BN == 64 ? 4 : (BN == 128 ? 3 : 2)) : (BN == 64 ? 8 : (BN == 128 ? 6 : 4));
   static constexpr int TMEM_COLS = 2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512);
+  static constexpr int EW = WE ? kEpiWarpsWide : kEpiWarps;  // epilogue warps
   static constexpr int WARP_BUF = TMAE ? 4 * 4096 : 4096;  // per epilogue warp
-  static constexpr int STAGING_BYTES = kEpiWarps * WARP_BUF;
+  static constexpr int STAGING_BYTES = EW * WARP_BUF;
   static constexpr int EBARS = TMAE ? 2 * kEpiWarps : 0;
   static constexpr int BAR_BYTES = 8 * ((XF ? 3 : 2) * STAGES + 4 + EBARS) + 16;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + BAR_BYTES;
@@ -456,13 +461,17 @@ __device__ __forceinline__ void xf_rows(const GemmParams& p, const XfParams& q, 
 // XF (with EPI_PLAIN): BatchNorm in the operand path (GemmParams::xf_*):
 // eight more warps transform each stage between the TMA's arrival (full) and
 // the MMAs (xready), see xf_rows.
-template <int BN, int EPI, bool XF = false>
-__global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
+// WE (with EPI_PLAIN, TMA stores): the wide epilogue, warps 2-17 in four
+// groups: group g drains accumulator g & 1, columns of half g >> 1.
+template <int BN, int EPI, bool XF = false, bool WE = false>
+__global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide : kGemmThreads), 1)
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapX,
            const __grid_constant__ CUtensorMap mapD, const __grid_constant__ GemmParams p) {
   constexpr bool BS = EPI != EPI_PLAIN, TMAE = EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, ADD = EPI == EPI_BS_ADD;
-  using Cfg = GemmCfg<BN, TMAE, XF>;
+  static_assert(!WE || (EPI == EPI_PLAIN && !XF && BN % 128 == 0), "the wide epilogue: plain, BN 128 or 256");
+  using Cfg = GemmCfg<BN, TMAE, XF, WE>;
+  constexpr int CS = WE ? 2 : 1;  // column halves per tile
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -485,7 +494,7 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&tempty[a]), 4 * CS);  // every warp that drains the accumulator arrives
     }
     for (int b = 0; b < Cfg::EBARS; ++b) mbar_init(smem_u32(&ebar[b]), 1);
     if (XF)
@@ -666,10 +675,12 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
       if (!ok) break;
     }
   } else {
-    // epilogue warps 2..9 -> TMEM sub-partitions 2, 3, 0, 1; group grp drains accumulator grp
+    // epilogue warps 2..9 (2..17 with WE) -> TMEM sub-partitions 2, 3, 0, 1, ...; group grp
+    // drains accumulator grp & 1, columns [c_begin, c_end) (the whole tile, or half of it)
     const int e = warp - 2, grp = e >> 2, sub = warp & 3;
     const int row = sub * 32 + lane;
-    const int acc = grp;
+    const int acc = grp & 1;
+    const int c_begin = WE ? (grp >> 1) * (BN / CS) : 0, c_end = c_begin + BN / CS;
     uint32_t acc_phase = 0;
     const uint32_t stg = smem_u32(staging) + (uint32_t)(e * Cfg::WARP_BUF);
     EpiStats stats;
@@ -680,7 +691,7 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
                            tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, lim, abort_flag, stats);
     const bool bstats = BS && p.st_mean && p.bs_x && p.tma_store;
     BwdIn bin;
-    for (int u = cid + grp * ncl; u < total && !TMAE; u += 2 * ncl) {
+    for (int u = cid + acc * ncl; u < total && !TMAE; u += 2 * ncl) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       int m0, n0, split, kb0, kb1;
       unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
@@ -700,7 +711,7 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
         const int nv = min(32, max(0, p.M - (m0 + sub * 32)));
         // 64-column chunks: TMEM -> registers -> 128B-swizzled staging -> TMA store
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 64) {
+        for (int c = c_begin; c < c_end; c += 64) {
           uint32_t r[64];
           tmem_ld16(tbase + c, r);
           tmem_ld16(tbase + c + 16, r + 16);
@@ -708,7 +719,7 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
           tmem_ld16(tbase + c + 48, r + 48);
           tmem_ld_wait();
           if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
-          if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
+          if (c + 64 >= c_end) {  // this warp's columns fully read: hand TMEM back before the stores
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
@@ -796,7 +807,7 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : kGemmThreads, 1)
       if (BS)
         stats.write_cta_bwd(p, staging, e, slot, n0, nch, lane, p.bs_levels);
       else
-        stats.write_cta(p, staging, e, slot, n0, nch, lane, cid % p.n_tiles == 0);
+        stats.write_cta(p, staging, e, slot, n0, nch, lane, cid % p.n_tiles == 0, Cfg::EW, BN / 64 / CS);
       if (blockIdx.x == 0 && e == 0 && lane == 0) {
         p.st_hdr[0] = ncl / p.n_tiles;
         p.st_hdr[1] = 5 + p.bs_levels + 3;
@@ -821,29 +832,29 @@ int gemm_smem_bytes(int BN) {
   }
 }
 
-template <int BN, int EPI = EPI_PLAIN, bool XF = false>
+template <int BN, int EPI = EPI_PLAIN, bool XF = false, bool WE = false>
 static cudaError_t set_smem_attr() {
   static bool attr_set[64] = {false};  // per device ordinal
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI, XF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI, XF, WE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF, WE>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
   return cudaSuccess;
 }
 
-template <int BN, int EPI, bool XF = false>
+template <int BN, int EPI, bool XF = false, bool WE = false>
 static cudaError_t launch_variant(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mC,
                                   const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
                                   cudaStream_t s) {
-  cudaError_t e = set_smem_attr<BN, EPI, XF>();
+  cudaError_t e = set_smem_attr<BN, EPI, XF, WE>();
   if (e != cudaSuccess) return e;
-  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF>::SMEM;
-  launch_pdl(k_gemm<BN, EPI, XF>, dim3(grid), dim3(XF ? kGemmThreadsXf : kGemmThreads), smem, s, mA, mB, mC, mX,
-             mD, p);
+  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF, WE>::SMEM;
+  launch_pdl(k_gemm<BN, EPI, XF, WE>, dim3(grid), dim3(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide : kGemmThreads)),
+             smem, s, mA, mB, mC, mX, mD, p);
   return counted_launches(1);
 }
 
@@ -857,6 +868,14 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     if (epi != EPI_PLAIN) return cudaErrorInvalidValue;
     return launch_variant<BN, EPI_PLAIN, true>(mA, mB, mC, mX, mD, p, grid, s);
   }
+  // the shortest reductions (one or two K-blocks per tile) with a plain
+  // epilogue: the wide epilogue, whose 16 warps drain a tile's two column
+  // halves at once -- there the epilogue is the bound (56x56 64->256 forward
+  // with statistics 117 -> 103 us); from four K-blocks on, the pipeline stages
+  // it gives up cost more (14x14 256->1024 forward 42.2 -> 44.0 us)
+  if constexpr (BN == 128 || BN == 256)
+    if (epi == EPI_PLAIN && p.tma_store && p.kb_per_split <= 2)
+      return launch_variant<BN, EPI_PLAIN, false, true>(mA, mB, mC, mX, mD, p, grid, s);
   switch (epi) {
     case EPI_PLAIN: return launch_variant<BN, EPI_PLAIN>(mA, mB, mC, mX, mD, p, grid, s);
     case EPI_BS: return launch_variant<BN, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);
