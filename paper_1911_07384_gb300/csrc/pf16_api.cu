@@ -313,6 +313,46 @@ Wgrad3Plan wgrad3_plan(const Shape& s) {
 }
 size_t wgrad3_parts_bytes(const Wgrad3Plan& w) { return round_up((size_t)w.chunks * 64 * 576 * 2, 256); }
 
+// The 3x3 / stride 1 / pad 1 weight gradient with K a multiple of 128 and C
+// of 64 on the wide halo engine (k_wgrad3x3_wide): a tile is one image row
+// of nb images of wi = W + 1 columns (at most 128 pixels), per_chunk tiles
+// (at most 32: 4,096 pixels) per FP16 accumulation.  The chunk length
+// minimises a makespan model on GB300's 152 SMs: rounds of units x chunk
+// length x ~0.42 us per tile (8 MMAs of 128 x 192 x 16) plus the partial
+// planes through the split-K tree at ~2 TB/s; at most 1,024 chunks.
+struct WideWgradPlan {
+  bool ok;
+  int wi, nb, types, per_chunk, chunks;
+  long long tiles;
+};
+WideWgradPlan wide_wgrad_plan(const Shape& s) {
+  WideWgradPlan w{};
+  if (s.kind != KIND_GENERIC || s.R != 3 || s.S != 3 || s.st != 1 || s.pad != 1 || s.K < 128 || s.K % 128 != 0 ||
+      s.C % 64 != 0 || s.W + 1 > 128)
+    return w;
+  w.wi = (int)s.W + 1;
+  w.nb = (int)std::min<long long>(128 / w.wi, s.N);
+  w.tiles = cdiv(s.N, (long long)w.nb) * s.H;
+  w.types = (int)(3 * (s.C / 64) * (s.K / 128));
+  const double plane_us = (double)s.K * 9 * s.C * 2 / 2.0e6;
+  double best = 1e300;
+  for (int len = 1; len <= 32; ++len) {
+    const long long chunks = cdiv(w.tiles, (long long)len);
+    if (chunks > 1024) continue;
+    const double t = (double)cdiv(chunks * w.types, 152ll) * len * 0.42 + (double)chunks * plane_us;
+    if (t < best) {
+      best = t;
+      w.per_chunk = len;
+      w.chunks = (int)chunks;
+    }
+  }
+  w.ok = best < 1e300 && (long long)w.chunks * w.types < (1ll << 30);
+  return w;
+}
+size_t wide_wgrad_parts_bytes(const Shape& s, const WideWgradPlan& w) {
+  return round_up((size_t)w.chunks * s.K * 9 * s.C * 2, 256);
+}
+
 size_t ws_fwd(const Shape& s) {
   if (s.kind != KIND_STEM) return 0;
   const long long kc = stem_kcol(s);
@@ -326,6 +366,8 @@ size_t ws_wgrad(const Shape& s) {
   if (sw.ok) return stem_s2d_bytes(s) + stem_wgrad_parts_bytes(sw) + 128 * 128 * 2;
   const Wgrad3Plan w3 = wgrad3_plan(s);
   if (w3.ok) return wgrad3_parts_bytes(w3);
+  const WideWgradPlan ww = wide_wgrad_plan(s);
+  if (ww.ok) return wide_wgrad_parts_bytes(s, ww);
   const WgradSplit w = wgrad_split(s);
   size_t b = 0;
   if (w.splits > 1 || s.kind == KIND_STEM) b += round_up((size_t)w.splits * s.K * w.ncols * 2, 256);
@@ -1087,6 +1129,50 @@ static int run_wgrad3x3(const Shape& s, const Wgrad3Plan& w3, const uint16_t* x,
   return PF16_OK;
 }
 
+// The 3x3 stride-1 weight gradient with K % 128 == 0 through
+// k_wgrad3x3_wide (layouts at wide_wgrad_plan), then the split-K tree
+// straight into dw.
+static int run_wgrad3x3_wide(const Shape& s, const WideWgradPlan& ww, const uint16_t* x, const uint16_t* dy,
+                             uint16_t* dw, void* work, int* status, int sms, cudaStream_t st, bool f32) {
+  const long long N = s.N, H = s.H, W = s.W, C = s.C, K = s.K;
+  uint16_t* parts = static_cast<uint16_t*>(work);
+  CUtensorMap mdy, mx;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  cuuint32_t box[4] = {64, (cuuint32_t)ww.wi, (cuuint32_t)ww.nb, 1};
+  // both maps (c, w, n, h) over an NHWC tensor
+  for (int m = 0; m < 2; ++m) {
+    const long long ch = m == 0 ? K : C;
+    const cuuint64_t pix = (cuuint64_t)ch * 2, row = (cuuint64_t)W * pix, img = (cuuint64_t)H * row;
+    cuuint64_t dims[4] = {(cuuint64_t)ch, (cuuint64_t)W, (cuuint64_t)N, (cuuint64_t)H};
+    cuuint64_t strides[3] = {pix, img, row};
+    void* base = const_cast<uint16_t*>(m == 0 ? dy : x);
+    if (g_encode_tiled(m == 0 ? &mdy : &mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, base, dims, strides, box, es,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return PF16_ERR_CUDA;
+  }
+  GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
+  p.idesc = idesc_f16(kBM, 192, true, true, f32);
+  p.M = (int)K;
+  p.halo_chunks = (int)(C / 64);
+  p.halo_wi = ww.wi;
+  p.halo_ipr = ww.nb;
+  p.halo_w = (int)W;
+  p.halo_h = (int)H;
+  p.num_kb = (int)ww.tiles;
+  p.kb_per_split = ww.per_chunk;
+  p.splits = ww.chunks;
+  p.m_tiles = ww.chunks * ww.types;
+  p.out = parts;
+  p.ldo = 9 * C;
+  const int grid = p.m_tiles < sms ? p.m_tiles : sms;
+  if (launch_wgrad3x3_wide(mdy, mx, p, grid, st) != cudaSuccess) return PF16_ERR_CUDA;
+  if (launch_splitk_reduce(parts, ww.chunks, K, (int)(9 * C), dw, 9 * C, (int)(9 * C), st) != cudaSuccess)
+    return PF16_ERR_CUDA;
+  return PF16_OK;
+}
+
 static int conv_wgrad_impl(const pf16_conv_desc* d, const uint16_t* x, const uint16_t* dy, uint16_t* dw,
                            void* ws, size_t ws_bytes, uint32_t flags, void* stream,
                            const pf16_bn_operand* bn = nullptr) {
@@ -1110,6 +1196,8 @@ static int conv_wgrad_impl(const pf16_conv_desc* d, const uint16_t* x, const uin
   if (sw.ok) return run_stem_wgrad(s, sw, x, dy, dw, ws, status, sms, st, f32);
   const Wgrad3Plan w3 = wgrad3_plan(s);
   if (w3.ok) return run_wgrad3x3(s, w3, x, dy, dw, ws, status, sms, st, f32);
+  const WideWgradPlan ww = wide_wgrad_plan(s);
+  if (ww.ok) return run_wgrad3x3_wide(s, ww, x, dy, dw, ws, status, sms, st, f32);
   const WgradSplit wsp = wgrad_split(s);
 
   GemmParams p = base_params(status);

@@ -243,6 +243,16 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mapA, const CUtensorMap& mapB, c
 // rows; forward statistics (optional) as k_gemm's plain epilogue.
 cudaError_t launch_gemm_halo_wide(int BN, const CUtensorMap& mapA, const CUtensorMap& mapB, const CUtensorMap& mapC,
                                   const GemmParams& p, int grid, cudaStream_t stream);
+// Wide halo weight gradient (pf16_halo.cu): 3x3 / stride 1 / pad 1 with
+// p.M = K output channels (a multiple of 128) and p.halo_chunks 64-channel
+// input chunks.  mDy / mX: 4-D tiled maps (c, w, n, h) over dy [N][H][W][K]
+// and x [N][H][W][C], boxes (64, halo_wi, halo_ipr, 1) with halo_wi = W + 1
+// (halo_w = W, halo_h = H).  p.num_kb tiles (image group g, row h at tile
+// g * H + h) in p.splits chunks of p.kb_per_split; p.m_tiles = p.splits x
+// 3 x halo_chunks x K / 128 units; chunk q's partial plane at p.out + q * K *
+// p.ldo (p.ldo = 9 * C), laid out as dw.
+cudaError_t launch_wgrad3x3_wide(const CUtensorMap& mDy, const CUtensorMap& mX, const GemmParams& p, int grid,
+                                 cudaStream_t stream);
 
 // ---------------------------------------------------------------------------
 // Memory-bound kernels (pf16_elementwise.cu).  All return cudaError_t of the

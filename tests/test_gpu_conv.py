@@ -187,8 +187,10 @@ def test_delta_kernel_wide_halo_bit_exact(orc, shape, tap):
     assert np.array_equal(f64(dx), V)
 
 
-@pytest.mark.parametrize("shape", [(2, 8, 8, 64, 128, 3, 3, 1, 1),    # im2col GEMM
-                                   (2, 9, 12, 64, 64, 3, 3, 1, 1)],  # halo weight gradient, odd P
+@pytest.mark.parametrize("shape", [(2, 8, 8, 64, 192, 3, 3, 1, 1),    # im2col GEMM
+                                   (2, 9, 12, 64, 64, 3, 3, 1, 1),    # halo weight gradient, odd P
+                                   (2, 8, 8, 64, 128, 3, 3, 1, 1),    # wide halo weight gradient
+                                   (3, 5, 15, 128, 256, 3, 3, 1, 1)],  # wide, three images per box
                          ids=ids)
 def test_delta_gradient_wgrad_bit_exact(orc, shape):
     """dy nonzero (= 1) at a single pixel per channel: every dw element is one
@@ -205,9 +207,33 @@ def test_delta_gradient_wgrad_bit_exact(orc, shape):
     assert np.array_equal(f64(dw), V)
 
 
+# The wide halo weight gradient (K a multiple of 128, 3x3 stride 1): boxes of
+# nb images of W + 1 columns, chunked FP16 accumulations and the split-K tree.
+WGRAD_WIDE = [
+    (2, 7, 7, 512, 512, 3, 3, 1, 1),     # 7x7: 8-column images, four output-channel tiles
+    (17, 2, 7, 64, 128, 3, 3, 1, 1),     # 16 images per box, the second box one image
+    (1, 3, 127, 64, 128, 3, 3, 1, 1),    # W + 1 = 128: windows read the zero tail
+    (1, 4, 60, 64, 128, 3, 3, 1, 1),     # one image of 61 columns per box
+    (8, 28, 28, 128, 128, 3, 3, 1, 1),   # several tiles per chunk, several chunks
+    (3, 5, 9, 128, 384, 3, 3, 1, 1),     # three output-channel tiles
+]
+
+
+@pytest.mark.parametrize("shape", WGRAD_WIDE, ids=ids)
+def test_conv_wgrad_wide(orc, shape):
+    N, H, W, C, K, R, S, st, pd = shape
+    x, w, dy, P, Q = inputs(shape, seed_cfg=6)
+    d = pf16.conv_desc(*shape)
+    dw = run_wgrad(d, x, dy)
+    V, A, T = orc.conv_wgrad(x, dy, *shape)
+    rel = assert_conv_close(dw, V, A, N * P * Q, "wgrad")
+    assert rel < 2.0 ** -6, rel
+
+
 CFG3 = [(256, 56, 56, 256, 64, 1, 1, 1, 0), (256, 28, 28, 512, 128, 1, 1, 1, 0),
         (256, 14, 14, 1024, 256, 1, 1, 1, 0), (256, 7, 7, 512, 2048, 1, 1, 1, 0),
-        (256, 56, 56, 64, 64, 3, 3, 1, 1)]  # the 3x3 64-channel layer: halo engines, 802,816-pixel weight gradient
+        (256, 56, 56, 64, 64, 3, 3, 1, 1),  # the 3x3 64-channel layer: halo engines, 802,816-pixel weight gradient
+        (256, 14, 14, 256, 256, 3, 3, 1, 1)]  # wide halo engines: forward, 50,176-pixel weight gradient
 
 
 @pytest.mark.parametrize("shape", CFG3, ids=ids)
@@ -234,7 +260,7 @@ def test_full_size_sampled(orc, shape):
 
 
 F32_SHAPES = [
-    (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col, reduction 2,304, 256-wide N tiles
+    (2, 14, 14, 256, 256, 3, 3, 1, 1),   # im2col forward, reduction 2,304, 256-wide N tiles
     (4, 14, 14, 256, 256, 3, 3, 1, 1),   # wide halo engine, four images per padded row
     (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine
     (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem: space-to-depth halo forward, stem weight gradient
