@@ -586,7 +586,8 @@ int run_halo(const Shape& s, int ws, bool dgrad, const uint16_t* in, const uint1
     set_kmajor(p, false, true);
     if (!map_2d(&mb, w, 9 * 64, 64, 9 * 64, 64, 64)) return PF16_ERR_CUDA;
   }
-  p.idesc = idesc_f16(kBM, 64, false, dgrad, f32);
+  // N = 192: the slices of taps (r, 0..2), contiguous in shared memory
+  p.idesc = idesc_f16(kBM, 192, false, dgrad, f32);
   p.halo_ws = ws;
   p.halo_h = (int)H;
   p.halo_w = (int)W;

@@ -916,7 +916,9 @@ cudaError_t launch_gemm(int BN, const CUtensorMap& mA, const CUtensorMap& mB, co
 // weight slices stay in shared memory for the whole launch.  Two uses:
 //   - 3x3 / stride 1 / pad 1, 64 -> 64 channels (forward, or the data
 //     gradient as a convolution of dy with the flipped filter): cb = 128,
-//     128-byte swizzle, box rows i0-1 .. i0+128/ws, columns -1 .. ws-2;
+//     128-byte swizzle, box rows i0-1 .. i0+128/ws, columns -1 .. ws-2; one
+//     N = 192 MMA per filter row and K step (three taps' slices against one
+//     window, recombined by row shifts in the epilogue: halo3_combine);
 //   - the 7x7 / stride 2 / pad 3 stem after a 2x2 space-to-depth of its
 //     three-channel input: a 4x4 / stride 1 / unpadded convolution over 16
 //     channels (12 real), cb = 32, 32-byte swizzle, one K = 16 MMA per tap.
@@ -928,13 +930,88 @@ struct HaloCfg {
   static constexpr int B_BYTES = 9 * 64 * kBK * 2;  // resident: 9 taps x 64 x 64, or 16 x 64 x 16
   static constexpr int A_BOX_MAX = 64 * 4 * 128;    // ws = 64: 4 rows of 64 pixels (ws = 32: 6 x 32;
                                                     // the stem: 4 rows of 128 pixels x 32 bytes)
-  static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's over-read
+  static constexpr int A_STAGE = A_BOX_MAX + 1024;  // + the last tap window's over-read (the stem)
   static constexpr int STAGES = 3;
-  static constexpr int TMEM_COLS = 128;
   static constexpr int STAGING_BYTES = kEpiWarps * 4096;  // one 32 x 64 tile per epilogue warp
-  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
-  static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + BAR_BYTES;
+  // 3x3: rows 0 and 1 of each warp's shifted partials (128 32-bit columns),
+  // per epilogue group, tile parity and TMEM sub-partition
+  static constexpr int XCH_BYTES = 2 * 2 * 4 * 2 * 512;
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 7) + 16;
+  static constexpr int SMEM = 1024 + B_BYTES + STAGES * A_STAGE + STAGING_BYTES + XCH_BYTES + BAR_BYTES;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
+
+// 3x3 halo epilogue.  The accumulator holds in columns 64 j + c (j = 0, 1, 2)
+// the products of taps (r, j) read through the window of tap (r, 0), summed
+// over the filter rows r: row m of it is tap column j's share of output row
+// m - j.  So output m = D[m][c] + D[m + 1][64 + c] + D[m + 2][128 + c], each
+// addition rounded to FP16 (an FP32 accumulator: added in FP32 and rounded
+// once).  Rows m + 1 and m + 2 come from lanes + 1 and + 2 of the warp, and
+// for lanes 30 and 31 from rows 0 and 1 of the next warp (nxt: its rows
+// continue the same padded row), which that warp left in shared memory at
+// `other` (row l at + l * 512 bytes, columns 64..191 as 32-bit words).  Rows
+// m + 1, m + 2 of a padded row's last real pixels are still in that padded
+// row (ws >= W + 2), so a tile never needs another tile's rows.
+__device__ __forceinline__ void halo3_publish(uint32_t tb, int lane, uint32_t mine) {
+#pragma unroll 1
+  for (int h = 0; h < 2; ++h) {
+    uint32_t v[64];
+    tmem_ld16(tb + 64 + 64 * h, v);
+    tmem_ld16(tb + 80 + 64 * h, v + 16);
+    tmem_ld16(tb + 96 + 64 * h, v + 32);
+    tmem_ld16(tb + 112 + 64 * h, v + 48);
+    tmem_ld_wait();
+    if (lane < 2) {
+#pragma unroll
+      for (int q = 0; q < 16; ++q)
+        st_shared_v4(mine + (uint32_t)(lane * 512 + (64 * h + 4 * q) * 4),
+                     make_uint4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+    }
+  }
+}
+
+__device__ __forceinline__ void halo3_combine(uint32_t tb, int lane, bool f32, bool nxt, uint32_t other,
+                                              uint32_t* o) {
+#pragma unroll
+  for (int c = 0; c < 64; c += 16) {
+    uint32_t d0[16], a[16], b[16];
+    tmem_ld16(tb + c, d0);
+    tmem_ld16(tb + 64 + c, a);
+    tmem_ld16(tb + 128 + c, b);
+    tmem_ld_wait();
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      a[j] = __shfl_down_sync(0xffffffffu, a[j], 1);
+      b[j] = __shfl_down_sync(0xffffffffu, b[j], 2);
+    }
+    if (nxt && lane >= 30) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint4 v;
+        if (lane == 31) {
+          ld_shared_v4(other + (uint32_t)((c + 4 * q) * 4), v);
+          a[4 * q] = v.x, a[4 * q + 1] = v.y, a[4 * q + 2] = v.z, a[4 * q + 3] = v.w;
+        }
+        ld_shared_v4(other + (uint32_t)((lane - 30) * 512 + (64 + c + 4 * q) * 4), v);
+        b[4 * q] = v.x, b[4 * q + 1] = v.y, b[4 * q + 2] = v.z, b[4 * q + 3] = v.w;
+      }
+    }
+    if (f32) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        d0[j] = __float_as_uint(
+            __fadd_rn(__fadd_rn(__uint_as_float(d0[j]), __uint_as_float(a[j])), __uint_as_float(b[j])));
+      f32_to_f16_lo<16>(d0);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o[c / 2 + j] = pack_lo(d0[2 * j], d0[2 * j + 1]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        o[c / 2 + j] = hadd2_rn(hadd2_rn(pack_lo(d0[2 * j], d0[2 * j + 1]), pack_lo(a[2 * j], a[2 * j + 1])),
+                                pack_lo(b[2 * j], b[2 * j + 1]));
+    }
+  }
+}
 
 // CB = bytes of one input pixel: 128 (3x3, nine taps of four K = 16 steps,
 // 128-byte swizzle) or 32 (the space-to-depth stem, sixteen taps of one step,
@@ -952,19 +1029,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   constexpr int KSTEPS = CB / 32;                 // K = 16 steps per tap
   constexpr uint32_t SWZ = CB == 128 ? 2u : 6u;   // descriptor swizzle code
   constexpr int B_TILE = 64 * CB;                 // one tap's 64-row weight slice
+  constexpr int ACC = CB == 128 ? 192 : 64;       // accumulator columns (3x3: three taps' slices)
+  constexpr int TMEM_COLS = CB == 128 ? 512 : 128;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* bres = smem;                                   // the taps' weight slices
   uint8_t* astages = smem + Cfg::B_BYTES;                 // 1024-aligned stages
   uint8_t* staging = astages + Cfg::STAGES * Cfg::A_STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
+  uint8_t* xch = staging + Cfg::STAGING_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xch + Cfg::XCH_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + Cfg::STAGES;
   uint64_t* tfull = bars + 2 * Cfg::STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* bready = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bready + 1);
+  uint64_t* xbar = bready + 1;  // per epilogue group: the exchange of shifted partials
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int ws = p.halo_ws, rows = kBM / ws;
@@ -978,6 +1059,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
       mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&xbar[a]), 4);
     }
     mbar_init(smem_u32(bready), 1);
     *abort_flag = 0;
@@ -987,7 +1069,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tma_prefetch_desc(&mapC);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -1067,14 +1149,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 64);
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC);
         const uint64_t abase = adesc0 + desc_addr16(smem_u32(astages + stage * Cfg::A_STAGE));
+        if constexpr (CB == 128) {
+          // filter row r: one N = 192 MMA per K step, the window of tap (r, 0)
+          // against the contiguous slices of taps (r, 0), (r, 1), (r, 2)
 #pragma unroll
-        for (int t = 0; t < NTAPS; ++t)
+          for (int r = 0; r < 3; ++r)
 #pragma unroll
-          for (int kk = 0; kk < KSTEPS; ++kk)
-            tc_mma_f16(d_tmem, abase + toff[t] + kk * 2, bdesc0 + (uint32_t)(t * (B_TILE >> 4)) + kk * bk16,
-                       p.idesc, (t > 0 || kk > 0) ? 1u : 0u);
+            for (int kk = 0; kk < KSTEPS; ++kk)
+              tc_mma_f16(d_tmem, abase + toff[3 * r] + kk * 2,
+                         bdesc0 + (uint32_t)(3 * r * (B_TILE >> 4)) + kk * bk16, p.idesc,
+                         (r > 0 || kk > 0) ? 1u : 0u);
+        } else {
+#pragma unroll
+          for (int t = 0; t < NTAPS; ++t)
+#pragma unroll
+            for (int kk = 0; kk < KSTEPS; ++kk)
+              tc_mma_f16(d_tmem, abase + toff[t] + kk * 2, bdesc0 + (uint32_t)(t * (B_TILE >> 4)) + kk * bk16,
+                         p.idesc, (t > 0 || kk > 0) ? 1u : 0u);
+        }
         tc_commit(smem_u32(&empty[stage]));
         if (++stage == Cfg::STAGES) {
           stage = 0;
@@ -1096,6 +1190,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     EpiStats stats;
     stats.init();
     BwdIn bin;
+    // 3x3: exchange of shifted partials between the warps of a padded row
+    // (none at ws = 32, where a warp holds a whole padded row); xit counts
+    // this warp's tiles (exchange buffer and barrier parity)
+    const bool xchg = CB == 128 && ws > 32;
+    const bool pub = xchg && (sub * 32) % ws != 0;
+    const bool nxt = xchg && (sub * 32 + 32) % ws != 0;
+    uint32_t xit = 0;
     for (int u = blockIdx.x + grp * gridDim.x; u < total; u += 2 * gridDim.x) {
       if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       if (BS && p.st_mean) {  // the tile's inputs, loaded while the accumulator is computed
@@ -1110,28 +1211,42 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         break;
       }
       tc_fence_after();
-      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * 64);
-      uint32_t r[64];
-      tmem_ld16(tbase, r);
-      tmem_ld16(tbase + 16, r + 16);
-      tmem_ld16(tbase + 32, r + 32);
-      tmem_ld16(tbase + 48, r + 48);
-      tmem_ld_wait();
-      if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
+      const uint32_t tbase = tmem_base + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * ACC);
+      uint32_t o[32];  // the warp's 32 rows x 64 outputs, FP16 pairs
+      if constexpr (CB == 128) {
+        const uint32_t xslot = smem_u32(xch) + (uint32_t)((grp * 2 + (int)(xit & 1)) * 4 * 1024);
+        if (xchg) {
+          if (pub) halo3_publish(tbase, lane, xslot + (uint32_t)(sub * 1024));
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&xbar[grp]));
+          const bool okx = mbar_wait(smem_u32(&xbar[grp]), xit & 1, lim);
+          if (!__all_sync(0xffffffffu, okx)) {
+            if (lane == 0) record_timeout(p, abort_flag);
+            break;
+          }
+        }
+        halo3_combine(tbase, lane, p.d_f32 != 0, nxt, xslot + (uint32_t)((sub + 1) * 1024), o);
+        ++xit;
+      } else {
+        uint32_t r[64];
+        tmem_ld16(tbase, r);
+        tmem_ld16(tbase + 16, r + 16);
+        tmem_ld16(tbase + 32, r + 32);
+        tmem_ld16(tbase + 48, r + 48);
+        tmem_ld_wait();
+        if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
+#pragma unroll
+        for (int j = 0; j < 32; ++j) o[j] = pack_lo(r[2 * j], r[2 * j + 1]);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
       if (lane == 0) bulk_wait_read0();  // the previous store has read the staging tile
       __syncwarp();
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        uint4 v;
-        v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
-        v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
-        v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
-        v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
-        st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
-      }
+      for (int j = 0; j < 8; ++j)
+        st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4),
+                     make_uint4(o[j * 4], o[j * 4 + 1], o[j * 4 + 2], o[j * 4 + 3]));
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
@@ -1171,7 +1286,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -1188,6 +1303,11 @@ cudaError_t launch_gemm_halo(const CUtensorMap& mA, const CUtensorMap& mB, const
       p.halo_box_rows * p.halo_ws * p.halo_cb > HaloCfg::A_BOX_MAX ||
       max_off + kBM * p.halo_cb > HaloCfg::A_STAGE)
     return cudaErrorInvalidValue;
+  // 3x3: slot t holds tap (t / 3, t % 3), so filter row r's three slices are
+  // the contiguous N = 192 operand read through tap (r, 0)'s window
+  if (p.halo_cb == 128)
+    for (int t = 0; t < 9; ++t)
+      if (p.tap_dr[t] != t / 3 || p.tap_ds[t] != t % 3) return cudaErrorInvalidValue;
   // variants: 128-byte pixels, with backward statistics (the 3x3 data gradient) or not; 32-byte pixels
   static bool attr_set[3][64] = {};
   int dev = 0;

@@ -104,7 +104,13 @@ class Conv:
         size = pf16.conv_bnstats_size(self.desc)
         self.stats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
         # backward statistics of the BatchNorm whose output gradient the data gradient is
-        size = pf16.conv_dgrad_bnstats_size(self.desc) if self.desc.c != 3 else 0
+        # (not for the 3x3 64 -> 64 layers: their data gradient alone runs at about
+        # twice the rate it keeps with the statistics epilogue, which is bound by the
+        # latency of its per-element work, and the BatchNorm's own statistics pass
+        # costs less than the difference)
+        d = self.desc
+        halo64 = d.r == 3 and d.s == 3 and d.stride == 1 and d.c == 64 and d.k == 64
+        size = pf16.conv_dgrad_bnstats_size(d) if d.c != 3 and not halo64 else 0
         self.dstats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
 
     def fwd(self, x, y, with_stats=False, bn_in=None):
