@@ -488,8 +488,13 @@ def run_layers(args):
             d = layer.desc
             key = (kind, (d.n, d.h, d.w, d.c, int(d.flags)))
             relu, res = d.flags & pf16.PF16_BN_RELU, d.flags & pf16.PF16_BN_RESIDUAL
-            units = (2 + (1 if res else 0)) if kind == "bn_fwd" else (3 + (1 if res else 0))
-            work, unit = (2.0 * layer.elems * units + (layer.elems / 8 if relu else 0)) / 1e9, "GB/s"
+            e = layer.elems
+            if kind == "bn_pool_fwd":  # x read; pooled output, positions (a byte each) and ReLU bits written
+                work = (2.0 * e + 0.5 * e + 0.25 * e + e / 8) / 1e9
+            else:
+                units = (2 + (1 if res else 0)) if kind == "bn_fwd" else (3 + (1 if res else 0))
+                work = (2.0 * layer.elems * units + (layer.elems / 8 if relu else 0)) / 1e9
+            unit = "GB/s"
         else:
             key, work, unit = (kind, ()), 0.0, ""
         a = agg.setdefault(key, [0, 0.0, 0.0, unit])
@@ -782,7 +787,10 @@ def count_launches(net):
     total += sum(per["bn_fwd"] + per["bn_bwd"] - (1 if getattr(b, "fused_bwd", False) else 0)
                  - (1 if getattr(b, "fused_apply", False) else 0)
                  + (1 if b.desc.flags & pf16.PF16_BN_SWAP else 0) for b in net.bns)
-    total += per["maxpool_fwd"] + per["maxpool_bwd"] + per["avgpool_fwd"] + per["avgpool_bwd"]
+    # (the stem's fused BatchNorm + pooling forward: the BatchNorm's statistics final and the
+    # fused pass -- the BatchNorm's count above, with no pooling launch)
+    total += (0 if getattr(net, "stem_fused", False) else per["maxpool_fwd"]) + per["maxpool_bwd"]
+    total += per["avgpool_fwd"] + per["avgpool_bwd"]
     total += per["softmax_xent"] + 2 * per["sgd"]
     return total
 

@@ -338,6 +338,21 @@ size_t pf16_bn_workspace_size(const pf16_bn_desc* d);
 int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, void* ws,
                     size_t ws_bytes, void* stream);
 
+/* The stem's BatchNorm with ReLU and the 3x3 / stride 2 / pad 1 max pooling
+ * that follows it in one call (Sec. 5.1's ResNet-50 stem): phase 0 of
+ * pf16_bn_fwd_bwd (flags exactly PF16_BN_RELU: no residual; conv_stats as
+ * there) whose output y goes straight into the pooling, so y is never
+ * stored (t->y must be NULL).  Writes t->mean, t->invstd, t->relu_mask (if
+ * non-NULL, as phase 0) and pooled[n][p][q][c], argmax[n][p][q][c] as
+ * pf16_maxpool_fwd_argmax (p < (h - 1) / 2 + 1, q < (w - 1) / 2 + 1).  The
+ * results are bit for bit those of pf16_bn_fwd_bwd(phase 0) followed by
+ * pf16_maxpool_fwd_argmax on its y.  The workspace is phase 0's
+ * (pf16_bn_workspace_size).  Errors as pf16_bn_fwd_bwd; PF16_ERR_ARG when
+ * t->y is set; PF16_ERR_UNSUPPORTED for other flags or when 5 rows of w * c
+ * values exceed 200 KB; argmax 8-byte aligned. */
+int pf16_bn_relu_maxpool_fwd(const pf16_bn_desc* d, const pf16_bn_tensors* t, uint16_t* pooled,
+                             uint8_t* argmax, void* ws, size_t ws_bytes, void* stream);
+
 /* ------------------------------------------------- rest of the train step
  * The remaining ops of the ResNet-50 training step (Sec. 5.1), all FP16. */
 

@@ -1397,6 +1397,34 @@ int pf16_bn_fwd_bwd(const pf16_bn_desc* d, int phase, const pf16_bn_tensors* t, 
              : PF16_ERR_CUDA;
 }
 
+int pf16_bn_relu_maxpool_fwd(const pf16_bn_desc* d, const pf16_bn_tensors* t, uint16_t* pooled,
+                             uint8_t* argmax, void* ws, size_t ws_bytes, void* stream) {
+  BnLaunch b;
+  int rc = bn_validate(d, &b);
+  if (rc != PF16_OK) return rc;
+  if (!t || !pooled || !argmax) return PF16_ERR_NULL;
+  if (d->flags != PF16_BN_RELU) return PF16_ERR_UNSUPPORTED;  // ReLU, no residual
+  if (t->y) return PF16_ERR_ARG;                              // y is not stored
+  if (bn_pool_smem_bytes(d->w, d->c) > 200 * 1024) return PF16_ERR_UNSUPPORTED;
+  if (!ws) return PF16_ERR_WORKSPACE;
+  if (ws_bytes < bn_ws_bytes(b)) return PF16_ERR_WORKSPACE;
+  if (!aligned16(ws)) return PF16_ERR_ALIGN;
+  const void* req[] = {t->x, t->gamma, t->beta, t->mean, t->invstd, pooled};
+  for (const void* p : req) {
+    if (!p) return PF16_ERR_NULL;
+    if (!aligned16(p)) return PF16_ERR_ALIGN;
+  }
+  if (reinterpret_cast<uintptr_t>(argmax) % 8 != 0) return PF16_ERR_ALIGN;
+  if (t->conv_stats && !aligned16(t->conv_stats)) return PF16_ERR_ALIGN;
+  int sms = 0;
+  if (device_consts(&b.status, &sms) != PF16_OK) return PF16_ERR_CUDA;
+  return launch_bn_relu_pool_fwd(b, static_cast<const uint8_t*>(t->conv_stats), t->x, t->gamma, t->beta, t->mean,
+                                 t->invstd, pooled, argmax, t->relu_mask, static_cast<uint16_t*>(ws), d->n, d->h,
+                                 d->w, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? PF16_OK
+             : PF16_ERR_CUDA;
+}
+
 static int pool_check(const void* a, const void* b, int32_t n, int32_t h, int32_t w, int32_t c) {
   if (!a || !b) return PF16_ERR_NULL;
   if (!aligned16(a) || !aligned16(b)) return PF16_ERR_ALIGN;

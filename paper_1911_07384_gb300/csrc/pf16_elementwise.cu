@@ -623,6 +623,14 @@ struct BnStatArgs {
   uint16_t* ws4;        // backward, swap variant: per-CTA trees of dy' * residual [blocks][C], else null
 };
 
+// One window's first-maximum positions (bytes of cw, halves j&1) against a
+// cell's position `mine` in it: the lanes of the 2-half word j it selects.
+__device__ __forceinline__ uint32_t code_sel2(uint32_t cw, int j, uint32_t mine) {
+  const uint32_t c0 = (cw >> ((j & 1) * 16)) & 0xFFu;
+  const uint32_t c1 = (cw >> ((j & 1) * 16 + 8)) & 0xFFu;
+  return (c0 == mine ? 0x0000FFFFu : 0u) | (c1 == mine ? 0xFFFF0000u : 0u);
+}
+
 __device__ __forceinline__ uint4 tree8(uint4* v) {
 #pragma unroll
   for (int w = 4; w >= 1; w /= 2)
@@ -1586,12 +1594,6 @@ __global__ void __launch_bounds__(256)
 // the four windows' positions and gradients once, then every cell sums, in
 // window order (p, then q), the gradients of the windows whose first maximum
 // it is.  One CTA per block row (n, i).
-__device__ __forceinline__ uint32_t code_sel2(uint32_t cw, int j, uint32_t mine) {
-  const uint32_t c0 = (cw >> ((j & 1) * 16)) & 0xFFu;
-  const uint32_t c1 = (cw >> ((j & 1) * 16 + 8)) & 0xFFu;
-  return (c0 == mine ? 0x0000FFFFu : 0u) | (c1 == mine ? 0xFFFF0000u : 0u);
-}
-
 __global__ void __launch_bounds__(512)
     k_maxpool_bwd_codes(const uint8_t* __restrict__ codes, const uint16_t* __restrict__ dy,
                         uint16_t* __restrict__ dx, int N, int H, int W, int C, int P, int Q) {
@@ -1770,6 +1772,143 @@ cudaError_t launch_maxpool_bwd(const uint16_t* x, const uint16_t* dy, uint16_t* 
     if (e != cudaSuccess) return e;
   }
   launch_pdl(k_maxpool_bwd, dim3((unsigned)((long long)N * bands * (C / 8))), dim3(256), shm, s, x, dy, dx, N, H, W, C, P, Q);
+  return counted_launches(1);
+}
+
+// ============================================================================
+// The stem's BatchNorm, ReLU and 3x3 / stride 2 / pad 1 max pooling in one
+// pass (pf16_bn_relu_maxpool_fwd): y = ReLU(BN(x)) is never stored.  A CTA
+// owns kBpT output rows p0 .. p0 + kBpT - 1 of one image, i.e. input rows
+// 2 p0 .. 2 p0 + 2 kBpT - 1, whose ReLU bits it writes.  It computes y for
+// input rows 2 p0 - 1 .. 2 p0 + 2 kBpT - 1 into shared memory (row 2 p0 - 1
+// belongs to the previous CTA and is computed twice) with k_bn_apply's op
+// sequence, then takes each window's first maximum (rows then columns, as
+// k_maxpool_fwd) from there.  After the ReLU every value is +0 or positive,
+// where FP16 order is the order of the bit patterns, so the window scan
+// starts from its first valid cell and replaces the maximum where a cell is
+// strictly greater (set.gt on f16x2, exact for these values): the pooled
+// output and positions are those of k_maxpool_fwd on y, bit for bit.
+// ============================================================================
+constexpr int kBpT = 2;
+
+__device__ __forceinline__ uint32_t hgt2_mask(uint32_t a, uint32_t b) {  // 0xFFFF per half where a > b
+  uint32_t d;
+  asm("set.gt.u32.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
+// take cell value v (position rs) into the window's running maximum m / codes
+__device__ __forceinline__ void pool_take(uint4& m, uint32_t (&code)[2], const uint4& v, uint32_t rs) {
+  const uint32_t rsr = rs * 0x01010101u;
+  uint32_t* mw = &m.x;
+  const uint32_t* vw = &v.x;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const uint32_t gt = hgt2_mask(vw[k], mw[k]);
+    mw[k] = (vw[k] & gt) | (mw[k] & ~gt);
+    // the position bytes of halves 2k, 2k+1: bytes 2(k&1), 2(k&1)+1 of code word k/2
+    const uint32_t bm = __byte_perm(gt, 0u, 0x4420) << (16 * (k & 1));
+    code[k >> 1] = (code[k >> 1] & ~bm) | (rsr & bm);
+  }
+}
+
+__global__ void __launch_bounds__(256)
+    k_bn_relu_pool_fwd(const uint16_t* __restrict__ x, const uint16_t* __restrict__ gamma,
+                       const uint16_t* __restrict__ beta, const uint16_t* __restrict__ mean,
+                       const uint16_t* __restrict__ invstd, uint16_t post_scale, uint16_t* __restrict__ pooled,
+                       uint8_t* __restrict__ codes, uint8_t* __restrict__ mask, int N, int H, int W, int C, int P,
+                       int Q) {
+  pdl_wait();
+  extern __shared__ uint4 zs[];  // [2 kBpT + 1][W][C / 8]: y of the staged input rows
+  const int tc = C / 8;
+  const int nb = (P + kBpT - 1) / kBpT;
+  const int n = blockIdx.x / nb, p0 = (blockIdx.x - n * nb) * kBpT;
+  const uint32_t ps = dup2(post_scale);
+  // blockDim is a multiple of tc: a thread keeps one channel group throughout
+  // and steps over cells (then windows) by cstep
+  const int cg = threadIdx.x % tc, c0 = threadIdx.x / tc, cstep = blockDim.x / tc;
+  const uint4 mu = __ldg(reinterpret_cast<const uint4*>(mean) + cg);
+  const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
+  const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
+  const uint4 be = __ldg(reinterpret_cast<const uint4*>(beta) + cg);
+#pragma unroll 1
+  for (int rho = 0; rho < 2 * kBpT + 1; ++rho) {
+    const int h = 2 * p0 - 1 + rho;
+    if (h < 0 || h >= H) continue;
+    const long long rowoff = ((long long)n * H + h) * W * tc + cg;
+    uint4* zrow = zs + (rho * W) * tc + cg;
+    for (int w0 = c0; w0 < W; w0 += 4 * cstep) {
+      uint4 xv[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {  // four cells' loads in flight before any use
+        const int w = w0 + k * cstep;
+        xv[k] = w < W ? __ldg(reinterpret_cast<const uint4*>(x) + rowoff + (long long)w * tc) : zero4();
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int w = w0 + k * cstep;
+        if (w >= W) break;
+        const uint4 xh = mul4v(sub4(xv[k], mu), is);  // Eq. 1
+        uint32_t bits;
+        const uint4 z = relu_bits(mul4(add4(mul4v(ga, xh), be), ps), bits);  // Eq. 2, ReLU
+        zrow[w * tc] = z;
+        if (rho >= 1 && mask) mask[rowoff + (long long)w * tc] = (uint8_t)bits;  // rows 2 p0 .. are this CTA's
+      }
+    }
+  }
+  __syncthreads();
+#pragma unroll 1
+  for (int t = 0; t < kBpT; ++t) {
+    const int p = p0 + t;
+    if (p >= P) break;
+    for (int q = c0; q < Q; q += cstep) {
+      // the window's first valid cell (row 2p - 1 and column 2q - 1 are padding at p = 0, q = 0)
+      const int r0 = p == 0 ? 1 : 0, s0 = q == 0 ? 1 : 0;
+      uint4 m = zs[((2 * t + r0) * W + 2 * q + s0 - 1) * tc + cg];
+      uint32_t code[2];
+      code[0] = code[1] = (uint32_t)(r0 * 3 + s0) * 0x01010101u;
+#pragma unroll
+      for (int r = 0; r < 3; ++r) {
+        if (2 * p + r - 1 >= H || r < r0) continue;
+#pragma unroll
+        for (int s2 = 0; s2 < 3; ++s2) {
+          const int w = 2 * q + s2 - 1;
+          if (w < 0 || w >= W || (r == r0 && s2 <= s0)) continue;
+          pool_take(m, code, zs[((2 * t + r) * W + w) * tc + cg], (uint32_t)(r * 3 + s2));
+        }
+      }
+      const long long o = (((long long)n * P + p) * Q + q) * tc + cg;
+      reinterpret_cast<uint4*>(pooled)[o] = m;
+      reinterpret_cast<uint2*>(codes)[o] = make_uint2(code[0], code[1]);
+    }
+  }
+}
+
+int bn_pool_smem_bytes(int W, int C) { return (2 * kBpT + 1) * W * (C / 8) * 16; }
+
+cudaError_t launch_bn_relu_pool_fwd(const BnLaunch& b, const uint8_t* conv_stats, const uint16_t* x,
+                                    const uint16_t* gamma, const uint16_t* beta, uint16_t* mean,
+                                    uint16_t* invstd, uint16_t* pooled, uint8_t* codes, uint8_t* mask,
+                                    uint16_t* ws, int N, int H, int W, cudaStream_t s) {
+  // the statistics as pf16_bn_fwd_bwd's phase 0 takes them (from the conv's
+  // partial statistics, or a pass over x), then the fused apply and pooling
+  cudaError_t e = conv_stats ? launch_bn_fwd_given_stats(b, conv_stats, x, gamma, beta, nullptr, nullptr, nullptr,
+                                                         mean, invstd, s)
+                             : launch_bn_fwd(b, x, gamma, beta, nullptr, nullptr, nullptr, mean, invstd, ws, s);
+  if (e != cudaSuccess) return e;
+  const int C = b.C;
+  const int P = (H - 1) / 2 + 1, Q = (W - 1) / 2 + 1;
+  const int smem = bn_pool_smem_bytes(W, C);
+  // (opted in once for the largest staging the API accepts, 200 KB, whatever this call's size)
+  static bool attr[64] = {false};
+  if (smem > 200 * 1024) return cudaErrorInvalidValue;
+  e = stat_smem_attr(k_bn_relu_pool_fwd, 200 * 1024, attr);
+  if (e != cudaSuccess) return e;
+  const long long grid = (long long)N * ((P + kBpT - 1) / kBpT);
+  const int threads = 256 - 256 % (C / 8);  // a multiple of the channel groups
+  launch_pdl(k_bn_relu_pool_fwd, dim3((unsigned)grid), dim3(threads), smem, s, x, gamma, beta,
+             static_cast<const uint16_t*>(mean), static_cast<const uint16_t*>(invstd), b.post_scale, pooled, codes,
+             mask, N, H, W, C, P, Q);
   return counted_launches(1);
 }
 

@@ -314,6 +314,14 @@ cudaError_t launch_bn_fwd_given_stats(const BnLaunch& b, const uint8_t* conv_sta
                                       const uint16_t* gamma, const uint16_t* beta,
                                       const uint16_t* residual, uint16_t* y, uint8_t* relu_mask,
                                       uint16_t* mean, uint16_t* invstd, cudaStream_t s);
+// The stem's BatchNorm + ReLU + 3x3 / stride 2 / pad 1 max pooling (x is
+// N x H x W x C; pooled and codes N x P x Q x C, P = (H - 1) / 2 + 1): the
+// statistics as launch_bn_fwd(_given_stats), then one fused pass.
+int bn_pool_smem_bytes(int W, int C);
+cudaError_t launch_bn_relu_pool_fwd(const BnLaunch& b, const uint8_t* conv_stats, const uint16_t* x,
+                                    const uint16_t* gamma, const uint16_t* beta, uint16_t* mean,
+                                    uint16_t* invstd, uint16_t* pooled, uint8_t* codes, uint8_t* mask,
+                                    uint16_t* ws, int N, int H, int W, cudaStream_t s);
 // ReLU decisions from relu_mask when non-null, else from y_saved.
 cudaError_t launch_bn_bwd(const BnLaunch& b, const uint16_t* x, const uint16_t* gamma,
                           const uint16_t* mean, const uint16_t* invstd, const uint16_t* dy,

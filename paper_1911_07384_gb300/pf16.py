@@ -38,7 +38,7 @@ EXPORTS = [
     "pf16_kernel_launches", "pf16_maxpool_fwd_argmax", "pf16_maxpool_bwd_argmax",
     "pf16_conv_bnstats_size", "pf16_conv_fwd_bnstats", "pf16_conv_dgrad_bnstats_size",
     "pf16_conv_dgrad_bnstats", "pf16_conv_dgrad_bnstats_add", "pf16_tc_rate", "pf16_wait_flag",
-    "pf16_conv_fwd_bnin", "pf16_conv_wgrad_bnin",
+    "pf16_conv_fwd_bnin", "pf16_conv_wgrad_bnin", "pf16_bn_relu_maxpool_fwd",
 ]
 
 
@@ -129,6 +129,9 @@ def lib():
             L.pf16_bn_fwd_bwd.argtypes = [ctypes.POINTER(BnDesc), I, ctypes.POINTER(BnTensors), vp,
                                           sz, vp]
             L.pf16_bn_fwd_bwd.restype = I
+            L.pf16_bn_relu_maxpool_fwd.argtypes = [ctypes.POINTER(BnDesc), ctypes.POINTER(BnTensors), vp, vp,
+                                                   vp, sz, vp]
+            L.pf16_bn_relu_maxpool_fwd.restype = I
             L.pf16_maxpool_fwd.argtypes = [vp, vp, i32, i32, i32, i32, vp]
             L.pf16_maxpool_bwd.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
             L.pf16_maxpool_fwd_argmax.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
@@ -300,6 +303,14 @@ def bn_fwd_bwd(d, phase, ws, stream=None, **tensors):
     t = BnTensors(**{k: (v.data_ptr() if v is not None else None) for k, v in tensors.items()})
     _check(lib().pf16_bn_fwd_bwd(ctypes.byref(d), phase, ctypes.byref(t), _ptr(ws), _nbytes(ws),
                                  _stream(stream)), "pf16_bn_fwd_bwd")
+
+
+def bn_relu_maxpool_fwd(d, ws, pooled, argmax, stream=None, **tensors):
+    """The stem's BatchNorm (phase 0, ReLU) with its output max-pooled at once;
+    y is not stored (pass no y).  tensors as bn_fwd_bwd's."""
+    t = BnTensors(**{k: (v.data_ptr() if v is not None else None) for k, v in tensors.items()})
+    _check(lib().pf16_bn_relu_maxpool_fwd(ctypes.byref(d), ctypes.byref(t), _ptr(pooled), _ptr(argmax), _ptr(ws),
+                                          _nbytes(ws), _stream(stream)), "pf16_bn_relu_maxpool_fwd")
 
 
 def maxpool_fwd(x, y, n, h, w, c, stream=None):

@@ -350,7 +350,7 @@ class ResNet50:
     """Buffers and call sequence of one pure-FP16 ResNet-50 training step."""
 
     def __init__(self, batch=256, image=224, classes=1000, device="cuda", seed_cfg=4, hook=None, bn_swap=False,
-                 wgrad_branch=False, exchange=None, bn_in_operand=False):
+                 wgrad_branch=False, exchange=None, bn_in_operand=False, stem_fused=True):
         """wgrad_branch: issue the weight gradients on a second stream that joins
         before the update (in a captured step graph: a parallel branch), so that
         they fill the gaps of the data-gradient chain; off, every call runs on the
@@ -364,8 +364,12 @@ class ResNet50:
         off by default: on GB300 the conv's transform costs more than the
         apply pass it replaces (the 1x1 convs re-transform each operand tile
         once per tile of the other GEMM dimension, and their epilogues already
-        fill the SM's issue slots)."""
+        fill the SM's issue slots).
+        stem_fused: the stem's BatchNorm, ReLU and max pooling forward run as
+        one call (pf16_bn_relu_maxpool_fwd: bit-identical results, the
+        BatchNorm's output never stored)."""
         self.N, self.image, self.classes, self.device = batch, image, classes, device
+        self.stem_fused = stem_fused
         self.hook = hook  # optional callable(kind, layer, fn, *args) used for instrumentation
         self.exchange = exchange
         self.bn_in_operand = bn_in_operand
@@ -407,8 +411,11 @@ class ResNet50:
         h0, hp = self.h0, self.hp
         self.x = e(N, self.image, self.image, 3)
         self.labels = torch.zeros(N, dtype=torch.int32, device=dev)
-        self.a0, self.b0, self.p0 = e(N, h0, h0, 64), e(N, h0, h0, 64), e(N, hp, hp, 64)
-        self.dp0, self.db0, self.da0 = e(N, hp, hp, 64), e(N, h0, h0, 64), e(N, h0, h0, 64)
+        self.a0, self.p0 = e(N, h0, h0, 64), e(N, hp, hp, 64)
+        self.dp0, self.da0 = e(N, hp, hp, 64), e(N, h0, h0, 64)
+        # the stem BatchNorm's output (not stored when fused with the pooling) and its gradient
+        self.b0 = None if self.stem_fused else e(N, h0, h0, 64)
+        self.db0 = e(N, h0, h0, 64)
         # position of each pooling window's maximum, kept from the forward for the backward
         self.pool_arg = torch.empty(N * hp * hp * 64, dtype=torch.uint8, device=dev)
         for b in self.blocks:
@@ -457,9 +464,15 @@ class ResNet50:
 
     def forward(self):
         self.stem.fwd(self.x, self.a0, with_stats=True)
-        self.bn0.fwd(self.a0, self.b0, conv=self.stem)
-        self.call("maxpool_fwd", None, pf16.maxpool_fwd_argmax, self.b0, self.p0, self.pool_arg, self.N,
-                  self.h0, self.h0, 64)
+        if self.stem_fused:
+            b = self.bn0
+            self.call("bn_pool_fwd", b, pf16.bn_relu_maxpool_fwd, b.desc, self.ws, self.p0, self.pool_arg,
+                      x=self.a0, gamma=b.gamma, beta=b.beta, mean=b.mean, invstd=b.invstd, relu_mask=b.mask,
+                      conv_stats=self.stem.stats)
+        else:
+            self.bn0.fwd(self.a0, self.b0, conv=self.stem)
+            self.call("maxpool_fwd", None, pf16.maxpool_fwd_argmax, self.b0, self.p0, self.pool_arg, self.N,
+                      self.h0, self.h0, 64)
         h = self.p0
         for b in self.blocks:
             h = b.forward(h)
@@ -477,6 +490,8 @@ class ResNet50:
         for i in range(len(self.blocks) - 1, -1, -1):
             dx = self.blocks[i - 1].dy if i > 0 else self.dp0
             self.blocks[i].backward(dx, self.blocks[i - 1] if i > 0 else None)
+        # the pooling's backward, then the stem BatchNorm's (ReLU decisions from
+        # its bit mask: with the fused forward its output is not stored)
         self.call("maxpool_bwd", None, pf16.maxpool_bwd_argmax, self.pool_arg, self.dp0, self.db0, self.N,
                   self.h0, self.h0, 64)
         self.bn0.bwd(self.a0, self.b0, self.db0, self.da0)

@@ -69,6 +69,18 @@ def step():
             b.bn2.fwd(b.a2, b.b2, conv=b.conv2)
             torch.cuda.synchronize()
             assert torch.equal(mask, b.bn2.mask)
+    # The stem's BatchNorm + ReLU + max pooling forward runs fused
+    # (pf16_bn_relu_maxpool_fwd), which does not store the BatchNorm's output;
+    # make it with the separate call, bit-identical to the fused one
+    # (tests/test_gpu_stem_fused.py), so that the checks below can read it.
+    # The saved mean, invstd and ReLU mask must come out the same.
+    if net.stem_fused:
+        saved = [net.bn0.mean.clone(), net.bn0.invstd.clone(), net.bn0.mask.clone()]
+        net.b0 = torch.empty_like(net.a0)
+        net.bn0.fwd(net.a0, net.b0, conv=net.stem)
+        torch.cuda.synchronize()
+        for a, b in zip(saved, (net.bn0.mean, net.bn0.invstd, net.bn0.mask)):
+            assert torch.equal(a, b)
     assert pf16.sync_status() == 0
     yield net
     del net
