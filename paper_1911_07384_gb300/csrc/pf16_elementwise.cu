@@ -976,6 +976,11 @@ __global__ void __launch_bounds__(kBnThreads + 32, kBwdCtasPerSm) k_bn_bwd_stats
 }
 
 constexpr int kFinalThreads = 256;
+static_assert(kFinalThreads == kBnStatSlots, "the slot finals load one slot per thread");
+__device__ __forceinline__ uint4 shfl_down4(uint4 v, int d) {
+  return make_uint4(__shfl_down_sync(0xffffffffu, v.x, d), __shfl_down_sync(0xffffffffu, v.y, d),
+                    __shfl_down_sync(0xffffffffu, v.z, d), __shfl_down_sync(0xffffffffu, v.w, d));
+}
 
 // One CTA per group of 8 channels: each thread merges a contiguous run of
 // per-CTA results (loaded together), then the threads are merged in pairs in
@@ -1129,12 +1134,52 @@ __global__ void __launch_bounds__(kFinalThreads)
   __shared__ uint4 smu[kFinalThreads], sv[kFinalThreads];
   __shared__ long long sn[kFinalThreads];
   const int cg = blockIdx.x, t = threadIdx.x;
-  const int S = *reinterpret_cast<const int*>(stats);
   const uint16_t* smean = reinterpret_cast<const uint16_t*>(stats + bnstat_off_mean());
   const uint16_t* svar = reinterpret_cast<const uint16_t*>(stats + bnstat_off_var(C));
   const int* scnt = reinterpret_cast<const int*>(stats + bnstat_off_cnt(C));
+  // slot t's node, loaded before the slot count is known (the buffer holds
+  // kBnStatSlots = kFinalThreads slots, so the loads stay inside it)
+  const uint4 pm = __ldg(reinterpret_cast<const uint4*>(smean + (long long)t * C) + cg);
+  const uint4 pv = __ldg(reinterpret_cast<const uint4*>(svar + (long long)t * C) + cg);
+  const long long pn = __ldg(scnt + t);
+  const int S = *reinterpret_cast<const int*>(stats);
   int sp2 = 1;
   while (sp2 < S) sp2 *= 2;
+  if (sp2 <= kFinalThreads) {
+    // one slot per thread and the same strided tree as below: its levels of
+    // 32 and more in shared memory, the rest by shuffles in warp 0
+    const MV node = t < S ? MV{pm, pv, pn} : MV{zero4(), zero4(), 0ll};
+    smu[t] = node.mu;
+    sv[t] = node.v;
+    sn[t] = node.n;
+    __syncthreads();
+    for (int half = sp2 / 2; half >= 32; half /= 2) {
+      if (t < half) {
+        const MV r = mv_merge(MV{smu[t], sv[t], sn[t]}, MV{smu[t + half], sv[t + half], sn[t + half]});
+        smu[t] = r.mu;
+        sv[t] = r.v;
+        sn[t] = r.n;
+      }
+      __syncthreads();
+    }
+    if (t >= 32) return;
+    MV r{smu[t], sv[t], sn[t]};
+    for (int half = sp2 / 2 < 16 ? sp2 / 2 : 16; half >= 1; half /= 2) {
+      const MV o{shfl_down4(r.mu, half), shfl_down4(r.v, half), __shfl_down_sync(0xffffffffu, r.n, half)};
+      if (t < half) r = mv_merge(r, o);
+    }
+    if (t == 0) {
+      const uint4 ve = add4(r.v, make_uint4(dup2(eps), dup2(eps), dup2(eps), dup2(eps)));
+      uint4 is;
+      const __half2* hv = reinterpret_cast<const __half2*>(&ve);
+      __half2* hi = reinterpret_cast<__half2*>(&is);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) hi[j] = h2rsqrt(hv[j]);
+      reinterpret_cast<uint4*>(mean_out)[cg] = r.mu;
+      reinterpret_cast<uint4*>(invstd_out)[cg] = is;
+    }
+    return;
+  }
   const int nthr = sp2 < kFinalThreads ? sp2 : kFinalThreads;
   const int seg = sp2 / nthr;
   if (t < nthr) {
@@ -1200,11 +1245,45 @@ __global__ void __launch_bounds__(kFinalThreads)
   pdl_wait();
   __shared__ uint4 s1[kFinalThreads], s2[kFinalThreads];
   const int tc = C / 8, cg = blockIdx.x, t = threadIdx.x;
-  const int S = reinterpret_cast<const int*>(stats)[0];
   const uint16_t* sd = reinterpret_cast<const uint16_t*>(stats + bnstat_off_mean());
   const uint16_t* sp = reinterpret_cast<const uint16_t*>(stats + bnstat_off_var(C));
+  // slot t's sums, loaded before the slot count is known (as the forward's final)
+  const uint4 p1 = __ldg(reinterpret_cast<const uint4*>(sd + (long long)t * C) + cg);
+  const uint4 p2 = __ldg(reinterpret_cast<const uint4*>(sp + (long long)t * C) + cg);
+  const int S = reinterpret_cast<const int*>(stats)[0];
   int sp2 = 1;
   while (sp2 < S) sp2 *= 2;
+  if (sp2 <= kFinalThreads) {
+    // one slot per thread and the same strided tree as below: its levels of
+    // 32 and more in shared memory, the rest by shuffles in warp 0
+    s1[t] = t < S ? p1 : zero4();
+    s2[t] = t < S ? p2 : zero4();
+    __syncthreads();
+    for (int half = sp2 / 2; half >= 32; half /= 2) {
+      if (t < half) {
+        s1[t] = add4(s1[t], s1[t + half]);
+        s2[t] = add4(s2[t], s2[t + half]);
+      }
+      __syncthreads();
+    }
+    if (t >= 32) return;
+    uint4 a1 = s1[t], a2 = s2[t];
+    for (int half = sp2 / 2 < 16 ? sp2 / 2 : 16; half >= 1; half /= 2) {
+      const uint4 o1 = shfl_down4(a1, half), o2 = shfl_down4(a2, half);
+      if (t < half) {
+        a1 = add4(a1, o1);
+        a2 = add4(a2, o2);
+      }
+    }
+    if (t == 0) {
+      const uint32_t ratio2 = dup2(ratio), ps = dup2(post_scale);
+      reinterpret_cast<uint4*>(mm)[cg] = ldexp_down4(mul4(a1, ratio2), mean_levels);
+      reinterpret_cast<uint4*>(mm)[tc + cg] = ldexp_down4(mul4(a2, ratio2), mean_levels);
+      reinterpret_cast<uint4*>(dbeta)[cg] = mul4(a1, ps);
+      reinterpret_cast<uint4*>(dgamma)[cg] = mul4(a2, ps);
+    }
+    return;
+  }
   const int nthr = sp2 < kFinalThreads ? sp2 : kFinalThreads;
   const int seg = sp2 / nthr;
   if (t < nthr) {
