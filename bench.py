@@ -765,6 +765,21 @@ def kernel_roofline(pk, reps=10):
             "peak_src": f"{pk['src']} HBM copy"}
 
 
+def one_phase_launch(d):
+    """Whether the library runs a stride-2 data gradient's four stride phases
+    as one launch: every phase has taps, and all share the output grid and
+    the first dy row / column they read (as the library's planner decides)."""
+    if d.stride != 2 or d.r == 1:
+        return False
+
+    def axis(n, k, ph):
+        offs = [(ph + d.pad - r) // 2 for r in range(k) if (ph + d.pad - r) % 2 == 0]
+        return (-(-(n - ph) // 2), min(offs)) if offs else None
+
+    phases = [(axis(d.h, d.r, ph), axis(d.w, d.s, pw)) for ph in (0, 1) for pw in (0, 1)]
+    return all(a is not None and b is not None for a, b in phases) and len(set(phases)) == 1
+
+
 def count_launches(net):
     """Kernels of one step, counted by replaying the call sequence with a hook."""
     from paper_1911_07384_gb300 import pf16
@@ -777,7 +792,7 @@ def count_launches(net):
         stem = d.c == 3
         total += 1 + (1 if stem else 0)                      # fwd (+ the stem's space-to-depth)
         if not stem:
-            phases = d.stride * d.stride if d.r > 1 else 1
+            phases = d.stride * d.stride if d.r > 1 and not one_phase_launch(d) else 1
             total += phases  # dgrad (a strided 1x1 also zero-fills dx, by a memset node)
         ws = pf16.conv_workspace_size(d, pf16.PF16_PASS_WGRAD)
         total += 1 + (1 if ws else 0) + (2 if stem else 0)  # wgrad (+ split-K reduce, + the stem's s2d, scatter)
@@ -850,7 +865,8 @@ def conv_roofline(net, stream, reps=3):
         # gradients of other kernels (k_stem_wgrad, k_wgrad3x3_halo)
         wg = wgrad_is_gemm(d.h, d.w, d.c, d.k, d.r, d.s, d.stride, d.pad)
         byts += one * ((1 if stem else 2) + (1 if wg else 0))
-        gemms += 1 + (0 if stem else (d.stride * d.stride if d.r > 1 else 1)) + (1 if wg else 0)
+        dg = 1 if d.r == 1 or one_phase_launch(d) else d.stride * d.stride
+        gemms += 1 + (0 if stem else dg) + (1 if wg else 0)
     out = {"ms": ms, "gflop": gflop, "tflops": gflop / ms, "by_pass": {}, "bytes_per_launch": byts / gemms}
     for k, (t, f) in by_pass.items():
         out["by_pass"][k] = {"ms": t / reps, "tflops": (f / reps) / 1e9 / (t / reps) if t else None}

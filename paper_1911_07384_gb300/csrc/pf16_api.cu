@@ -515,6 +515,73 @@ void set_stats(GemmParams& p, void* stats, long long C) {
   p.st_cnt = reinterpret_cast<int*>(b + bnstat_off_cnt(C));
 }
 
+// Every stride phase of a stride-2 data gradient in one launch, when the four
+// phases share their output grid and im2col origin (even H and W with the
+// usual padding: the ResNet layers) and reach every position.  The units are
+// ordered by phase, the phases by falling tap count, so that the round-robin
+// schedule ends on the shortest tiles.  PF16_ERR_UNSUPPORTED: the phases
+// differ; the caller launches them one by one.
+int run_dgrad_phases(const Shape& s, const uint16_t* dy, const uint16_t* w, uint16_t* dx, int* status, int sms,
+                     cudaStream_t st, bool f32, bool accum, int BN) {
+  Phase f[4];
+  int order[4] = {0, 1, 2, 3}, taps = 0;
+  for (int q = 0; q < 4; ++q) {
+    f[q] = make_phase(s, q >> 1, q & 1);
+    if (f[q].empty()) return PF16_ERR_UNSUPPORTED;
+    taps += f[q].nr * f[q].ns;
+  }
+  if (taps > kMaxTaps) return PF16_ERR_UNSUPPORTED;
+  const int amin = *std::min_element(f[0].ar, f[0].ar + f[0].nr), bmin = *std::min_element(f[0].bs, f[0].bs + f[0].ns);
+  for (int q = 1; q < 4; ++q) {
+    const int a = *std::min_element(f[q].ar, f[q].ar + f[q].nr), b = *std::min_element(f[q].bs, f[q].bs + f[q].ns);
+    if (f[q].gh != f[0].gh || f[q].gw != f[0].gw || a != amin || b != bmin) return PF16_ERR_UNSUPPORTED;
+  }
+  std::stable_sort(order, order + 4, [&](int x, int y) { return f[x].nr * f[x].ns > f[y].nr * f[y].ns; });
+  const int gh = f[0].gh, gw = f[0].gw;
+  GemmParams p = base_params(status);
+  p.d_f32 = f32 ? 1 : 0;
+  CUtensorMap ma, mb;
+  p.M = (int)(s.N * gh * gw);
+  p.N = (int)s.C;
+  p.a_mode = LD_IM2COL_K;
+  p.b_mode = LD_TAP3D_MN;
+  set_kmajor(p, true, false);
+  set_mnmajor(p, false, true);
+  p.ga = PixGrid{gh, gw, 1, amin, bmin};
+  if (!map_im2col(&ma, dy, (int)s.N, (int)s.P, (int)s.Q, (int)s.K, amin, bmin, gh, gw, 1, kBM))
+    return PF16_ERR_CUDA;
+  if (!map_3d(&mb, w, s.C, s.R * s.S, s.K, s.C * 2, s.R * s.S * s.C * 2, 64, 1, 64)) return PF16_ERR_CUDA;
+  p.a_cpt = p.b_cpt = (int)(s.K / 64);
+  int t = 0;
+  for (int k = 0; k < 4; ++k) {
+    const Phase& g = f[order[k]];
+    p.ph_kb[k] = t * p.a_cpt;
+    p.ph_h[k] = (int8_t)(order[k] >> 1);
+    p.ph_w[k] = (int8_t)(order[k] & 1);
+    for (int i = 0; i < g.nr; ++i)
+      for (int j = 0; j < g.ns; ++j, ++t) {
+        p.tap_dr[t] = (int8_t)(g.ar[i] - amin);
+        p.tap_ds[t] = (int8_t)(g.bs[j] - bmin);
+        p.tap_w[t] = (int8_t)(g.rr[i] * s.S + g.ss[j]);
+      }
+  }
+  p.ph_kb[4] = t * p.a_cpt;
+  p.ntaps = t;
+  p.num_kb = p.ph_kb[4];
+  p.nphase = 4;
+  p.splits = 4;
+  p.out = dx;
+  p.ldo = s.C;
+  p.out_mode = accum ? OUT_ACCUM : OUT_STORE;
+  p.remap = 1;
+  p.rm_gh = gh;
+  p.rm_gw = gw;
+  p.rm_H = (int)s.H;
+  p.rm_W = (int)s.W;
+  p.rm_step = 2;
+  return run(BN, ma, mb, p, sms, st);
+}
+
 int check_common(const void* a, const void* b, const void* c) {
   if (!a || !b || !c) return PF16_ERR_NULL;
   if (!aligned16(a) || !aligned16(b) || !aligned16(c)) return PF16_ERR_ALIGN;
@@ -960,6 +1027,10 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
   bool any_empty = false;
   for (int ph = 0; ph < s.st; ++ph)
     for (int pw = 0; pw < s.st; ++pw) any_empty |= make_phase(s, ph, pw).empty();
+  if (s.st == 2 && !any_empty) {
+    const int rc2 = run_dgrad_phases(s, dy, w, dx, status, sms, st, f32, accum, BN);
+    if (rc2 != PF16_ERR_UNSUPPORTED) return rc2;
+  }
   if (any_empty && !accum && launch_fill_zero(dx, dx_elems, st) != cudaSuccess)
     return PF16_ERR_CUDA;
   for (int ph = 0; ph < s.st; ++ph)

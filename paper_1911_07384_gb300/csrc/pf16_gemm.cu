@@ -192,8 +192,13 @@ __device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0,
   const int mt = rem / p.n_tiles;
   m0 = mt * kBM;
   n0 = (rem - mt * p.n_tiles) * BN;
-  kb0 = split * p.kb_per_split;
-  kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+  if (p.nphase > 1) {  // the split index is the stride phase
+    kb0 = p.ph_kb[split];
+    kb1 = p.ph_kb[split + 1];
+  } else {
+    kb0 = split * p.kb_per_split;
+    kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+  }
 }
 
 __device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int split) {
@@ -205,8 +210,8 @@ __device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int spl
     const int n = m / per;
     const int rem = m - n * per;
     const int i = rem / p.rm_gw, j = rem - (rem / p.rm_gw) * p.rm_gw;
-    row = ((long long)n * p.rm_H + (long long)(i * p.rm_step + p.rm_ph)) * p.rm_W +
-          (j * p.rm_step + p.rm_pw);
+    const int ph = p.nphase > 1 ? p.ph_h[split] : p.rm_ph, pw = p.nphase > 1 ? p.ph_w[split] : p.rm_pw;
+    row = ((long long)n * p.rm_H + (long long)(i * p.rm_step + ph)) * p.rm_W + (j * p.rm_step + pw);
   } else {
     row = m;
   }
@@ -678,7 +683,6 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
     // epilogue warps 2..9 (2..17 with WE) -> TMEM sub-partitions 2, 3, 0, 1, ...; group grp
     // drains accumulator grp & 1, columns [c_begin, c_end) (the whole tile, or half of it)
     const int e = warp - 2, grp = e >> 2, sub = warp & 3;
-    const int row = sub * 32 + lane;
     const int acc = grp & 1;
     const int c_begin = WE ? (grp >> 1) * (BN / CS) : 0, c_end = c_begin + BN / CS;
     uint32_t acc_phase = 0;
@@ -759,42 +763,68 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
         acc_phase ^= 1;
         continue;
       }
-      const int m = m0 + row;
-      const bool row_ok = m < p.M;
-      uint16_t* orow = row_ok ? out_row(p, m, split) : nullptr;
+      // Rows remapped to strided positions (a stride phase): each 64-column
+      // chunk goes through the warp's 128B-swizzled staging tile, then lane l
+      // moves 16 bytes (columns 8 (l % 8) ..) of rows l / 8 + 4 i, i < 8: a
+      // warp instruction writes four whole 128-byte row segments.
+      const int rq = lane >> 3, cj = lane & 7;
+      uint16_t* orow[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int m = m0 + sub * 32 + rq + 4 * i;
+        orow[i] = m < p.M ? out_row(p, m, split) : nullptr;
+      }
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        uint32_t r[32];
+      for (int c = 0; c < BN; c += 64) {
+        uint32_t r[64];
         tmem_ld16(tbase + c, r);
         tmem_ld16(tbase + c + 16, r + 16);
+        tmem_ld16(tbase + c + 32, r + 32);
+        tmem_ld16(tbase + c + 48, r + 48);
         tmem_ld_wait();
-        if (p.d_f32) f32_to_f16_lo<32>(r);  // FP32 accumulator: one rounding to FP16
-        if (row_ok) {
+        if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
+        if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+        }
+        __syncwarp();  // every lane is done reading the previous chunk from the staging tile
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            const int n = n0 + c + g * 8;
-            if (n + 8 <= p.N) {
-              uint4 v;
-              v.x = pack_lo(r[g * 8 + 0], r[g * 8 + 1]);
-              v.y = pack_lo(r[g * 8 + 2], r[g * 8 + 3]);
-              v.z = pack_lo(r[g * 8 + 4], r[g * 8 + 5]);
-              v.w = pack_lo(r[g * 8 + 6], r[g * 8 + 7]);
-              uint4* dst = reinterpret_cast<uint4*>(orow + n);
-              if (p.out_mode == OUT_ACCUM) {
-                const uint4 o = *dst;
-                v.x = hadd2_rn(o.x, v.x);
-                v.y = hadd2_rn(o.y, v.y);
-                v.z = hadd2_rn(o.z, v.z);
-                v.w = hadd2_rn(o.w, v.w);
-              }
-              *dst = v;
+        for (int j = 0; j < 8; ++j) {
+          uint4 v;
+          v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
+          v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
+          v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
+          v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
+          st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
+        }
+        __syncwarp();
+        const int n = n0 + c + 8 * cj;
+        if (n + 8 <= p.N) {
+          uint4 v[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int rr = rq + 4 * i;
+            ld_shared_v4(stg + rr * 128 + ((cj ^ (rr & 7)) << 4), v[i]);
+          }
+          if (p.out_mode == OUT_ACCUM) {
+            uint4 o[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              o[i] = orow[i] ? *reinterpret_cast<const uint4*>(orow[i] + n) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              v[i].x = hadd2_rn(o[i].x, v[i].x);
+              v[i].y = hadd2_rn(o[i].y, v[i].y);
+              v[i].z = hadd2_rn(o[i].z, v[i].z);
+              v[i].w = hadd2_rn(o[i].w, v[i].w);
             }
           }
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (orow[i]) *reinterpret_cast<uint4*>(orow[i] + n) = v[i];
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
       acc_phase ^= 1;
     }
     if (p.tma_store && lane == 0) bulk_wait0();

@@ -102,6 +102,13 @@ struct GemmParams {
   long long ldo;          // output row stride (elements)
   int remap;              // rows -> strided positions of a stride phase
   int rm_gh, rm_gw, rm_H, rm_W, rm_step, rm_ph, rm_pw;
+  // All stride phases of a data gradient in one launch (nphase > 1, with
+  // remap and splits = nphase): a unit's split index is its phase f, whose
+  // K-blocks are [ph_kb[f], ph_kb[f + 1]) of the phases' concatenated tap
+  // lists and whose rows land at (i * rm_step + ph_h[f], j * rm_step + ph_w[f]).
+  int nphase;
+  int ph_kb[5];
+  int8_t ph_h[4], ph_w[4];
   // MMA
   uint32_t idesc;
   int d_f32;              // FP32 accumulator in TMEM (PF16_F32_ACCUM), rounded once to FP16 in the epilogue

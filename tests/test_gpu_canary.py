@@ -43,6 +43,7 @@ def intact_ws(buf, nbytes):
 SHAPES = [
     (1, 7, 7, 64, 64, 3, 3, 1, 1),       # halo engine, one partial tile
     (2, 9, 9, 64, 128, 3, 3, 2, 1),      # strided 3x3, unequal stride phases
+    (3, 10, 12, 128, 64, 3, 3, 2, 1),    # strided 3x3, even size: the four phases in one launch
     (2, 13, 13, 128, 256, 1, 1, 2, 0),   # strided 1x1
     (3, 10, 10, 192, 320, 3, 3, 1, 1),   # partial N tile
     (2, 31, 29, 3, 64, 7, 7, 2, 3),      # stem, odd H and W

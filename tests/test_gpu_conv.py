@@ -21,6 +21,8 @@ SHAPES = [
     (3, 16, 30, 64, 64, 3, 3, 1, 1),     # halo engine, W + 2 = 32 exactly
     (1, 7, 7, 64, 64, 3, 3, 1, 1),       # one partial M tile
     (2, 9, 9, 64, 128, 3, 3, 2, 1),      # strided 3x3, odd size: unequal stride phases
+    (3, 14, 14, 128, 128, 3, 3, 2, 1),   # strided 3x3, even size: the four phases in one launch, ragged M tile
+    (2, 10, 12, 192, 64, 3, 3, 2, 1),    # the same with H != W and a partial N tile
     (2, 14, 14, 256, 64, 1, 1, 1, 0),    # 1x1 GEMM
     (2, 14, 14, 64, 256, 1, 1, 1, 0),
     (2, 13, 13, 128, 256, 1, 1, 2, 0),   # strided 1x1 projection, odd size
@@ -122,6 +124,7 @@ def test_stem_full_width_sampled(orc):
 
 @pytest.mark.parametrize("shape", [(2, 9, 9, 64, 128, 3, 3, 1, 1), (2, 10, 10, 64, 64, 1, 1, 2, 0),
                                    (2, 11, 11, 64, 64, 3, 3, 2, 1), (2, 12, 10, 64, 64, 3, 3, 1, 1),
+                                   (2, 12, 12, 64, 64, 3, 3, 2, 1),
                                    (2, 32, 32, 3, 64, 7, 7, 2, 3)],
                          ids=ids)
 def test_accumulate_flag(orc, shape):
