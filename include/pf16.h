@@ -126,10 +126,14 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
  * The CTAs' nodes go to `stats` (stats_bytes >= pf16_conv_dgrad_bnstats_size(d),
  * 16-byte aligned, caller-owned, no initial contents needed);
  * pf16_bn_fwd_bwd phase 1 takes it through pf16_bn_tensors.conv_stats and
- * skips its statistics pass over dy and x.  Requires stride 1 (dx rows in
- * pixel order) and c a multiple of 64 (PF16_ERR_UNSUPPORTED otherwise; the
- * size function then returns 0); x, mean, invstd 16-byte aligned, relu_mask
- * 8-byte aligned. */
+ * skips its statistics pass over dy and x.  Requires c a multiple of 64 and
+ * either stride 1 or a stride-2 filter larger than 1x1 whose four stride
+ * phases all receive taps and share their output grid and first dy row and
+ * column (for 3x3 with pad 1: even h and w, as in ResNet; the phases then run
+ * as one GEMM whose rows land at scattered pixels, and the warps' rows are
+ * those rows);
+ * PF16_ERR_UNSUPPORTED otherwise, and the size function then returns 0.
+ * x, mean, invstd 16-byte aligned, relu_mask 8-byte aligned. */
 typedef struct {
   const uint16_t* x;         /* the BatchNorm's input, n x h x w x c */
   const uint8_t* relu_mask;  /* its ReLU decisions (bit mask), or NULL: no ReLU */

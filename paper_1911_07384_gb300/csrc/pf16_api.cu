@@ -479,11 +479,17 @@ int run(int BN, const CUtensorMap& a, const CUtensorMap& b, GemmParams& p, int s
   }
   // backward statistics: the BatchNorm input (and the addend) enter the
   // epilogue as TMA tiles of the output's 32 x 64 boxes
+  // (remapped rows -- a stride phase -- read it by plain loads instead)
   CUtensorMap mx = c, md = c;
   if (p.bs_x) {
-    if (!p.tma_store || p.out_mode != OUT_STORE) return PF16_ERR_UNSUPPORTED;
-    if (!map_2d(&mx, p.bs_x, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
-    if (p.add_src && !map_2d(&md, p.add_src, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+    if (p.out_mode != OUT_STORE) return PF16_ERR_UNSUPPORTED;
+    if (p.remap) {
+      if (p.add_src) return PF16_ERR_UNSUPPORTED;
+    } else {
+      if (!p.tma_store) return PF16_ERR_UNSUPPORTED;
+      if (!map_2d(&mx, p.bs_x, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+      if (p.add_src && !map_2d(&md, p.add_src, p.N, p.M, p.ldo, 64, 32)) return PF16_ERR_CUDA;
+    }
   }
   int grid = (int)std::min<long long>(units, sms);
   if (p.st_mean) {
@@ -521,25 +527,38 @@ void set_stats(GemmParams& p, void* stats, long long C) {
 // ordered by phase, the phases by falling tap count, so that the round-robin
 // schedule ends on the shortest tiles.  PF16_ERR_UNSUPPORTED: the phases
 // differ; the caller launches them one by one.
-int run_dgrad_phases(const Shape& s, const uint16_t* dy, const uint16_t* w, uint16_t* dx, int* status, int sms,
-                     cudaStream_t st, bool f32, bool accum, int BN) {
-  Phase f[4];
-  int order[4] = {0, 1, 2, 3}, taps = 0;
+bool phases_one_launch(const Shape& s, Phase* f = nullptr) {
+  Phase g[4];
+  if (!f) f = g;
+  if (s.kind == KIND_STEM || s.st != 2 || (s.R == 1 && s.S == 1)) return false;
+  int taps = 0;
   for (int q = 0; q < 4; ++q) {
     f[q] = make_phase(s, q >> 1, q & 1);
-    if (f[q].empty()) return PF16_ERR_UNSUPPORTED;
+    if (f[q].empty()) return false;
     taps += f[q].nr * f[q].ns;
   }
-  if (taps > kMaxTaps) return PF16_ERR_UNSUPPORTED;
+  if (taps > kMaxTaps) return false;
   const int amin = *std::min_element(f[0].ar, f[0].ar + f[0].nr), bmin = *std::min_element(f[0].bs, f[0].bs + f[0].ns);
   for (int q = 1; q < 4; ++q) {
     const int a = *std::min_element(f[q].ar, f[q].ar + f[q].nr), b = *std::min_element(f[q].bs, f[q].bs + f[q].ns);
-    if (f[q].gh != f[0].gh || f[q].gw != f[0].gw || a != amin || b != bmin) return PF16_ERR_UNSUPPORTED;
+    if (f[q].gh != f[0].gh || f[q].gw != f[0].gw || a != amin || b != bmin) return false;
   }
+  return true;
+}
+
+int run_dgrad_phases(const Shape& s, const uint16_t* dy, const uint16_t* w, uint16_t* dx, int* status, int sms,
+                     cudaStream_t st, bool f32, bool accum, int BN, void* stats = nullptr,
+                     const pf16_bn_source* bn = nullptr) {
+  Phase f[4];
+  int order[4] = {0, 1, 2, 3};
+  if (!phases_one_launch(s, f)) return PF16_ERR_UNSUPPORTED;
+  const int amin = *std::min_element(f[0].ar, f[0].ar + f[0].nr), bmin = *std::min_element(f[0].bs, f[0].bs + f[0].ns);
   std::stable_sort(order, order + 4, [&](int x, int y) { return f[x].nr * f[x].ns > f[y].nr * f[y].ns; });
   const int gh = f[0].gh, gw = f[0].gw;
   GemmParams p = base_params(status);
   p.d_f32 = f32 ? 1 : 0;
+  set_stats(p, stats, s.C);  // the four phases together cover every pixel once
+  if (stats) set_bwd_stats(p, bn);
   CUtensorMap ma, mb;
   p.M = (int)(s.N * gh * gw);
   p.N = (int)s.C;
@@ -963,7 +982,7 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
     if (!aligned16(stats) || !aligned16(bn->x) || !aligned16(bn->mean) || !aligned16(bn->invstd) ||
         (reinterpret_cast<uintptr_t>(bn->relu_mask) & 7u) != 0)
       return PF16_ERR_ALIGN;
-    if (s.C % 64 != 0 || s.st != 1) return PF16_ERR_UNSUPPORTED;
+    if (s.C % 64 != 0 || (s.st != 1 && !phases_one_launch(s))) return PF16_ERR_UNSUPPORTED;
     if (stats_bytes < bnstat_bytes(s.C)) return PF16_ERR_WORKSPACE;
   }
   if (add) {
@@ -1027,10 +1046,7 @@ static int conv_dgrad_impl(const pf16_conv_desc* d, const uint16_t* dy, const ui
   bool any_empty = false;
   for (int ph = 0; ph < s.st; ++ph)
     for (int pw = 0; pw < s.st; ++pw) any_empty |= make_phase(s, ph, pw).empty();
-  if (s.st == 2 && !any_empty) {
-    const int rc2 = run_dgrad_phases(s, dy, w, dx, status, sms, st, f32, accum, BN);
-    if (rc2 != PF16_ERR_UNSUPPORTED) return rc2;
-  }
+  if (phases_one_launch(s)) return run_dgrad_phases(s, dy, w, dx, status, sms, st, f32, accum, BN, stats, bn);
   if (any_empty && !accum && launch_fill_zero(dx, dx_elems, st) != cudaSuccess)
     return PF16_ERR_CUDA;
   for (int ph = 0; ph < s.st; ++ph)
@@ -1090,7 +1106,8 @@ int pf16_conv_dgrad(const pf16_conv_desc* d, const uint16_t* dy, const uint16_t*
 
 size_t pf16_conv_dgrad_bnstats_size(const pf16_conv_desc* d) {
   Shape s;
-  if (conv_shape(d, &s) != PF16_OK || s.kind == KIND_STEM || s.C % 64 != 0 || s.st != 1) return 0;
+  if (conv_shape(d, &s) != PF16_OK || s.kind == KIND_STEM || s.C % 64 != 0) return 0;
+  if (s.st != 1 && !phases_one_launch(s)) return 0;
   return bnstat_bytes(s.C);
 }
 

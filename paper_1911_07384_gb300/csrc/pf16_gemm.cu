@@ -201,17 +201,23 @@ __device__ __forceinline__ void unit_decode(const GemmParams& p, int u, int& m0,
   }
 }
 
+// Pixel row of GEMM row m of a stride phase (remap): grid point (n, i, j) ->
+// (n, i * step + ph, j * step + pw).
+__device__ __forceinline__ long long remap_row(const GemmParams& p, int m, int split) {
+  const int per = p.rm_gh * p.rm_gw;
+  const int n = m / per;
+  const int rem = m - n * per;
+  const int i = rem / p.rm_gw, j = rem - (rem / p.rm_gw) * p.rm_gw;
+  const int ph = p.nphase > 1 ? p.ph_h[split] : p.rm_ph, pw = p.nphase > 1 ? p.ph_w[split] : p.rm_pw;
+  return ((long long)n * p.rm_H + (long long)(i * p.rm_step + ph)) * p.rm_W + (j * p.rm_step + pw);
+}
+
 __device__ __forceinline__ uint16_t* out_row(const GemmParams& p, int m, int split) {
   long long row;
   if (p.out_mode == OUT_PARTIAL) {
     row = (long long)split * p.M + m;
   } else if (p.remap) {
-    const int per = p.rm_gh * p.rm_gw;
-    const int n = m / per;
-    const int rem = m - n * per;
-    const int i = rem / p.rm_gw, j = rem - (rem / p.rm_gw) * p.rm_gw;
-    const int ph = p.nphase > 1 ? p.ph_h[split] : p.rm_ph, pw = p.nphase > 1 ? p.ph_w[split] : p.rm_pw;
-    row = ((long long)n * p.rm_H + (long long)(i * p.rm_step + ph)) * p.rm_W + (j * p.rm_step + pw);
+    row = remap_row(p, m, split);
   } else {
     row = m;
   }
@@ -227,10 +233,13 @@ struct ChunkIn {
   uint2 m, am;
   uint32_t mu2, is2;
 
+  // row0: the tile's first row; prow >= 0: instead, the pixel row of row `lane`
+  // (scattered rows of a stride phase), -1 past the tensor
   template <bool ADD>
-  __device__ __forceinline__ void load(const GemmParams& p, long long row0, int col0, int lane) {
-    const long long r = row0 + lane;
-    const bool in = r < p.M;
+  __device__ __forceinline__ void load(const GemmParams& p, long long row0, int col0, int lane,
+                                       long long prow = -2) {
+    const long long r = prow == -2 ? row0 + lane : prow;
+    const bool in = prow == -2 ? r < p.M : prow >= 0;
     const long long mo = r * (p.N / 8) + col0 / 8;
     m = make_uint2(0xFFFFFFFFu, 0xFFFFFFFFu);
     if (p.bs_mask && in) m = __ldg(reinterpret_cast<const uint2*>(p.bs_mask + mo));
@@ -251,16 +260,22 @@ struct ChunkIn {
 // (ChunkIn) are loaded as far ahead.  With ADD the chunk's output is
 // rn(result + addend) where the addend's mask bit is set (rn(result + 0)
 // elsewhere), and the statistics are taken of that sum.
-template <int BN, bool ADD>
+// REMAP (rows at the scattered pixels of a stride phase; no ADD): every lane
+// fetches 16-byte pieces of x's rows with cp.async into the swizzled X[b]
+// (the barrier then expects 32 arrivals), and the chunk leaves S[b] by plain
+// stores of whole 128-byte row segments instead of a TMA store.
+template <int BN, bool ADD, bool REMAP>
 __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorMap* mapC, const CUtensorMap* mapX,
                                             const CUtensorMap* mapD, uint8_t* wbuf, uint64_t* wbar,
                                             uint64_t* tfull, uint64_t* tempty, uint32_t tmem_base, int acc, int sub,
                                             int lane, int u0, int ustep, int total, uint64_t lim,
                                             volatile int* abort_flag, EpiStats& stats) {
+  static_assert(!(ADD && REMAP), "the addend's rows are in pixel order");
   if (u0 >= total) return;
   const uint32_t S0 = smem_u32(wbuf), X0 = S0 + 2 * 4096;
   const uint32_t B0 = smem_u32(wbar);
   const uint32_t tx = ADD ? 2 * 4096 : 4096;
+  const int rq = lane >> 3, cj = lane & 7;  // REMAP: rows rq + 4 i, 16-byte column cj
   // lane 0: the chunk index whose loads are in flight in each buffer (-1: none)
   int pend[2] = {-1, -1};
   auto issue = [&](int b, int row0, int col0, int q) {
@@ -269,12 +284,35 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
     if (ADD) tma_load_2d(S0 + b * 4096, mapD, B0 + 8 * b, col0, row0);
     pend[b] = q;
   };
+  // REMAP, all lanes: rows of the chunk whose row `lane` is at pixel row prow (-1: past the tensor)
+  auto issue_rows = [&](int b, long long prow, int col0, int q) {
+    const uint32_t xb = X0 + b * 4096;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int rr = rq + 4 * i;
+      const long long pr = __shfl_sync(0xffffffffu, prow, rr);
+      if (pr >= 0) cp_async_16(xb + rr * 128 + ((cj ^ (rr & 7)) << 4), p.bs_x + pr * p.ldo + col0 + 8 * cj);
+    }
+    cp_async_mbar_arrive_noinc(B0 + 8 * b);
+    if (lane == 0) pend[b] = q;
+  };
+  // REMAP: the pixel row of row `lane` of the tile at m (-1 past the tensor)
+  auto pixel_row = [&](int m, int sp) -> long long {
+    const int mr = m + sub * 32 + lane;
+    return mr < p.M ? remap_row(p, mr, sp) : -1ll;
+  };
   int u = u0, m0, n0, split, kb0, kb1;
   unit_decode(p, u, m0, n0, split, kb0, kb1, BN);
   int c = 0;
-  if (lane == 0) issue(0, m0 + sub * 32, n0, 0);
+  long long prow = 0, prow2 = 0;
+  if constexpr (REMAP) {
+    prow = pixel_row(m0, split);
+    issue_rows(0, prow, n0, 0);
+  } else if (lane == 0) {
+    issue(0, m0 + sub * 32, n0, 0);
+  }
   ChunkIn cur, nxt;
-  cur.load<ADD>(p, (long long)(m0 + sub * 32), n0, lane);
+  cur.load<ADD>(p, (long long)(m0 + sub * 32), n0, lane, REMAP ? prow : -2);
   uint32_t acc_phase = 0, tbase = 0;
   int nv = 0;
   for (int q = 0;; ++q) {
@@ -301,12 +339,15 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
     const bool more = u2 < total;
     if (more) {
       __syncwarp();  // every lane is done reading buffer b ^ 1 (chunk q - 1)
-      if (lane == 0) {
+      if constexpr (REMAP) {
+        prow2 = last ? pixel_row(m2, split) : prow;
+        issue_rows(b ^ 1, prow2, n2 + c2, q + 1);
+      } else if (lane == 0) {
         bulk_wait_read0();         // chunk q - 1's store has read S[b ^ 1]
         fence_proxy_async_smem();  // the warp's reads of X[b ^ 1] before the copy's writes
         issue(b ^ 1, m2 + sub * 32, n2 + c2, q + 1);
       }
-      nxt.load<ADD>(p, (long long)(m2 + sub * 32), n2 + c2, lane);
+      nxt.load<ADD>(p, (long long)(m2 + sub * 32), n2 + c2, lane, REMAP ? prow2 : -2);
     }
     uint32_t r[64];
     tmem_ld16(tbase + c, r);
@@ -350,11 +391,24 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
       }
       st_shared_v4(addr, v);
     }
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      tma_store_2d(mapC, S, n0 + c, m0 + sub * 32);
-      bulk_commit();
+    if constexpr (REMAP) {
+      __syncwarp();
+      const int n = n0 + c + 8 * cj;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = rq + 4 * i;
+        const long long pr = __shfl_sync(0xffffffffu, prow, rr);
+        uint4 v;
+        ld_shared_v4(S + rr * 128 + ((cj ^ (rr & 7)) << 4), v);
+        if (pr >= 0 && n + 8 <= p.N) *reinterpret_cast<uint4*>(p.out + pr * p.ldo + n) = v;
+      }
+    } else {
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(mapC, S, n0 + c, m0 + sub * 32);
+        bulk_commit();
+      }
     }
     if (p.st_mean && nv > 0) stats.leaf_bwd_tile(c / 64, S, X, lane, nv, cur.m, cur.mu2, cur.is2);
     if (last) {
@@ -363,6 +417,7 @@ __device__ __forceinline__ void epilogue_bs(const GemmParams& p, const CUtensorM
     }
     if (!more) break;
     cur = nxt;
+    prow = prow2;
     u = u2;
     c = c2;
     m0 = m2;
@@ -463,6 +518,8 @@ __device__ __forceinline__ void xf_rows(const GemmParams& p, const XfParams& q, 
 //   EPI_BS_TMA: the same statistics from TMA-fed tiles (epilogue_bs; for short
 //     reductions, whose epilogue is the bound);
 //   EPI_BS_ADD: EPI_BS_TMA plus the addend (GemmParams::add_src).
+//   EPI_BS_REMAP: EPI_BS_TMA for the scattered rows of a stride phase (x by
+//     cp.async, the output by plain stores).
 // XF (with EPI_PLAIN): BatchNorm in the operand path (GemmParams::xf_*):
 // eight more warps transform each stage between the TMA's arrival (full) and
 // the MMAs (xready), see xf_rows.
@@ -473,7 +530,8 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
     k_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
            const __grid_constant__ CUtensorMap mapC, const __grid_constant__ CUtensorMap mapX,
            const __grid_constant__ CUtensorMap mapD, const __grid_constant__ GemmParams p) {
-  constexpr bool BS = EPI != EPI_PLAIN, TMAE = EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, ADD = EPI == EPI_BS_ADD;
+  constexpr bool BS = EPI != EPI_PLAIN, ADD = EPI == EPI_BS_ADD, REMAP = EPI == EPI_BS_REMAP;
+  constexpr bool TMAE = EPI == EPI_BS_TMA || ADD || REMAP;
   static_assert(!WE || (EPI == EPI_PLAIN && !XF && BN % 128 == 0), "the wide epilogue: plain, BN 128 or 256");
   using Cfg = GemmCfg<BN, TMAE, XF, WE>;
   constexpr int CS = WE ? 2 : 1;  // column halves per tile
@@ -501,7 +559,8 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
       mbar_init(smem_u32(&tfull[a]), 1);
       mbar_init(smem_u32(&tempty[a]), 4 * CS);  // every warp that drains the accumulator arrives
     }
-    for (int b = 0; b < Cfg::EBARS; ++b) mbar_init(smem_u32(&ebar[b]), 1);
+    // (a stride phase's x rows arrive by every lane's cp.async: 32 arrivals)
+    for (int b = 0; b < Cfg::EBARS; ++b) mbar_init(smem_u32(&ebar[b]), REMAP ? 32 : 1);
     if (XF)
       for (int s = 0; s < Cfg::STAGES; ++s) mbar_init(smem_u32(&xready[s]), kXfWarps);
     *abort_flag = 0;
@@ -690,9 +749,9 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
     EpiStats stats;
     stats.init();
     // tcgen05.ld is warp-collective: every exit decision below is warp-uniform
-    if constexpr (TMAE)  // (the host launches these only with TMA stores of rows in pixel order)
-      epilogue_bs<BN, ADD>(p, &mapC, &mapX, &mapD, staging + e * Cfg::WARP_BUF, ebar + 2 * e, tfull, tempty,
-                           tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, lim, abort_flag, stats);
+    if constexpr (TMAE)  // (rows in pixel order with TMA stores, or the scattered rows of a stride phase)
+      epilogue_bs<BN, ADD, REMAP>(p, &mapC, &mapX, &mapD, staging + e * Cfg::WARP_BUF, ebar + 2 * e, tfull, tempty,
+                                  tmem_base, acc, sub, lane, cid + grp * ncl, 2 * ncl, total, lim, abort_flag, stats);
     const bool bstats = BS && p.st_mean && p.bs_x && p.tma_store;
     BwdIn bin;
     for (int u = cid + acc * ncl; u < total && !TMAE; u += 2 * ncl) {
@@ -763,66 +822,68 @@ __global__ void __launch_bounds__(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide :
         acc_phase ^= 1;
         continue;
       }
-      // Rows remapped to strided positions (a stride phase): each 64-column
-      // chunk goes through the warp's 128B-swizzled staging tile, then lane l
-      // moves 16 bytes (columns 8 (l % 8) ..) of rows l / 8 + 4 i, i < 8: a
-      // warp instruction writes four whole 128-byte row segments.
-      const int rq = lane >> 3, cj = lane & 7;
-      uint16_t* orow[8];
+      if constexpr (!XF) {  // (the operand-transform variants never take remapped rows)
+        // Rows remapped to strided positions (a stride phase): each 64-column
+        // chunk goes through the warp's 128B-swizzled staging tile, then lane l
+        // moves 16 bytes (columns 8 (l % 8) ..) of rows l / 8 + 4 i, i < 8: a
+        // warp instruction writes four whole 128-byte row segments.
+        const int rq = lane >> 3, cj = lane & 7;
+        uint16_t* orow[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int m = m0 + sub * 32 + rq + 4 * i;
-        orow[i] = m < p.M ? out_row(p, m, split) : nullptr;
-      }
+        for (int i = 0; i < 8; ++i) {
+          const int m = m0 + sub * 32 + rq + 4 * i;
+          orow[i] = m < p.M ? out_row(p, m, split) : nullptr;
+        }
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 64) {
-        uint32_t r[64];
-        tmem_ld16(tbase + c, r);
-        tmem_ld16(tbase + c + 16, r + 16);
-        tmem_ld16(tbase + c + 32, r + 32);
-        tmem_ld16(tbase + c + 48, r + 48);
-        tmem_ld_wait();
-        if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
-        if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
-        }
-        __syncwarp();  // every lane is done reading the previous chunk from the staging tile
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          uint4 v;
-          v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
-          v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
-          v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
-          v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
-          st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
-        }
-        __syncwarp();
-        const int n = n0 + c + 8 * cj;
-        if (n + 8 <= p.N) {
-          uint4 v[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int rr = rq + 4 * i;
-            ld_shared_v4(stg + rr * 128 + ((cj ^ (rr & 7)) << 4), v[i]);
+        for (int c = 0; c < BN; c += 64) {
+          uint32_t r[64];
+          tmem_ld16(tbase + c, r);
+          tmem_ld16(tbase + c + 16, r + 16);
+          tmem_ld16(tbase + c + 32, r + 32);
+          tmem_ld16(tbase + c + 48, r + 48);
+          tmem_ld_wait();
+          if (p.d_f32) f32_to_f16_lo<64>(r);  // FP32 accumulator: one rounding to FP16
+          if (c + 64 >= BN) {  // accumulator fully read: hand TMEM back before the stores
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
           }
-          if (p.out_mode == OUT_ACCUM) {
-            uint4 o[8];
+          __syncwarp();  // every lane is done reading the previous chunk from the staging tile
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-              o[i] = orow[i] ? *reinterpret_cast<const uint4*>(orow[i] + n) : make_uint4(0u, 0u, 0u, 0u);
+          for (int j = 0; j < 8; ++j) {
+            uint4 v;
+            v.x = pack_lo(r[j * 8 + 0], r[j * 8 + 1]);
+            v.y = pack_lo(r[j * 8 + 2], r[j * 8 + 3]);
+            v.z = pack_lo(r[j * 8 + 4], r[j * 8 + 5]);
+            v.w = pack_lo(r[j * 8 + 6], r[j * 8 + 7]);
+            st_shared_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), v);
+          }
+          __syncwarp();
+          const int n = n0 + c + 8 * cj;
+          if (n + 8 <= p.N) {
+            uint4 v[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-              v[i].x = hadd2_rn(o[i].x, v[i].x);
-              v[i].y = hadd2_rn(o[i].y, v[i].y);
-              v[i].z = hadd2_rn(o[i].z, v[i].z);
-              v[i].w = hadd2_rn(o[i].w, v[i].w);
+              const int rr = rq + 4 * i;
+              ld_shared_v4(stg + rr * 128 + ((cj ^ (rr & 7)) << 4), v[i]);
             }
-          }
+            if (p.out_mode == OUT_ACCUM) {
+              uint4 o[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            if (orow[i]) *reinterpret_cast<uint4*>(orow[i] + n) = v[i];
+              for (int i = 0; i < 8; ++i)
+                o[i] = orow[i] ? *reinterpret_cast<const uint4*>(orow[i] + n) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                v[i].x = hadd2_rn(o[i].x, v[i].x);
+                v[i].y = hadd2_rn(o[i].y, v[i].y);
+                v[i].z = hadd2_rn(o[i].z, v[i].z);
+                v[i].w = hadd2_rn(o[i].w, v[i].w);
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              if (orow[i]) *reinterpret_cast<uint4*>(orow[i] + n) = v[i];
+          }
         }
       }
       acc_phase ^= 1;
@@ -869,7 +930,7 @@ static cudaError_t set_smem_attr() {
   cudaGetDevice(&dev);
   if (dev < 64 && !attr_set[dev]) {
     cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI, XF, WE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF, WE>::SMEM);
+                                         GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD || EPI == EPI_BS_REMAP, XF, WE>::SMEM);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
@@ -882,7 +943,7 @@ static cudaError_t launch_variant(const CUtensorMap& mA, const CUtensorMap& mB, 
                                   cudaStream_t s) {
   cudaError_t e = set_smem_attr<BN, EPI, XF, WE>();
   if (e != cudaSuccess) return e;
-  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD, XF, WE>::SMEM;
+  constexpr int smem = GemmCfg<BN, EPI == EPI_BS_TMA || EPI == EPI_BS_ADD || EPI == EPI_BS_REMAP, XF, WE>::SMEM;
   launch_pdl(k_gemm<BN, EPI, XF, WE>, dim3(grid), dim3(XF ? kGemmThreadsXf : (WE ? kGemmThreadsWide : kGemmThreads)),
              smem, s, mA, mB, mC, mX, mD, p);
   return counted_launches(1);
@@ -893,7 +954,8 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
                                const CUtensorMap& mX, const CUtensorMap& mD, const GemmParams& p, int grid,
                                cudaStream_t s) {
   const int epi = gemm_epilogue(p);
-  if (epi != EPI_PLAIN && (!p.tma_store || p.out_mode != OUT_STORE)) return cudaErrorInvalidValue;
+  if (epi != EPI_PLAIN && p.out_mode != OUT_STORE) return cudaErrorInvalidValue;
+  if (epi != EPI_PLAIN && !p.tma_store && !(epi == EPI_BS_REMAP && p.remap)) return cudaErrorInvalidValue;
   if (p.xf_operand) {
     if (epi != EPI_PLAIN) return cudaErrorInvalidValue;
     return launch_variant<BN, EPI_PLAIN, true>(mA, mB, mC, mX, mD, p, grid, s);
@@ -911,6 +973,7 @@ static cudaError_t launch_bn_t(const CUtensorMap& mA, const CUtensorMap& mB, con
     case EPI_BS: return launch_variant<BN, EPI_BS>(mA, mB, mC, mX, mD, p, grid, s);
     case EPI_BS_TMA: return launch_variant<BN, EPI_BS_TMA>(mA, mB, mC, mX, mD, p, grid, s);
     case EPI_BS_ADD: return launch_variant<BN, EPI_BS_ADD>(mA, mB, mC, mX, mD, p, grid, s);
+    case EPI_BS_REMAP: return launch_variant<BN, EPI_BS_REMAP>(mA, mB, mC, mX, mD, p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

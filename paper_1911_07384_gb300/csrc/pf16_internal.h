@@ -193,11 +193,12 @@ __host__ __device__ inline size_t bnstat_bytes(long long C) {
 // K-blocks per tile: there the epilogue's traffic is the bound) and always
 // with an addend; else their inputs go through registers, which leaves the
 // main loop all of its pipeline stages.
-enum GemmEpi : int { EPI_PLAIN = 0, EPI_BS = 1, EPI_BS_TMA = 2, EPI_BS_ADD = 3 };
+enum GemmEpi : int { EPI_PLAIN = 0, EPI_BS = 1, EPI_BS_TMA = 2, EPI_BS_ADD = 3, EPI_BS_REMAP = 4 };
 constexpr int kTmaEpiMaxKb = 8;
 inline int gemm_epilogue(const GemmParams& p) {
   if (!p.bs_x) return EPI_PLAIN;
   if (p.add_src) return EPI_BS_ADD;
+  if (p.remap) return EPI_BS_REMAP;  // scattered rows: x by cp.async into the same double buffers
   return p.kb_per_split <= kTmaEpiMaxKb ? EPI_BS_TMA : EPI_BS;
 }
 

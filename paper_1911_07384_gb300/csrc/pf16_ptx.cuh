@@ -151,6 +151,17 @@ __device__ __forceinline__ void bulk_load_1d(uint32_t dst, const void* src, uint
       "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
       : "memory");
 }
+// 16 bytes global -> shared through L2 (cp.async), tracked by the thread's
+// async-copy state (addresses 16-byte aligned)
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(reinterpret_cast<uint64_t>(src))
+               : "memory");
+}
+// an arrival on the mbarrier once every cp.async this thread issued before has
+// landed; .noinc: the barrier's expected arrival count includes it
+__device__ __forceinline__ void cp_async_mbar_arrive_noinc(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
 __device__ __forceinline__ void ld_shared_v4(uint32_t addr, uint4& v) {
   asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)

@@ -108,9 +108,14 @@ class Conv:
         # twice the rate it keeps with the statistics epilogue, which is bound by the
         # latency of its per-element work, and the BatchNorm's own statistics pass
         # costs less than the difference)
+        # Stride-2 data gradients take them only where dx is large: at 56x56x128 (batch
+        # 256) the fused epilogue (160 us) undercuts the plain data gradient plus the
+        # BatchNorm's own statistics pass (115 + 74 us); at 28x28x256 the two are even
+        # and at 14x14x512 the separate pass is cheaper.
         d = self.desc
         halo64 = d.r == 3 and d.s == 3 and d.stride == 1 and d.c == 64 and d.k == 64
-        size = pf16.conv_dgrad_bnstats_size(d) if d.c != 3 and not halo64 else 0
+        small_strided = d.stride != 1 and d.n * d.h * d.w * d.c < (1 << 26)
+        size = pf16.conv_dgrad_bnstats_size(d) if d.c != 3 and not halo64 and not small_strided else 0
         self.dstats = torch.empty(size, dtype=torch.uint8, device=a.w.device) if size else None
 
     def fwd(self, x, y, with_stats=False, bn_in=None):
@@ -127,7 +132,7 @@ class Conv:
 
     def dgrad(self, dy, dx, accumulate=False, bn=None, add=None):
         """bn: (BN layer, its input x) when dx is that BatchNorm's output gradient and
-        this layer can take its backward statistics (stride 1); see BN.bwd(conv=).
+        this layer takes its backward statistics (see bind); see BN.bwd(conv=).
         add (with bn, 1x1 only): (tensor, bit mask) added to the data gradient where
         the mask's bit is set -- an identity shortcut's share of dx."""
         if bn is not None and add is not None:

@@ -71,10 +71,13 @@ def test_conv_validation_errors():
               None) == pf16.PF16_ERR_ALIGN
     nox = pf16.BnSource(None, None, FAKE, FAKE)
     assert dg(ctypes.byref(good), FAKE, FAKE, FAKE, None, 0, ctypes.byref(nox), FAKE, sz, None) == pf16.PF16_ERR_NULL
-    s2 = pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 2, 1)
-    assert pf16.conv_dgrad_bnstats_size(s2) == 0
-    assert dg(ctypes.byref(s2), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, sz,
-              None) == pf16.PF16_ERR_UNSUPPORTED
+    # stride 2: the four stride phases must share their grid (even sizes with 3x3 / pad 1)
+    assert pf16.conv_dgrad_bnstats_size(pf16.conv_desc(2, 8, 8, 64, 64, 3, 3, 2, 1)) == sz
+    for s2 in (pf16.conv_desc(2, 9, 9, 64, 64, 3, 3, 2, 1), pf16.conv_desc(2, 8, 9, 64, 64, 3, 3, 2, 1),
+               pf16.conv_desc(2, 8, 8, 64, 64, 1, 1, 2, 0)):
+        assert pf16.conv_dgrad_bnstats_size(s2) == 0
+        assert dg(ctypes.byref(s2), FAKE, FAKE, FAKE, None, 0, ctypes.byref(src), FAKE, sz,
+                  None) == pf16.PF16_ERR_UNSUPPORTED
     # ... plus a masked addend: 1x1 stride 1 only, no overlap with dx
     da = L.pf16_conv_dgrad_bnstats_add
     one = pf16.conv_desc(2, 8, 8, 256, 64, 1, 1, 1, 0)

@@ -97,6 +97,10 @@ BWD_SHAPES = [
     ((1, 7, 7, 64, 64, 3, 3, 1, 1), True),       # one partial tile (49 rows)
     ((2, 7, 7, 256, 1024, 1, 1, 1, 0), True),    # long reduction (16 K-blocks): register-fed epilogue
     ((4, 14, 14, 256, 128, 1, 1, 1, 0), True),   # short reduction, many tiles per CTA: TMA-fed epilogue
+    ((3, 14, 14, 128, 128, 3, 3, 2, 1), True),   # strided 3x3, even size: the four stride phases in one
+                                                 # launch, scattered rows, ragged last tile of each phase
+    ((2, 10, 12, 64, 64, 3, 3, 2, 1), False),    # the same with H != W and no ReLU
+    ((2, 14, 14, 512, 512, 3, 3, 2, 1), True),   # the same with two n-tiles
 ]
 
 
@@ -167,14 +171,19 @@ def check_bn_bwd_from_stats(orc, bd, bws, tx, tg, tm, ti, ty, tmask, dx, stats, 
     assert np.all(np.abs(f64(host(tdg)) - dgo) <= tol_g), float(np.max(np.abs(f64(host(tdg)) - dgo) / tol_g))
 
 
-def test_conv_dgrad_bnstats_rejects_strided():
-    d = pf16.conv_desc(2, 14, 14, 64, 64, 3, 3, 2, 1)
+@pytest.mark.parametrize("shape", [(2, 13, 13, 64, 64, 3, 3, 2, 1),    # odd size: unequal stride phases
+                                   (2, 14, 14, 64, 64, 1, 1, 2, 0)],   # strided 1x1: positions no tap reaches
+                         ids=ids)
+def test_conv_dgrad_bnstats_rejects_strided(shape):
+    N, H, W, C, K, R, S, st, pd = shape
+    P, Q = (H + 2 * pd - R) // st + 1, (W + 2 * pd - S) // st + 1
+    d = pf16.conv_desc(*shape)
     assert pf16.conv_dgrad_bnstats_size(d) == 0
     stats = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
-    t = empty16(2 * 14 * 14 * 64)
+    t = empty16(N * H * W * C)
     with pytest.raises(pf16.PF16Error):
-        pf16.conv_dgrad_bnstats(d, empty16(2 * 7 * 7 * 64), empty16(64 * 9 * 64), t, t, None, empty16(64),
-                                empty16(64), stats)
+        pf16.conv_dgrad_bnstats(d, empty16(N * P * Q * K), empty16(K * R * S * C), t, t, None, empty16(C),
+                                empty16(C), stats)
 
 
 ADD_SHAPES = [
