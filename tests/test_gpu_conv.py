@@ -268,6 +268,8 @@ F32_SHAPES = [
     (2, 28, 28, 64, 64, 3, 3, 1, 1),     # halo engine
     (2, 32, 32, 3, 64, 7, 7, 2, 3),      # stem: space-to-depth halo forward, stem weight gradient
     (2, 14, 14, 64, 256, 1, 1, 1, 0),    # dense 1x1
+    (2, 12, 12, 128, 128, 3, 3, 2, 1),   # strided 3x3: the four stride phases in one launch, scattered rows
+    (2, 9, 9, 64, 128, 3, 3, 2, 1),      # strided 3x3, odd size: one launch per phase
 ]
 
 
