@@ -1663,6 +1663,12 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+__device__ __forceinline__ uint32_t heq2_mask(uint32_t a, uint32_t b) {  // 0xFFFF per half where a == b
+  uint32_t d;
+  asm("set.eq.u32.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
 // Backward from the recorded positions.  Input cells (2i + a, 2j + b),
 // a, b in {0, 1}, are covered exactly by the windows p in {i, i+1}, q in
 // {j, j+1} (cell row 2i only by p = i, cell column 2j only by q = j), so one
@@ -1691,6 +1697,17 @@ __global__ void __launch_bounds__(512)
         cd[a][b] = ok ? __ldg(reinterpret_cast<const uint2*>(codes) + oi) : make_uint2(~0u, ~0u);
         g[a][b] = ok ? __ldg(reinterpret_cast<const uint4*>(dy) + oi) : make_uint4(0, 0, 0, 0);
       }
+    // each window's positions widened to one 16-bit lane per channel (word k:
+    // channels 2k, 2k + 1), compared as binary16 bit patterns: 0..8 and 0xFF
+    // are zero or subnormal, so f16x2 equality is equality of the codes
+    uint32_t cw16[2][2][4];
+#pragma unroll
+    for (int a = 0; a < 2; ++a)
+#pragma unroll
+      for (int b = 0; b < 2; ++b)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          cw16[a][b][k] = __byte_perm(k < 2 ? cd[a][b].x : cd[a][b].y, 0u, (k & 1) ? 0x4342 : 0x4140);
 #pragma unroll
     for (int ch = 0; ch < 2; ++ch) {
       const int h = 2 * i + ch;
@@ -1706,15 +1723,13 @@ __global__ void __launch_bounds__(512)
 #pragma unroll
           for (int b = 0; b < 2; ++b) {
             if (b > cw) break;
-            // the cell's position in window (i + a, j + b), in every byte: row
-            // ch - 2a + 1, column cw - 2b + 1; the bytes of the window's
-            // positions that match it, spread to the halves of each 2-channel word
-            const uint32_t mine = (uint32_t)((ch - 2 * a + 1) * 3 + (cw - 2 * b + 1)) * 0x01010101u;
-            const uint32_t mx = __vcmpeq4(cd[a][b].x, mine), my = __vcmpeq4(cd[a][b].y, mine);
+            // the cell's position in window (i + a, j + b): row ch - 2a + 1,
+            // column cw - 2b + 1, in both halves
+            const uint32_t mine = (uint32_t)((ch - 2 * a + 1) * 3 + (cw - 2 * b + 1)) * 0x00010001u;
             const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g[a][b]);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-              const uint32_t sel = __byte_perm(k < 2 ? mx : my, 0u, (k & 1) ? 0x3322 : 0x1100);
+              const uint32_t sel = heq2_mask(cw16[a][b][k], mine);
               if (sel) acc[k] = hadd2_rn(acc[k], gw[k] & sel);
             }
           }
