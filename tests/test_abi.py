@@ -154,3 +154,22 @@ def test_wait_flag_validation_errors():
     assert L.pf16_wait_flag(None, 1, 1000, None) == pf16.PF16_ERR_NULL
     assert L.pf16_wait_flag(FAKE_MIS, 1, 1000, None) == pf16.PF16_ERR_ALIGN
     assert L.pf16_wait_flag(FAKE, 1, 10_000_000_001, None) == pf16.PF16_ERR_ARG
+
+
+def test_launch_plan_agrees_with_the_library():
+    """bench.py counts one data-gradient launch for a stride-2 filter when the
+    library runs its four stride phases as one GEMM -- exactly the layers for
+    which the library also offers the fused backward statistics."""
+    import bench
+
+    seen = set()
+    for h, w in [(8, 8), (9, 9), (12, 10), (13, 14), (56, 56), (7, 7)]:
+        for r in (1, 3, 5, 7):
+            for pad in range(r):
+                if (h + 2 * pad - r) < 0 or (w + 2 * pad - r) < 0:
+                    continue
+                d = pf16.conv_desc(2, h, w, 64, 64, r, r, 2, pad)
+                one = bench.one_phase_launch(d)
+                assert one == (pf16.conv_dgrad_bnstats_size(d) > 0), (h, w, r, pad)
+                seen.add(one)
+    assert seen == {True, False}
