@@ -1924,28 +1924,42 @@ __global__ void __launch_bounds__(256)
   const uint4 is = __ldg(reinterpret_cast<const uint4*>(invstd) + cg);
   const uint4 ga = __ldg(reinterpret_cast<const uint4*>(gamma) + cg);
   const uint4 be = __ldg(reinterpret_cast<const uint4*>(beta) + cg);
+  // two staged rows at a time, four cells of each: eight loads in flight before any use
 #pragma unroll 1
-  for (int rho = 0; rho < 2 * kBpT + 1; ++rho) {
-    const int h = 2 * p0 - 1 + rho;
-    if (h < 0 || h >= H) continue;
-    const long long rowoff = ((long long)n * H + h) * W * tc + cg;
-    uint4* zrow = zs + (rho * W) * tc + cg;
+  for (int rho0 = 0; rho0 < 2 * kBpT + 1; rho0 += 2) {
+    bool rv[2];
+    long long rowoff[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int h = 2 * p0 - 1 + rho0 + e;
+      rv[e] = rho0 + e < 2 * kBpT + 1 && h >= 0 && h < H;
+      rowoff[e] = ((long long)n * H + (rv[e] ? h : 0)) * W * tc + cg;
+    }
     for (int w0 = c0; w0 < W; w0 += 4 * cstep) {
-      uint4 xv[4];
+      uint4 xv[2][4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {  // four cells' loads in flight before any use
-        const int w = w0 + k * cstep;
-        xv[k] = w < W ? __ldg(reinterpret_cast<const uint4*>(x) + rowoff + (long long)w * tc) : zero4();
-      }
+      for (int e = 0; e < 2; ++e)
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int w = w0 + k * cstep;
-        if (w >= W) break;
-        const uint4 xh = mul4v(sub4(xv[k], mu), is);  // Eq. 1
-        uint32_t bits;
-        const uint4 z = relu_bits(mul4(add4(mul4v(ga, xh), be), ps), bits);  // Eq. 2, ReLU
-        zrow[w * tc] = z;
-        if (rho >= 1 && mask) mask[rowoff + (long long)w * tc] = (uint8_t)bits;  // rows 2 p0 .. are this CTA's
+        for (int k = 0; k < 4; ++k) {
+          const int w = w0 + k * cstep;
+          xv[e][k] = (rv[e] && w < W) ? __ldg(reinterpret_cast<const uint4*>(x) + rowoff[e] + (long long)w * tc)
+                                      : zero4();
+        }
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        if (!rv[e]) continue;
+        const int rho = rho0 + e;
+        uint4* zrow = zs + (rho * W) * tc + cg;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int w = w0 + k * cstep;
+          if (w >= W) break;
+          const uint4 xh = mul4v(sub4(xv[e][k], mu), is);  // Eq. 1
+          uint32_t bits;
+          const uint4 z = relu_bits(mul4(add4(mul4v(ga, xh), be), ps), bits);  // Eq. 2, ReLU
+          zrow[w * tc] = z;
+          if (rho >= 1 && mask) mask[rowoff[e] + (long long)w * tc] = (uint8_t)bits;  // rows 2 p0 .. are this CTA's
+        }
       }
     }
   }
